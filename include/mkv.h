@@ -1,0 +1,241 @@
+/*
+ * mkv.h -- C ABI of the MomentKV hot path on one GB300 (sm_103a).
+ *
+ * MomentKV (arXiv 2606.01563) keeps, for every attention head, a summary of
+ * the KV pairs evicted from the cache -- the count n, key mean mu_k, value
+ * mean mu_v and value-key cross-covariance C -- and uses it twice: to choose
+ * which tokens to evict (moment residual, Eq. residual) and to add back a
+ * closed-form first-order estimate of the evicted tokens' attention output
+ * (Eqs. fhat, jensen, fused).  Three calls cover the data-parallel path:
+ *
+ *   mkv_compress      prefill: window scores, budget top-k, moment filter,
+ *                     evicted-set moments                    (Sec. 5.1, 4.2)
+ *   mkv_decode_step   attention over the retained cache merged with the
+ *                     moment term in one normaliser     (Algorithm 1 Phase 2)
+ *   mkv_evict_append  append a token and evict one at a time down to the
+ *                     budget by the moment-informed score (Algorithm 1 Phase 1)
+ *
+ * Conventions shared by every call
+ *  - Pointers are DEVICE pointers unless a comment says otherwise; the
+ *    caller allocates and owns every buffer.  The library never allocates or
+ *    frees device memory.
+ *  - bf16 tensors are IEEE bfloat16 stored as 16-bit words; fp32 is IEEE
+ *    binary32.  All tensors are dense, row-major, with the shapes given.
+ *  - Index conventions: b batch, h_kv KV head, g = group (query heads per KV
+ *    head), query head j uses KV head j / g, d = head_dim in {64, 128},
+ *    scale = 1/sqrt(d).  A "unit" is one (batch, KV head) pair.
+ *  - Calls are asynchronous and ordered on `stream` (a cudaStream_t; NULL is
+ *    the legacy default stream).  Host-side validation failures return an
+ *    error and launch nothing.  Errors the kernels detect (capacity overflow
+ *    on append, empty attention, a bounded wait that ran out) are written to
+ *    an error word inside the workspace and read by mkv_get_device_error.
+ *  - A workspace serves one stream at a time; two calls that overlap on the
+ *    GPU must not share one.
+ */
+#ifndef MKV_H
+#define MKV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define MKV_API __attribute__((visibility("default")))
+#else
+#define MKV_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  MKV_OK = 0,
+  MKV_ERR_INVALID_ARG = 1, /* null pointer, bad parameter, empty attention  */
+  MKV_ERR_SHAPE = 2,       /* unsupported or inconsistent sizes             */
+  MKV_ERR_CAPACITY = 3,    /* cache capacity too small                      */
+  MKV_ERR_CUDA = 4,        /* a CUDA runtime call failed                    */
+  MKV_ERR_TIMEOUT = 5,     /* a bounded device-side wait ran out            */
+  MKV_ERR_UNSUPPORTED = 6, /* head_dim or group outside the built kernels   */
+  MKV_ERR_WORKSPACE = 7    /* workspace missing, too small or misaligned    */
+} mkv_status;
+
+/* Attention geometry of one layer.  head_dim in {64, 128}; group in {1,2,4,8}. */
+typedef struct {
+  int32_t batch;
+  int32_t n_kv_heads;
+  int32_t group;
+  int32_t head_dim;
+} mkv_geom;
+
+/*
+ * Evicted-set moments, one set per unit (Sec. 4.1, App. A.1).
+ *   n    int32 [b, h_kv]          number of evicted tokens n_e
+ *   mu_k fp32  [b, h_kv, d]       key mean    k_bar = s_k / n_e
+ *   mu_v fp32  [b, h_kv, d]       value mean  v_bar = s_v / n_e
+ *   C    fp32  [b, h_kv, d, d]    C[a][c] = S_tilde[a][c] / n_e with
+ *                                 S_tilde = sum_E v (k - k_bar)^T (Eq. app_S_tilde):
+ *                                 row a indexes value dims, column c key dims.
+ * n = 0 means "no evicted token" (the other fields are then ignored); a
+ * zero-filled struct is the state at the start of a generation (Sec. 5.1).
+ */
+typedef struct {
+  int32_t* n;
+  float* mu_k;
+  float* mu_v;
+  float* C;
+} mkv_moments;
+
+/*
+ * Retained KV cache, one slab per unit.
+ *   K, V  bf16  [b, h_kv, capacity, d]   rows 0..len-1 are in use
+ *   pos   int32 [b, h_kv, capacity]      absolute position of each row; rows
+ *                                        are kept in ascending position order
+ *   len   int32 [b, h_kv]                rows in use
+ *   seen  int32 [b, h_kv]                tokens seen so far; an appended token
+ *                                        takes position `seen`, then seen += 1
+ */
+typedef struct {
+  void* K;
+  void* V;
+  int32_t* pos;
+  int32_t* len;
+  int32_t* seen;
+  int32_t capacity;
+} mkv_cache;
+
+/* Prefill compression parameters (SnapKV protocol of Sec. 5.1 plus the
+ * moment filter of Sec. 4.2). */
+typedef struct {
+  int32_t budget;      /* L: rows kept per unit (includes sink and window)   */
+  int32_t window;      /* w: observation window = the last w positions        */
+  int32_t sink;        /* leading positions always kept (the paper keeps 1)   */
+  int32_t keep_window; /* 1: the w window positions are always kept           */
+  int32_t pool;        /* adjacent-token chunk size for scores, 1 = off (Sec. 5.1 uses 4) */
+  int32_t mi;          /* 1: moment-informed second stage; 0: window scores only */
+  int32_t causal;      /* 1: window query i (position T-w+i) sees keys t <= T-w+i */
+  float tau;           /* clamp |S_tilde_ab| < tau to 0 in the residual (App. C.2) */
+} mkv_compress_params;
+
+/* Optional outputs of mkv_compress for inspection; any field may be NULL. */
+typedef struct {
+  float* scores;       /* fp32 [b, h_kv, T] pooled window scores s_t               */
+  float* score2;       /* fp32 [b, h_kv, T] s_t * ||r_t|| (mi=1); protected rows 0 */
+  int32_t* idx_stage1; /* int32 [b, h_kv, budget] first-stage retained positions    */
+} mkv_compress_diag;
+
+/* Decode parameters (Algorithm 1 Phase 2, Table 4, App. C.2). */
+typedef struct {
+  int32_t correction; /* 1: merge the moment term; 0: plain attention over R   */
+  int32_t order;      /* 1: f_hat_E = v_bar + S_tilde q/(n sqrt d); 0: v_bar only */
+  float tau;          /* clamp |S_tilde_ab| < tau to 0 before S_tilde q         */
+} mkv_decode_params;
+
+/* Human-readable name of a status code (static string). */
+MKV_API const char* mkv_status_str(mkv_status s);
+
+/* Library ABI version (major * 10000 + minor * 100 + patch). */
+MKV_API int32_t mkv_version(void);
+
+/*
+ * Bytes of device workspace mkv_compress needs for this geometry and T.
+ * Returns 0 if the arguments are invalid.  The workspace needs no
+ * initialisation.
+ */
+MKV_API size_t mkv_compress_workspace_size(mkv_geom geom, int32_t T, const mkv_compress_params* p);
+
+/*
+ * Prefill compression of one layer (Sec. 5.1 protocol, Sec. 4.2 moments).
+ *   K, V   bf16 [b, h_kv, T, d]       keys and values of the whole prompt
+ *   Q_obs  bf16 [b, h_kv, g, w, d]    the last w queries of each query head
+ * Per unit:
+ *   1. logits l_{h,i,t} = scale q_{h,i} . k_t over the g*w window rows
+ *      (causal: row i sees t <= T-w+i); s_t = sum over rows of softmax; pooled
+ *      into aligned chunks of `pool` tokens.
+ *   2. R0 = protected (sink, and the window if keep_window) plus the
+ *      budget-|protected| highest s_t; ties keep the lower position.
+ *   3. if mi: moments M0 of E0 = all \ R0; r_t = v_t - mu_v0 - scale C0' k_t
+ *      with C0' = C0 clamped where |n0 C0| < tau (Eq. residual); score2 =
+ *      s_t ||r_t||; R = protected plus the top of score2, same tie rule.
+ *      if !mi: R = R0.
+ *   4. writes the retained rows of R to out_cache in ascending position
+ *      (K, V, pos), len = |R|, seen = T, and the moments of E = all \ R to
+ *      out_mom (overwritten).  If T <= budget every token is kept and n = 0.
+ * Requirements: budget >= sink + (keep_window ? w : 0), 1 <= w <= T,
+ * out_cache->capacity >= min(T, budget), T <= 1,048,576.
+ */
+MKV_API mkv_status mkv_compress(mkv_geom geom, int32_t T, const void* K, const void* V, const void* Q_obs,
+                        const mkv_compress_params* p, const mkv_cache* out_cache,
+                        const mkv_moments* out_mom, const mkv_compress_diag* diag,
+                        void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * Bytes of device workspace mkv_decode_step needs for this geometry and cache
+ * capacity on the current device.  Returns 0 if the arguments are invalid.
+ * The workspace must be zero-filled before its first use; every call leaves
+ * it ready for the next one.
+ */
+MKV_API size_t mkv_decode_workspace_size(mkv_geom geom, int32_t capacity);
+
+/*
+ * One decode step for every unit (Algorithm 1: append, then Phase 2).
+ *   q             bf16 [b, g*h_kv, d]   this step's queries
+ *   k_new, v_new  bf16 [b, h_kv, d]     optional (both NULL or both set): the
+ *                                       new token is appended at row len with
+ *                                       position seen before attending.
+ *   out           fp32 [b, g*h_kv, d]   corrected output f_hat(q) (Eq. fused)
+ *   lse           fp32 [b, g*h_kv]      optional: natural log of the merged
+ *                                       normaliser, log(Z_R + Z_hat_E), or log
+ *                                       Z_R when no correction applies.
+ * For each query head: (m_R, l_R, o_R) over the retained rows; if
+ * correction && n > 0: log Z_hat_E = log n + scale q.mu_k (Eq. jensen),
+ * f_hat_E = mu_v + scale C' q (order 1, C' clamped as in mkv_compress) or
+ * mu_v (order 0), w_R from a log-sum-exp of log Z_R and log Z_hat_E
+ * (App. C.2), out = w_R o_R + (1 - w_R) f_hat_E.  With no retained row the
+ * output is f_hat_E; with neither rows nor moments the kernel records
+ * MKV_ERR_INVALID_ARG and writes zeros.  An append past capacity records
+ * MKV_ERR_CAPACITY, still attends over the new token, and leaves the cache
+ * unchanged.
+ */
+MKV_API mkv_status mkv_decode_step(mkv_geom geom, const void* q, const void* k_new, const void* v_new,
+                           const mkv_cache* cache, const mkv_moments* mom,
+                           const mkv_decode_params* p, float* out, float* lse,
+                           void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * Bytes of device workspace mkv_evict_append needs.  Returns 0 if invalid.
+ * The workspace needs no initialisation.
+ */
+MKV_API size_t mkv_evict_workspace_size(mkv_geom geom, int32_t capacity);
+
+/*
+ * Algorithm 1's append step and Phase 1 for every unit.
+ *   q             bf16 [b, g*h_kv, d]   queries whose attention weights score
+ *                                       the rows (alpha_j summed over the g
+ *                                       query heads of the unit)
+ *   k_new, v_new  bf16 [b, h_kv, d]     optional token appended first
+ * Then, while len > budget: recover v_bar and S_tilde = n C from the moments
+ * (zero if n = 0), clamp |S_tilde_ab| < tau to 0, alpha = sum over the group
+ * of softmax(scale q . k_j) over the current rows, r_j = v_j - v_bar -
+ * S_tilde k_j / (n sqrt d), score_j = alpha_j ||r_j||, evict the row with
+ * the smallest score (ties: the lower position), fold it into the moments
+ * (n+1; the equivalent of Eq. app_update on (n, mu_k, mu_v, C)) and remove
+ * it.  Surviving rows keep their ascending position order.
+ * Requirements: 0 <= budget, len + (k_new ? 1 : 0) <= capacity (else the
+ * kernel records MKV_ERR_CAPACITY and leaves the unit unchanged).
+ */
+MKV_API mkv_status mkv_evict_append(mkv_geom geom, const void* q, const void* k_new, const void* v_new,
+                            int32_t budget, const mkv_cache* cache, const mkv_moments* mom,
+                            float tau, void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * Synchronises `stream`, returns the first error a kernel recorded in this
+ * workspace since the last call (MKV_OK if none) and clears it.  `info`
+ * (host pointer, may be NULL) receives a detail word (e.g. the unit index).
+ */
+MKV_API mkv_status mkv_get_device_error(void* workspace, void* stream, int32_t* info);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MKV_H */

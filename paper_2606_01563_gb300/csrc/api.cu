@@ -1,0 +1,224 @@
+// C-ABI entry points declared in include/mkv.h: argument validation,
+// workspace sizing and kernel dispatch.  No allocation, no global state
+// beyond a per-device cache of the SM count.
+#include <cuda_runtime.h>
+
+#include "common.cuh"
+#include "kernels.h"
+
+using namespace mkv;
+
+namespace {
+
+int num_sms_current() {
+  static int cache[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 148;
+  if (dev >= 0 && dev < 64 && cache[dev] > 0) return cache[dev];
+  int n = 0;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
+  if (dev >= 0 && dev < 64) cache[dev] = n;
+  return n;
+}
+
+bool geom_ok(const mkv_geom& g) {
+  return g.batch >= 1 && g.n_kv_heads >= 1 && (g.head_dim == 64 || g.head_dim == 128) &&
+         (g.group == 1 || g.group == 2 || g.group == 4 || g.group == 8) &&
+         (long)g.batch * g.n_kv_heads <= 65535L * 64;
+}
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+bool cache_ok(const mkv_cache* c) {
+  return c && c->K && c->V && c->pos && c->len && c->seen && c->capacity >= 1 && aligned(c->K, 16) &&
+         aligned(c->V, 16);
+}
+
+bool moments_ok(const mkv_moments* m) {
+  return m && m->n && m->mu_k && m->mu_v && m->C && aligned(m->C, 16) && aligned(m->mu_k, 4) &&
+         aligned(m->mu_v, 4);
+}
+
+int protected_count_host(int T, int W, int sink, int keep_window) {
+  const int s = sink < T ? sink : T;
+  const int w = keep_window ? (W < T ? W : T) : 0;
+  const int overlap = s - (T - w) > 0 ? s - (T - w) : 0;
+  return s + w - overlap;
+}
+
+mkv_status cuda_status(cudaError_t e) { return e == cudaSuccess ? MKV_OK : MKV_ERR_CUDA; }
+
+}  // namespace
+
+extern "C" {
+
+const char* mkv_status_str(mkv_status s) {
+  switch (s) {
+    case MKV_OK: return "ok";
+    case MKV_ERR_INVALID_ARG: return "invalid argument";
+    case MKV_ERR_SHAPE: return "unsupported or inconsistent shape";
+    case MKV_ERR_CAPACITY: return "cache capacity exceeded";
+    case MKV_ERR_CUDA: return "CUDA runtime error";
+    case MKV_ERR_TIMEOUT: return "device-side wait timed out";
+    case MKV_ERR_UNSUPPORTED: return "unsupported head_dim or group";
+    case MKV_ERR_WORKSPACE: return "workspace missing, too small or misaligned";
+  }
+  return "unknown status";
+}
+
+int32_t mkv_version(void) { return 100; }
+
+// ------------------------------------------------------------------ decode
+size_t mkv_decode_workspace_size(mkv_geom geom, int32_t capacity) {
+  if (!geom_ok(geom) || capacity < 1) return 0;
+  return decode_workspace_bytes(geom, capacity, num_sms_current());
+}
+
+mkv_status mkv_decode_step(mkv_geom geom, const void* q, const void* k_new, const void* v_new,
+                           const mkv_cache* cache, const mkv_moments* mom, const mkv_decode_params* p,
+                           float* out, float* lse, void* workspace, size_t workspace_bytes, void* stream) {
+  if (!geom_ok(geom)) return (geom.head_dim == 64 || geom.head_dim == 128) ? MKV_ERR_SHAPE : MKV_ERR_UNSUPPORTED;
+  if (!q || !out || !p || !cache_ok(cache)) return MKV_ERR_INVALID_ARG;
+  if ((k_new == nullptr) != (v_new == nullptr)) return MKV_ERR_INVALID_ARG;
+  if (p->correction != 0 && p->correction != 1) return MKV_ERR_INVALID_ARG;
+  if (p->order != 0 && p->order != 1) return MKV_ERR_INVALID_ARG;
+  if (p->correction && !moments_ok(mom)) return MKV_ERR_INVALID_ARG;
+  if (!(p->tau >= 0.f)) return MKV_ERR_INVALID_ARG;
+  const int sms = num_sms_current();
+  const size_t need = decode_workspace_bytes(geom, cache->capacity, sms);
+  if (!workspace || workspace_bytes < need || !aligned(workspace, 256)) return MKV_ERR_WORKSPACE;
+  DecodeArgs a{};
+  a.q = q;
+  a.k_new = k_new;
+  a.v_new = v_new;
+  a.K = cache->K;
+  a.V = cache->V;
+  a.pos = cache->pos;
+  a.len = cache->len;
+  a.seen = cache->seen;
+  a.cap = cache->capacity;
+  a.n = p->correction ? mom->n : nullptr;
+  a.mu_k = p->correction ? mom->mu_k : nullptr;
+  a.mu_v = p->correction ? mom->mu_v : nullptr;
+  a.C = p->correction ? mom->C : nullptr;
+  a.correction = p->correction;
+  a.order = p->order;
+  a.tau = p->tau;
+  a.out = out;
+  a.lse = lse;
+  a.batch = geom.batch;
+  a.n_kv = geom.n_kv_heads;
+  decode_carve(a, geom, cache->capacity, sms, workspace);
+  return cuda_status(launch_decode(a, geom.head_dim, geom.group, static_cast<cudaStream_t>(stream)));
+}
+
+// ------------------------------------------------------------------- evict
+size_t mkv_evict_workspace_size(mkv_geom geom, int32_t capacity) {
+  if (!geom_ok(geom) || capacity < 1 || capacity > 65536) return 0;
+  return evict_workspace_bytes(geom, capacity);
+}
+
+mkv_status mkv_evict_append(mkv_geom geom, const void* q, const void* k_new, const void* v_new, int32_t budget,
+                            const mkv_cache* cache, const mkv_moments* mom, float tau, void* workspace,
+                            size_t workspace_bytes, void* stream) {
+  if (!geom_ok(geom)) return (geom.head_dim == 64 || geom.head_dim == 128) ? MKV_ERR_SHAPE : MKV_ERR_UNSUPPORTED;
+  if (!q || !cache_ok(cache) || !moments_ok(mom) || budget < 0 || !(tau >= 0.f)) return MKV_ERR_INVALID_ARG;
+  if ((k_new == nullptr) != (v_new == nullptr)) return MKV_ERR_INVALID_ARG;
+  if (cache->capacity > 65536) return MKV_ERR_SHAPE;
+  const size_t need = evict_workspace_bytes(geom, cache->capacity);
+  if (!workspace || workspace_bytes < need || !aligned(workspace, 256)) return MKV_ERR_WORKSPACE;
+  EvictArgs a{};
+  a.q = q;
+  a.k_new = k_new;
+  a.v_new = v_new;
+  a.K = cache->K;
+  a.V = cache->V;
+  a.pos = cache->pos;
+  a.len = cache->len;
+  a.seen = cache->seen;
+  a.cap = cache->capacity;
+  a.n = mom->n;
+  a.mu_k = mom->mu_k;
+  a.mu_v = mom->mu_v;
+  a.C = mom->C;
+  a.budget = budget;
+  a.tau = tau;
+  a.batch = geom.batch;
+  a.n_kv = geom.n_kv_heads;
+  evict_carve(a, geom, cache->capacity, workspace);
+  return cuda_status(launch_evict(a, geom.head_dim, geom.group, static_cast<cudaStream_t>(stream)));
+}
+
+// ---------------------------------------------------------------- compress
+static mkv_status compress_params_ok(const mkv_geom& geom, int32_t T, const mkv_compress_params* p) {
+  if (!geom_ok(geom)) return (geom.head_dim == 64 || geom.head_dim == 128) ? MKV_ERR_SHAPE : MKV_ERR_UNSUPPORTED;
+  if (!p || T < 1 || T > (1 << 20) || p->budget < 1 || p->window < 1 || p->window > T || p->sink < 0)
+    return MKV_ERR_INVALID_ARG;
+  if ((p->keep_window != 0 && p->keep_window != 1) || (p->mi != 0 && p->mi != 1) ||
+      (p->causal != 0 && p->causal != 1) || !(p->tau >= 0.f))
+    return MKV_ERR_INVALID_ARG;
+  if (!(p->pool == 1 || p->pool == 2 || p->pool == 4 || p->pool == 8 || p->pool == 16 || p->pool == 32))
+    return MKV_ERR_INVALID_ARG;
+  if ((long)geom.group * p->window > 1024) return MKV_ERR_SHAPE;
+  if (T > p->budget && protected_count_host(T, p->window, p->sink, p->keep_window) > p->budget)
+    return MKV_ERR_INVALID_ARG;
+  return MKV_OK;
+}
+
+size_t mkv_compress_workspace_size(mkv_geom geom, int32_t T, const mkv_compress_params* p) {
+  if (compress_params_ok(geom, T, p) != MKV_OK) return 0;
+  return compress_workspace_bytes(geom, T, *p, num_sms_current());
+}
+
+mkv_status mkv_compress(mkv_geom geom, int32_t T, const void* K, const void* V, const void* Q_obs,
+                        const mkv_compress_params* p, const mkv_cache* out_cache, const mkv_moments* out_mom,
+                        const mkv_compress_diag* diag, void* workspace, size_t workspace_bytes, void* stream) {
+  mkv_status st = compress_params_ok(geom, T, p);
+  if (st != MKV_OK) return st;
+  if (!K || !V || !Q_obs || !cache_ok(out_cache) || !moments_ok(out_mom)) return MKV_ERR_INVALID_ARG;
+  if (!aligned(K, 16) || !aligned(V, 16) || !aligned(Q_obs, 16)) return MKV_ERR_INVALID_ARG;
+  const int32_t keep = T < p->budget ? T : p->budget;
+  if (out_cache->capacity < keep) return MKV_ERR_CAPACITY;
+  const int sms = num_sms_current();
+  const size_t need = compress_workspace_bytes(geom, T, *p, sms);
+  if (!workspace || workspace_bytes < need || !aligned(workspace, 256)) return MKV_ERR_WORKSPACE;
+  CompressArgs a{};
+  a.K = K;
+  a.V = V;
+  a.Q = Q_obs;
+  a.T = T;
+  a.budget = p->budget;
+  a.window = p->window;
+  a.sink = p->sink;
+  a.keep_window = p->keep_window;
+  a.pool = p->pool;
+  a.mi = p->mi;
+  a.causal = p->causal;
+  a.tau = p->tau;
+  a.cache = *out_cache;
+  a.mom = *out_mom;
+  a.diag_scores = diag ? diag->scores : nullptr;
+  a.diag_score2 = diag ? diag->score2 : nullptr;
+  a.diag_idx1 = diag ? diag->idx_stage1 : nullptr;
+  a.ws = workspace;
+  a.batch = geom.batch;
+  a.n_kv = geom.n_kv_heads;
+  return cuda_status(launch_compress(a, geom, workspace_bytes, sms, static_cast<cudaStream_t>(stream)));
+}
+
+// ------------------------------------------------------------------ errors
+mkv_status mkv_get_device_error(void* workspace, void* stream, int32_t* info) {
+  if (!workspace) return MKV_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  ErrorWord w{};
+  if (cudaMemcpyAsync(&w, workspace, sizeof(w), cudaMemcpyDeviceToHost, s) != cudaSuccess) return MKV_ERR_CUDA;
+  if (cudaStreamSynchronize(s) != cudaSuccess) return MKV_ERR_CUDA;
+  if (w.code != 0) {
+    if (cudaMemsetAsync(workspace, 0, sizeof(w), s) != cudaSuccess) return MKV_ERR_CUDA;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return MKV_ERR_CUDA;
+  }
+  if (info) *info = w.info;
+  return static_cast<mkv_status>(w.code);
+}
+
+}  // extern "C"

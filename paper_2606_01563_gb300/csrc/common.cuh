@@ -1,0 +1,139 @@
+// Shared device helpers for the MomentKV kernels (sm_103a).
+//
+// Every workspace starts with a 256-byte header holding the device error
+// word: [0] status code (first error wins), [1] detail word.  Kernels record
+// into it instead of trapping; mkv_get_device_error reads and clears it.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/mkv.h"
+
+namespace mkv {
+
+constexpr size_t kHeaderBytes = 256;
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
+// Upper bound on polls of one mbarrier phase before a wait gives up.  Each
+// poll is a try_wait that may itself suspend for a while, so this is well
+// over a second -- far beyond any legitimate copy latency.
+constexpr uint32_t kMaxPolls = 1u << 22;
+
+struct ErrorWord {
+  uint32_t code;
+  int32_t info;
+};
+
+__device__ __forceinline__ void record_error(void* ws, uint32_t code, int32_t info) {
+  ErrorWord* e = reinterpret_cast<ErrorWord*>(ws);
+  if (atomicCAS(&e->code, 0u, code) == 0u) {
+    atomicExch(reinterpret_cast<int*>(&e->info), info);
+  }
+}
+
+__host__ __device__ __forceinline__ size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// ---------------------------------------------------------------- mbarrier
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_fence_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_addr(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Bounded wait on one phase; returns false if it gave up.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+  for (uint32_t i = 0; i < kMaxPolls; ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+  }
+  return false;
+}
+
+// ------------------------------------------------------- bulk async copies
+// 1-D bulk copy global -> shared completing on an mbarrier (TMA engine).
+// dst, src 16-byte aligned; bytes a multiple of 16.
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          smem_addr(dst)),
+      "l"(src), "r"(bytes), "r"(smem_addr(bar))
+      : "memory");
+}
+
+// ----------------------------------------------------------------- numeric
+__device__ __forceinline__ float fast_exp2(float x) { return exp2f(x); }
+
+// Order-preserving map of a float to uint32 (larger float -> larger key).
+__device__ __forceinline__ uint32_t float_key(float f) {
+  uint32_t u = __float_as_uint(f);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+// Load N consecutive bf16 as floats (N in {2, 4, 8}); p must be aligned to 2N bytes.
+template <int N>
+__device__ __forceinline__ void load_bf16(const __nv_bfloat16* p, float* out) {
+  if constexpr (N == 2) {
+    __nv_bfloat162 v = *reinterpret_cast<const __nv_bfloat162*>(p);
+    out[0] = __low2float(v);
+    out[1] = __high2float(v);
+  } else if constexpr (N == 4) {
+    uint2 raw = *reinterpret_cast<const uint2*>(p);
+    __nv_bfloat162 a = *reinterpret_cast<__nv_bfloat162*>(&raw.x);
+    __nv_bfloat162 b = *reinterpret_cast<__nv_bfloat162*>(&raw.y);
+    out[0] = __low2float(a);
+    out[1] = __high2float(a);
+    out[2] = __low2float(b);
+    out[3] = __high2float(b);
+  } else {
+    uint4 raw = *reinterpret_cast<const uint4*>(p);
+    const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      __nv_bfloat162 v = *reinterpret_cast<const __nv_bfloat162*>(&w[i]);
+      out[2 * i] = __low2float(v);
+      out[2 * i + 1] = __high2float(v);
+    }
+  }
+}
+
+}  // namespace mkv

@@ -1,0 +1,105 @@
+// Internal launcher interface between the C-ABI layer (api.cu) and the kernels.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "../../include/mkv.h"
+
+namespace mkv {
+
+// ------------------------------------------------------------------ decode
+struct DecodeArgs {
+  const void* q;      // bf16 [b, Hkv*G, D]
+  const void* k_new;  // bf16 [b, Hkv, D] or null
+  const void* v_new;
+  void* K;            // bf16 [b, Hkv, cap, D]
+  void* V;
+  int32_t* pos;
+  int32_t* len;
+  int32_t* seen;
+  int32_t cap;
+  const int32_t* n;
+  const float* mu_k;
+  const float* mu_v;
+  const float* C;
+  int32_t correction;
+  int32_t order;
+  float tau;
+  float* out;
+  float* lse;
+  void* ws;            // workspace header (error word)
+  uint32_t* counters;  // [units]
+  float* partial;      // [units][S][G][D+4]
+  float* fhat;         // [units][G][D]
+  int32_t batch;
+  int32_t n_kv;
+  int32_t S;
+};
+
+constexpr int kDecodeTile = 32;  // tokens per pipeline stage
+
+int decode_splits(const mkv_geom& g, int32_t capacity, int num_sms);
+size_t decode_workspace_bytes(const mkv_geom& g, int32_t capacity, int num_sms);
+// Carves the workspace and fills the ws/counters/partial/fhat fields.
+void decode_carve(DecodeArgs& a, const mkv_geom& g, int32_t capacity, int num_sms, void* ws);
+cudaError_t launch_decode(const DecodeArgs& a, int head_dim, int group, cudaStream_t stream);
+
+// ------------------------------------------------------------------- evict
+struct EvictArgs {
+  const void* q;      // bf16 [b, Hkv*G, D]
+  const void* k_new;  // bf16 [b, Hkv, D] or null
+  const void* v_new;
+  void* K;
+  void* V;
+  int32_t* pos;
+  int32_t* len;
+  int32_t* seen;
+  int32_t cap;
+  int32_t* n;
+  float* mu_k;
+  float* mu_v;
+  float* C;
+  int32_t budget;
+  float tau;
+  void* ws;
+  float* scratch;  // [units][cap] logits / scores
+  int32_t batch;
+  int32_t n_kv;
+};
+
+size_t evict_workspace_bytes(const mkv_geom& g, int32_t capacity);
+void evict_carve(EvictArgs& a, const mkv_geom& g, int32_t capacity, void* ws);
+cudaError_t launch_evict(const EvictArgs& a, int head_dim, int group, cudaStream_t stream);
+
+// ---------------------------------------------------------------- compress
+struct CompressArgs {
+  const void* K;      // bf16 [b, Hkv, T, D]
+  const void* V;
+  const void* Q;      // bf16 [b, Hkv, G, w, D]
+  int32_t T;
+  int32_t budget;
+  int32_t window;
+  int32_t sink;
+  int32_t keep_window;
+  int32_t pool;
+  int32_t mi;
+  int32_t causal;
+  float tau;
+  mkv_cache cache;
+  mkv_moments mom;
+  float* diag_scores;
+  float* diag_score2;
+  int32_t* diag_idx1;
+  void* ws;
+  int32_t batch;
+  int32_t n_kv;
+};
+
+size_t compress_workspace_bytes(const mkv_geom& g, int32_t T, const mkv_compress_params& p,
+                                int num_sms);
+cudaError_t launch_compress(const CompressArgs& a, const mkv_geom& g, size_t ws_bytes, int num_sms,
+                            cudaStream_t stream);
+
+}  // namespace mkv

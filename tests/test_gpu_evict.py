@@ -1,0 +1,113 @@
+"""Moment-informed eviction (Algorithm 1 append + Phase 1) on the GPU against
+the fp64 oracle, through the C ABI: the evicted positions (exact wherever the
+oracle's argmin gap exceeds 1e-5), the surviving rows in order, and the
+updated moments (1e-4 relative)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2606_01563_gb300 import mkv
+from paper_2606_01563_gb300.inputs import bf16_round
+from gpu_util import GAP_EXACT, assert_moment_close, bf16, f32, host, i32
+
+pytestmark = pytest.mark.gpu
+
+
+def setup(rng, b, H, G, D, lens, cap, n_evicted0):
+    """Cache rows and moments that come from a real evicted set of size n_evicted0."""
+    st = {"K": bf16_round(1.5 * rng.standard_normal((b, H, cap, D))),
+          "V": bf16_round(rng.standard_normal((b, H, cap, D))),
+          "lens": np.array(lens, np.int32).reshape(b, H),
+          "q": bf16_round(2.0 * rng.standard_normal((b, H * G, D))),
+          "kn": bf16_round(1.5 * rng.standard_normal((b, H, D))),
+          "vn": bf16_round(rng.standard_normal((b, H, D)))}
+    n = np.zeros((b, H), np.int32)
+    mk = np.zeros((b, H, D), np.float32)
+    mv = np.zeros((b, H, D), np.float32)
+    C = np.zeros((b, H, D, D), np.float32)
+    for bi in range(b):
+        for h in range(H):
+            ne = n_evicted0[bi * H + h]
+            if ne:
+                m = O.moments_of(bf16_round(1.5 * rng.standard_normal((ne, D))),
+                                 bf16_round(rng.standard_normal((ne, D))))
+                n[bi, h], mk[bi, h], mv[bi, h], C[bi, h] = m.n, m.mu_k, m.mu_v, m.C
+    st.update(n=n, mu_k=mk, mu_v=mv, C=C, cap=cap)
+    return st
+
+
+def run_case(st, b, H, G, D, budget, new, tau=1e-6):
+    g = mkv.geom(b, H, G, D)
+    cap = st["cap"]
+    pos0 = np.broadcast_to(np.arange(cap, dtype=np.int32) * 3, (b, H, cap)).copy()
+    cache = mkv.Cache(bf16(st["K"]), bf16(st["V"]), i32(pos0), i32(st["lens"]), i32(np.full((b, H), 10 ** 6)))
+    mom = mkv.Moments(i32(st["n"]), f32(st["mu_k"]), f32(st["mu_v"]), f32(st["C"]))
+    ws = mkv.alloc_workspace(mkv.mkv_evict_workspace_size(g, cap))
+    mkv.mkv_evict_append(g, bf16(st["q"]), bf16(st["kn"]) if new else None, bf16(st["vn"]) if new else None,
+                         budget, cache, mom, tau, ws)
+    code, info = mkv.mkv_get_device_error(ws)
+    gpu = dict(K=host(cache.K), V=host(cache.V), pos=host(cache.pos), len=host(cache.len), seen=host(cache.seen),
+               n=host(mom.n), mu_k=host(mom.mu_k), mu_v=host(mom.mu_v), C=host(mom.C), code=code, info=info)
+    refs = {}
+    for bi in range(b):
+        for h in range(H):
+            L = st["lens"][bi, h]
+            m = O.Moments(int(st["n"][bi, h]), st["mu_k"][bi, h], st["mu_v"][bi, h], st["C"][bi, h])
+            refs[bi, h] = O.evict_append(st["q"][bi, h * G:(h + 1) * G], st["K"][bi, h, :L], st["V"][bi, h, :L],
+                                         pos0[bi, h, :L], m, budget, tau,
+                                         st["kn"][bi, h] if new else None, st["vn"][bi, h] if new else None,
+                                         10 ** 6 if new else None)
+    return gpu, refs
+
+
+def check(gpu, refs, st, budget):
+    assert gpu["code"] == 0
+    for (bi, h), r in refs.items():
+        if r.gaps:
+            assert min(r.gaps) > GAP_EXACT, "fixture has a near-tie; pick another seed"
+        L = len(r.pos)
+        assert gpu["len"][bi, h] == L
+        np.testing.assert_array_equal(gpu["pos"][bi, h, :L], r.pos)
+        np.testing.assert_array_equal(gpu["K"][bi, h, :L], r.K)
+        np.testing.assert_array_equal(gpu["V"][bi, h, :L], r.V)
+        assert gpu["n"][bi, h] == r.moments.n
+        if r.moments.n:
+            assert_moment_close(gpu["mu_k"][bi, h], r.moments.mu_k, "mu_k")
+            assert_moment_close(gpu["mu_v"][bi, h], r.moments.mu_v, "mu_v")
+            assert_moment_close(gpu["C"][bi, h], r.moments.C, "C")
+
+
+@pytest.mark.parametrize("new", [False, True])
+def test_evict_tiny(new):
+    rng = np.random.default_rng(21)
+    st = setup(rng, 1, 2, 2, 64, [40, 33], 48, [0, 25])
+    gpu, refs = run_case(st, 1, 2, 2, 64, 24, new)
+    check(gpu, refs, st, 24)
+    if new:
+        np.testing.assert_array_equal(gpu["seen"], np.full((1, 2), 10 ** 6 + 1))
+
+
+@pytest.mark.parametrize("G", [1, 4, 8])
+def test_evict_llama_periodic(G):
+    """Budget 128 with 64 tokens appended since the last eviction: 64 evictions."""
+    rng = np.random.default_rng(22 + G)
+    H = 8 if G != 8 else 2
+    st = setup(rng, 1, H, G, 128, [191] * H, 200, [2000] * (H // 2) + [0] * (H - H // 2))
+    gpu, refs = run_case(st, 1, H, G, 128, 128, True)
+    check(gpu, refs, st, 128)
+
+
+def test_nothing_to_evict_only_appends():
+    rng = np.random.default_rng(23)
+    st = setup(rng, 2, 2, 2, 64, [10, 3, 0, 7], 16, [0, 1, 2, 3])
+    gpu, refs = run_case(st, 2, 2, 2, 64, 12, True)
+    check(gpu, refs, st, 12)
+
+
+def test_capacity_overflow_leaves_unit_unchanged():
+    rng = np.random.default_rng(24)
+    st = setup(rng, 1, 2, 2, 64, [16, 5], 16, [0, 4])
+    gpu, refs = run_case(st, 1, 2, 2, 64, 4, True)
+    assert gpu["code"] == 3 and gpu["info"] == 0
+    assert gpu["len"][0, 0] == 16 and gpu["len"][0, 1] == 4

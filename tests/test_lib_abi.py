@@ -1,0 +1,124 @@
+"""The C-ABI library builds, loads and exports every entry point include/mkv.h
+declares; host-side validation rejects bad arguments before touching the
+GPU.  Runs on the CPU (no kernel is launched)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2606_01563_gb300 import mkv
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def L():
+    if not os.path.exists(mkv.LIB_PATH):
+        from paper_2606_01563_gb300 import build
+        build.build()
+    return mkv.lib()
+
+
+def declared_functions():
+    src = open(os.path.join(ROOT, "include", "mkv.h")).read()
+    return sorted(set(re.findall(r"MKV_API\s+[\w\s\*]+?\b(mkv_\w+)\s*\(", src)))
+
+
+def test_every_declared_symbol_is_exported(L):
+    names = declared_functions()
+    assert len(names) == 9, names
+    assert set(names) == set(mkv.EXPORTS)
+    for n in names:
+        assert hasattr(L, n), n
+
+
+def test_version_and_status_strings(L):
+    assert mkv.mkv_version() == 100
+    for code in range(8):
+        assert mkv.mkv_status_str(code)
+    assert mkv.mkv_status_str(99) == "unknown status"
+
+
+FAKE = 1 << 20  # never dereferenced: validation fails before any launch
+
+
+def fake_cache(cap=64):
+    return mkv.mkv_cache(FAKE, FAKE, FAKE, FAKE, FAKE, cap)
+
+
+def fake_moments():
+    return mkv.mkv_moments(FAKE, FAKE, FAKE, FAKE)
+
+
+def decode(L, g, q=FAKE, kn=None, vn=None, cache=None, mom=None, p=None, out=FAKE, ws=FAKE, wsb=1 << 30):
+    cache = cache or fake_cache()
+    mom = mom or fake_moments()
+    p = p or mkv.mkv_decode_params(1, 1, 1e-6)
+    return L.mkv_decode_step(g, q, kn, vn, ctypes.byref(cache), ctypes.byref(mom), ctypes.byref(p), out, None,
+                             ws, wsb, None)
+
+
+def test_decode_validation(L):
+    g = mkv.geom(1, 2, 4, 128)
+    assert decode(L, mkv.geom(1, 2, 4, 96)) == 6            # head_dim unsupported
+    assert decode(L, mkv.geom(1, 2, 3, 128)) == 2           # group unsupported
+    assert decode(L, mkv.geom(0, 2, 4, 128)) == 2           # empty batch
+    assert decode(L, g, q=None) == 1
+    assert decode(L, g, out=None) == 1
+    assert decode(L, g, kn=FAKE) == 1                        # k_new without v_new
+    assert decode(L, g, p=mkv.mkv_decode_params(1, 2, 0.0)) == 1   # order
+    assert decode(L, g, p=mkv.mkv_decode_params(1, 1, -1.0)) == 1  # tau
+    assert decode(L, g, cache=mkv.mkv_cache(FAKE, FAKE, FAKE, FAKE, FAKE, 0)) == 1
+    assert decode(L, g, cache=mkv.mkv_cache(FAKE + 2, FAKE, FAKE, FAKE, FAKE, 64)) == 1  # misaligned K
+    assert decode(L, g, ws=None) == 7
+    assert decode(L, g, wsb=16) == 7
+    assert decode(L, g, ws=FAKE + 8) == 7                    # misaligned workspace
+
+
+def test_workspace_sizes(L):
+    g = mkv.geom(2, 8, 4, 128)
+    assert L.mkv_decode_workspace_size(g, 576) > 256
+    assert L.mkv_decode_workspace_size(mkv.geom(2, 8, 4, 80), 576) == 0
+    assert L.mkv_evict_workspace_size(g, 576) >= 256 + 2 * 8 * 4 * 576 * 4
+    assert L.mkv_evict_workspace_size(g, 70000) == 0
+    p = mkv.mkv_compress_params(512, 32, 1, 1, 1, 1, 1, 1e-6)
+    assert L.mkv_compress_workspace_size(g, 8192, ctypes.byref(p)) > 2 * 8 * 8192 * 4
+    bad = mkv.mkv_compress_params(16, 32, 1, 1, 1, 1, 1, 1e-6)  # budget < protected
+    assert L.mkv_compress_workspace_size(g, 8192, ctypes.byref(bad)) == 0
+
+
+def compress(L, g, T, p, cache=None, ws=FAKE, wsb=1 << 30, K=FAKE):
+    cache = cache or fake_cache(1024)
+    mom = fake_moments()
+    return L.mkv_compress(g, T, K, FAKE, FAKE, ctypes.byref(p), ctypes.byref(cache), ctypes.byref(mom), None,
+                          ws, wsb, None)
+
+
+def test_compress_validation(L):
+    g = mkv.geom(1, 2, 2, 64)
+    P = lambda **kw: mkv.mkv_compress_params(**{**dict(budget=128, window=16, sink=1, keep_window=1, pool=1,
+                                                        mi=1, causal=1, tau=1e-6), **kw})
+    assert compress(L, g, 1024, P(budget=10)) == 1            # budget below sink + window
+    assert compress(L, g, 1024, P(window=0)) == 1
+    assert compress(L, g, 8, P(window=16)) == 1               # window longer than the prompt
+    assert compress(L, g, 1024, P(pool=3)) == 1
+    assert compress(L, g, 1024, P(mi=2)) == 1
+    assert compress(L, g, 0, P()) == 1
+    assert compress(L, g, 1024, P(), cache=fake_cache(100)) == 3   # capacity < budget
+    assert compress(L, g, 1024, P(), K=None) == 1
+    assert compress(L, g, 1024, P(), wsb=1024) == 7
+    assert compress(L, mkv.geom(1, 2, 2, 100), 1024, P()) == 6
+
+
+def test_evict_validation(L):
+    g = mkv.geom(1, 2, 2, 64)
+    c, m = fake_cache(), fake_moments()
+    run = lambda **kw: L.mkv_evict_append(kw.get("g", g), kw.get("q", FAKE), None, None, kw.get("budget", 8),
+                                          ctypes.byref(c), ctypes.byref(m), kw.get("tau", 0.0),
+                                          kw.get("ws", FAKE), kw.get("wsb", 1 << 30), None)
+    assert run(budget=-1) == 1
+    assert run(q=None) == 1
+    assert run(tau=float("nan")) == 1
+    assert run(wsb=8) == 7
+    assert run(g=mkv.geom(1, 2, 5, 64)) == 2
