@@ -202,6 +202,35 @@ MKV_API mkv_status mkv_decode_step(mkv_geom geom, const void* q, const void* k_n
                            void* workspace, size_t workspace_bytes, void* stream);
 
 /*
+ * mkv_decode_step without a workspace argument.  The paper has no
+ * counterpart: this is a deployment variant for callers that cannot
+ * allocate device memory when they decode -- a plugin that its host engine
+ * gives only input and output buffers, a server whose device memory another
+ * allocator reserved at start-up, or a latency-critical path that cannot
+ * accept cudaMalloc's implicit device synchronisation.
+ * Arguments, computation and outputs are those of mkv_decode_step.  The
+ * split-K scratch (error word, ticket counters, partial states, moment rows)
+ * is a fixed 4 MiB device array inside the library, held by every GPU that
+ * loads it until the process exits; this call allocates nothing and frees
+ * nothing.
+ *  - The first call on a device sets up that device (looks up the array's
+ *    address, zeroes it, synchronises the device); make that first call before
+ *    any stream capture.
+ *  - Geometries whose scratch would exceed 4 MiB even with one split per unit
+ *    (b * h_kv * g * (d + 4) * 4 bytes plus the moment rows) are rejected with
+ *    MKV_ERR_WORKSPACE before anything runs; smaller ones use as many splits
+ *    as fit.
+ *  - Every call shares the array: calls that overlap on the GPU (e.g. on two
+ *    streams) race and give wrong results.  Serialise them.
+ *  - Errors the kernel detects are recorded in the array's error word, which
+ *    this call does not expose; the outputs in those cases are as described
+ *    for mkv_decode_step.
+ */
+MKV_API mkv_status mkv_decode_step_noalloc(mkv_geom geom, const void* q, const void* k_new, const void* v_new,
+                                           const mkv_cache* cache, const mkv_moments* mom,
+                                           const mkv_decode_params* p, float* out, float* lse, void* stream);
+
+/*
  * Bytes of device workspace mkv_evict_append needs.  Returns 0 if invalid.
  * The workspace needs no initialisation.
  */

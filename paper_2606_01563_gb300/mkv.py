@@ -51,7 +51,7 @@ STATUS = {0: "MKV_OK", 1: "MKV_ERR_INVALID_ARG", 2: "MKV_ERR_SHAPE", 3: "MKV_ERR
 
 EXPORTS = ("mkv_status_str", "mkv_version", "mkv_compress_workspace_size", "mkv_compress",
            "mkv_decode_workspace_size", "mkv_decode_step", "mkv_evict_workspace_size",
-           "mkv_evict_append", "mkv_get_device_error")
+           "mkv_evict_append", "mkv_get_device_error", "mkv_decode_step_noalloc")
 
 
 class MKVError(RuntimeError):
@@ -86,6 +86,10 @@ def lib():
         L.mkv_decode_step.argtypes = [mkv_geom, c_vp, c_vp, c_vp, ctypes.POINTER(mkv_cache),
                                       ctypes.POINTER(mkv_moments), ctypes.POINTER(mkv_decode_params),
                                       c_vp, c_vp, c_vp, ctypes.c_size_t, c_vp]
+        L.mkv_decode_step_noalloc.restype = c_i32
+        L.mkv_decode_step_noalloc.argtypes = [mkv_geom, c_vp, c_vp, c_vp, ctypes.POINTER(mkv_cache),
+                                              ctypes.POINTER(mkv_moments), ctypes.POINTER(mkv_decode_params),
+                                              c_vp, c_vp, c_vp]
         L.mkv_evict_workspace_size.restype = ctypes.c_size_t
         L.mkv_evict_workspace_size.argtypes = [mkv_geom, c_i32]
         L.mkv_evict_append.restype = c_i32
@@ -209,6 +213,17 @@ def mkv_decode_step(g, q, k_new, v_new, cache: Cache, mom: Moments | None, p: mk
                                  ctypes.byref(m) if m is not None else None, ctypes.byref(p), _ptr(out),
                                  _ptr(lse), _ptr(ws), ws.numel(), _stream(stream))
     _check(code, "mkv_decode_step")
+
+
+def mkv_decode_step_noalloc(g, q, k_new, v_new, cache: Cache, mom: Moments | None, p: mkv_decode_params, out,
+                            lse, stream=None):
+    """mkv_decode_step with the library's fixed device scratch instead of a workspace."""
+    c = cache.c()
+    m = mom.c() if mom is not None else None
+    code = lib().mkv_decode_step_noalloc(g, _ptr(q), _ptr(k_new), _ptr(v_new), ctypes.byref(c),
+                                         ctypes.byref(m) if m is not None else None, ctypes.byref(p), _ptr(out),
+                                         _ptr(lse), _stream(stream))
+    _check(code, "mkv_decode_step_noalloc")
 
 
 def mkv_evict_append(g, q, k_new, v_new, budget, cache: Cache, mom: Moments, tau, ws, stream=None):

@@ -27,7 +27,7 @@ def declared_functions():
 
 def test_every_declared_symbol_is_exported(L):
     names = declared_functions()
-    assert len(names) == 9, names
+    assert len(names) == 10, names
     assert set(names) == set(mkv.EXPORTS)
     for n in names:
         assert hasattr(L, n), n
