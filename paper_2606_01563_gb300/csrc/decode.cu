@@ -163,8 +163,8 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a) {
   __nv_bfloat16* sV = sK + kStages * kTT * D;
   __nv_bfloat16* sNew = sV + kStages * kTT * D;  // [2][D]: new k, new v
   __shared__ float sQ[G * D];                      // q * scale * log2(e)
-  __shared__ float sRed[4][G][D + 2];
   __shared__ float sSbar[G];
+  __shared__ float sM[G], sL[G];
   __shared__ __align__(8) uint64_t bars[kStages];
   __shared__ int sTicket;
 
@@ -216,35 +216,52 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a) {
   __syncthreads();
 
   // ---- moment rows: f_hat_E[h][row] = mu_v[row] + scale * sum_c C'[row][c] q_h[c]
+  // (each warp keeps RB rows' loads in flight before reducing them)
   if (use_m && a.order == 1) {
+    constexpr int RB = 4;
     const int rpc = (D + a.S - 1) / a.S;
     const int r0 = s * rpc, r1 = min(D, r0 + rpc);
     const float tau = a.tau;
     const float nf = static_cast<float>(n_e);
-    for (int row = r0 + warp; row < r1; row += 4) {
-      const float* Crow = a.C + ((size_t)u * D + row) * D + lane * DPL;
-      float cv[DPL];
-      if constexpr (DPL == 4) {
-        const float4 t = __ldg(reinterpret_cast<const float4*>(Crow));
-        cv[0] = t.x; cv[1] = t.y; cv[2] = t.z; cv[3] = t.w;
-      } else {
-        const float2 t = __ldg(reinterpret_cast<const float2*>(Crow));
-        cv[0] = t.x; cv[1] = t.y;
+    for (int base = r0 + warp; base < r1; base += 4 * RB) {
+      float cv[RB][DPL];
+      float mv[RB];
+#pragma unroll
+      for (int k = 0; k < RB; ++k) {
+        const int row = base + 4 * k;
+        mv[k] = 0.f;
+#pragma unroll
+        for (int i = 0; i < DPL; ++i) cv[k][i] = 0.f;
+        if (row < r1) {
+          const float* Crow = a.C + ((size_t)u * D + row) * D + lane * DPL;
+          if constexpr (DPL == 4) {
+            const float4 t = __ldg(reinterpret_cast<const float4*>(Crow));
+            cv[k][0] = t.x; cv[k][1] = t.y; cv[k][2] = t.z; cv[k][3] = t.w;
+          } else {
+            const float2 t = __ldg(reinterpret_cast<const float2*>(Crow));
+            cv[k][0] = t.x; cv[k][1] = t.y;
+          }
+          if (lane == 0) mv[k] = __ldg(a.mu_v + (size_t)u * D + row);
+        }
       }
 #pragma unroll
-      for (int i = 0; i < DPL; ++i) cv[i] = (fabsf(cv[i] * nf) < tau) ? 0.f : cv[i];
-      float acc[G];
+      for (int k = 0; k < RB; ++k) {
+        const int row = base + 4 * k;
+        if (row >= r1) break;  // warp-uniform
 #pragma unroll
-      for (int h = 0; h < G; ++h) {
-        acc[h] = 0.f;
+        for (int i = 0; i < DPL; ++i) cv[k][i] = (fabsf(cv[k][i] * nf) < tau) ? 0.f : cv[k][i];
+        float acc[G];
 #pragma unroll
-        for (int i = 0; i < DPL; ++i) acc[h] = fmaf(cv[i], sQ[h * D + lane * DPL + i], acc[h]);
-        acc[h] = warp_sum(acc[h]);
-      }
-      if (lane == 0) {
-        const float mv = a.mu_v[(size_t)u * D + row];
+        for (int h = 0; h < G; ++h) {
+          acc[h] = 0.f;
 #pragma unroll
-        for (int h = 0; h < G; ++h) a.fhat[((size_t)u * G + h) * D + row] = mv + acc[h] * (1.f / kLog2e);
+          for (int i = 0; i < DPL; ++i) acc[h] = fmaf(cv[k][i], sQ[h * D + lane * DPL + i], acc[h]);
+          acc[h] = warp_sum(acc[h]);
+        }
+        if (lane == 0) {
+#pragma unroll
+          for (int h = 0; h < G; ++h) a.fhat[((size_t)u * G + h) * D + row] = mv[k] + acc[h] * (1.f / kLog2e);
+        }
       }
     }
   }
@@ -300,14 +317,16 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a) {
     if (warp == 0) process_rows<D, G>(st, qr, sNew, sNew + D, 0, 1, lane);
   }
 
-  // ---- merge the 4 warps into this CTA's partial record
+  // ---- merge the 4 warps into this CTA's partial record (through the free tile ring)
+  float* sRed = reinterpret_cast<float*>(dsmem);  // [4][G][D + 2]
+  __syncthreads();
 #pragma unroll
   for (int h = 0; h < G; ++h) {
 #pragma unroll
-    for (int i = 0; i < DPL; ++i) sRed[warp][h][lane * DPL + i] = st.o[h][i];
+    for (int i = 0; i < DPL; ++i) sRed[(warp * G + h) * (D + 2) + lane * DPL + i] = st.o[h][i];
     if (lane == 0) {
-      sRed[warp][h][D] = st.m[h];
-      sRed[warp][h][D + 1] = st.l[h];
+      sRed[(warp * G + h) * (D + 2) + D] = st.m[h];
+      sRed[(warp * G + h) * (D + 2) + D + 1] = st.l[h];
     }
   }
   __syncthreads();
@@ -316,14 +335,15 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a) {
     const int h = idx / D, dd = idx % D;
     float M = -INFINITY;
 #pragma unroll
-    for (int w = 0; w < 4; ++w) M = fmaxf(M, sRed[w][h][D]);
+    for (int w = 0; w < 4; ++w) M = fmaxf(M, sRed[(w * G + h) * (D + 2) + D]);
     float o = 0.f, l = 0.f;
     if (M != -INFINITY) {
 #pragma unroll
       for (int w = 0; w < 4; ++w) {
-        const float f = fast_exp2(sRed[w][h][D] - M);
-        o = fmaf(f, sRed[w][h][dd], o);
-        l = fmaf(f, sRed[w][h][D + 1], l);
+        const float* rw = sRed + (w * G + h) * (D + 2);
+        const float f = fast_exp2(rw[D] - M);
+        o = fmaf(f, rw[dd], o);
+        l = fmaf(f, rw[D + 1], l);
       }
     }
     part[h * PS + dd] = o;
@@ -352,47 +372,77 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a) {
   }
   __syncthreads();
 
+  // combine the S partial records: per-(split, head) weights in shared
+  // memory, then each thread accumulates 4 output dims with all loads in flight
   const float* pu = a.partial + (size_t)u * a.S * G * PS;
-  for (int idx = tid; idx < G * D; idx += kThreads) {
-    const int h = idx / D, dd = idx % D;
+  float* sW = reinterpret_cast<float*>(dsmem);  // [S][G] max, then weight
+  float* sLs = sW + a.S * G;                    // [S][G] sums
+  __syncthreads();
+  for (int i = tid; i < a.S * G; i += kThreads) {
+    sW[i] = __ldcg(pu + (size_t)i * PS + D);
+    sLs[i] = __ldcg(pu + (size_t)i * PS + D + 1);
+  }
+  __syncthreads();
+  if (tid < G) {
     float M = -INFINITY;
-    for (int sp = 0; sp < a.S; ++sp) M = fmaxf(M, __ldcg(pu + ((size_t)sp * G + h) * PS + D));
-    float o = 0.f, l = 0.f;
-    if (M != -INFINITY) {
-      for (int sp = 0; sp < a.S; ++sp) {
-        const float* rec = pu + ((size_t)sp * G + h) * PS;
-        const float ls = __ldcg(rec + D + 1);
-        if (ls > 0.f) {
-          const float f = fast_exp2(__ldcg(rec + D) - M);
-          l = fmaf(ls, f, l);
-          o = fmaf(f, __ldcg(rec + dd), o);
-        }
-      }
+    for (int sp = 0; sp < a.S; ++sp)
+      if (sLs[sp * G + tid] > 0.f) M = fmaxf(M, sW[sp * G + tid]);
+    float l = 0.f;
+    if (M != -INFINITY)
+      for (int sp = 0; sp < a.S; ++sp)
+        if (sLs[sp * G + tid] > 0.f) l = fmaf(sLs[sp * G + tid], fast_exp2(sW[sp * G + tid] - M), l);
+    sM[tid] = M;
+    sL[tid] = l;
+  }
+  __syncthreads();
+  for (int i = tid; i < a.S * G; i += kThreads) {
+    const float M = sM[i % G];
+    sW[i] = (sLs[i] > 0.f && M != -INFINITY) ? fast_exp2(sW[i] - M) : 0.f;
+  }
+  __syncthreads();
+  for (int slot = tid; slot < G * (D / 4); slot += kThreads) {
+    const int h = slot / (D / 4), d0 = (slot % (D / 4)) * 4;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 4
+    for (int sp = 0; sp < a.S; ++sp) {
+      const float w = sW[sp * G + h];
+      const float4 o = __ldcg(reinterpret_cast<const float4*>(pu + ((size_t)sp * G + h) * PS + d0));
+      acc.x = fmaf(w, o.x, acc.x);
+      acc.y = fmaf(w, o.y, acc.y);
+      acc.z = fmaf(w, o.z, acc.z);
+      acc.w = fmaf(w, o.w, acc.w);
     }
+    const float l = sL[h];
     const bool have_r = l > 0.f;
-    const float aR = have_r ? M * kLn2 + logf(l) : -INFINITY;
-    const float oR = have_r ? o / l : 0.f;
-    float res, lse;
+    const float aR = have_r ? sM[h] * kLn2 + logf(l) : -INFINITY;
+    const float inv_l = have_r ? 1.f / l : 0.f;
+    const float oR[4] = {acc.x * inv_l, acc.y * inv_l, acc.z * inv_l, acc.w * inv_l};
+    float res[4], lse = aR;
     if (use_m) {
       const float e = logf(static_cast<float>(n_e)) + sSbar[h];
-      const float fh = (a.order == 1) ? __ldcg(a.fhat + ((size_t)u * G + h) * D + dd) : a.mu_v[(size_t)u * D + dd];
+      float fh[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k)
+        fh[k] = (a.order == 1) ? __ldcg(a.fhat + ((size_t)u * G + h) * D + d0 + k) : a.mu_v[(size_t)u * D + d0 + k];
       if (have_r) {
         const float top = fmaxf(aR, e);
         const float wr = expf(aR - top), we = expf(e - top);
         const float wR = wr / (wr + we);
-        res = wR * oR + (1.f - wR) * fh;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) res[k] = wR * oR[k] + (1.f - wR) * fh[k];
         lse = top + logf(wr + we);
       } else {
-        res = fh;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) res[k] = fh[k];
         lse = e;
       }
     } else {
-      if (!have_r && dd == 0 && h == 0) record_error(a.ws, MKV_ERR_INVALID_ARG, u);
-      res = oR;
-      lse = aR;
+      if (!have_r && d0 == 0 && h == 0) record_error(a.ws, MKV_ERR_INVALID_ARG, u);
+#pragma unroll
+      for (int k = 0; k < 4; ++k) res[k] = oR[k];
     }
-    a.out[((size_t)u * G + h) * D + dd] = res;
-    if (a.lse != nullptr && dd == 0) a.lse[(size_t)u * G + h] = lse;
+    *reinterpret_cast<float4*>(a.out + ((size_t)u * G + h) * D + d0) = make_float4(res[0], res[1], res[2], res[3]);
+    if (a.lse != nullptr && d0 == 0) a.lse[(size_t)u * G + h] = lse;
   }
 
   if (has_new) {

@@ -68,7 +68,10 @@ struct EvictArgs {
   int32_t budget;
   float tau;
   void* ws;
-  float* scratch;  // [units][cap] logits / scores
+  float* scratch;  // [units][G][cap] logits (single-CTA kernel)
+  void* stage;     // [units][cap] rows staged by the cluster kernel's compaction
+  int32_t rows_max;  // cluster kernel: rows per CTA slice = ceil(cap / CTAs per unit)
+  int32_t kv_smem;   // cluster kernel: the slice's K/V rows are cached in shared memory
   int32_t batch;
   int32_t n_kv;
 };

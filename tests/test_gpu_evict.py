@@ -111,3 +111,30 @@ def test_capacity_overflow_leaves_unit_unchanged():
     gpu, refs = run_case(st, 1, 2, 2, 64, 4, True)
     assert gpu["code"] == 3 and gpu["info"] == 0
     assert gpu["len"][0, 0] == 16 and gpu["len"][0, 1] == 4
+
+
+@pytest.mark.parametrize("tau", [0.0, 1e-6, 0.05, 0.5])
+def test_evict_clamp_paths(tau):
+    """Moments from a handful of evicted tokens make n C entries O(1), so a large
+    tau clamps a visible share of them: few entries exercise the incremental
+    correction list, many exercise the direct clamped product."""
+    rng = np.random.default_rng(31)
+    st = setup(rng, 1, 2, 2, 64, [60, 45], 64, [3, 5])
+    gpu, refs = run_case(st, 1, 2, 2, 64, 30, True, tau=tau)
+    check(gpu, refs, st, 30)
+
+
+def test_evict_large_capacity_fallback():
+    """A capacity whose row slices do not fit in shared memory runs the
+    single-CTA kernel; results are the same."""
+    rng = np.random.default_rng(32)
+    st = setup(rng, 1, 1, 4, 128, [2300], 2400, [500])
+    gpu, refs = run_case(st, 1, 1, 4, 128, 2260, False)
+    check(gpu, refs, st, 2260)
+
+
+def test_evict_budget_zero_and_batch():
+    rng = np.random.default_rng(33)
+    st = setup(rng, 2, 2, 1, 64, [9, 17, 1, 30], 32, [0, 2, 0, 7])
+    gpu, refs = run_case(st, 2, 2, 1, 64, 0, False)
+    check(gpu, refs, st, 0)
