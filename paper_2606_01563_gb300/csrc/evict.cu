@@ -347,60 +347,94 @@ __global__ void __launch_bounds__(kThreads) evict_kernel(const EvictArgs a) {
   }
 }
 
-constexpr int kCL = 8;          // CTAs per unit (one cluster)
+constexpr int kCL = 8;           // CTAs per unit (one cluster)
+constexpr int kCT = 1024;        // threads per CTA of the cluster kernel
+constexpr int kCW = kCT / 32;    // warps per CTA
+constexpr int kLPR = 8;          // lanes per row
+constexpr int kRPW = 32 / kLPR;  // rows per warp per pass
+constexpr int kRowsPerPass = kCW * kRPW;
+constexpr int kMaxClamp = 64;    // clamped entries corrected incrementally
+constexpr int kTW = 4;           // warps that run the 32x32 tile transposes
+// dynamic shared memory available next to the kernel's ~30 KB of static arrays
+constexpr size_t kSmemBudget = 192 * 1024;
 
 // Bytes of staging per unit (K and V rows, positions), padded so that every
 // unit's block starts on a 256-byte boundary.
 __host__ __device__ inline size_t stage_stride(int cap, int D) {
   return align_up((size_t)cap * (4 * (size_t)D + 4), 256);
 }
-constexpr int kMaxClamp = 64;   // clamped entries corrected incrementally
-constexpr size_t kSmemBudget = 220 * 1024;
 
 template <int D, int G>
 struct ClusterLayout {
-  size_t Ct, Y, lg, kbuf, Ks, Vs, alive, total;
-  __host__ __device__ ClusterLayout(int R, int kv) {
+  size_t Ct, Y, lg, Ks, Vs, alive, total;
+  // R rows per slice; cap rows per unit (logits and alive flags cover the unit)
+  __host__ __device__ ClusterLayout(int R, int cap, int kv) {
     size_t off = 0;
     Ct = off; off += (size_t)D * D * 4;
     Y = off; off += (size_t)R * D * 4;
-    lg = off; off += align_up((size_t)G * R * 4, 16);
-    kbuf = off; off += (size_t)kWarps * kRowsPerGroup * D * 4;
+    lg = off; off += align_up((size_t)G * cap * 4, 16);
     Ks = off; off += kv ? (size_t)R * D * 2 : 0;
     Vs = off; off += kv ? (size_t)R * D * 2 : 0;
-    alive = off; off += align_up((size_t)R, 16);
+    alive = off; off += align_up((size_t)cap, 16);
     total = off;
   }
 };
 
+// A row is handled by a group of 8 lanes; lane q of the group owns the
+// value/key dims of float4 chunks q, q+8, q+16, ... (NC = D/32 chunks), so
+// the 8 lanes of a row touch 8 different bank groups.
+template <int D>
+__device__ __forceinline__ int chunk_dim(int q, int c) { return (q + 8 * c) * 4; }
+
+__device__ __forceinline__ float group_sum(float v) {
+  v += __shfl_xor_sync(kFull, v, 1);
+  v += __shfl_xor_sync(kFull, v, 2);
+  v += __shfl_xor_sync(kFull, v, 4);
+  return v;
+}
+
+template <int D>
+__device__ __forceinline__ void load4_bf16(const __nv_bfloat16* p, float* o) { load_bf16<4>(p, o); }
+
 template <int D, int G>
-__global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kThreads)
+__global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
     evict_cluster_kernel(const EvictArgs a) {
-  constexpr int DPL = D / 32;
+  constexpr int NC = D / 32;
   extern __shared__ __align__(16) uint8_t dsmem[];
   const int R = a.rows_max;
-  const ClusterLayout<D, G> lay(R, a.kv_smem);
-  float* Ct = reinterpret_cast<float*>(dsmem + lay.Ct);      // Ct[c*D + r] = C[r][c]
-  float* Y = reinterpret_cast<float*>(dsmem + lay.Y);        // [R][D] y_j = C k_j
-  float* lg = reinterpret_cast<float*>(dsmem + lay.lg);      // [G][R] logits
-  float* kbuf = reinterpret_cast<float*>(dsmem + lay.kbuf);  // [warps][4][D]
-  uint8_t* alive = dsmem + lay.alive;                        // [R]
-  __shared__ float s_mu_k[D], s_mu_v[D], s_dk[D], s_dv[D];
-  __shared__ float s_q[G][D];
-  __shared__ float s_red[kWarps][G];
+  const ClusterLayout<D, G> lay(R, a.cap, a.kv_smem);
+  float* Ct = reinterpret_cast<float*>(dsmem + lay.Ct);  // Ct[c*D + r] = C[r][c]
+  float* Y = reinterpret_cast<float*>(dsmem + lay.Y);    // [R][D] y_j = C k_j of this slice
+  float* lg = reinterpret_cast<float*>(dsmem + lay.lg);  // [G][cap] logits of every row of the unit
+  uint8_t* alive_all = dsmem + lay.alive;                // [cap] alive flags of the unit
+  __shared__ __align__(16) float s_mu_k[D];
+  __shared__ __align__(16) float s_mu_v[D];
+  __shared__ __align__(16) float s_dk[D];
+  __shared__ __align__(16) float s_dv[D];
+  __shared__ __align__(16) float s_q[G][D];
+  __shared__ float s_red[kCW][G], s_red2[kCW][G];
   __shared__ float s_M[G], s_Z[G];
-  __shared__ float ex_ml[2 * G];       // this CTA's per-head (max, sum), read by the cluster
-  __shared__ unsigned long long ex_best;
+  __shared__ int s_js;
+  // published to the cluster, double-buffered by iteration parity: this CTA's
+  // best (score, row) key and that row's k and v
+  __shared__ unsigned long long ex_best[2];
+  __shared__ __align__(16) __nv_bfloat16 ex_row[2][2 * D];
+  __shared__ __align__(16) __nv_bfloat16 s_cand[kCL][2 * D];  // every rank's candidate row
+  __shared__ unsigned long long s_keys[kCL];
   __shared__ int ex_cnt;
-  __shared__ unsigned long long s_bestw[kWarps];
+  __shared__ unsigned long long s_bestw[kCW];
   __shared__ uint32_t s_zidx[kMaxClamp];
   __shared__ float s_zval[kMaxClamp];
   __shared__ int s_nz;
+  __shared__ float s_tile[kTW][32 * 33];  // transpose staging (setup / write-back)
+  __shared__ float s_invZ[G];
 
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = static_cast<int>(cluster.block_rank());
   const int u = blockIdx.x / kCL;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int q = lane & 7;                      // lane within its row group
+  const int rsub = warp * kRPW + (lane >> 3);  // row of this group within a pass
   const size_t row0 = (size_t)u * a.cap;
   __nv_bfloat16* Kg = reinterpret_cast<__nv_bfloat16*>(a.K) + row0 * D;
   __nv_bfloat16* Vg = reinterpret_cast<__nv_bfloat16*>(a.V) + row0 * D;
@@ -419,7 +453,7 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kThreads)
   if (has_new && len_in >= j0 && len_in < j1) {  // the owning CTA appends the token
     const __nv_bfloat16* kn = reinterpret_cast<const __nv_bfloat16*>(a.k_new) + (size_t)u * D;
     const __nv_bfloat16* vn = reinterpret_cast<const __nv_bfloat16*>(a.v_new) + (size_t)u * D;
-    for (int i = tid; i < D; i += kThreads) {
+    for (int i = tid; i < D; i += kCT) {
       Kg[(size_t)len_in * D + i] = kn[i];
       Vg[(size_t)len_in * D + i] = vn[i];
     }
@@ -436,94 +470,131 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kThreads)
   }
 
   int n = a.n[u];
-  for (int idx = tid; idx < D * D; idx += kThreads) {
-    const int r = idx / D, c = idx % D;
-    Ct[c * D + r] = (n > 0) ? a.C[(size_t)u * D * D + idx] : 0.f;
+  {
+    // Ct[c][r] = C[r][c]: each warp moves 32x32 tiles through a padded buffer
+    // so that both the global reads and the shared-memory writes are dense
+    float* tb = s_tile[warp % kTW];
+    for (int t = warp; warp < kTW && t < (D / 32) * (D / 32); t += kTW) {
+      const int r0 = (t / (D / 32)) * 32, c0 = (t % (D / 32)) * 32;
+      for (int i = 0; i < 32; ++i)
+        tb[i * 33 + lane] = (n > 0) ? a.C[(size_t)u * D * D + (size_t)(r0 + i) * D + c0 + lane] : 0.f;
+      __syncwarp();
+      for (int i = 0; i < 32; ++i) Ct[(size_t)(c0 + i) * D + r0 + lane] = tb[lane * 33 + i];
+      __syncwarp();
+    }
   }
-  for (int i = tid; i < D; i += kThreads) {
+  for (int i = tid; i < D; i += kCT) {
     s_mu_k[i] = (n > 0) ? a.mu_k[(size_t)u * D + i] : 0.f;
     s_mu_v[i] = (n > 0) ? a.mu_v[(size_t)u * D + i] : 0.f;
   }
   const float scale = rsqrtf(static_cast<float>(D));
   const __nv_bfloat16* qg = reinterpret_cast<const __nv_bfloat16*>(a.q) + (size_t)u * G * D;
-  for (int i = tid; i < G * D; i += kThreads) s_q[i / D][i % D] = __bfloat162float(qg[i]) * scale;
-  // this slice's rows (global or cached in shared memory)
+  for (int i = tid; i < G * D; i += kCT) s_q[i / D][i % D] = __bfloat162float(qg[i]) * scale;
   const __nv_bfloat16* Kr = Kg + (size_t)j0 * D;
   const __nv_bfloat16* Vr = Vg + (size_t)j0 * D;
   if (a.kv_smem) {
     __nv_bfloat16* Ks = reinterpret_cast<__nv_bfloat16*>(dsmem + lay.Ks);
     __nv_bfloat16* Vs = reinterpret_cast<__nv_bfloat16*>(dsmem + lay.Vs);
-    for (int idx = tid; idx < nr * (D / 8); idx += kThreads) {
+    for (int idx = tid; idx < nr * (D / 8); idx += kCT) {
       reinterpret_cast<uint4*>(Ks)[idx] = reinterpret_cast<const uint4*>(Kr)[idx];
       reinterpret_cast<uint4*>(Vs)[idx] = reinterpret_cast<const uint4*>(Vr)[idx];
     }
     Kr = Ks;
     Vr = Vs;
   }
-  for (int r = tid; r < R; r += kThreads) alive[r] = r < nr ? 1 : 0;
+  for (int j = tid; j < a.cap; j += kCT) alive_all[j] = j < len ? 1 : 0;
   if (tid == 0) s_nz = 0;
   __syncthreads();
+  const uint8_t* alive = alive_all + j0;  // this slice's flags
 
-  // logits and y_j = C k_j for the slice
-  for (int r = warp; r < nr; r += kWarps) {
-    float kf[DPL];
-    load_bf16<DPL>(Kr + (size_t)r * D + lane * DPL, kf);
+  // ---- logits of every row of the unit (8 lanes per row, read from global)
+  for (int base = 0; base < len; base += kRowsPerPass) {
+    const int j = base + rsub;
+    const bool ok = j < len;
+    float kf[NC][4];
+#pragma unroll
+    for (int c = 0; c < NC; ++c) {
+      if (ok) load4_bf16<D>(Kg + (size_t)j * D + chunk_dim<D>(q, c), kf[c]);
+      else kf[c][0] = kf[c][1] = kf[c][2] = kf[c][3] = 0.f;
+    }
 #pragma unroll
     for (int h = 0; h < G; ++h) {
       float acc = 0.f;
 #pragma unroll
-      for (int i = 0; i < DPL; ++i) acc = fmaf(s_q[h][lane * DPL + i], kf[i], acc);
-      acc = warp_sum(acc);
-      if (lane == 0) lg[h * R + r] = acc;
+      for (int c = 0; c < NC; ++c) {
+        const float4 q4 = *reinterpret_cast<const float4*>(&s_q[h][chunk_dim<D>(q, c)]);
+        acc = fmaf(q4.x, kf[c][0], fmaf(q4.y, kf[c][1], fmaf(q4.z, kf[c][2], fmaf(q4.w, kf[c][3], acc))));
+      }
+      acc = group_sum(acc);
+      if (ok && q == 0) lg[h * a.cap + j] = acc;
     }
   }
-  float* kb = kbuf + warp * kRowsPerGroup * D;
-  for (int g0 = warp * kRowsPerGroup; g0 < nr; g0 += kWarps * kRowsPerGroup) {
+  __syncthreads();
+  // softmax is shift-invariant: keep e_hj = exp(l_hj - M0_h) with M0_h the
+  // largest logit of the unit at the start, so that every iteration's
+  // normaliser is a plain sum over the surviving rows
+  {
+    float mx[G];
 #pragma unroll
-    for (int r = 0; r < kRowsPerGroup; ++r) {
-      float kf[DPL];
-      if (g0 + r < nr) {
-        load_bf16<DPL>(Kr + (size_t)(g0 + r) * D + lane * DPL, kf);
-      } else {
+    for (int h = 0; h < G; ++h) mx[h] = -INFINITY;
+    for (int jj = tid; jj < len; jj += kCT)
 #pragma unroll
-        for (int i = 0; i < DPL; ++i) kf[i] = 0.f;
-      }
+      for (int h = 0; h < G; ++h) mx[h] = fmaxf(mx[h], lg[h * a.cap + jj]);
 #pragma unroll
-      for (int i = 0; i < DPL; ++i) kb[r * D + lane * DPL + i] = kf[i];
+    for (int h = 0; h < G; ++h) {
+      mx[h] = warp_max(mx[h]);
+      if (lane == 0) s_red[warp][h] = mx[h];
     }
-    __syncwarp();
-    float y[kRowsPerGroup][DPL];
+    __syncthreads();
+    if (warp == 0) {
 #pragma unroll
-    for (int r = 0; r < kRowsPerGroup; ++r)
+      for (int h = 0; h < G; ++h) {
+        const float m = warp_max(s_red[lane][h]);
+        if (lane == 0) s_M[h] = m;
+      }
+    }
+    __syncthreads();
+    for (int jj = tid; jj < len; jj += kCT)
 #pragma unroll
-      for (int i = 0; i < DPL; ++i) y[r][i] = 0.f;
+      for (int h = 0; h < G; ++h) lg[h * a.cap + jj] = expf(lg[h * a.cap + jj] - s_M[h]);
+  }
+  // ---- y_j = C k_j for this slice
+  for (int base = 0; base < nr; base += kRowsPerPass) {
+    const int r = base + rsub;
+    const bool ok = r < nr;
     if (n > 0) {
-#pragma unroll 4
-      for (int c = 0; c < D; ++c) {
-        float cv[DPL];
+      float y[NC][4];
 #pragma unroll
-        for (int i = 0; i < DPL; ++i) cv[i] = Ct[c * D + lane * DPL + i];
+      for (int c = 0; c < NC; ++c) y[c][0] = y[c][1] = y[c][2] = y[c][3] = 0.f;
+      if (ok) {
+        for (int kc = 0; kc < D; ++kc) {
+          const float kv = __bfloat162float(Kr[(size_t)r * D + kc]);
 #pragma unroll
-        for (int r = 0; r < kRowsPerGroup; ++r) {
-          const float kc = kb[r * D + c];
-#pragma unroll
-          for (int i = 0; i < DPL; ++i) y[r][i] = fmaf(cv[i], kc, y[r][i]);
+          for (int c = 0; c < NC; ++c) {
+            const float4 c4 = *reinterpret_cast<const float4*>(Ct + kc * D + chunk_dim<D>(q, c));
+            y[c][0] = fmaf(c4.x, kv, y[c][0]);
+            y[c][1] = fmaf(c4.y, kv, y[c][1]);
+            y[c][2] = fmaf(c4.z, kv, y[c][2]);
+            y[c][3] = fmaf(c4.w, kv, y[c][3]);
+          }
         }
       }
-    }
+      if (ok) {
 #pragma unroll
-    for (int r = 0; r < kRowsPerGroup; ++r)
-      if (g0 + r < nr) {
-#pragma unroll
-        for (int i = 0; i < DPL; ++i) Y[(size_t)(g0 + r) * D + lane * DPL + i] = y[r][i];
+        for (int c = 0; c < NC; ++c)
+          *reinterpret_cast<float4*>(Y + (size_t)r * D + chunk_dim<D>(q, c)) = make_float4(y[c][0], y[c][1], y[c][2], y[c][3]);
       }
-    __syncwarp();
+    } else if (ok) {
+#pragma unroll
+      for (int c = 0; c < NC; ++c)
+        *reinterpret_cast<float4*>(Y + (size_t)r * D + chunk_dim<D>(q, c)) = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
   }
   // clamp list for the initial moments: entries with 0 < |n C_ab| < tau
   const float tau = a.tau;
   if (n > 0 && tau > 0.f) {
     const float nf = static_cast<float>(n);
-    for (int idx = tid; idx < D * D; idx += kThreads) {
+    for (int idx = tid; idx < D * D; idx += kCT) {
       const float c = Ct[idx];
       if (c != 0.f && fabsf(c * nf) < tau) {
         const int k = atomicAdd(&s_nz, 1);
@@ -538,34 +609,16 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kThreads)
 
   const int n_evict = len - a.budget;
   for (int e = 0; e < n_evict; ++e) {
-    // ---- phase A: per-head softmax normaliser over the whole unit
+    // ---- phase A: per-head softmax normaliser over every surviving row of
+    // the unit: Z_h = sum of e_hj (every CTA holds all of them: no exchange)
     {
-      float mx[G], zs[G];
-#pragma unroll
-      for (int h = 0; h < G; ++h) mx[h] = -INFINITY;
-      for (int r = tid; r < nr; r += kThreads)
-        if (alive[r]) {
-#pragma unroll
-          for (int h = 0; h < G; ++h) mx[h] = fmaxf(mx[h], lg[h * R + r]);
-        }
-#pragma unroll
-      for (int h = 0; h < G; ++h) {
-        mx[h] = warp_max(mx[h]);
-        if (lane == 0) s_red[warp][h] = mx[h];
-      }
-      __syncthreads();
-      if (tid < G) {
-        float m = -INFINITY;
-        for (int w = 0; w < kWarps; ++w) m = fmaxf(m, s_red[w][tid]);
-        s_M[tid] = m;
-      }
-      __syncthreads();
+      float zs[G];
 #pragma unroll
       for (int h = 0; h < G; ++h) zs[h] = 0.f;
-      for (int r = tid; r < nr; r += kThreads)
-        if (alive[r]) {
+      for (int jj = tid; jj < len; jj += kCT)
+        if (alive_all[jj]) {
 #pragma unroll
-          for (int h = 0; h < G; ++h) zs[h] += expf(lg[h * R + r] - s_M[h]);
+          for (int h = 0; h < G; ++h) zs[h] += lg[h * a.cap + jj];
         }
 #pragma unroll
       for (int h = 0; h < G; ++h) {
@@ -573,132 +626,198 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kThreads)
         if (lane == 0) s_red[warp][h] = zs[h];
       }
       __syncthreads();
-      if (tid < G) {
-        float z = 0.f;
-        for (int w = 0; w < kWarps; ++w) z += s_red[w][tid];
-        ex_ml[tid] = s_M[tid];
-        ex_ml[G + tid] = z;
+      if (warp == 0) {
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+          const float z = warp_sum(s_red[lane][h]);
+          if (lane == 0) s_invZ[h] = 1.f / z;
+        }
       }
+      __syncthreads();
     }
-    cluster.sync();
-    if (tid < G) {
-      float M = -INFINITY;
-      for (int r = 0; r < kCL; ++r) M = fmaxf(M, cluster.map_shared_rank(ex_ml, r)[tid]);
-      float Z = 0.f;
-      for (int r = 0; r < kCL; ++r) {
-        const float* rm = cluster.map_shared_rank(ex_ml, r);
-        if (rm[tid] != -INFINITY) Z += rm[G + tid] * expf(rm[tid] - M);
-      }
-      s_M[tid] = M;
-      s_Z[tid] = Z;
-    }
-    __syncthreads();
 
-    // ---- phase B: scores of this slice, local argmin
+    // ---- phase B: scores of this slice, local argmin (8 lanes per row)
     const float rs = (n > 0) ? scale : 0.f;
     const int nz = s_nz;
     const bool direct = nz > kMaxClamp;
     const float nf = static_cast<float>(n);
     unsigned long long best = ~0ull;
-    for (int r = warp; r < nr; r += kWarps) {
-      if (!alive[r]) continue;  // warp-uniform
-      float yv[DPL], vf[DPL];
-      load_bf16<DPL>(Vr + (size_t)r * D + lane * DPL, vf);
-      if (!direct) {
+    for (int base = 0; base < nr; base += kRowsPerPass) {
+      const int r = base + rsub;
+      const bool ok = (r < nr) && alive[r];
+      float ss = 0.f;
+      if (ok) {
+        if (!direct) {
 #pragma unroll
-        for (int i = 0; i < DPL; ++i) yv[i] = Y[(size_t)r * D + lane * DPL + i];
-        for (int z = 0; z < nz; ++z) {  // y'_a -= C_ab k_b for clamped (a, b)
-          const uint32_t idx = s_zidx[z];
-          const int cb = static_cast<int>(idx / D), ra = static_cast<int>(idx % D);
-          if (ra / DPL == lane) yv[ra % DPL] -= s_zval[z] * __bfloat162float(Kr[(size_t)r * D + cb]);
-        }
-      } else {
-        float kf[DPL];
-        load_bf16<DPL>(Kr + (size_t)r * D + lane * DPL, kf);
+          for (int c = 0; c < NC; ++c) {
+            const int d0 = chunk_dim<D>(q, c);
+            float4 y4 = *reinterpret_cast<const float4*>(Y + (size_t)r * D + d0);
+            for (int z = 0; z < nz; ++z) {  // y'_a -= C_ab k_b for clamped (a, b)
+              const int kb = static_cast<int>(s_zidx[z] / D), va = static_cast<int>(s_zidx[z] % D);
+              if (va >= d0 && va < d0 + 4) {
+                const float corr = s_zval[z] * __bfloat162float(Kr[(size_t)r * D + kb]);
+                const int o = va - d0;
+                if (o == 0) y4.x -= corr;
+                else if (o == 1) y4.y -= corr;
+                else if (o == 2) y4.z -= corr;
+                else y4.w -= corr;
+              }
+            }
+            float vf[4];
+            load4_bf16<D>(Vr + (size_t)r * D + d0, vf);
+            const float4 m4 = *reinterpret_cast<const float4*>(s_mu_v + d0);
+            const float r0 = vf[0] - m4.x - rs * y4.x, r1 = vf[1] - m4.y - rs * y4.y;
+            const float r2 = vf[2] - m4.z - rs * y4.z, r3 = vf[3] - m4.w - rs * y4.w;
+            ss = fmaf(r0, r0, fmaf(r1, r1, fmaf(r2, r2, fmaf(r3, r3, ss))));
+          }
+        } else {
+          float y[NC][4];
 #pragma unroll
-        for (int i = 0; i < DPL; ++i) yv[i] = 0.f;
-        for (int c = 0; c < D; ++c) {
-          const float kc = __shfl_sync(kFull, kf[c % DPL], c / DPL);
+          for (int c = 0; c < NC; ++c) y[c][0] = y[c][1] = y[c][2] = y[c][3] = 0.f;
+          for (int kc = 0; kc < D; ++kc) {
+            const float kv = __bfloat162float(Kr[(size_t)r * D + kc]);
 #pragma unroll
-          for (int i = 0; i < DPL; ++i) {
-            float cv = Ct[c * D + lane * DPL + i];
-            cv = (fabsf(cv * nf) < tau) ? 0.f : cv;
-            yv[i] = fmaf(cv, kc, yv[i]);
+            for (int c = 0; c < NC; ++c) {
+              const float4 c4 = *reinterpret_cast<const float4*>(Ct + kc * D + chunk_dim<D>(q, c));
+              y[c][0] = fmaf((fabsf(c4.x * nf) < tau) ? 0.f : c4.x, kv, y[c][0]);
+              y[c][1] = fmaf((fabsf(c4.y * nf) < tau) ? 0.f : c4.y, kv, y[c][1]);
+              y[c][2] = fmaf((fabsf(c4.z * nf) < tau) ? 0.f : c4.z, kv, y[c][2]);
+              y[c][3] = fmaf((fabsf(c4.w * nf) < tau) ? 0.f : c4.w, kv, y[c][3]);
+            }
+          }
+#pragma unroll
+          for (int c = 0; c < NC; ++c) {
+            const int d0 = chunk_dim<D>(q, c);
+            float vf[4];
+            load4_bf16<D>(Vr + (size_t)r * D + d0, vf);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              const float rr = vf[i] - s_mu_v[d0 + i] - rs * y[c][i];
+              ss = fmaf(rr, rr, ss);
+            }
           }
         }
       }
-      float ss = 0.f;
+      ss = group_sum(ss);
+      if (ok && q == 0) {
+        float alpha = 0.f;
 #pragma unroll
-      for (int i = 0; i < DPL; ++i) {
-        const float rr = vf[i] - s_mu_v[lane * DPL + i] - rs * yv[i];
-        ss = fmaf(rr, rr, ss);
+        for (int h = 0; h < G; ++h) alpha = fmaf(lg[h * a.cap + j0 + r], s_invZ[h], alpha);
+        const float score = alpha * sqrtf(ss);
+        const unsigned long long key =
+            (static_cast<unsigned long long>(__float_as_uint(score)) << 32) | static_cast<unsigned>(j0 + r);
+        best = key < best ? key : best;
       }
-      ss = warp_sum(ss);
-      float alpha = 0.f;
-#pragma unroll
-      for (int h = 0; h < G; ++h) alpha += expf(lg[h * R + r] - s_M[h]) / s_Z[h];
-      const float score = alpha * sqrtf(ss);
-      const unsigned long long key =
-          (static_cast<unsigned long long>(__float_as_uint(score)) << 32) | static_cast<unsigned>(j0 + r);
-      best = key < best ? key : best;
     }
     best = shfl_min_u64(best);
     if (lane == 0) s_bestw[warp] = best;
     __syncthreads();
-    if (tid == 0) {
-      unsigned long long b = s_bestw[0];
-      for (int w = 1; w < kWarps; ++w) b = s_bestw[w] < b ? s_bestw[w] : b;
-      ex_best = b;
-      s_nz = 0;
+    const int par = e & 1;
+    if (warp == 0) {
+      unsigned long long b = s_bestw[lane];
+      b = shfl_min_u64(b);
+      if (lane == 0) {
+        ex_best[par] = b;
+        s_nz = 0;
+      }
+      // publish the candidate row's k and v next to its key
+      const int jb = (b == ~0ull) ? -1 : static_cast<int>(b & 0xffffffffu) - j0;
+      if (jb >= 0 && lane < D / 8) {
+        reinterpret_cast<uint4*>(ex_row[par])[lane] = reinterpret_cast<const uint4*>(Kr + (size_t)jb * D)[lane];
+        reinterpret_cast<uint4*>(ex_row[par] + D)[lane] = reinterpret_cast<const uint4*>(Vr + (size_t)jb * D)[lane];
+      }
     }
     cluster.sync();
-    unsigned long long gb = ~0ull;
-    for (int r = 0; r < kCL; ++r) {
-      const unsigned long long v = *cluster.map_shared_rank(&ex_best, r);
-      gb = v < gb ? v : gb;
+    // every rank's key and candidate row in one round of remote reads
+    if (tid < kCL) s_keys[tid] = cluster.map_shared_rank(ex_best, tid)[par];
+    if (tid >= 32 && tid < 32 + kCL * (D / 4)) {
+      const int t = tid - 32, rk = t / (D / 4), i = t % (D / 4);
+      reinterpret_cast<uint4*>(s_cand[rk])[i] =
+          reinterpret_cast<const uint4*>(cluster.map_shared_rank(&ex_row[par][0], rk))[i];
     }
-    const int js = static_cast<int>(gb & 0xffffffffu);
+    __syncthreads();
+    if (tid == 0) {
+      unsigned long long b = s_keys[0];
+      int w = 0;
+      for (int r2 = 1; r2 < kCL; ++r2)
+        if (s_keys[r2] < b) {
+          b = s_keys[r2];
+          w = r2;
+        }
+      s_js = static_cast<int>(b & 0xffffffffu) | (w << 24);
+    }
+    __syncthreads();
+    const int js = s_js & 0xffffff, wr = s_js >> 24;
 
     // ---- phase C: fold row j* into the moments, update y for the slice
     const float n1 = static_cast<float>(n + 1);
-    for (int i = tid; i < D; i += kThreads) {
-      const float kx = __bfloat162float(Kg[(size_t)js * D + i]);
-      const float vx = __bfloat162float(Vg[(size_t)js * D + i]);
-      const float dk = kx - s_mu_k[i];
-      s_mu_k[i] += dk / n1;
-      const float mv = s_mu_v[i] + (vx - s_mu_v[i]) / n1;
-      s_mu_v[i] = mv;
-      s_dk[i] = dk;
-      s_dv[i] = vx - mv;
-    }
-    if (tid == 0 && js >= j0 && js < j1) alive[js - j0] = 0;
-    __syncthreads();
-    const float keep = static_cast<float>(n) / n1;
     const float inv = 1.f / n1;
-    for (int idx = tid; idx < D * D; idx += kThreads) {
-      const int c = idx / D, r = idx % D;  // Ct[c][r] = C[r][c]
-      const float v = keep * Ct[idx] + inv * s_dv[r] * s_dk[c];
-      Ct[idx] = v;
-      if (tau > 0.f && v != 0.f && fabsf(v * n1) < tau) {
-        const int k = atomicAdd(&s_nz, 1);
-        if (k < kMaxClamp) {
-          s_zidx[k] = static_cast<uint32_t>(idx);
-          s_zval[k] = v;
-        }
+    if (tid < D) {
+      const float kx = __bfloat162float(s_cand[wr][tid]);
+      const float vx = __bfloat162float(s_cand[wr][D + tid]);
+      const float dk = kx - s_mu_k[tid];
+      s_mu_k[tid] = fmaf(dk, inv, s_mu_k[tid]);
+      const float mv = fmaf(vx - s_mu_v[tid], inv, s_mu_v[tid]);
+      s_mu_v[tid] = mv;
+      s_dk[tid] = dk * inv;  // scaled by 1/(n+1) for the rank-1 terms below
+      s_dv[tid] = vx - mv;
+    }
+    if (tid == 0) alive_all[js] = 0;
+    __syncthreads();
+    const float keep = static_cast<float>(n) * inv;
+    const float thr = tau * inv;  // |C_ab| < tau / (n+1)  <=>  |(n+1) C_ab| < tau
+    for (int i4 = tid; i4 < D * D / 4; i4 += kCT) {
+      const int c = (i4 * 4) / D, r = (i4 * 4) % D;  // Ct[c][r..r+3] = C[r..r+3][c]
+      float4 v = reinterpret_cast<float4*>(Ct)[i4];
+      const float kd = s_dk[c];
+      const float4 dv = *reinterpret_cast<const float4*>(s_dv + r);
+      v.x = fmaf(keep, v.x, kd * dv.x);
+      v.y = fmaf(keep, v.y, kd * dv.y);
+      v.z = fmaf(keep, v.z, kd * dv.z);
+      v.w = fmaf(keep, v.w, kd * dv.w);
+      reinterpret_cast<float4*>(Ct)[i4] = v;
+      const bool any = (fabsf(v.x) < thr) | (fabsf(v.y) < thr) | (fabsf(v.z) < thr) | (fabsf(v.w) < thr);
+      if (any) {
+        const float vv[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          if (vv[k] != 0.f && fabsf(vv[k] * n1) < tau) {
+            const int slot = atomicAdd(&s_nz, 1);
+            if (slot < kMaxClamp) {
+              s_zidx[slot] = static_cast<uint32_t>(i4 * 4 + k);
+              s_zval[slot] = vv[k];
+            }
+          }
       }
     }
-    for (int r = warp; r < nr; r += kWarps) {
-      if (!alive[r]) continue;
-      float kf[DPL];
-      load_bf16<DPL>(Kr + (size_t)r * D + lane * DPL, kf);
+    for (int base = 0; base < nr; base += kRowsPerPass) {
+      const int r = base + rsub;
+      const bool ok = (r < nr) && alive[r];
+      float kf[NC][4];
       float dot = 0.f;
+      if (ok) {
 #pragma unroll
-      for (int i = 0; i < DPL; ++i) dot = fmaf(s_dk[lane * DPL + i], kf[i], dot);
-      dot = warp_sum(dot) * inv;
+        for (int c = 0; c < NC; ++c) {
+          const int d0 = chunk_dim<D>(q, c);
+          load4_bf16<D>(Kr + (size_t)r * D + d0, kf[c]);
+          const float4 k4 = *reinterpret_cast<const float4*>(s_dk + d0);
+          dot = fmaf(k4.x, kf[c][0], fmaf(k4.y, kf[c][1], fmaf(k4.z, kf[c][2], fmaf(k4.w, kf[c][3], dot))));
+        }
+      }
+      dot = group_sum(dot);
+      if (ok) {
 #pragma unroll
-      for (int i = 0; i < DPL; ++i) {
-        float* yp = Y + (size_t)r * D + lane * DPL + i;
-        *yp = keep * *yp + dot * s_dv[lane * DPL + i];
+        for (int c = 0; c < NC; ++c) {
+          const int d0 = chunk_dim<D>(q, c);
+          float4* yp = reinterpret_cast<float4*>(Y + (size_t)r * D + d0);
+          float4 y4 = *yp;
+          const float4 dv = *reinterpret_cast<const float4*>(s_dv + d0);
+          y4.x = fmaf(keep, y4.x, dot * dv.x);
+          y4.y = fmaf(keep, y4.y, dot * dv.y);
+          y4.z = fmaf(keep, y4.z, dot * dv.z);
+          y4.w = fmaf(keep, y4.w, dot * dv.w);
+          *yp = y4;
+        }
       }
     }
     n += 1;
@@ -708,13 +827,14 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kThreads)
   // ---- ordered compaction across the cluster through the staging buffer
   {
     int cnt = 0;
-    for (int r = tid; r < nr; r += kThreads) cnt += alive[r];
-    cnt = static_cast<int>(warp_sum(static_cast<float>(cnt)));
+    for (int r = tid; r < nr; r += kCT) cnt += alive[r];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) cnt += __shfl_xor_sync(kFull, cnt, o);
     if (lane == 0) s_red[warp][0] = static_cast<float>(cnt);
     __syncthreads();
     if (tid == 0) {
       int c = 0;
-      for (int w = 0; w < kWarps; ++w) c += static_cast<int>(s_red[w][0]);
+      for (int w = 0; w < kCW; ++w) c += static_cast<int>(s_red[w][0]);
       ex_cnt = c;
     }
   }
@@ -726,50 +846,44 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kThreads)
   __nv_bfloat16* SK = reinterpret_cast<__nv_bfloat16*>(st);
   __nv_bfloat16* SV = SK + (size_t)a.cap * D;
   int32_t* SP = reinterpret_cast<int32_t*>(SV + (size_t)a.cap * D);
-  if (warp == 0) {
-    int run = base;
-    for (int c0 = 0; c0 < nr; c0 += 32) {
-      const bool al = (c0 + lane < nr) && alive[c0 + lane];
-      const unsigned m = __ballot_sync(kFull, al);
-      if (al) SP[run + __popc(m & ((1u << lane) - 1u))] = Pg[j0 + c0 + lane];
-      run += __popc(m);
+  for (int c0 = 0; c0 < nr; c0 += 32) {
+    // warp w moves row c0 + w of this chunk (32 warps = 32 rows)
+    const bool al = (c0 + lane < nr) && alive[c0 + lane];
+    const unsigned m = __ballot_sync(kFull, al);
+    int before = 0;  // survivors in earlier chunks
+    for (int c1 = 0; c1 < c0; c1 += 32) {
+      const bool a1 = (c1 + lane < nr) && alive[c1 + lane];
+      before += __popc(__ballot_sync(kFull, a1));
     }
-  }
-  {
-    // rows: each warp copies survivors; destination = base + rank among survivors
-    for (int c0 = 0; c0 < nr; c0 += 32) {
-      const bool al = (c0 + lane < nr) && alive[c0 + lane];
-      const unsigned m = __ballot_sync(kFull, al);
-      int before = 0;  // survivors in earlier chunks
-      for (int c1 = 0; c1 < c0; c1 += 32) {
-        const bool a1 = (c1 + lane < nr) && alive[c1 + lane];
-        before += __popc(__ballot_sync(kFull, a1));
+    const int bit = warp;
+    if ((m >> bit) & 1u) {
+      const int r = c0 + bit;
+      const int dst = base + before + __popc(m & ((1u << bit) - 1u));
+      for (int i = lane; i < D / 8; i += 32) {
+        reinterpret_cast<uint4*>(SK + (size_t)dst * D)[i] = reinterpret_cast<const uint4*>(Kr + (size_t)r * D)[i];
+        reinterpret_cast<uint4*>(SV + (size_t)dst * D)[i] = reinterpret_cast<const uint4*>(Vr + (size_t)r * D)[i];
       }
-      for (int bit = warp; bit < 32; bit += kWarps) {
-        if (!((m >> bit) & 1u)) continue;
-        const int r = c0 + bit;
-        const int dst = base + before + __popc(m & ((1u << bit) - 1u));
-        for (int i = lane; i < D / 8; i += 32) {
-          reinterpret_cast<uint4*>(SK + (size_t)dst * D)[i] = reinterpret_cast<const uint4*>(Kr + (size_t)r * D)[i];
-          reinterpret_cast<uint4*>(SV + (size_t)dst * D)[i] = reinterpret_cast<const uint4*>(Vr + (size_t)r * D)[i];
-        }
-      }
+      if (lane == 0) SP[dst] = Pg[j0 + r];
     }
   }
   __threadfence();
   cluster.sync();
-  for (int idx = tid; idx < mine * (D / 8); idx += kThreads) {
+  for (int idx = tid; idx < mine * (D / 8); idx += kCT) {
     const int row = base + idx / (D / 8), i = idx % (D / 8);
     reinterpret_cast<uint4*>(Kg + (size_t)row * D)[i] = reinterpret_cast<const uint4*>(SK + (size_t)row * D)[i];
     reinterpret_cast<uint4*>(Vg + (size_t)row * D)[i] = reinterpret_cast<const uint4*>(SV + (size_t)row * D)[i];
   }
-  for (int r = tid; r < mine; r += kThreads) Pg[base + r] = SP[base + r];
+  for (int r = tid; r < mine; r += kCT) Pg[base + r] = SP[base + r];
   if (rank == 0) {
-    for (int idx = tid; idx < D * D; idx += kThreads) {
-      const int r = idx / D, c = idx % D;
-      a.C[(size_t)u * D * D + idx] = Ct[c * D + r];
+    float* tb = s_tile[warp % kTW];
+    for (int t = warp; warp < kTW && t < (D / 32) * (D / 32); t += kTW) {
+      const int c0 = (t / (D / 32)) * 32, r0 = (t % (D / 32)) * 32;
+      for (int i = 0; i < 32; ++i) tb[i * 33 + lane] = Ct[(size_t)(c0 + i) * D + r0 + lane];
+      __syncwarp();
+      for (int i = 0; i < 32; ++i) a.C[(size_t)u * D * D + (size_t)(r0 + i) * D + c0 + lane] = tb[lane * 33 + i];
+      __syncwarp();
     }
-    for (int i = tid; i < D; i += kThreads) {
+    for (int i = tid; i < D; i += kCT) {
       a.mu_k[(size_t)u * D + i] = s_mu_k[i];
       a.mu_v[(size_t)u * D + i] = s_mu_v[i];
     }
@@ -784,13 +898,13 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kThreads)
 template <int D, int G>
 size_t cluster_smem(int cap, int* kv) {
   const int R = (cap + kCL - 1) / kCL;
-  const size_t with_kv = ClusterLayout<D, G>(R, 1).total;
+  const size_t with_kv = ClusterLayout<D, G>(R, cap, 1).total;
   if (with_kv <= kSmemBudget) {
     *kv = 1;
     return with_kv;
   }
   *kv = 0;
-  return ClusterLayout<D, G>(R, 0).total;
+  return ClusterLayout<D, G>(R, cap, 0).total;
 }
 
 template <int D, int G>
@@ -804,7 +918,7 @@ cudaError_t launch_dg(const EvictArgs& a0, cudaStream_t stream) {
     cudaError_t e = cudaFuncSetAttribute(evict_cluster_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(csm));
     if (e != cudaSuccess) return e;
-    evict_cluster_kernel<D, G><<<a.batch * a.n_kv * kCL, kThreads, csm, stream>>>(a);
+    evict_cluster_kernel<D, G><<<a.batch * a.n_kv * kCL, kCT, csm, stream>>>(a);
     return cudaGetLastError();
   }
   const size_t smem = (size_t)D * D * 4 + (size_t)kWarps * kRowsPerGroup * D * 4 + align_up(a.cap, 16);
