@@ -5,9 +5,13 @@
 // into it instead of trapping; mkv_get_device_error reads and clears it.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
+#include <cudaTypedefs.h>
 #include <stdint.h>
+
+#include <mutex>
 
 #include "../../include/mkv.h"
 
@@ -86,6 +90,50 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
           smem_addr(dst)),
       "l"(src), "r"(bytes), "r"(smem_addr(bar))
       : "memory");
+}
+
+// 2-D tiled bulk copy (TMA) global -> shared through a tensor map; x is the
+// inner (element) coordinate and must be a multiple of 16 bytes' worth of
+// elements, y the row.  Out-of-range elements are filled with zeros.
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int x, int y, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+          smem_addr(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar))
+      : "memory");
+}
+
+// Host: encode a row-major bf16 matrix [rows][inner] (row stride in bytes) as a
+// 2-D tensor map with a box of box_rows x box_inner elements and the 128-byte
+// swizzle (box_inner * 2 <= 128).  Returns false if the driver refuses it.
+inline bool encode_tmap_bf16(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows,
+                             uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_rows) {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  if (fn == nullptr) return false;
+  const cuuint64_t dims[2] = {inner, rows};
+  const cuuint64_t strides[1] = {row_stride_bytes};
+  const cuuint32_t box[2] = {box_inner, box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Byte offset of element (r, c) in a tile of `rows` rows stored as boxes of 64
+// bf16 columns (128 B per row) with the 128-byte swizzle: within each 8-row
+// group, the 16-byte chunk index is XORed with (row mod 8).
+__device__ __forceinline__ uint32_t swz_off(int r, int c, int rows) {
+  const int box = c >> 6, cc = c & 63;
+  return static_cast<uint32_t>(box * rows * 128 + r * 128 + ((((cc >> 3) ^ (r & 7))) << 4) + (cc & 7) * 2);
 }
 
 // ----------------------------------------------------------------- numeric

@@ -3,15 +3,19 @@
 //
 // Grid (S, h_kv, b): every CTA serves all G query heads of one KV head
 // (GQA grouping, so K/V rows are read once per unit) over one contiguous
-// split of the retained rows.  Rows stream from HBM through a 4-stage ring of
-// shared-memory tiles filled by 1-D bulk copies (TMA engine, mbarrier
-// completion); compute is an online softmax per head.  The moment term
-// S_tilde q / (n sqrt d) is spread over the same CTAs: CTA s computes rows
-// [s*D/S, ...) of C'q for all G heads, so C (64 KB fp32 at d=128) is read once
-// per unit, concurrently with the K/V stream.  The last CTA of a unit to
-// finish (atomic ticket, no waiting) merges the S partial (m, l, o) states and
-// the moment pseudo-partial (log n + scale q.mu_k, f_hat_E) with a
-// log-sum-exp and writes the output; it also performs the append.
+// split of the retained rows.  Rows stream from HBM through a 3-stage ring of
+// 64-row tiles, each filled by 2-D TMA tensor copies (boxes of 64 rows x 64
+// columns, 128-byte swizzle, mbarrier completion); the swizzle makes every
+// shared-memory fragment load below bank-conflict-free.  Each warp takes 16
+// rows of a tile: S = Q K^T and O += P V run on the tensor cores
+// (mma.m16n8k16, bf16 in, fp32 accumulate) with the G query heads as the M
+// rows; P is split into bf16 hi + lo parts so the mixing weights keep ~16
+// bits.  The moment term S_tilde q / (n sqrt d) is spread over the same CTAs:
+// CTA s computes rows [s*D/S, ...) of C'q for all G heads, so C (64 KB fp32
+// at d=128) is read once per unit, concurrently with the K/V stream.  The last
+// CTA of a unit to finish (atomic ticket, no waiting) merges the S partial
+// (m, l, o) records with the moment pseudo-partial (log n + scale q.mu_k,
+// f_hat_E) by log-sum-exp and writes the output; it also performs the append.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -19,150 +23,117 @@ namespace mkv {
 
 namespace {
 
-constexpr int kThreads = 128;  // 4 warps, 8 tokens of each tile per warp
-constexpr int kStages = 4;
+constexpr int kThreads = 128;  // 4 warps x 16 rows of each 64-row tile
+constexpr int kStages = 3;
 constexpr int kTT = kDecodeTile;
 constexpr unsigned kFull = 0xffffffffu;
 
-// Butterfly transpose-reduction: each lane holds N partial sums (N = 8*G,
-// value index = token*G + head); afterwards lane l holds the full sums of
-// value indices [l*R, l*R+R) with R = max(1, N/32) (for N < 32 lanes that
-// differ only in the low bits hold copies: index = l >> log2(32/N)).
-template <int N>
-__device__ __forceinline__ void transpose_reduce(float (&v)[N], int lane) {
-#pragma unroll
-  for (int k = 0; k < 5; ++k) {
-    const int off = 16 >> k;
-    const int half = (N >> k) / 2;
-    if (half >= 1) {
-      const bool upper = (lane & off) != 0;
-#pragma unroll
-      for (int i = 0; i < (N >> (k + 1)); ++i) {
-        const float send = upper ? v[i] : v[i + (N >> (k + 1))];
-        const float keep = upper ? v[i + (N >> (k + 1))] : v[i];
-        v[i] = keep + __shfl_xor_sync(kFull, send, off);
-      }
-    } else {
-      v[0] += __shfl_xor_sync(kFull, v[0], off);
-    }
-  }
+__device__ __forceinline__ void mma_bf16(float (&d)[4], uint32_t a0, uint32_t a2, uint32_t b0, uint32_t b1) {
+  // A rows 8..15 are zero (at most 8 query heads per KV head): registers a1, a3 = 0
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(0u), "r"(a2), "r"(0u), "r"(b0), "r"(b1));
 }
 
-// Lane that holds (token j, head h) after transpose_reduce, and which of its
-// R values it is.
-template <int G>
-__device__ __forceinline__ int src_lane(int j, int h) {
-  if constexpr (G == 1) return j << 2;
-  else if constexpr (G == 2) return (j << 2) | (h << 1);
-  else if constexpr (G == 4) return (j << 2) | h;
-  else return (j << 2) | (h >> 1);
+__device__ __forceinline__ void ldsm_x4_trans(uint32_t (&r)[4], const void* p) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(smem_addr(p)));
 }
 
-template <int G>
-__device__ __forceinline__ int my_head(int lane, int r) {
-  if constexpr (G == 1) return 0;
-  else if constexpr (G == 2) return (lane >> 1) & 1;
-  else if constexpr (G == 4) return lane & 3;
-  else return ((lane & 3) << 1) | r;
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
 }
 
-template <int D, int G>
+// Per-warp online-softmax state for head g = lane/4 (meaningful when g < G):
+// running max m (log2 domain), sum l, and O[g][nt*8 + 2t + {0,1}] in o[nt][0..1].
+template <int D>
 struct WarpState {
-  static constexpr int DPL = D / 32;
-  float m[G];  // running max, log2 domain, replicated across lanes
-  float l[G];  // running sum, replicated
-  float o[G][DPL];
+  float m, l;
+  float o[D / 8][4];
 };
 
-// Process up to 8 rows (this warp's slice of a tile) of K/V in shared memory.
+// 16 rows [row0, row0 + 16) of a shared-memory tile; rows >= `rows` are masked.
 template <int D, int G>
-__device__ __forceinline__ void process_rows(WarpState<D, G>& st, const float (&qr)[G][D / 32],
-                                             const __nv_bfloat16* tK, const __nv_bfloat16* tV,
-                                             int row0, int rows, int lane) {
-  constexpr int DPL = D / 32;
-  constexpr int N = 8 * G;
-  constexpr int R = (N >= 32) ? N / 32 : 1;
-  float v[N];
+__device__ __forceinline__ void process16(WarpState<D>& st, const uint32_t (&qa)[D / 16][2],
+                                          const uint8_t* tK, const uint8_t* tV, int row0, int rows,
+                                          float qscale, int lane) {
+  const int g = lane >> 2, t = lane & 3;
+  float s[2][4];
 #pragma unroll
-  for (int j = 0; j < 8; ++j) {
-    float kf[DPL];
-    if (row0 + j < rows) {
-      load_bf16<DPL>(tK + (row0 + j) * D + lane * DPL, kf);
-    } else {
+  for (int nt = 0; nt < 2; ++nt) {
+    s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
+    const int r = row0 + nt * 8 + g;
 #pragma unroll
-      for (int i = 0; i < DPL; ++i) kf[i] = 0.f;
-    }
-#pragma unroll
-    for (int h = 0; h < G; ++h) {
-      float acc = 0.f;
-#pragma unroll
-      for (int i = 0; i < DPL; ++i) acc = fmaf(qr[h][i], kf[i], acc);
-      v[j * G + h] = acc;
+    for (int kk = 0; kk < D / 16; ++kk) {
+      const uint32_t b0 = *reinterpret_cast<const uint32_t*>(tK + swz_off(r, kk * 16 + 2 * t, kTT));
+      const uint32_t b1 = *reinterpret_cast<const uint32_t*>(tK + swz_off(r, kk * 16 + 8 + 2 * t, kTT));
+      mma_bf16(s[nt], qa[kk][0], qa[kk][1], b0, b1);
     }
   }
-  transpose_reduce<N>(v, lane);
-
-  const int j = lane >> 2;
-  const bool valid = (row0 + j) < rows;
-  float sc[R], tmax[R];
+  float x[4];
 #pragma unroll
-  for (int r = 0; r < R; ++r) {
-    sc[r] = valid ? v[r] : -INFINITY;
-    tmax[r] = sc[r];
+  for (int nt = 0; nt < 2; ++nt)
 #pragma unroll
-    for (int off = 4; off <= 16; off <<= 1) tmax[r] = fmaxf(tmax[r], __shfl_xor_sync(kFull, tmax[r], off));
-  }
-  // every lane learns every head's new running max and rescale factor
-  float mnew[G], alpha[G];
-#pragma unroll
-  for (int h = 0; h < G; ++h) {
-    const float tm = __shfl_sync(kFull, tmax[(G == 8) ? (h & 1) : 0], src_lane<G>(0, h));
-    mnew[h] = fmaxf(st.m[h], tm);
-    alpha[h] = (mnew[h] == -INFINITY) ? 1.f : fast_exp2(st.m[h] - mnew[h]);
-  }
-  float p[R], ls[R];
-#pragma unroll
-  for (int r = 0; r < R; ++r) {
-    const int hh = my_head<G>(lane, r);
-    float mm = 0.f;
-#pragma unroll
-    for (int h = 0; h < G; ++h) mm = (h == hh) ? mnew[h] : mm;
-    p[r] = valid ? fast_exp2(sc[r] - mm) : 0.f;
-    ls[r] = p[r];
-#pragma unroll
-    for (int off = 4; off <= 16; off <<= 1) ls[r] += __shfl_xor_sync(kFull, ls[r], off);
-  }
-#pragma unroll
-  for (int h = 0; h < G; ++h) {
-    const float lt = __shfl_sync(kFull, ls[(G == 8) ? (h & 1) : 0], src_lane<G>(0, h));
-    st.l[h] = st.l[h] * alpha[h] + lt;
-    st.m[h] = mnew[h];
-#pragma unroll
-    for (int i = 0; i < DPL; ++i) st.o[h][i] *= alpha[h];
-  }
-#pragma unroll
-  for (int jj = 0; jj < 8; ++jj) {
-    if (row0 + jj >= rows) break;  // warp-uniform
-    float vf[DPL];
-    load_bf16<DPL>(tV + (row0 + jj) * D + lane * DPL, vf);
-#pragma unroll
-    for (int h = 0; h < G; ++h) {
-      const float pj = __shfl_sync(kFull, p[(G == 8) ? (h & 1) : 0], src_lane<G>(jj, h));
-#pragma unroll
-      for (int i = 0; i < DPL; ++i) st.o[h][i] = fmaf(pj, vf[i], st.o[h][i]);
+    for (int j = 0; j < 2; ++j) {
+      const int tok = row0 + nt * 8 + 2 * t + j;
+      x[nt * 2 + j] = (tok < rows) ? s[nt][j] * qscale : -INFINITY;
     }
+  float tmax = fmaxf(fmaxf(x[0], x[1]), fmaxf(x[2], x[3]));
+  tmax = fmaxf(tmax, __shfl_xor_sync(kFull, tmax, 1));
+  tmax = fmaxf(tmax, __shfl_xor_sync(kFull, tmax, 2));
+  const float mnew = fmaxf(st.m, tmax);
+  const float alpha = (mnew == -INFINITY) ? 1.f : fast_exp2(st.m - mnew);
+  float p[4], ps = 0.f;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    p[i] = (x[i] == -INFINITY) ? 0.f : fast_exp2(x[i] - mnew);
+    ps += p[i];
+  }
+  ps += __shfl_xor_sync(kFull, ps, 1);
+  ps += __shfl_xor_sync(kFull, ps, 2);
+  st.l = st.l * alpha + ps;
+  st.m = mnew;
+#pragma unroll
+  for (int nt = 0; nt < D / 8; ++nt) {
+    st.o[nt][0] *= alpha;
+    st.o[nt][1] *= alpha;
+  }
+  // P as bf16 hi + lo (A operand: tokens 2t, 2t+1 and 8+2t, 8+2t+1 of row g)
+  const uint32_t ph0 = pack_bf16(p[0], p[1]), ph2 = pack_bf16(p[2], p[3]);
+  const float r0 = p[0] - __bfloat162float(__float2bfloat16_rn(p[0]));
+  const float r1 = p[1] - __bfloat162float(__float2bfloat16_rn(p[1]));
+  const float r2 = p[2] - __bfloat162float(__float2bfloat16_rn(p[2]));
+  const float r3 = p[3] - __bfloat162float(__float2bfloat16_rn(p[3]));
+  const uint32_t pl0 = pack_bf16(r0, r1), pl2 = pack_bf16(r2, r3);
+  const int mi = lane >> 3, mr = lane & 7;
+  const int vr = row0 + (mi & 1) * 8 + mr;
+#pragma unroll
+  for (int np = 0; np < D / 16; ++np) {
+    uint32_t vb[4];
+    ldsm_x4_trans(vb, tV + swz_off(vr, np * 16 + (mi >> 1) * 8, kTT));
+    mma_bf16(st.o[2 * np], ph0, ph2, vb[0], vb[1]);
+    mma_bf16(st.o[2 * np], pl0, pl2, vb[0], vb[1]);
+    mma_bf16(st.o[2 * np + 1], ph0, ph2, vb[2], vb[3]);
+    mma_bf16(st.o[2 * np + 1], pl0, pl2, vb[2], vb[3]);
   }
 }
 
 template <int D, int G>
-__global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a) {
+__global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, const __grid_constant__ CUtensorMap tmK,
+                                                          const __grid_constant__ CUtensorMap tmV) {
   constexpr int DPL = D / 32;
   constexpr int PS = D + 4;  // partial record: o[D], m (log2 domain), l
-  extern __shared__ __align__(128) uint8_t dsmem[];
-  __nv_bfloat16* sK = reinterpret_cast<__nv_bfloat16*>(dsmem);
-  __nv_bfloat16* sV = sK + kStages * kTT * D;
-  __nv_bfloat16* sNew = sV + kStages * kTT * D;  // [2][D]: new k, new v
-  __shared__ float sQ[G * D];                      // q * scale * log2(e)
+  constexpr int kTileBytes = kTT * D * 2;
+  extern __shared__ __align__(128) uint8_t dsmem_raw[];
+  // the 128-byte swizzle pattern repeats every 1024 bytes: align the ring to it
+  uint8_t* dsmem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dsmem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sK = dsmem;                          // [stage][box][kTT][128 B]
+  uint8_t* sV = dsmem + kStages * kTileBytes;
+  __shared__ float sQ[G * D];  // q * scale * log2(e)
   __shared__ float sSbar[G];
   __shared__ float sM[G], sL[G];
   __shared__ __align__(8) uint64_t bars[kStages];
@@ -190,16 +161,18 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a) {
   const bool own_new = has_new && t_begin <= len0 && len0 < t_end;
   const int n_tiles = (n_cached + kTT - 1) / kTT;
 
-  const __nv_bfloat16* Kg = reinterpret_cast<const __nv_bfloat16*>(a.K) + ((size_t)u * a.cap + t_begin) * D;
-  const __nv_bfloat16* Vg = reinterpret_cast<const __nv_bfloat16*>(a.V) + ((size_t)u * a.cap + t_begin) * D;
-
+  // one thread fills a stage: a 64-row box per 64 columns, for K and for V
+  // (rows past the unit's slab belong to the next unit or are zero-filled by
+  // the TMA unit; they are masked below)
+  const int row_base = u * a.cap + t_begin;
   auto issue = [&](int it) {
     const int st = it % kStages;
-    const int rows = min(kTT, n_cached - it * kTT);
-    const uint32_t bytes = static_cast<uint32_t>(rows) * D * 2u;
-    mbar_arrive_expect_tx(&bars[st], 2u * bytes);
-    bulk_g2s(sK + st * kTT * D, Kg + (size_t)it * kTT * D, bytes, &bars[st]);
-    bulk_g2s(sV + st * kTT * D, Vg + (size_t)it * kTT * D, bytes, &bars[st]);
+    mbar_arrive_expect_tx(&bars[st], 2u * kTileBytes);
+#pragma unroll
+    for (int bx = 0; bx < D / 64; ++bx) {
+      tma_load_2d(sK + st * kTileBytes + bx * kTT * 128, &tmK, bx * 64, row_base + it * kTT, &bars[st]);
+      tma_load_2d(sV + st * kTileBytes + bx * kTT * 128, &tmV, bx * 64, row_base + it * kTT, &bars[st]);
+    }
   };
 
   if (tid == 0) {
@@ -212,8 +185,28 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a) {
   }
 
   const __nv_bfloat16* qg = reinterpret_cast<const __nv_bfloat16*>(a.q) + ((size_t)u * G) * D;
+  // Q as the A operand: rows = heads (g = lane/4 < G), 16 dims per k-step
+  uint32_t qa[D / 16][2];
+  {
+    const int g = lane >> 2, t = lane & 3;
+#pragma unroll
+    for (int kk = 0; kk < D / 16; ++kk) {
+      qa[kk][0] = (g < G) ? *reinterpret_cast<const uint32_t*>(qg + g * D + kk * 16 + 2 * t) : 0u;
+      qa[kk][1] = (g < G) ? *reinterpret_cast<const uint32_t*>(qg + g * D + kk * 16 + 8 + 2 * t) : 0u;
+    }
+  }
   for (int i = tid; i < G * D; i += kThreads) sQ[i] = __bfloat162float(qg[i]) * (scale * kLog2e);
   __syncthreads();
+
+  // scale * q . mu_k for every head (every CTA; the last one uses it)
+  if (use_m) {
+    for (int h = warp; h < G; h += 4) {
+      float acc = 0.f;
+      for (int c = lane; c < D; c += 32) acc = fmaf(sQ[h * D + c], __ldg(a.mu_k + (size_t)u * D + c), acc);
+      acc = warp_sum(acc);
+      if (lane == 0) sSbar[h] = acc * (1.f / kLog2e);
+    }
+  }
 
   // ---- moment rows: f_hat_E[h][row] = mu_v[row] + scale * sum_c C'[row][c] q_h[c]
   // (each warp keeps RB rows' loads in flight before reducing them)
@@ -235,11 +228,11 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a) {
         if (row < r1) {
           const float* Crow = a.C + ((size_t)u * D + row) * D + lane * DPL;
           if constexpr (DPL == 4) {
-            const float4 t = __ldg(reinterpret_cast<const float4*>(Crow));
-            cv[k][0] = t.x; cv[k][1] = t.y; cv[k][2] = t.z; cv[k][3] = t.w;
+            const float4 t4 = __ldg(reinterpret_cast<const float4*>(Crow));
+            cv[k][0] = t4.x; cv[k][1] = t4.y; cv[k][2] = t4.z; cv[k][3] = t4.w;
           } else {
-            const float2 t = __ldg(reinterpret_cast<const float2*>(Crow));
-            cv[k][0] = t.x; cv[k][1] = t.y;
+            const float2 t2 = __ldg(reinterpret_cast<const float2*>(Crow));
+            cv[k][0] = t2.x; cv[k][1] = t2.y;
           }
           if (lane == 0) mv[k] = __ldg(a.mu_v + (size_t)u * D + row);
         }
@@ -267,29 +260,31 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a) {
   }
 
   // ---- retained rows
-  WarpState<D, G> st;
-  float qr[G][DPL];
+  WarpState<D> st;
+  st.m = -INFINITY;
+  st.l = 0.f;
 #pragma unroll
-  for (int h = 0; h < G; ++h) {
-    st.m[h] = -INFINITY;
-    st.l[h] = 0.f;
-#pragma unroll
-    for (int i = 0; i < DPL; ++i) {
-      st.o[h][i] = 0.f;
-      qr[h][i] = sQ[h * D + lane * DPL + i];
-    }
-  }
+  for (int nt = 0; nt < D / 8; ++nt) st.o[nt][0] = st.o[nt][1] = st.o[nt][2] = st.o[nt][3] = 0.f;
+  const float qscale = scale * kLog2e;
   bool ok = true;
   int it = 0;
   for (; it < n_tiles; ++it) {
     const int stg = it % kStages;
+    const int rows = min(kTT, n_cached - it * kTT);
     const bool got = mbar_wait(&bars[stg], (it / kStages) & 1);
     if (!__syncthreads_and(got)) {
       ok = false;
       break;
     }
-    const int rows = min(kTT, n_cached - it * kTT);
-    process_rows<D, G>(st, qr, sK + stg * kTT * D, sV + stg * kTT * D, warp * 8, rows, lane);
+    if (rows < kTT) {  // ragged tile: zero the unused V rows (P is 0 there, V must be finite)
+      for (int i = tid; i < (kTT - rows) * (D / 8); i += kThreads) {
+        const int r = rows + i / (D / 8), c = (i % (D / 8)) * 8;  // whole rows: layout-free
+        *reinterpret_cast<uint4*>(sV + stg * kTileBytes + (c >> 6) * kTT * 128 + r * 128 + (c & 63) * 2) =
+            make_uint4(0u, 0u, 0u, 0u);
+      }
+      __syncthreads();
+    }
+    process16<D, G>(st, qa, sK + stg * kTileBytes, sV + stg * kTileBytes, warp * 16, rows, qscale, lane);
     __syncthreads();
     if (tid == 0 && it + kStages < n_tiles) issue(it + kStages);
   }
@@ -300,33 +295,39 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a) {
       for (int j = it; j < min(n_tiles, it + kStages); ++j) (void)mbar_wait(&bars[j % kStages], (j / kStages) & 1);
     }
     __syncthreads();
+    st.m = -INFINITY;
+    st.l = 0.f;
 #pragma unroll
-    for (int h = 0; h < G; ++h) {
-      st.m[h] = -INFINITY;
-      st.l[h] = 0.f;
-    }
+    for (int nt = 0; nt < D / 8; ++nt) st.o[nt][0] = st.o[nt][1] = 0.f;
   }
-  if (own_new) {
+  if (own_new) {  // the appended token: row 0 of stage 0 (free now), rows 1..15 zero
     const __nv_bfloat16* kn = reinterpret_cast<const __nv_bfloat16*>(a.k_new) + (size_t)u * D;
     const __nv_bfloat16* vn = reinterpret_cast<const __nv_bfloat16*>(a.v_new) + (size_t)u * D;
-    for (int i = tid; i < D; i += kThreads) {
-      sNew[i] = kn[i];
-      sNew[D + i] = vn[i];
+    for (int i = tid; i < 16 * D; i += kThreads) {
+      const int r = i / D, c = i % D;
+      *reinterpret_cast<__nv_bfloat16*>(sK + swz_off(r, c, kTT)) = (r == 0) ? kn[c] : __float2bfloat16_rn(0.f);
+      *reinterpret_cast<__nv_bfloat16*>(sV + swz_off(r, c, kTT)) = (r == 0) ? vn[c] : __float2bfloat16_rn(0.f);
     }
     __syncthreads();
-    if (warp == 0) process_rows<D, G>(st, qr, sNew, sNew + D, 0, 1, lane);
+    if (warp == 0) process16<D, G>(st, qa, sK, sV, 0, 1, qscale, lane);
   }
 
   // ---- merge the 4 warps into this CTA's partial record (through the free tile ring)
   float* sRed = reinterpret_cast<float*>(dsmem);  // [4][G][D + 2]
   __syncthreads();
+  {
+    const int g = lane >> 2, t = lane & 3;
+    if (g < G) {
+      float* rw = sRed + (warp * G + g) * (D + 2);
 #pragma unroll
-  for (int h = 0; h < G; ++h) {
-#pragma unroll
-    for (int i = 0; i < DPL; ++i) sRed[(warp * G + h) * (D + 2) + lane * DPL + i] = st.o[h][i];
-    if (lane == 0) {
-      sRed[(warp * G + h) * (D + 2) + D] = st.m[h];
-      sRed[(warp * G + h) * (D + 2) + D + 1] = st.l[h];
+      for (int nt = 0; nt < D / 8; ++nt) {
+        rw[nt * 8 + 2 * t] = st.o[nt][0];
+        rw[nt * 8 + 2 * t + 1] = st.o[nt][1];
+      }
+      if (t == 0) {
+        rw[D] = st.m;
+        rw[D + 1] = st.l;
+      }
     }
   }
   __syncthreads();
@@ -362,25 +363,24 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a) {
   __threadfence();
   if (tid == 0) a.counters[u] = 0u;
 
-  if (use_m) {
-    for (int h = warp; h < G; h += 4) {
-      float acc = 0.f;
-      for (int c = lane; c < D; c += 32) acc = fmaf(sQ[h * D + c], a.mu_k[(size_t)u * D + c], acc);
-      acc = warp_sum(acc);
-      if (lane == 0) sSbar[h] = acc * (1.f / kLog2e);  // scale * q . mu_k
-    }
-  }
-  __syncthreads();
-
-  // combine the S partial records: per-(split, head) weights in shared
-  // memory, then each thread accumulates 4 output dims with all loads in flight
+  // combine the S partial records: stage them in shared memory with one round
+  // of loads when they fit in the (free) tile ring, else read them in place
   const float* pu = a.partial + (size_t)u * a.S * G * PS;
-  float* sW = reinterpret_cast<float*>(dsmem);  // [S][G] max, then weight
-  float* sLs = sW + a.S * G;                    // [S][G] sums
+  const size_t rec_floats = (size_t)a.S * G * PS;
+  const bool staged = rec_floats * 4 + 2 * a.S * G * 4 <= (size_t)kStages * 2 * kTileBytes;
+  float* sP = reinterpret_cast<float*>(dsmem);
+  const float* src = pu;
+  if (staged) {
+    for (size_t i = tid; i < rec_floats / 4; i += kThreads)
+      reinterpret_cast<float4*>(sP)[i] = __ldcg(reinterpret_cast<const float4*>(pu) + i);
+    src = sP;
+  }
+  float* sW = staged ? sP + rec_floats : sP;  // [S][G] max, then weight
+  float* sLs = sW + a.S * G;                  // [S][G] sums
   __syncthreads();
   for (int i = tid; i < a.S * G; i += kThreads) {
-    sW[i] = __ldcg(pu + (size_t)i * PS + D);
-    sLs[i] = __ldcg(pu + (size_t)i * PS + D + 1);
+    sW[i] = staged ? src[(size_t)i * PS + D] : __ldcg(src + (size_t)i * PS + D);
+    sLs[i] = staged ? src[(size_t)i * PS + D + 1] : __ldcg(src + (size_t)i * PS + D + 1);
   }
   __syncthreads();
   if (tid < G) {
@@ -402,11 +402,18 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a) {
   __syncthreads();
   for (int slot = tid; slot < G * (D / 4); slot += kThreads) {
     const int h = slot / (D / 4), d0 = (slot % (D / 4)) * 4;
+    float fh[4];
+    if (use_m) {
+#pragma unroll
+      for (int k = 0; k < 4; ++k)
+        fh[k] = (a.order == 1) ? __ldcg(a.fhat + ((size_t)u * G + h) * D + d0 + k) : a.mu_v[(size_t)u * D + d0 + k];
+    }
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll 4
     for (int sp = 0; sp < a.S; ++sp) {
       const float w = sW[sp * G + h];
-      const float4 o = __ldcg(reinterpret_cast<const float4*>(pu + ((size_t)sp * G + h) * PS + d0));
+      const float* rec = src + ((size_t)sp * G + h) * PS + d0;
+      const float4 o = staged ? *reinterpret_cast<const float4*>(rec) : __ldcg(reinterpret_cast<const float4*>(rec));
       acc.x = fmaf(w, o.x, acc.x);
       acc.y = fmaf(w, o.y, acc.y);
       acc.z = fmaf(w, o.z, acc.z);
@@ -420,10 +427,6 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a) {
     float res[4], lse = aR;
     if (use_m) {
       const float e = logf(static_cast<float>(n_e)) + sSbar[h];
-      float fh[4];
-#pragma unroll
-      for (int k = 0; k < 4; ++k)
-        fh[k] = (a.order == 1) ? __ldcg(a.fhat + ((size_t)u * G + h) * D + d0 + k) : a.mu_v[(size_t)u * D + d0 + k];
       if (have_r) {
         const float top = fmaxf(aR, e);
         const float wr = expf(aR - top), we = expf(e - top);
@@ -468,13 +471,19 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a) {
 
 template <int D, int G>
 cudaError_t launch_dg(const DecodeArgs& a, cudaStream_t stream) {
-  const size_t smem = (size_t)(2 * kStages * kTT * D + 2 * D) * sizeof(__nv_bfloat16);
+  const size_t smem = (size_t)2 * kStages * kTT * D * 2 + 1024;  // + alignment slack
   // per-device function attribute; setting it again is harmless
   cudaError_t e = cudaFuncSetAttribute(decode_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
+  // the cache slabs of all units as one [units * cap][D] matrix
+  const uint64_t rows = (uint64_t)a.batch * a.n_kv * a.cap;
+  CUtensorMap tmK, tmV;
+  if (!encode_tmap_bf16(&tmK, a.K, D, rows, (uint64_t)D * 2, 64, kTT) ||
+      !encode_tmap_bf16(&tmV, a.V, D, rows, (uint64_t)D * 2, 64, kTT))
+    return cudaErrorInvalidValue;
   dim3 grid(a.S, a.n_kv, a.batch);
-  decode_kernel<D, G><<<grid, kThreads, smem, stream>>>(a);
+  decode_kernel<D, G><<<grid, kThreads, smem, stream>>>(a, tmK, tmV);
   return cudaGetLastError();
 }
 

@@ -38,7 +38,7 @@ struct DecodeArgs {
   int32_t S;
 };
 
-constexpr int kDecodeTile = 32;  // tokens per pipeline stage
+constexpr int kDecodeTile = 64;  // tokens per pipeline stage
 
 int decode_splits(const mkv_geom& g, int32_t capacity, int num_sms);
 size_t decode_workspace_bytes(const mkv_geom& g, int32_t capacity, int num_sms);
