@@ -142,6 +142,45 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
   const int s = blockIdx.x, kv = blockIdx.y, b = blockIdx.z;
   const int u = b * a.n_kv + kv;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const float scale = rsqrtf(static_cast<float>(D));
+
+  // ---- loads that do not depend on the cache length go out first
+  const __nv_bfloat16* qg = reinterpret_cast<const __nv_bfloat16*>(a.q) + ((size_t)u * G) * D;
+  uint32_t qa[D / 16][2];  // Q as the A operand: rows = heads (g = lane/4 < G), 16 dims per k-step
+  {
+    const int g = lane >> 2, t = lane & 3;
+#pragma unroll
+    for (int kk = 0; kk < D / 16; ++kk) {
+      qa[kk][0] = (g < G) ? *reinterpret_cast<const uint32_t*>(qg + g * D + kk * 16 + 2 * t) : 0u;
+      qa[kk][1] = (g < G) ? *reinterpret_cast<const uint32_t*>(qg + g * D + kk * 16 + 8 + 2 * t) : 0u;
+    }
+  }
+  const bool corr = a.correction != 0 && a.n != nullptr;
+  constexpr int RB = 4;  // moment rows per warp whose loads are in flight together
+  const int rpc = (D + a.S - 1) / a.S;
+  const int r0 = s * rpc, r1 = min(D, r0 + rpc);
+  float cv[RB][DPL], mvr[RB], muk[DPL];
+#pragma unroll
+  for (int k = 0; k < RB; ++k) {
+    const int row = r0 + warp + 4 * k;
+    mvr[k] = 0.f;
+#pragma unroll
+    for (int i = 0; i < DPL; ++i) cv[k][i] = 0.f;
+    if (corr && a.order == 1 && row < r1) {
+      const float* Crow = a.C + ((size_t)u * D + row) * D + lane * DPL;
+      if constexpr (DPL == 4) {
+        const float4 t4 = __ldg(reinterpret_cast<const float4*>(Crow));
+        cv[k][0] = t4.x; cv[k][1] = t4.y; cv[k][2] = t4.z; cv[k][3] = t4.w;
+      } else {
+        const float2 t2 = __ldg(reinterpret_cast<const float2*>(Crow));
+        cv[k][0] = t2.x; cv[k][1] = t2.y;
+      }
+      mvr[k] = __ldg(a.mu_v + (size_t)u * D + row);
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < DPL; ++i) muk[i] = corr ? __ldg(a.mu_k + (size_t)u * D + lane * DPL + i) : 0.f;
+  const int n_e = corr ? a.n[u] : 0;
   int len0 = a.len[u];
   if (len0 < 0 || len0 > a.cap) {  // corrupt cache state: never read past the slab
     if (tid == 0 && s == 0) record_error(a.ws, MKV_ERR_CAPACITY, u);
@@ -149,9 +188,7 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
   }
   const bool has_new = a.k_new != nullptr;
   const int L = len0 + (has_new ? 1 : 0);
-  const int n_e = (a.correction != 0 && a.n != nullptr) ? a.n[u] : 0;
   const bool use_m = n_e > 0;
-  const float scale = rsqrtf(static_cast<float>(D));
 
   const int tiles_total = (L + kTT - 1) / kTT;
   const int tiles_per = (tiles_total + a.S - 1) / a.S;
@@ -178,82 +215,55 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
   if (tid == 0) {
     for (int i = 0; i < kStages; ++i) mbar_init(&bars[i], 1);
     mbar_fence_init();
-  }
-  __syncthreads();
-  if (tid == 0) {
     for (int i = 0; i < min(kStages, n_tiles); ++i) issue(i);
-  }
-
-  const __nv_bfloat16* qg = reinterpret_cast<const __nv_bfloat16*>(a.q) + ((size_t)u * G) * D;
-  // Q as the A operand: rows = heads (g = lane/4 < G), 16 dims per k-step
-  uint32_t qa[D / 16][2];
-  {
-    const int g = lane >> 2, t = lane & 3;
-#pragma unroll
-    for (int kk = 0; kk < D / 16; ++kk) {
-      qa[kk][0] = (g < G) ? *reinterpret_cast<const uint32_t*>(qg + g * D + kk * 16 + 2 * t) : 0u;
-      qa[kk][1] = (g < G) ? *reinterpret_cast<const uint32_t*>(qg + g * D + kk * 16 + 8 + 2 * t) : 0u;
-    }
   }
   for (int i = tid; i < G * D; i += kThreads) sQ[i] = __bfloat162float(qg[i]) * (scale * kLog2e);
   __syncthreads();
 
-  // scale * q . mu_k for every head (every CTA; the last one uses it)
   if (use_m) {
+    // scale * q . mu_k for every head (every CTA; the last one uses it)
     for (int h = warp; h < G; h += 4) {
       float acc = 0.f;
-      for (int c = lane; c < D; c += 32) acc = fmaf(sQ[h * D + c], __ldg(a.mu_k + (size_t)u * D + c), acc);
+#pragma unroll
+      for (int i = 0; i < DPL; ++i) acc = fmaf(sQ[h * D + lane * DPL + i], muk[i], acc);
       acc = warp_sum(acc);
       if (lane == 0) sSbar[h] = acc * (1.f / kLog2e);
     }
-  }
-
-  // ---- moment rows: f_hat_E[h][row] = mu_v[row] + scale * sum_c C'[row][c] q_h[c]
-  // (each warp keeps RB rows' loads in flight before reducing them)
-  if (use_m && a.order == 1) {
-    constexpr int RB = 4;
-    const int rpc = (D + a.S - 1) / a.S;
-    const int r0 = s * rpc, r1 = min(D, r0 + rpc);
-    const float tau = a.tau;
-    const float nf = static_cast<float>(n_e);
-    for (int base = r0 + warp; base < r1; base += 4 * RB) {
-      float cv[RB][DPL];
-      float mv[RB];
+    // moment rows: f_hat_E[h][row] = mu_v[row] + scale * sum_c C'[row][c] q_h[c]
+    if (a.order == 1) {
+      const float tau = a.tau;
+      const float nf = static_cast<float>(n_e);
+      for (int base = r0 + warp; base < r1; base += 4 * RB) {
+        if (base != r0 + warp) {  // rows beyond the first batch (few splits): load now
 #pragma unroll
-      for (int k = 0; k < RB; ++k) {
-        const int row = base + 4 * k;
-        mv[k] = 0.f;
+          for (int k = 0; k < RB; ++k) {
+            const int row = base + 4 * k;
+            if (row < r1) {
+              const float* Crow = a.C + ((size_t)u * D + row) * D + lane * DPL;
 #pragma unroll
-        for (int i = 0; i < DPL; ++i) cv[k][i] = 0.f;
-        if (row < r1) {
-          const float* Crow = a.C + ((size_t)u * D + row) * D + lane * DPL;
-          if constexpr (DPL == 4) {
-            const float4 t4 = __ldg(reinterpret_cast<const float4*>(Crow));
-            cv[k][0] = t4.x; cv[k][1] = t4.y; cv[k][2] = t4.z; cv[k][3] = t4.w;
-          } else {
-            const float2 t2 = __ldg(reinterpret_cast<const float2*>(Crow));
-            cv[k][0] = t2.x; cv[k][1] = t2.y;
+              for (int i = 0; i < DPL; ++i) cv[k][i] = __ldg(Crow + i);
+              mvr[k] = __ldg(a.mu_v + (size_t)u * D + row);
+            }
           }
-          if (lane == 0) mv[k] = __ldg(a.mu_v + (size_t)u * D + row);
         }
-      }
 #pragma unroll
-      for (int k = 0; k < RB; ++k) {
-        const int row = base + 4 * k;
-        if (row >= r1) break;  // warp-uniform
+        for (int k = 0; k < RB; ++k) {
+          const int row = base + 4 * k;
+          if (row >= r1) break;  // warp-uniform
 #pragma unroll
-        for (int i = 0; i < DPL; ++i) cv[k][i] = (fabsf(cv[k][i] * nf) < tau) ? 0.f : cv[k][i];
-        float acc[G];
+          for (int i = 0; i < DPL; ++i) cv[k][i] = (fabsf(cv[k][i] * nf) < tau) ? 0.f : cv[k][i];
+          float acc[G];
 #pragma unroll
-        for (int h = 0; h < G; ++h) {
-          acc[h] = 0.f;
+          for (int h = 0; h < G; ++h) {
+            acc[h] = 0.f;
 #pragma unroll
-          for (int i = 0; i < DPL; ++i) acc[h] = fmaf(cv[k][i], sQ[h * D + lane * DPL + i], acc[h]);
-          acc[h] = warp_sum(acc[h]);
-        }
-        if (lane == 0) {
+            for (int i = 0; i < DPL; ++i) acc[h] = fmaf(cv[k][i], sQ[h * D + lane * DPL + i], acc[h]);
+            acc[h] = warp_sum(acc[h]);
+          }
+          if (lane == 0) {
 #pragma unroll
-          for (int h = 0; h < G; ++h) a.fhat[((size_t)u * G + h) * D + row] = mv[k] + acc[h] * (1.f / kLog2e);
+            for (int h = 0; h < G; ++h) a.fhat[((size_t)u * G + h) * D + row] = mvr[k] + acc[h] * (1.f / kLog2e);
+          }
         }
       }
     }
@@ -310,6 +320,14 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
     }
     __syncthreads();
     if (warp == 0) process16<D, G>(st, qa, sK, sV, 0, 1, qscale, lane);
+    if (len0 + 1 <= a.cap) {  // nobody reads this cache row during the step
+      __nv_bfloat16* Kd = reinterpret_cast<__nv_bfloat16*>(a.K) + ((size_t)u * a.cap + len0) * D;
+      __nv_bfloat16* Vd = reinterpret_cast<__nv_bfloat16*>(a.V) + ((size_t)u * a.cap + len0) * D;
+      for (int i = tid; i < D; i += kThreads) {
+        Kd[i] = kn[i];
+        Vd[i] = vn[i];
+      }
+    }
   }
 
   // ---- merge the 4 warps into this CTA's partial record (through the free tile ring)
@@ -367,16 +385,24 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
   // of loads when they fit in the (free) tile ring, else read them in place
   const float* pu = a.partial + (size_t)u * a.S * G * PS;
   const size_t rec_floats = (size_t)a.S * G * PS;
-  const bool staged = rec_floats * 4 + 2 * a.S * G * 4 <= (size_t)kStages * 2 * kTileBytes;
+  const bool staged = rec_floats * 4 + (2 * a.S * G + G * D) * 4 <= (size_t)kStages * 2 * kTileBytes;
   float* sP = reinterpret_cast<float*>(dsmem);
   const float* src = pu;
+  float* sF = sP;  // [G][D] f_hat_E rows (or mu_v for order 0)
   if (staged) {
+    sF = sP + rec_floats;
     for (size_t i = tid; i < rec_floats / 4; i += kThreads)
       reinterpret_cast<float4*>(sP)[i] = __ldcg(reinterpret_cast<const float4*>(pu) + i);
+    if (use_m) {
+      for (int i = tid; i < G * D / 4; i += kThreads)
+        reinterpret_cast<float4*>(sF)[i] =
+            (a.order == 1) ? __ldcg(reinterpret_cast<const float4*>(a.fhat + (size_t)u * G * D) + i)
+                           : __ldg(reinterpret_cast<const float4*>(a.mu_v + (size_t)u * D) + (i % (D / 4)));
+    }
     src = sP;
   }
-  float* sW = staged ? sP + rec_floats : sP;  // [S][G] max, then weight
-  float* sLs = sW + a.S * G;                  // [S][G] sums
+  float* sW = staged ? sF + G * D : sP;  // [S][G] max, then weight
+  float* sLs = sW + a.S * G;             // [S][G] sums
   __syncthreads();
   for (int i = tid; i < a.S * G; i += kThreads) {
     sW[i] = staged ? src[(size_t)i * PS + D] : __ldcg(src + (size_t)i * PS + D);
@@ -406,7 +432,9 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
     if (use_m) {
 #pragma unroll
       for (int k = 0; k < 4; ++k)
-        fh[k] = (a.order == 1) ? __ldcg(a.fhat + ((size_t)u * G + h) * D + d0 + k) : a.mu_v[(size_t)u * D + d0 + k];
+        fh[k] = staged ? sF[h * D + d0 + k]
+                       : ((a.order == 1) ? __ldcg(a.fhat + ((size_t)u * G + h) * D + d0 + k)
+                                         : a.mu_v[(size_t)u * D + d0 + k]);
     }
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll 4
@@ -448,23 +476,13 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
     if (a.lse != nullptr && d0 == 0) a.lse[(size_t)u * G + h] = lse;
   }
 
-  if (has_new) {
+  if (has_new && tid == 0) {  // the row itself was written by the CTA that attended to it
     if (len0 + 1 > a.cap) {
-      if (tid == 0) record_error(a.ws, MKV_ERR_CAPACITY, u);
+      record_error(a.ws, MKV_ERR_CAPACITY, u);
     } else {
-      const __nv_bfloat16* kn = reinterpret_cast<const __nv_bfloat16*>(a.k_new) + (size_t)u * D;
-      const __nv_bfloat16* vn = reinterpret_cast<const __nv_bfloat16*>(a.v_new) + (size_t)u * D;
-      __nv_bfloat16* Kd = reinterpret_cast<__nv_bfloat16*>(a.K) + ((size_t)u * a.cap + len0) * D;
-      __nv_bfloat16* Vd = reinterpret_cast<__nv_bfloat16*>(a.V) + ((size_t)u * a.cap + len0) * D;
-      for (int i = tid; i < D; i += kThreads) {
-        Kd[i] = kn[i];
-        Vd[i] = vn[i];
-      }
-      if (tid == 0) {
-        a.pos[(size_t)u * a.cap + len0] = a.seen[u];
-        a.seen[u] = a.seen[u] + 1;
-        a.len[u] = len0 + 1;
-      }
+      a.pos[(size_t)u * a.cap + len0] = a.seen[u];
+      a.seen[u] = a.seen[u] + 1;
+      a.len[u] = len0 + 1;
     }
   }
 }
