@@ -1,44 +1,58 @@
 // Prefill compression (Sec. 5.1 SnapKV protocol with the moment filter of
 // Sec. 4.2, read as two data-parallel selection stages).
 //
-// Launch sequence per call (all on one stream):
-//   stats    (chunk, unit)  window-row online (max, sum) of the causal logits
-//                           l = scale q . k, and the chunk's centred moments
-//                           (n_c, mean k, mean v, co-moment M_c = sum (v-mv)(k-mk)^T)
-//   scores   (chunk, unit)  s_t = sum over rows of exp(l - m_row) / l_row,
-//                           pooled into aligned chunks of `pool` tokens
-//   select   (unit)         R0 = protected + top-k(s)   (radix select, ties
-//                           to the lower position), mean k/v of R0
-//   moments  (rows, unit)   moments of E0 = all \ R0: multi-way Chan merge of
-//                           the chunk moments minus R0's own centred moments
-//   residual (chunk, unit)  score2_t = s_t ||v_t - mu_v0 - scale C0' k_t||
-//   select   (unit)         R = protected + top-k(score2)
-//   moments  (rows, unit)   moments of E = all \ R -> caller's mkv_moments
-//   gather   (rows, unit)   retained rows of R, ascending, -> caller's cache
+// Launch sequence per call (one stream):
+//   stats_tc  (chunk, unit)  window logits Q_obs K^T on the tensor cores ->
+//                            online (max, sum) of each causal window row; the
+//                            covariance V^T K accumulated in TMEM and the column
+//                            sums -> the chunk's centred moments
+//   scores_tc (chunk, unit)  logits again (token-major) -> s_t = sum over rows
+//                            of exp(l - m_row) / l_row, pooled
+//   select    (unit)         R0 = protected + top-k(s) (radix select, ties to the
+//                            lower position); R0's rows gathered densely
+//   stats_tc  (unit)         moments of the gathered R0 rows (no logits)
+//   finalize  (rows, unit)   M0 = moments(all) - moments(R0) (Chan merges)
+//   residual_tc (chunk, unit) Y = K C0'^T on the tensor cores (C0' split into
+//                            three bf16 parts) -> score2 = s_t ||v - mu_v0 - scale y||
+//   select    (unit)         R = protected + top-k(score2), gathered into the cache
+//   stats_tc  (unit)         moments of the retained rows
+//   finalize  (rows, unit)   moments of E = all \ R -> caller's mkv_moments
+//
+// The tensor-core kernels are warp-specialised: warp 0 issues the TMA copies
+// (3-D tensor maps over per-unit slabs: rows past a unit's end read as zeros),
+// warp 1 owns TMEM and issues tcgen05.mma, warps 2-5 run the epilogue; stages
+// hand over through mbarriers whose waits are all bounded.  Head dims below
+// 128 use the same 128-wide MMAs: the missing 64-column box is zero-filled.
 #include "common.cuh"
 #include "kernels.h"
+#include "tc.cuh"
 
 namespace mkv {
 
 namespace {
 
-constexpr int kTT = 32;  // tokens per tile (one per lane)
+constexpr int kTok = 128;                   // tokens per tile
+constexpr int kDP = 128;                    // padded head dim of every MMA
+constexpr int kTileBytes = kTok * kDP * 2;  // one [128 x 128] bf16 tile: 2 boxes of 16 KB
+constexpr int kBoxBytes = kTok * 128;
+constexpr int kTcThreads = 192;  // warp 0 TMA, warp 1 MMA, warps 2..5 epilogue
+constexpr int kSelThreads = 1024;
 constexpr unsigned kFull = 0xffffffffu;
 
 struct Layout {
-  int D, G, W, RW;  // head dim, group, window, window rows = G*W
+  int D, G, W, RW, RWb;  // head dim, group, window, window rows = G*W, 128-row blocks of them
   int T, B;
   int units, n_chunks, chunk;
-  size_t rec;  // floats per chunk-moment record: 4 + 2D + D*D (padded)
-  // carved pointers
-  float* rowpart;   // [units][n_chunks][RW][2]
-  float* mpart;     // [units][n_chunks][rec]
-  float* s;         // [units][T]
-  float* s2;        // [units][T]
-  int32_t* idx0;    // [units][B]
-  int32_t* idx1;    // [units][B]
-  float* rmean;     // [units][2][4 + 2D]   n_R, mean k, mean v of R0 / R
-  float* m0;        // [units][4 + 2D + D*D] n0, mu_k0, mu_v0, C0
+  size_t rec;         // floats per moment record: 4 + 2D + D*D (padded)
+  float* rowpart;     // [units][n_chunks][RW][2]  (max in log2 units, sum)
+  float* mpart;       // [units][n_chunks][rec]    all-token chunk moments
+  float* rpart;       // [units][rec]              retained-set moments
+  float* s;           // [units][T]
+  float* s2;          // [units][T]
+  int32_t* idx;       // [units][B]
+  __nv_bfloat16* gK;  // [units][B][D] rows of R0
+  __nv_bfloat16* gV;
+  float* m0;  // [units][rec] moments of E0
 };
 
 __host__ __device__ inline size_t rec_floats(int D) { return align_up(4 + 2 * (size_t)D + (size_t)D * D, 4); }
@@ -49,14 +63,15 @@ Layout make_layout(const mkv_geom& g, int T, int B, int W, int num_sms) {
   L.G = g.group;
   L.W = W;
   L.RW = g.group * W;
+  L.RWb = (L.RW + 127) / 128;
   L.T = T;
   L.B = B;
   L.units = g.batch * g.n_kv_heads;
-  long target = (2L * num_sms + L.units - 1) / L.units;
-  long tiles = (T + kTT - 1) / kTT;
-  if (target > tiles) target = tiles;
-  if (target < 1) target = 1;
-  L.chunk = static_cast<int>(((tiles + target - 1) / target) * kTT);
+  long per = num_sms / L.units;  // one resident CTA per SM: fill the machine once
+  const long tiles = (T + kTok - 1) / kTok;
+  if (per < 1) per = 1;
+  if (per > tiles) per = tiles;
+  L.chunk = static_cast<int>(((tiles + per - 1) / per) * kTok);
   L.n_chunks = (T + L.chunk - 1) / L.chunk;
   L.rec = rec_floats(L.D);
   return L;
@@ -73,18 +88,14 @@ size_t carve(Layout& L, void* ws) {
   const size_t U = L.units;
   L.rowpart = reinterpret_cast<float*>(take(U * L.n_chunks * L.RW * 2 * sizeof(float)));
   L.mpart = reinterpret_cast<float*>(take(U * L.n_chunks * L.rec * sizeof(float)));
+  L.rpart = reinterpret_cast<float*>(take(U * L.rec * sizeof(float)));
   L.s = reinterpret_cast<float*>(take(U * (size_t)L.T * sizeof(float)));
   L.s2 = reinterpret_cast<float*>(take(U * (size_t)L.T * sizeof(float)));
-  L.idx0 = reinterpret_cast<int32_t*>(take(U * (size_t)L.B * sizeof(int32_t)));
-  L.idx1 = reinterpret_cast<int32_t*>(take(U * (size_t)L.B * sizeof(int32_t)));
-  L.rmean = reinterpret_cast<float*>(take(U * 2 * (4 + 2 * (size_t)L.D) * sizeof(float)));
-  L.m0 = reinterpret_cast<float*>(take(U * rec_floats(L.D) * sizeof(float)));
+  L.idx = reinterpret_cast<int32_t*>(take(U * (size_t)L.B * sizeof(int32_t)));
+  L.gK = reinterpret_cast<__nv_bfloat16*>(take(U * (size_t)L.B * L.D * 2));
+  L.gV = reinterpret_cast<__nv_bfloat16*>(take(U * (size_t)L.B * L.D * 2));
+  L.m0 = reinterpret_cast<float*>(take(U * L.rec * sizeof(float)));
   return off;
-}
-
-// Is window row r = h*W + i allowed to see token t?
-__device__ __forceinline__ bool visible(int t, int i, int T, int W, int causal) {
-  return !causal || t <= T - W + i;
 }
 
 __device__ __forceinline__ bool is_protected(int t, int T, int W, int sink, int keep_window) {
@@ -98,226 +109,524 @@ __host__ __device__ __forceinline__ int protected_count(int T, int W, int sink, 
   return s + w - overlap;
 }
 
-// Load a [kTT][D] bf16 tile (rows t0..t0+rows-1) into fp32 shared memory with
-// row stride D+1 (conflict-free both along rows and along columns).
-template <int D>
-__device__ __forceinline__ void load_tile(float* dst, const __nv_bfloat16* src, int rows, int tid, int nthr) {
-  for (int idx = tid; idx < kTT * (D / 2); idx += nthr) {
-    const int r = idx / (D / 2), c2 = (idx % (D / 2)) * 2;
-    float2 f = make_float2(0.f, 0.f);
-    if (r < rows) f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(src + (size_t)r * D + c2));
-    dst[r * (D + 1) + c2] = f.x;
-    dst[r * (D + 1) + c2 + 1] = f.y;
-  }
+// bf16 element (r, c) of a [128 x 128] tile held as two 64-column boxes with
+// the 128-byte swizzle (the TMA layout).
+__device__ __forceinline__ float tile_at(const uint8_t* tile, int r, int c) {
+  return __bfloat162float(*reinterpret_cast<const __nv_bfloat16*>(tile + swz_off(r, c, kTok)));
 }
 
-// Logits of 4 window rows (qT holds q*scale*log2e transposed, [D][RWpad]) for
-// the 32 tokens of a tile, one token per lane.
-template <int D>
-__device__ __forceinline__ void logits4(float (&acc)[4], const float* qT, int RWp, int r0, const float* tK,
-                                        int lane) {
-#pragma unroll
-  for (int i = 0; i < 4; ++i) acc[i] = 0.f;
-#pragma unroll 8
-  for (int c = 0; c < D; ++c) {
-    const float kc = tK[lane * (D + 1) + c];
-    const float4 q4 = *reinterpret_cast<const float4*>(qT + c * RWp + r0);
-    acc[0] = fmaf(q4.x, kc, acc[0]);
-    acc[1] = fmaf(q4.y, kc, acc[1]);
-    acc[2] = fmaf(q4.z, kc, acc[2]);
-    acc[3] = fmaf(q4.w, kc, acc[3]);
-  }
+__device__ __forceinline__ void epi_sync() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+
+// Pipeline wait that gives up after the bounded poll count: records the
+// timeout once and raises the CTA's abort flag so that no other role waits on.
+__device__ __forceinline__ bool pwait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, void* ws, int u) {
+  if (*abort_flag) return false;
+  if (mbar_wait(bar, parity)) return true;
+  *abort_flag = 1;
+  record_error(ws, MKV_ERR_TIMEOUT, u);
+  return false;
 }
 
-// ----------------------------------------------------------------- stats
-template <int D>
-__global__ void __launch_bounds__(256) stats_kernel(const CompressArgs a, const Layout L) {
-  constexpr int NT = 256;
-  extern __shared__ __align__(16) float sm[];
-  const int RWp = align_up(L.RW, 4);
-  float* qT = sm;                          // [D][RWp]
-  float* tK = qT + D * RWp;                // [32][D+1]
-  float* tV = tK + kTT * (D + 1);          // [32][D+1]
-  float* rowm = tV + kTT * (D + 1);        // [RWp]
-  float* rowl = rowm + RWp;                // [RWp]
+struct TcArgs {
+  int n_rows;  // rows of each unit's slab that take part
+  int chunk;   // rows per CTA (multiple of kTok)
+  int n_chunks;
+  int D, RW, RWb, W, T, causal, sink, keep_window, pool;
+  float qscale;  // scale * log2(e)
+  float tau;
+  float* rowpart;
+  float* mrec;  // moment records, [units][n_chunks][rec]
+  const float* s_in;
+  float* s_out;
+  float* diag;
+  const float* m0;
+  void* ws;
+};
+
+// --------------------------------------------------------------- stats_tc
+// LOGITS = 1: window-row statistics and chunk moments of the prompt;
+// LOGITS = 0: moments only (a dense row set).
+template <int LOGITS>
+__global__ void __launch_bounds__(kTcThreads, 1)
+    stats_tc(const TcArgs p, const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+             const __grid_constant__ CUtensorMap tmQ) {
+  constexpr int kS = 2;
+  extern __shared__ __align__(1024) uint8_t smraw[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sK = sm;                        // [kS][128 x 128]
+  uint8_t* sV = sm + kS * kTileBytes;      // [kS][128 x 128]
+  uint8_t* sQ = sm + 2 * kS * kTileBytes;  // [2 boxes][RWb*128 rows][128 B]
+  __shared__ __align__(8) uint64_t full[kS], empty[kS], lfull, lempty, qfull, sdone;
+  __shared__ uint32_t tmem_base;
+  __shared__ int abort_flag;
+  __shared__ float sum_k[kDP], sum_v[kDP];
+
   const int chunk = blockIdx.x, u = blockIdx.y;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int t_begin = chunk * L.chunk;
-  const int t_end = min(L.T, t_begin + L.chunk);
-  const float qs = rsqrtf(static_cast<float>(D)) * kLog2e;
+  const int t_begin = chunk * p.chunk;
+  const int t_end = min(p.n_rows, t_begin + p.chunk);
+  const int n_tiles = (max(0, t_end - t_begin) + kTok - 1) / kTok;
+  const int RWb = p.RWb;
+  volatile int* abrt = &abort_flag;
 
-  const __nv_bfloat16* Qg = reinterpret_cast<const __nv_bfloat16*>(a.Q) + (size_t)u * L.RW * D;
-  for (int idx = tid; idx < D * RWp; idx += NT) {
-    const int c = idx / RWp, r = idx % RWp;
-    qT[idx] = (r < L.RW) ? __bfloat162float(Qg[(size_t)r * D + c]) * qs : 0.f;
+  if (tid == 0) {
+    for (int i = 0; i < kS; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], 1 + 4);  // MMA commit + the 4 epilogue warps (column sums)
+    }
+    mbar_init(&lfull, 1);
+    mbar_init(&lempty, 4);
+    mbar_init(&qfull, 1);
+    mbar_init(&sdone, 1);
+    abort_flag = 0;
+    mbar_fence_init();
   }
-  for (int r = tid; r < RWp; r += NT) {
-    rowm[r] = -INFINITY;
-    rowl[r] = 0.f;
-  }
-  // S accumulator: thread owns an (D/16) x 8 block: rows a0.., cols c0..
-  constexpr int AR = D / 16;  // 8 at D=128, 4 at D=64
-  const int a0 = (tid / 16) * AR, c0 = (tid % 16) * (D / 16);
-  constexpr int CC = D / 16;
-  float S[AR][CC];
-#pragma unroll
-  for (int i = 0; i < AR; ++i)
-#pragma unroll
-    for (int j = 0; j < CC; ++j) S[i][j] = 0.f;
-  float colsum = 0.f;  // tid < D: sum k[:, tid]; D <= tid < 2D: sum v[:, tid-D]
+  if (warp == 1) tmem_alloc(&tmem_base, 512);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tm = tmem_base;
 
-  const __nv_bfloat16* Kg = reinterpret_cast<const __nv_bfloat16*>(a.K) + (size_t)u * L.T * D;
-  const __nv_bfloat16* Vg = reinterpret_cast<const __nv_bfloat16*>(a.V) + (size_t)u * L.T * D;
-  for (int t0 = t_begin; t0 < t_end; t0 += kTT) {
-    const int rows = min(kTT, t_end - t0);
-    __syncthreads();
-    load_tile<D>(tK, Kg + (size_t)t0 * D, rows, tid, NT);
-    load_tile<D>(tV, Vg + (size_t)t0 * D, rows, tid, NT);
-    __syncthreads();
-    // window-row statistics: each warp takes groups of 4 rows
-    const int t = t0 + lane;
-    for (int r0 = warp * 4; r0 < L.RW; r0 += 32) {
-      float acc[4];
-      logits4<D>(acc, qT, RWp, r0, tK, lane);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const int r = r0 + i;
-        if (r >= L.RW) break;
-        const bool ok = lane < rows && visible(t, r % L.W, L.T, L.W, a.causal);
-        const float x = ok ? acc[i] : -INFINITY;
-        const float mt = warp_max(x);
-        if (mt == -INFINITY) continue;
-        const float mo = rowm[r];
-        const float mn = fmaxf(mo, mt);
-        const float p = ok ? fast_exp2(x - mn) : 0.f;
-        const float ps = warp_sum(p);
-        if (lane == 0) {
-          rowl[r] = rowl[r] * fast_exp2(mo - mn) + ps;
-          rowm[r] = mn;
+  if (warp == 0) {
+    if (lane == 0) {  // ---- producer
+      if (LOGITS) {
+        mbar_arrive_expect_tx(&qfull, 2u * RWb * kBoxBytes);
+        for (int bx = 0; bx < 2; ++bx) tma_load_3d(sQ + bx * RWb * kBoxBytes, &tmQ, bx * 64, 0, u, &qfull);
+      }
+      for (int i = 0; i < n_tiles; ++i) {
+        const int s = i % kS, j = i / kS;
+        if (j >= 1 && !pwait(&empty[s], (j - 1) & 1, abrt, p.ws, u)) break;
+        mbar_arrive_expect_tx(&full[s], 2u * kTileBytes);
+        for (int bx = 0; bx < 2; ++bx) {
+          tma_load_3d(sK + s * kTileBytes + bx * kBoxBytes, &tmK, bx * 64, t_begin + i * kTok, u, &full[s]);
+          tma_load_3d(sV + s * kTileBytes + bx * kBoxBytes, &tmV, bx * 64, t_begin + i * kTok, u, &full[s]);
         }
-        __syncwarp();
       }
     }
-    // moment sums
-    for (int tt = 0; tt < rows; ++tt) {
-      float va[AR], kc[CC];
-#pragma unroll
-      for (int i = 0; i < AR; ++i) va[i] = tV[tt * (D + 1) + a0 + i];
-#pragma unroll
-      for (int j = 0; j < CC; ++j) kc[j] = tK[tt * (D + 1) + c0 + j];
-#pragma unroll
-      for (int i = 0; i < AR; ++i)
-#pragma unroll
-        for (int j = 0; j < CC; ++j) S[i][j] = fmaf(va[i], kc[j], S[i][j]);
+  } else if (warp == 1) {
+    if (lane == 0) {  // ---- MMA issuer
+      const uint32_t idL = idesc_bf16(128, 128, 0, 0);  // logits: rows x tokens, both K-major
+      const uint32_t idS = idesc_bf16(128, 128, 1, 1);  // V^T K: both MN-major (reduction over tokens)
+      const uint32_t aQ = smem_addr(sQ);
+      const bool ok = !LOGITS || pwait(&qfull, 0, abrt, p.ws, u);
+      for (int i = 0; ok && i < n_tiles; ++i) {
+        const int s = i % kS, j = i / kS;
+        if (!pwait(&full[s], j & 1, abrt, p.ws, u)) break;
+        tc_fence_after();
+        const uint32_t aK = smem_addr(sK + s * kTileBytes), aV = smem_addr(sV + s * kTileBytes);
+        if (LOGITS) {
+          if (i >= 1 && !pwait(&lempty, (i - 1) & 1, abrt, p.ws, u)) break;
+          tc_fence_after();
+          for (int rb = 0; rb < RWb; ++rb)
+            for (int kk = 0; kk < 8; ++kk) {
+              const uint64_t dq =
+                  sdesc_sw128(aQ + (kk >> 2) * RWb * kBoxBytes + rb * kBoxBytes + (kk & 3) * 32, 16, 1024);
+              const uint64_t dk = sdesc_sw128(aK + (kk >> 2) * kBoxBytes + (kk & 3) * 32, 16, 1024);
+              umma_bf16(tm + rb * 128, dq, dk, idL, kk > 0 ? 1u : 0u);
+            }
+          umma_commit(&lfull);
+        }
+        for (int kk = 0; kk < 8; ++kk) {
+          const uint64_t dv = sdesc_sw128(aV + kk * 2048, kBoxBytes, 1024);
+          const uint64_t dk = sdesc_sw128(aK + kk * 2048, kBoxBytes, 1024);
+          umma_bf16(tm + 256, dv, dk, idS, (i > 0 || kk > 0) ? 1u : 0u);
+        }
+        umma_commit(&empty[s]);
+      }
+      umma_commit(&sdone);
     }
-    if (tid < D) {
-      for (int tt = 0; tt < rows; ++tt) colsum += tK[tt * (D + 1) + tid];
-    } else if (tid < 2 * D) {
-      for (int tt = 0; tt < rows; ++tt) colsum += tV[tt * (D + 1) + tid - D];
+  } else {
+    // ---- epilogue: warps 2..5; TMEM lane quarter qd = warp % 4
+    const int et = tid - 64, qd = warp & 3;
+    const uint32_t lane_base = static_cast<uint32_t>(qd * 32) << 16;
+    float sk = 0.f, sv = 0.f;
+    float m[2] = {-INFINITY, -INFINITY}, l[2] = {0.f, 0.f};
+    for (int i = 0; i < n_tiles; ++i) {
+      const int s = i % kS, j = i / kS;
+      if (!pwait(&full[s], j & 1, abrt, p.ws, u)) break;
+      if (et < p.D) {  // column sums (rows past the slab's end are zero-filled)
+        const uint8_t* tk = sK + s * kTileBytes;
+        const uint8_t* tv = sV + s * kTileBytes;
+#pragma unroll 8
+        for (int r = 0; r < kTok; ++r) {
+          sk += tile_at(tk, r, et);
+          sv += tile_at(tv, r, et);
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty[s]);
+      if (LOGITS) {
+        if (!pwait(&lfull, i & 1, abrt, p.ws, u)) break;
+        tc_fence_after();
+        for (int rb = 0; rb < RWb; ++rb) {
+          const int r = rb * 128 + qd * 32 + lane;  // window row of this thread
+          const int wi = r % p.W;
+          const int tmax_vis = p.causal ? p.T - p.W + wi : 0x7fffffff;
+          for (int c0 = 0; c0 < kTok; c0 += 32) {
+            float x[32];
+            tmem_ld32(tm + lane_base + rb * 128 + c0, x);
+            const int t0 = t_begin + i * kTok + c0;
+            float mx = -INFINITY;
+#pragma unroll
+            for (int jj = 0; jj < 32; ++jj) {
+              const int t = t0 + jj;
+              x[jj] = (t < t_end && t <= tmax_vis) ? x[jj] * p.qscale : -INFINITY;
+              mx = fmaxf(mx, x[jj]);
+            }
+            const float mn = fmaxf(m[rb], mx);
+            if (mn != -INFINITY) {
+              float acc = 0.f;
+#pragma unroll
+              for (int jj = 0; jj < 32; ++jj) acc += fast_exp2(x[jj] - mn);
+              l[rb] = l[rb] * fast_exp2(m[rb] - mn) + acc;
+              m[rb] = mn;
+            }
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&lempty);
+      }
     }
-  }
-  __syncthreads();
-  float* rp = L.rowpart + ((size_t)u * L.n_chunks + chunk) * L.RW * 2;
-  for (int r = tid; r < L.RW; r += NT) {
-    rp[2 * r] = rowm[r];
-    rp[2 * r + 1] = rowl[r];
-  }
-  // centred co-moment of this chunk
-  float* rec = L.mpart + ((size_t)u * L.n_chunks + chunk) * L.rec;
-  const float nc = static_cast<float>(t_end - t_begin);
-  float* sums = tK;  // reuse: [0..D) sum k, [D..2D) sum v
-  if (tid < 2 * D) sums[tid] = colsum;
-  __syncthreads();
-  if (tid == 0) rec[0] = nc;
-  if (tid < D) {
-    rec[4 + tid] = sums[tid] / nc;
-    rec[4 + D + tid] = sums[D + tid] / nc;
-  }
+    if (LOGITS) {
+      for (int rb = 0; rb < RWb; ++rb) {
+        const int r = rb * 128 + qd * 32 + lane;
+        if (r < p.RW) {
+          float* rp = p.rowpart + (((size_t)u * p.n_chunks + chunk) * p.RW + r) * 2;
+          rp[0] = m[rb];
+          rp[1] = l[rb];
+        }
+      }
+    }
+    sum_k[et] = sk;
+    sum_v[et] = sv;
+    epi_sync();
+    const bool got = pwait(&sdone, 0, abrt, p.ws, u);
+    tc_fence_after();
+    const float nc = static_cast<float>(max(0, t_end - t_begin));
+    float* rec = p.mrec + ((size_t)u * p.n_chunks + chunk) * rec_floats(p.D);
+    const int a = qd * 32 + lane;  // value dim = TMEM lane
+    for (int c0 = 0; c0 < kDP; c0 += 32) {
+      float srow[32];
+      tmem_ld32(tm + lane_base + 256 + c0, srow);
+      if (a < p.D && nc > 0.f) {
 #pragma unroll
-  for (int i = 0; i < AR; ++i)
-#pragma unroll
-    for (int j = 0; j < CC; ++j)
-      rec[4 + 2 * D + (size_t)(a0 + i) * D + c0 + j] = S[i][j] - sums[D + a0 + i] * sums[c0 + j] / nc;
+        for (int jj = 0; jj < 32; ++jj) {
+          const int c = c0 + jj;
+          if (c < p.D) rec[4 + 2 * p.D + (size_t)a * p.D + c] = srow[jj] - sum_v[a] * sum_k[c] / nc;
+        }
+      }
+    }
+    if (et < p.D) {
+      rec[4 + et] = nc > 0.f ? sum_k[et] / nc : 0.f;
+      rec[4 + p.D + et] = nc > 0.f ? sum_v[et] / nc : 0.f;
+    }
+    if (et == 0) rec[0] = got ? nc : 0.f;
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tm, 512);
+  }
 }
 
-// ----------------------------------------------------------------- scores
-template <int D>
-__global__ void __launch_bounds__(256) scores_kernel(const CompressArgs a, const Layout L) {
-  constexpr int NT = 256;
-  extern __shared__ __align__(16) float sm[];
-  const int RWp = align_up(L.RW, 4);
-  float* qT = sm;                  // [D][RWp]
-  float* tK = qT + D * RWp;        // [32][D+1]
-  float* rowm = tK + kTT * (D + 1);
-  float* rowil = rowm + RWp;       // 1 / l
-  float* part = rowil + RWp;       // [8][32]
+// -------------------------------------------------------------- scores_tc
+__global__ void __launch_bounds__(kTcThreads, 1)
+    scores_tc(const TcArgs p, const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmQ) {
+  constexpr int kS = 3;
+  extern __shared__ __align__(1024) uint8_t smraw[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sK = sm;                    // [kS][128 x 128]
+  uint8_t* sQ = sm + kS * kTileBytes;  // [2 boxes][RWb*128][128 B]
+  __shared__ __align__(8) uint64_t full[kS], empty[kS], lfull[2], lempty[2], qfull;
+  __shared__ uint32_t tmem_base;
+  __shared__ int abort_flag;
+  __shared__ float s_m[256], s_il[256];
+
   const int chunk = blockIdx.x, u = blockIdx.y;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int t_begin = chunk * L.chunk;
-  const int t_end = min(L.T, t_begin + L.chunk);
-  const float qs = rsqrtf(static_cast<float>(D)) * kLog2e;
-  const __nv_bfloat16* Qg = reinterpret_cast<const __nv_bfloat16*>(a.Q) + (size_t)u * L.RW * D;
-  for (int idx = tid; idx < D * RWp; idx += NT) {
-    const int c = idx / RWp, r = idx % RWp;
-    qT[idx] = (r < L.RW) ? __bfloat162float(Qg[(size_t)r * D + c]) * qs : 0.f;
+  const int t_begin = chunk * p.chunk;
+  const int t_end = min(p.n_rows, t_begin + p.chunk);
+  const int n_tiles = (max(0, t_end - t_begin) + kTok - 1) / kTok;
+  const int RWb = p.RWb, RWp = RWb * 128;
+  volatile int* abrt = &abort_flag;
+
+  if (tid == 0) {
+    for (int i = 0; i < kS; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&lfull[i], 1);
+      mbar_init(&lempty[i], 4);
+    }
+    mbar_init(&qfull, 1);
+    abort_flag = 0;
+    mbar_fence_init();
   }
-  // merge the per-chunk row statistics
-  const float* rp = L.rowpart + (size_t)u * L.n_chunks * L.RW * 2;
-  for (int r = tid; r < RWp; r += NT) {
-    float m = -INFINITY, l = 0.f;
-    if (r < L.RW) {
-      for (int c = 0; c < L.n_chunks; ++c) m = fmaxf(m, rp[((size_t)c * L.RW + r) * 2]);
-      for (int c = 0; c < L.n_chunks; ++c) {
-        const float mc = rp[((size_t)c * L.RW + r) * 2];
-        if (mc != -INFINITY) l += rp[((size_t)c * L.RW + r) * 2 + 1] * fast_exp2(mc - m);
+  if (warp == 1) tmem_alloc(&tmem_base, 512);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tm = tmem_base;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      mbar_arrive_expect_tx(&qfull, 2u * RWb * kBoxBytes);
+      for (int bx = 0; bx < 2; ++bx) tma_load_3d(sQ + bx * RWb * kBoxBytes, &tmQ, bx * 64, 0, u, &qfull);
+      for (int i = 0; i < n_tiles; ++i) {
+        const int s = i % kS, j = i / kS;
+        if (j >= 1 && !pwait(&empty[s], (j - 1) & 1, abrt, p.ws, u)) break;
+        mbar_arrive_expect_tx(&full[s], kTileBytes);
+        for (int bx = 0; bx < 2; ++bx)
+          tma_load_3d(sK + s * kTileBytes + bx * kBoxBytes, &tmK, bx * 64, t_begin + i * kTok, u, &full[s]);
       }
     }
-    rowm[r] = m;
-    rowil[r] = (l > 0.f) ? 1.f / l : 0.f;
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t id = idesc_bf16(128, RWp, 0, 0);  // tokens x window rows, both K-major
+      const uint32_t aQ = smem_addr(sQ);
+      const bool ok = pwait(&qfull, 0, abrt, p.ws, u);
+      for (int i = 0; ok && i < n_tiles; ++i) {
+        const int s = i % kS, j = i / kS, b = i & 1;
+        if (!pwait(&full[s], j & 1, abrt, p.ws, u)) break;
+        if (i >= 2 && !pwait(&lempty[b], ((i >> 1) - 1) & 1, abrt, p.ws, u)) break;
+        tc_fence_after();
+        const uint32_t aK = smem_addr(sK + s * kTileBytes);
+        for (int kk = 0; kk < 8; ++kk) {
+          const uint64_t dk = sdesc_sw128(aK + (kk >> 2) * kBoxBytes + (kk & 3) * 32, 16, 1024);
+          const uint64_t dq = sdesc_sw128(aQ + (kk >> 2) * RWb * kBoxBytes + (kk & 3) * 32, 16, 1024);
+          umma_bf16(tm + b * 256, dk, dq, id, kk > 0 ? 1u : 0u);
+        }
+        umma_commit(&lfull[b]);
+        umma_commit(&empty[s]);
+      }
+    }
+  } else {
+    const int et = tid - 64, qd = warp & 3;
+    const uint32_t lane_base = static_cast<uint32_t>(qd * 32) << 16;
+    // merged row statistics of every window row
+    for (int r = et; r < RWp; r += 128) {
+      float M = -INFINITY, Lsum = 0.f;
+      if (r < p.RW) {
+        for (int c = 0; c < p.n_chunks; ++c)
+          M = fmaxf(M, p.rowpart[(((size_t)u * p.n_chunks + c) * p.RW + r) * 2]);
+        if (M != -INFINITY)
+          for (int c = 0; c < p.n_chunks; ++c) {
+            const float* rp = p.rowpart + (((size_t)u * p.n_chunks + c) * p.RW + r) * 2;
+            if (rp[0] != -INFINITY) Lsum += rp[1] * fast_exp2(rp[0] - M);
+          }
+      }
+      s_m[r] = M;
+      s_il[r] = Lsum > 0.f ? 1.f / Lsum : 0.f;
+    }
+    epi_sync();
+    for (int i = 0; i < n_tiles; ++i) {
+      const int b = i & 1;
+      if (!pwait(&lfull[b], (i >> 1) & 1, abrt, p.ws, u)) break;
+      tc_fence_after();
+      const int t = t_begin + i * kTok + qd * 32 + lane;  // token of this thread (TMEM lane)
+      float acc = 0.f;
+      for (int c0 = 0; c0 < RWp; c0 += 32) {
+        float x[32];
+        tmem_ld32(tm + lane_base + b * 256 + c0, x);
+#pragma unroll
+        for (int jj = 0; jj < 32; ++jj) {
+          const int r = c0 + jj;
+          if (r < p.RW && (!p.causal || t <= p.T - p.W + r % p.W))
+            acc += fast_exp2(x[jj] * p.qscale - s_m[r]) * s_il[r];
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&lempty[b]);
+      for (int o = 1; o < p.pool; o <<= 1) acc += __shfl_xor_sync(kFull, acc, o);  // aligned chunks
+      if (t < t_end) {
+        p.s_out[(size_t)u * p.T + t] = acc;
+        if (p.diag) p.diag[(size_t)u * p.T + t] = acc;
+      }
+    }
   }
-  const __nv_bfloat16* Kg = reinterpret_cast<const __nv_bfloat16*>(a.K) + (size_t)u * L.T * D;
-  float* s_out = L.s + (size_t)u * L.T;
-  for (int t0 = t_begin; t0 < t_end; t0 += kTT) {
-    const int rows = min(kTT, t_end - t0);
-    __syncthreads();
-    load_tile<D>(tK, Kg + (size_t)t0 * D, rows, tid, NT);
-    __syncthreads();
-    const int t = t0 + lane;
-    float colp = 0.f;
-    for (int r0 = warp * 4; r0 < L.RW; r0 += 32) {
-      float acc[4];
-      logits4<D>(acc, qT, RWp, r0, tK, lane);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const int r = r0 + i;
-        if (r < L.RW && lane < rows && visible(t, r % L.W, L.T, L.W, a.causal))
-          colp += fast_exp2(acc[i] - rowm[r]) * rowil[r];
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tm, 512);
+  }
+}
+
+// ------------------------------------------------------------ residual_tc
+__global__ void __launch_bounds__(kTcThreads, 1)
+    residual_tc(const TcArgs p, const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV) {
+  constexpr int kS = 2;
+  extern __shared__ __align__(1024) uint8_t smraw[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sK = sm;                        // [kS][128 x 128]
+  uint8_t* sV = sm + kS * kTileBytes;      // [kS][128 x 128]
+  uint8_t* sC = sm + 2 * kS * kTileBytes;  // [3 parts][128 x 128]: C0' = hi + mid + lo
+  __shared__ __align__(8) uint64_t full[kS], empty[kS], yfull[2], yempty[2];
+  __shared__ uint32_t tmem_base;
+  __shared__ int abort_flag;
+  __shared__ float s_mv[kDP];
+
+  const int chunk = blockIdx.x, u = blockIdx.y;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int t_begin = chunk * p.chunk;
+  const int t_end = min(p.n_rows, t_begin + p.chunk);
+  const int n_tiles = (max(0, t_end - t_begin) + kTok - 1) / kTok;
+  volatile int* abrt = &abort_flag;
+  const int D = p.D;
+  const float* m0 = p.m0 + (size_t)u * rec_floats(D);
+
+  if (tid == 0) {
+    for (int i = 0; i < kS; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], 1 + 4);  // MMA commit + the 4 epilogue warps (value rows)
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&yfull[i], 1);
+      mbar_init(&yempty[i], 4);
+    }
+    abort_flag = 0;
+    mbar_fence_init();
+    // the first stages' copies go out while C0' is being prepared
+    for (int i = 0; i < min(kS, n_tiles); ++i) {
+      mbar_arrive_expect_tx(&full[i], 2u * kTileBytes);
+      for (int bx = 0; bx < 2; ++bx) {
+        tma_load_3d(sK + i * kTileBytes + bx * kBoxBytes, &tmK, bx * 64, t_begin + i * kTok, u, &full[i]);
+        tma_load_3d(sV + i * kTileBytes + bx * kBoxBytes, &tmV, bx * 64, t_begin + i * kTok, u, &full[i]);
       }
     }
-    part[warp * 32 + lane] = colp;
-    __syncthreads();
-    if (warp == 0) {
-      float sum = 0.f;
+  }
+  if (warp == 1) tmem_alloc(&tmem_base, 256);
+  if (warp >= 2) {
+    // C0' (clamped where |n0 C0| < tau) as three bf16 parts in the K-major
+    // swizzled layout: row a = value dim (N), 128-byte rows over key dims (K)
+    const int a = tid - 64;
+    const float n0 = m0[0];
+    const float tau = p.tau;
+    for (int c = 0; c < kDP; c += 2) {
+      float v0 = 0.f, v1 = 0.f;
+      if (n0 > 0.f && a < D) {
+        if (c < D) v0 = m0[4 + 2 * D + (size_t)a * D + c];
+        if (c + 1 < D) v1 = m0[4 + 2 * D + (size_t)a * D + c + 1];
+        if (fabsf(v0 * n0) < tau) v0 = 0.f;
+        if (fabsf(v1 * n0) < tau) v1 = 0.f;
+      }
+      float r0 = v0, r1 = v1;
 #pragma unroll
-      for (int w = 0; w < 8; ++w) sum += part[w * 32 + lane];
-      // pool into aligned chunks of `pool` tokens (pool divides 32, tiles are aligned)
-      for (int o = 1; o < a.pool; o <<= 1) sum += __shfl_xor_sync(kFull, sum, o);
-      if (lane < rows) {
-        s_out[t] = sum;
-        if (a.diag_scores) a.diag_scores[(size_t)u * L.T + t] = sum;
+      for (int part = 0; part < 3; ++part) {
+        const __nv_bfloat16 h0 = __float2bfloat16_rn(r0), h1 = __float2bfloat16_rn(r1);
+        __nv_bfloat162 hv;
+        hv.x = h0;
+        hv.y = h1;
+        *reinterpret_cast<__nv_bfloat162*>(sC + part * kTileBytes + swz_off(a, c, kTok)) = hv;
+        r0 -= __bfloat162float(h0);
+        r1 -= __bfloat162float(h1);
       }
     }
+    s_mv[a] = (n0 > 0.f && a < D) ? m0[4 + D + a] : 0.f;
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // generic writes -> tensor-core reads
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tm = tmem_base;
+  const float scale = rsqrtf(static_cast<float>(D));
+
+  if (warp == 0) {
+    if (lane == 0) {
+      for (int i = kS; i < n_tiles; ++i) {
+        const int s = i % kS, j = i / kS;
+        if (!pwait(&empty[s], (j - 1) & 1, abrt, p.ws, u)) break;
+        mbar_arrive_expect_tx(&full[s], 2u * kTileBytes);
+        for (int bx = 0; bx < 2; ++bx) {
+          tma_load_3d(sK + s * kTileBytes + bx * kBoxBytes, &tmK, bx * 64, t_begin + i * kTok, u, &full[s]);
+          tma_load_3d(sV + s * kTileBytes + bx * kBoxBytes, &tmV, bx * 64, t_begin + i * kTok, u, &full[s]);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t id = idesc_bf16(128, 128, 0, 0);
+      const uint32_t aC = smem_addr(sC);
+      for (int i = 0; i < n_tiles; ++i) {
+        const int s = i % kS, j = i / kS, b = i & 1;
+        if (!pwait(&full[s], j & 1, abrt, p.ws, u)) break;
+        if (i >= 2 && !pwait(&yempty[b], ((i >> 1) - 1) & 1, abrt, p.ws, u)) break;
+        tc_fence_after();
+        const uint32_t aK = smem_addr(sK + s * kTileBytes);
+        for (int part = 0; part < 3; ++part)
+          for (int kk = 0; kk < 8; ++kk) {
+            const uint64_t dk = sdesc_sw128(aK + (kk >> 2) * kBoxBytes + (kk & 3) * 32, 16, 1024);
+            const uint64_t dc =
+                sdesc_sw128(aC + part * kTileBytes + (kk >> 2) * kBoxBytes + (kk & 3) * 32, 16, 1024);
+            umma_bf16(tm + b * 128, dk, dc, id, (part > 0 || kk > 0) ? 1u : 0u);
+          }
+        umma_commit(&yfull[b]);
+        umma_commit(&empty[s]);
+      }
+    }
+  } else {
+    const int qd = warp & 3;
+    const uint32_t lane_base = static_cast<uint32_t>(qd * 32) << 16;
+    const int row = qd * 32 + lane;  // token within the tile = TMEM lane
+    for (int i = 0; i < n_tiles; ++i) {
+      const int s = i % kS, j = i / kS, b = i & 1;
+      if (!pwait(&yfull[b], (i >> 1) & 1, abrt, p.ws, u)) break;
+      if (!pwait(&full[s], j & 1, abrt, p.ws, u)) break;
+      tc_fence_after();
+      const uint8_t* tv = sV + s * kTileBytes;
+      float ss = 0.f;
+      for (int c0 = 0; c0 < kDP; c0 += 32) {
+        float y[32];
+        tmem_ld32(tm + lane_base + b * 128 + c0, y);
+        if (c0 < D) {
+#pragma unroll
+          for (int jj = 0; jj < 32; jj += 8) {
+            const uint4 raw = *reinterpret_cast<const uint4*>(tv + swz_off(row, c0 + jj, kTok));
+            const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const float2 vv = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[e]));
+              const int c = c0 + jj + 2 * e;
+              const float r0 = vv.x - s_mv[c] - scale * y[jj + 2 * e];
+              const float r1 = vv.y - s_mv[c + 1] - scale * y[jj + 2 * e + 1];
+              ss = fmaf(r0, r0, fmaf(r1, r1, ss));
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(&yempty[b]);
+        mbar_arrive(&empty[s]);
+      }
+      const int t = t_begin + i * kTok + row;
+      if (t < t_end) {
+        const float v =
+            is_protected(t, p.T, p.W, p.sink, p.keep_window) ? 0.f : p.s_in[(size_t)u * p.T + t] * sqrtf(ss);
+        p.s_out[(size_t)u * p.T + t] = v;
+        if (p.diag) p.diag[(size_t)u * p.T + t] = v;
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tm, 256);
   }
 }
 
 // ----------------------------------------------------------------- select
 // One CTA (1024 threads) per unit: R = protected + the k highest keys among
-// the other positions (ties to the lower position).  Writes R ascending to
-// idx_out[u][0..B) and (n_R, mean k, mean v) of R to rmean_out.
-constexpr int kSelThreads = 1024;
-
+// the other positions (ties to the lower position), written ascending; the
+// rows of R are gathered into dst_K/dst_V [unit][dst_cap][D] (with positions,
+// length and tokens seen when the destination is a cache).
 __device__ __forceinline__ int block_excl_scan(int flag, int* wsum, int* total) {
-  // flag in {0,1}; returns exclusive prefix count in thread order
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const unsigned m = __ballot_sync(kFull, flag);
   const int in_warp = __popc(m & ((1u << lane) - 1u));
@@ -331,7 +640,7 @@ __device__ __forceinline__ int block_excl_scan(int flag, int* wsum, int* total) 
       const int y = __shfl_up_sync(kFull, x, o);
       if (lane >= o) x += y;
     }
-    wsum[lane] = x - v;  // exclusive
+    wsum[lane] = x - v;
     if (lane == 31) *total = x;
   }
   __syncthreads();
@@ -340,41 +649,77 @@ __device__ __forceinline__ int block_excl_scan(int flag, int* wsum, int* total) 
   return r;
 }
 
-template <int D>
-__global__ void __launch_bounds__(kSelThreads) select_kernel(const CompressArgs a, const Layout L,
-                                                             const float* scores, int32_t* idx_out,
-                                                             float* rmean_out, int32_t* diag_idx) {
+struct SelectArgs {
+  const float* scores;  // [units][T]
+  int T, W, B, sink, keep_window, D;
+  const __nv_bfloat16* K;  // prompt [units][T][D]
+  const __nv_bfloat16* V;
+  int32_t* idx;          // [units][B] retained positions (workspace)
+  int32_t* diag_idx;     // optional copy
+  __nv_bfloat16* dst_K;  // [units][dst_cap][D]
+  __nv_bfloat16* dst_V;
+  int dst_cap;
+  int32_t* dst_pos;  // optional cache bookkeeping
+  int32_t* dst_len;
+  int32_t* dst_seen;
+};
+
+__global__ void __launch_bounds__(kSelThreads) select_kernel(const SelectArgs a) {
   __shared__ uint32_t hist[256];
+  __shared__ uint32_t whist[8][256];  // private histograms for groups of 4 warps (less contention)
   __shared__ int wsum[32];
   __shared__ int tot;
   __shared__ uint32_t s_prefix;
   __shared__ int s_need;
-  const int u = blockIdx.x, tid = threadIdx.x;
-  const int T = L.T, W = L.W;
-  const float* sc = scores + (size_t)u * T;
-  const int k = L.B - protected_count(T, W, a.sink, a.keep_window);  // >= 0 (validated), < candidates
+  const int u = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int T = a.T, W = a.W;
+  const float* sc = a.scores + (size_t)u * T;
+  const int k = a.B - protected_count(T, W, a.sink, a.keep_window);  // >= 0 (validated), < candidates
 
   uint32_t prefix = 0, pmask = 0;
   int need = k;
   if (k > 0) {
     for (int pass = 0; pass < 4; ++pass) {
       const int shift = 24 - 8 * pass;
-      for (int i = tid; i < 256; i += kSelThreads) hist[i] = 0;
+      for (int i = tid; i < 8 * 256; i += kSelThreads) (&whist[0][0])[i] = 0;
       __syncthreads();
+      uint32_t* wh = whist[warp & 7];
       for (int t = tid; t < T; t += kSelThreads) {
         if (is_protected(t, T, W, a.sink, a.keep_window)) continue;
         const uint32_t key = float_key(sc[t]);
-        if ((key & pmask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+        if ((key & pmask) == prefix) atomicAdd(&wh[(key >> shift) & 255u], 1u);
       }
       __syncthreads();
-      if (tid == 0) {
-        int cum = 0, dg = 0;
-        for (dg = 255; dg > 0; --dg) {
-          if (cum + static_cast<int>(hist[dg]) >= need) break;
-          cum += hist[dg];
+      for (int i = tid; i < 256; i += kSelThreads) {
+        uint32_t c = 0;
+#pragma unroll
+        for (int g = 0; g < 8; ++g) c += whist[g][i];
+        hist[i] = c;
+      }
+      __syncthreads();
+      if (warp == 0) {  // the digit where the descending cumulative count reaches `need`
+        int cnt[8], tot8 = 0;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          cnt[e] = static_cast<int>(hist[255 - (lane * 8 + e)]);
+          tot8 += cnt[e];
         }
-        s_need = need - cum;
-        s_prefix = prefix | (static_cast<uint32_t>(dg) << shift);
+        int incl = tot8;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const int y = __shfl_up_sync(kFull, incl, o);
+          if (lane >= o) incl += y;
+        }
+        const int excl = incl - tot8;
+        if (excl < need && incl >= need) {
+          int cum = excl, e = 0;
+          for (; e < 7; ++e) {
+            if (cum + cnt[e] >= need) break;
+            cum += cnt[e];
+          }
+          s_need = need - cum;
+          s_prefix = prefix | (static_cast<uint32_t>(255 - (lane * 8 + e)) << shift);
+        }
       }
       __syncthreads();
       need = s_need;
@@ -383,9 +728,8 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const CompressArgs 
       __syncthreads();
     }
   }
-  // ascending output: selected = protected | key > K* | (key == K* and tie rank < need)
   int ties_before = 0, sel_before = 0;
-  int32_t* out = idx_out + (size_t)u * L.B;
+  int32_t* out = a.idx + (size_t)u * a.B;
   for (int base = 0; base < T; base += kSelThreads) {
     const int t = base + tid;
     bool prot = false, tie = false, gt = false;
@@ -404,80 +748,74 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const CompressArgs 
     const int sel_total = tot;
     if (sel) {
       const int o = sel_before + sr;
-      if (o < L.B) {
+      if (o < a.B) {
         out[o] = t;
-        if (diag_idx) diag_idx[(size_t)u * L.B + o] = t;
+        if (a.diag_idx) a.diag_idx[(size_t)u * a.B + o] = t;
       }
     }
     ties_before += tie_total;
     sel_before += sel_total;
   }
   __syncthreads();
-  // mean key / value of R (thread c < D: key dim c; D <= thread < 2D: value dim)
-  if (rmean_out) {
-    float* rm = rmean_out + (size_t)u * (4 + 2 * D);
-    const int nR = min(sel_before, L.B);
-    if (tid < 2 * D) {
-      const bool isv = tid >= D;
-      const int c = isv ? tid - D : tid;
-      const __nv_bfloat16* X = reinterpret_cast<const __nv_bfloat16*>(isv ? a.V : a.K) + (size_t)u * T * D;
-      float acc = 0.f;
-      for (int i = 0; i < nR; ++i) acc += __bfloat162float(X[(size_t)out[i] * D + c]);
-      rm[4 + tid] = acc / static_cast<float>(nR);
-    }
-    if (tid == 0) rm[0] = static_cast<float>(nR);
+  // gather the retained rows (16-byte chunks)
+  const int D = a.D;
+  const int per_row = D / 8;
+  for (int i = tid; i < a.B * per_row; i += kSelThreads) {
+    const int r = i / per_row, c = i % per_row;
+    const int t = min(max(out[r], 0), T - 1);  // never read outside the unit's slab
+    const size_t src = ((size_t)u * T + t) * D;
+    const size_t dst = ((size_t)u * a.dst_cap + r) * D;
+    reinterpret_cast<uint4*>(a.dst_K + dst)[c] = reinterpret_cast<const uint4*>(a.K + src)[c];
+    reinterpret_cast<uint4*>(a.dst_V + dst)[c] = reinterpret_cast<const uint4*>(a.V + src)[c];
+  }
+  if (a.dst_pos)
+    for (int r = tid; r < a.B; r += kSelThreads) a.dst_pos[(size_t)u * a.dst_cap + r] = out[r];
+  if (tid == 0 && a.dst_len) {
+    a.dst_len[u] = a.B;
+    a.dst_seen[u] = T;
   }
 }
 
-// ---------------------------------------------------------------- moments
-// Moments of E = all \ R for 8 rows (value dims) of C per CTA.
-template <int D>
-__global__ void __launch_bounds__(256) moments_kernel(const CompressArgs a, const Layout L, const int32_t* idx,
-                                                      const float* rmean, float* out_rec, mkv_moments out_mom,
-                                                      int final_out) {
+// --------------------------------------------------------------- finalize
+// Moments of E = all \ R for 8 value dims (rows of C) per CTA: the all-token
+// co-moment is the multi-way Chan merge of the chunk records; R's centred
+// record is removed with the reverse pairwise formula.
+__global__ void __launch_bounds__(256) finalize_kernel(const Layout L, float* out_rec, mkv_moments out_mom,
+                                                       int final_out) {
   constexpr int NT = 256, RB = 8;
-  __shared__ float mk[D], mv[D], mkR[D], mvR[D];
+  __shared__ float mk[kDP], mv[kDP], mkR[kDP], mvR[kDP];
   __shared__ float s_n;
+  const int D = L.D;
   const int rb = blockIdx.x, u = blockIdx.y, tid = threadIdx.x;
-  const float* recs = L.mpart + (size_t)u * L.n_chunks * L.rec;
-  // totals over all tokens
+  const size_t rf = rec_floats(D);
+  const float* recs = L.mpart + (size_t)u * L.n_chunks * rf;
+  const float* rR = L.rpart + (size_t)u * rf;
   if (tid < 2 * D) {
     float num = 0.f, n = 0.f;
     for (int c = 0; c < L.n_chunks; ++c) {
-      const float nc = recs[(size_t)c * L.rec];
+      const float nc = recs[(size_t)c * rf];
       n += nc;
-      num += nc * recs[(size_t)c * L.rec + 4 + tid];
+      num += nc * recs[(size_t)c * rf + 4 + tid];
     }
     if (tid < D) mk[tid] = num / n;
     else mv[tid - D] = num / n;
     if (tid == 0) s_n = n;
   }
-  const float* rm = rmean + (size_t)u * (4 + 2 * D);
   if (tid < D) {
-    mkR[tid] = rm[4 + tid];
-    mvR[tid] = rm[4 + D + tid];
+    mkR[tid] = rR[4 + tid];
+    mvR[tid] = rR[4 + D + tid];
   }
   __syncthreads();
-  const float n = s_n, nR = rm[0], nE = n - nR;
-  const __nv_bfloat16* Kg = reinterpret_cast<const __nv_bfloat16*>(a.K) + (size_t)u * L.T * D;
-  const __nv_bfloat16* Vg = reinterpret_cast<const __nv_bfloat16*>(a.V) + (size_t)u * L.T * D;
-  const int32_t* ix = idx + (size_t)u * L.B;
-  const int nRi = static_cast<int>(nR);
+  const float n = s_n, nR = rR[0], nE = n - nR;
   for (int e = tid; e < RB * D; e += NT) {
     const int ar = rb * RB + e / D, c = e % D;
-    // all-token co-moment: multi-way Chan merge of the chunk records
     float M = 0.f;
     for (int ch = 0; ch < L.n_chunks; ++ch) {
-      const float* r = recs + (size_t)ch * L.rec;
+      const float* r = recs + (size_t)ch * rf;
       const float nc = r[0];
-      M += r[4 + 2 * D + (size_t)ar * D + c] + nc * (r[4 + D + ar] - mv[ar]) * (r[4 + c] - mk[c]);
+      if (nc > 0.f) M += r[4 + 2 * D + (size_t)ar * D + c] + nc * (r[4 + D + ar] - mv[ar]) * (r[4 + c] - mk[c]);
     }
-    // retained-set co-moment
-    float MR = 0.f;
-    for (int i = 0; i < nRi; ++i) {
-      const size_t row = (size_t)ix[i] * D;
-      MR = fmaf(__bfloat162float(Vg[row + ar]) - mvR[ar], __bfloat162float(Kg[row + c]) - mkR[c], MR);
-    }
+    const float MR = rR[4 + 2 * D + (size_t)ar * D + c];
     float CE = 0.f, mkE_c = 0.f, mvE_a = 0.f;
     if (nE > 0.f) {
       mkE_c = (n * mk[c] - nR * mkR[c]) / nE;
@@ -487,10 +825,10 @@ __global__ void __launch_bounds__(256) moments_kernel(const CompressArgs a, cons
     }
     if (final_out) {
       out_mom.C[((size_t)u * D + ar) * D + c] = CE;
-      if (c == 0) out_mom.mu_v[(size_t)u * D + ar] = (nE > 0.f) ? mvE_a : 0.f;
-      if (rb == 0 && e < D) out_mom.mu_k[(size_t)u * D + c] = (nE > 0.f) ? mkE_c : 0.f;
+      if (c == 0) out_mom.mu_v[(size_t)u * D + ar] = mvE_a;
+      if (rb == 0 && e < D) out_mom.mu_k[(size_t)u * D + c] = mkE_c;
     } else {
-      float* o = out_rec + (size_t)u * rec_floats(D);
+      float* o = out_rec + (size_t)u * rf;
       o[4 + 2 * D + (size_t)ar * D + c] = CE;
       if (c == 0) o[4 + D + ar] = mvE_a;
       if (rb == 0 && e < D) o[4 + c] = mkE_c;
@@ -498,155 +836,154 @@ __global__ void __launch_bounds__(256) moments_kernel(const CompressArgs a, cons
   }
   if (rb == 0 && tid == 0) {
     if (final_out) out_mom.n[u] = static_cast<int32_t>(nE);
-    else out_rec[(size_t)u * rec_floats(D)] = nE;
+    else out_rec[(size_t)u * rf] = nE;
   }
 }
 
-// --------------------------------------------------------------- residual
+// ---------------------------------------------------------- keep-all path
 template <int D>
-__global__ void __launch_bounds__(256) residual_kernel(const CompressArgs a, const Layout L) {
-  constexpr int NT = 256;
-  extern __shared__ __align__(16) float sm[];
-  float* Ct = sm;                   // [D][D] C0' transposed: Ct[c][a]
-  float* tK = Ct + D * D;           // [32][D+1]
-  float* part = tK + kTT * (D + 1); // [8][32]
-  __shared__ float mv0[D];
-  const int chunk = blockIdx.x, u = blockIdx.y;
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int t_begin = chunk * L.chunk;
-  const int t_end = min(L.T, t_begin + L.chunk);
-  const float* m0 = L.m0 + (size_t)u * rec_floats(D);
-  const float n0 = m0[0];
-  const float tau = a.tau;
-  for (int idx = tid; idx < D * D; idx += NT) {
-    const int ar = idx / D, c = idx % D;
-    float cv = (n0 > 0.f) ? m0[4 + 2 * D + idx] : 0.f;
-    if (fabsf(cv * n0) < tau) cv = 0.f;
-    Ct[c * D + ar] = cv;
-  }
-  if (tid < D) mv0[tid] = (n0 > 0.f) ? m0[4 + D + tid] : 0.f;
-  const float scale = rsqrtf(static_cast<float>(D));
-  const __nv_bfloat16* Kg = reinterpret_cast<const __nv_bfloat16*>(a.K) + (size_t)u * L.T * D;
-  const __nv_bfloat16* Vg = reinterpret_cast<const __nv_bfloat16*>(a.V) + (size_t)u * L.T * D;
-  const float* s = L.s + (size_t)u * L.T;
-  float* s2 = L.s2 + (size_t)u * L.T;
-  constexpr int AW = D / 8;  // output dims per warp
-  for (int t0 = t_begin; t0 < t_end; t0 += kTT) {
-    const int rows = min(kTT, t_end - t0);
-    __syncthreads();
-    load_tile<D>(tK, Kg + (size_t)t0 * D, rows, tid, NT);
-    __syncthreads();
-    float y[AW];
-#pragma unroll
-    for (int i = 0; i < AW; ++i) y[i] = 0.f;
-    const int a0 = warp * AW;
-#pragma unroll 4
-    for (int c = 0; c < D; ++c) {
-      const float kc = tK[lane * (D + 1) + c];
-#pragma unroll
-      for (int i = 0; i < AW; i += 4) {
-        const float4 c4 = *reinterpret_cast<const float4*>(Ct + c * D + a0 + i);
-        y[i] = fmaf(c4.x, kc, y[i]);
-        y[i + 1] = fmaf(c4.y, kc, y[i + 1]);
-        y[i + 2] = fmaf(c4.z, kc, y[i + 2]);
-        y[i + 3] = fmaf(c4.w, kc, y[i + 3]);
-      }
-    }
-    const int t = t0 + lane;
-    float ss = 0.f;
-    if (lane < rows) {
-      const __nv_bfloat16* vrow = Vg + (size_t)t * D + a0;
-#pragma unroll
-      for (int i = 0; i < AW; ++i) {
-        const float r = __bfloat162float(vrow[i]) - mv0[a0 + i] - scale * y[i];
-        ss = fmaf(r, r, ss);
-      }
-    }
-    part[warp * 32 + lane] = ss;
-    __syncthreads();
-    if (warp == 0 && lane < rows) {
-      float tot = 0.f;
-#pragma unroll
-      for (int w = 0; w < 8; ++w) tot += part[w * 32 + lane];
-      const float v = is_protected(t, L.T, L.W, a.sink, a.keep_window) ? 0.f : s[t] * sqrtf(tot);
-      s2[t] = v;
-      if (a.diag_score2) a.diag_score2[(size_t)u * L.T + t] = v;
-    }
-  }
-}
-
-// ----------------------------------------------------------------- gather
-template <int D>
-__global__ void __launch_bounds__(256) gather_kernel(const CompressArgs a, const Layout L, const int32_t* idx,
-                                                     int count, int keep_all) {
+__global__ void __launch_bounds__(256) keep_all_kernel(const CompressArgs a, int T) {
   const int u = blockIdx.y;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int i = blockIdx.x * 8 + warp;
-  if (i < count) {
-    const int t = keep_all ? i : idx[(size_t)u * L.B + i];
-    const __nv_bfloat16* Ks = reinterpret_cast<const __nv_bfloat16*>(a.K) + ((size_t)u * L.T + t) * D;
-    const __nv_bfloat16* Vs = reinterpret_cast<const __nv_bfloat16*>(a.V) + ((size_t)u * L.T + t) * D;
+  if (i < T) {
+    const __nv_bfloat16* Ks = reinterpret_cast<const __nv_bfloat16*>(a.K) + ((size_t)u * T + i) * D;
+    const __nv_bfloat16* Vs = reinterpret_cast<const __nv_bfloat16*>(a.V) + ((size_t)u * T + i) * D;
     __nv_bfloat16* Kd = reinterpret_cast<__nv_bfloat16*>(a.cache.K) + ((size_t)u * a.cache.capacity + i) * D;
     __nv_bfloat16* Vd = reinterpret_cast<__nv_bfloat16*>(a.cache.V) + ((size_t)u * a.cache.capacity + i) * D;
     for (int c = lane * 2; c < D; c += 64) {
       *reinterpret_cast<__nv_bfloat162*>(Kd + c) = *reinterpret_cast<const __nv_bfloat162*>(Ks + c);
       *reinterpret_cast<__nv_bfloat162*>(Vd + c) = *reinterpret_cast<const __nv_bfloat162*>(Vs + c);
     }
-    if (lane == 0) a.cache.pos[(size_t)u * a.cache.capacity + i] = t;
+    if (lane == 0) a.cache.pos[(size_t)u * a.cache.capacity + i] = i;
   }
-  if (blockIdx.x == 0 && threadIdx.x == 0) {
-    a.cache.len[u] = count;
-    a.cache.seen[u] = L.T;
-  }
-  if (keep_all && blockIdx.x == 0) {
-    // nothing evicted: zero moments
+  if (blockIdx.x == 0) {
+    if (threadIdx.x == 0) {
+      a.cache.len[u] = T;
+      a.cache.seen[u] = T;
+      a.mom.n[u] = 0;
+    }
     for (int e = threadIdx.x; e < D * D; e += blockDim.x) a.mom.C[(size_t)u * D * D + e] = 0.f;
     for (int e = threadIdx.x; e < D; e += blockDim.x) {
       a.mom.mu_k[(size_t)u * D + e] = 0.f;
       a.mom.mu_v[(size_t)u * D + e] = 0.f;
     }
-    if (threadIdx.x == 0) a.mom.n[u] = 0;
   }
 }
 
-template <int D>
+// ------------------------------------------------------------------- host
+constexpr size_t kStatsSmem = 1024 + 2 * 2 * kTileBytes + 2 * 2 * kBoxBytes;  // K, V stages + Q (RWb <= 2)
+constexpr size_t kScoresSmem = 1024 + 3 * kTileBytes + 2 * 2 * kBoxBytes;
+constexpr size_t kResidualSmem = 1024 + 2 * 2 * kTileBytes + 3 * kTileBytes;
+
 cudaError_t run(const CompressArgs& a, const mkv_geom& g, int num_sms, cudaStream_t st) {
   Layout L = make_layout(g, a.T, a.budget, a.window, num_sms);
   carve(L, a.ws);
-  cudaError_t e;
-  const dim3 cg(L.n_chunks, L.units);
-  const int RWp = static_cast<int>(align_up(L.RW, 4));
-  const bool keep_all = a.T <= a.budget;
-  if (!keep_all || a.diag_scores != nullptr) {  // nothing to select when keep_all: score only if asked
-    const size_t sm_stats = (size_t)(D * RWp + 2 * kTT * (D + 1) + 2 * RWp) * sizeof(float);
-    e = cudaFuncSetAttribute(stats_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_stats);
-    if (e != cudaSuccess) return e;
-    stats_kernel<D><<<cg, 256, sm_stats, st>>>(a, L);
-    const size_t sm_scores = (size_t)(D * RWp + kTT * (D + 1) + 2 * RWp + 8 * 32) * sizeof(float);
-    e = cudaFuncSetAttribute(scores_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_scores);
-    if (e != cudaSuccess) return e;
-    scores_kernel<D><<<cg, 256, sm_scores, st>>>(a, L);
+  const int D = g.head_dim, T = a.T, B = a.budget, U = L.units;
+  const bool keep_all = T <= B;
+  cudaError_t e = cudaSuccess;
+  auto attr = [](const void* f, size_t bytes) {
+    return cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes));
+  };
+  if ((e = attr((const void*)stats_tc<1>, kStatsSmem)) != cudaSuccess) return e;
+  if ((e = attr((const void*)stats_tc<0>, kStatsSmem)) != cudaSuccess) return e;
+  if ((e = attr((const void*)scores_tc, kScoresSmem)) != cudaSuccess) return e;
+  if ((e = attr((const void*)residual_tc, kResidualSmem)) != cudaSuccess) return e;
+
+  CUtensorMap tmK, tmV, tmQ, tmGK, tmGV, tmCK, tmCV;
+  const uint64_t rs = (uint64_t)D * 2;
+  bool ok = encode_tmap_bf16_3d(&tmK, a.K, D, T, U, rs, (uint64_t)T * rs, kTok) &&
+            encode_tmap_bf16_3d(&tmV, a.V, D, T, U, rs, (uint64_t)T * rs, kTok) &&
+            encode_tmap_bf16_3d(&tmQ, a.Q, D, L.RW, U, rs, (uint64_t)L.RW * rs, L.RWb * 128);
+  if (!keep_all)
+    ok = ok && encode_tmap_bf16_3d(&tmGK, L.gK, D, B, U, rs, (uint64_t)B * rs, kTok) &&
+         encode_tmap_bf16_3d(&tmGV, L.gV, D, B, U, rs, (uint64_t)B * rs, kTok) &&
+         encode_tmap_bf16_3d(&tmCK, a.cache.K, D, B, U, rs, (uint64_t)a.cache.capacity * rs, kTok) &&
+         encode_tmap_bf16_3d(&tmCV, a.cache.V, D, B, U, rs, (uint64_t)a.cache.capacity * rs, kTok);
+  if (!ok) return cudaErrorInvalidValue;
+
+  TcArgs tp{};
+  tp.D = D;
+  tp.RW = L.RW;
+  tp.RWb = L.RWb;
+  tp.W = a.window;
+  tp.T = T;
+  tp.causal = a.causal;
+  tp.sink = a.sink;
+  tp.keep_window = a.keep_window;
+  tp.pool = a.pool;
+  tp.qscale = rsqrtf(static_cast<float>(D)) * kLog2e;
+  tp.tau = a.tau;
+  tp.ws = a.ws;
+  const dim3 cg(L.n_chunks, U);
+
+  if (!keep_all || a.diag_scores != nullptr) {
+    TcArgs p1 = tp;
+    p1.n_rows = T;
+    p1.chunk = L.chunk;
+    p1.n_chunks = L.n_chunks;
+    p1.rowpart = L.rowpart;
+    p1.mrec = L.mpart;
+    stats_tc<1><<<cg, kTcThreads, kStatsSmem, st>>>(p1, tmK, tmV, tmQ);
+    TcArgs p2 = p1;
+    p2.s_out = L.s;
+    p2.diag = a.diag_scores;
+    scores_tc<<<cg, kTcThreads, kScoresSmem, st>>>(p2, tmK, tmQ);
   }
   if (keep_all) {
-    gather_kernel<D><<<dim3((a.T + 7) / 8, L.units), 256, 0, st>>>(a, L, nullptr, a.T, 1);
+    if (D == 128) keep_all_kernel<128><<<dim3((T + 7) / 8, U), 256, 0, st>>>(a, T);
+    else keep_all_kernel<64><<<dim3((T + 7) / 8, U), 256, 0, st>>>(a, T);
     return cudaGetLastError();
   }
-  select_kernel<D><<<L.units, kSelThreads, 0, st>>>(a, L, L.s, L.idx0, L.rmean, a.diag_idx1);
-  const int32_t* final_idx = L.idx0;
-  const float* final_rmean = L.rmean;
+
+  SelectArgs sa{};
+  sa.T = T;
+  sa.W = a.window;
+  sa.B = B;
+  sa.sink = a.sink;
+  sa.keep_window = a.keep_window;
+  sa.D = D;
+  sa.K = static_cast<const __nv_bfloat16*>(a.K);
+  sa.V = static_cast<const __nv_bfloat16*>(a.V);
+  sa.idx = L.idx;
+  TcArgs rset = tp;  // moments of a dense row set: one chunk per unit
+  rset.n_rows = B;
+  rset.chunk = static_cast<int>(align_up(B, kTok));
+  rset.n_chunks = 1;
+  rset.mrec = L.rpart;
+
   if (a.mi) {
-    moments_kernel<D><<<dim3(D / 8, L.units), 256, 0, st>>>(a, L, L.idx0, L.rmean, L.m0, a.mom, 0);
-    const size_t sm_res = (size_t)(D * D + kTT * (D + 1) + 8 * 32) * sizeof(float);
-    e = cudaFuncSetAttribute(residual_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_res);
-    if (e != cudaSuccess) return e;
-    residual_kernel<D><<<cg, 256, sm_res, st>>>(a, L);
-    float* rm1 = L.rmean + (size_t)L.units * (4 + 2 * D);
-    select_kernel<D><<<L.units, kSelThreads, 0, st>>>(a, L, L.s2, L.idx1, rm1, nullptr);
-    final_idx = L.idx1;
-    final_rmean = rm1;
+    SelectArgs s0 = sa;
+    s0.scores = L.s;
+    s0.diag_idx = a.diag_idx1;
+    s0.dst_K = L.gK;
+    s0.dst_V = L.gV;
+    s0.dst_cap = B;
+    select_kernel<<<U, kSelThreads, 0, st>>>(s0);
+    stats_tc<0><<<dim3(1, U), kTcThreads, kStatsSmem, st>>>(rset, tmGK, tmGV, tmQ);
+    finalize_kernel<<<dim3(D / 8, U), 256, 0, st>>>(L, L.m0, a.mom, 0);
+    TcArgs r = tp;
+    r.n_rows = T;
+    r.chunk = L.chunk;
+    r.n_chunks = L.n_chunks;
+    r.m0 = L.m0;
+    r.s_in = L.s;
+    r.s_out = L.s2;
+    r.diag = a.diag_score2;
+    residual_tc<<<cg, kTcThreads, kResidualSmem, st>>>(r, tmK, tmV);
   }
-  moments_kernel<D><<<dim3(D / 8, L.units), 256, 0, st>>>(a, L, final_idx, final_rmean, nullptr, a.mom, 1);
-  gather_kernel<D><<<dim3((a.budget + 7) / 8, L.units), 256, 0, st>>>(a, L, final_idx, a.budget, 0);
+  SelectArgs s1 = sa;
+  s1.scores = a.mi ? L.s2 : L.s;
+  s1.diag_idx = a.mi ? nullptr : a.diag_idx1;
+  s1.dst_K = static_cast<__nv_bfloat16*>(a.cache.K);
+  s1.dst_V = static_cast<__nv_bfloat16*>(a.cache.V);
+  s1.dst_cap = a.cache.capacity;
+  s1.dst_pos = a.cache.pos;
+  s1.dst_len = a.cache.len;
+  s1.dst_seen = a.cache.seen;
+  select_kernel<<<U, kSelThreads, 0, st>>>(s1);
+  stats_tc<0><<<dim3(1, U), kTcThreads, kStatsSmem, st>>>(rset, tmCK, tmCV, tmQ);
+  finalize_kernel<<<dim3(D / 8, U), 256, 0, st>>>(L, nullptr, a.mom, 1);
   return cudaGetLastError();
 }
 
@@ -660,9 +997,8 @@ size_t compress_workspace_bytes(const mkv_geom& g, int32_t T, const mkv_compress
 cudaError_t launch_compress(const CompressArgs& a, const mkv_geom& g, size_t ws_bytes, int num_sms,
                             cudaStream_t stream) {
   (void)ws_bytes;
-  if (g.head_dim == 128) return run<128>(a, g, num_sms, stream);
-  if (g.head_dim == 64) return run<64>(a, g, num_sms, stream);
-  return cudaErrorInvalidValue;
+  if (g.head_dim != 128 && g.head_dim != 64) return cudaErrorInvalidValue;
+  return run(a, g, num_sms, stream);
 }
 
 }  // namespace mkv
