@@ -156,6 +156,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   uint8_t* sK = sm;                        // [kS][128 x 128]
   uint8_t* sV = sm + kS * kTileBytes;      // [kS][128 x 128]
   uint8_t* sQ = sm + 2 * kS * kTileBytes;  // [2 boxes][RWb*128 rows][128 B]
+  uint8_t* sOnes = sQ + 2 * 2 * kBoxBytes;  // [2 boxes][16 rows][128 B] of bf16 1.0
   __shared__ __align__(8) uint64_t full[kS], empty[kS], lfull, lempty, qfull, sdone;
   __shared__ uint32_t tmem_base;
   __shared__ int abort_flag;
@@ -172,7 +173,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   if (tid == 0) {
     for (int i = 0; i < kS; ++i) {
       mbar_init(&full[i], 1);
-      mbar_init(&empty[i], 1 + 4);  // MMA commit + the 4 epilogue warps (column sums)
+      mbar_init(&empty[i], 1);  // the stage is free once its MMAs have completed
     }
     mbar_init(&lfull, 1);
     mbar_init(&lempty, 4);
@@ -182,6 +183,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     mbar_fence_init();
   }
   if (warp == 1) tmem_alloc(&tmem_base, 512);
+  if (warp >= 2) {  // the ones operand of the column sums K^T 1 and V^T 1
+    for (int i = tid - 64; i < 2 * 16 * 128 / 16; i += 128)
+      reinterpret_cast<uint4*>(sOnes)[i] = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u);
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -207,7 +213,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (lane == 0) {  // ---- MMA issuer
       const uint32_t idL = idesc_bf16(128, 128, 0, 0);  // logits: rows x tokens, both K-major
       const uint32_t idS = idesc_bf16(128, 128, 1, 1);  // V^T K: both MN-major (reduction over tokens)
-      const uint32_t aQ = smem_addr(sQ);
+      const uint32_t id1 = idesc_bf16(128, 16, 1, 0);   // X^T 1: X MN-major, ones K-major
+      const uint32_t aQ = smem_addr(sQ), a1 = smem_addr(sOnes);
       const bool ok = !LOGITS || pwait(&qfull, 0, abrt, p.ws, u);
       for (int i = 0; ok && i < n_tiles; ++i) {
         const int s = i % kS, j = i / kS;
@@ -229,7 +236,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         for (int kk = 0; kk < 8; ++kk) {
           const uint64_t dv = sdesc_sw128(aV + kk * 2048, kBoxBytes, 1024);
           const uint64_t dk = sdesc_sw128(aK + kk * 2048, kBoxBytes, 1024);
-          umma_bf16(tm + 256, dv, dk, idS, (i > 0 || kk > 0) ? 1u : 0u);
+          const uint64_t d1 = sdesc_sw128(a1 + (kk >> 2) * 2048 + (kk & 3) * 32, 16, 1024);
+          const uint32_t acc = (i > 0 || kk > 0) ? 1u : 0u;
+          umma_bf16(tm + 256, dv, dk, idS, acc);
+          umma_bf16(tm + 384, dk, d1, id1, acc);  // column sums of K (lane = key dim)
+          umma_bf16(tm + 400, dv, d1, id1, acc);  // column sums of V (lane = value dim)
         }
         umma_commit(&empty[s]);
       }
@@ -239,40 +250,39 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     // ---- epilogue: warps 2..5; TMEM lane quarter qd = warp % 4
     const int et = tid - 64, qd = warp & 3;
     const uint32_t lane_base = static_cast<uint32_t>(qd * 32) << 16;
-    float sk = 0.f, sv = 0.f;
     float m[2] = {-INFINITY, -INFINITY}, l[2] = {0.f, 0.f};
-    for (int i = 0; i < n_tiles; ++i) {
-      const int s = i % kS, j = i / kS;
-      if (!pwait(&full[s], j & 1, abrt, p.ws, u)) break;
-      if (et < p.D) {  // column sums (rows past the slab's end are zero-filled)
-        const uint8_t* tk = sK + s * kTileBytes;
-        const uint8_t* tv = sV + s * kTileBytes;
-#pragma unroll 8
-        for (int r = 0; r < kTok; ++r) {
-          sk += tile_at(tk, r, et);
-          sv += tile_at(tv, r, et);
-        }
-      }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&empty[s]);
-      if (LOGITS) {
-        if (!pwait(&lfull, i & 1, abrt, p.ws, u)) break;
-        tc_fence_after();
-        for (int rb = 0; rb < RWb; ++rb) {
-          const int r = rb * 128 + qd * 32 + lane;  // window row of this thread
-          const int wi = r % p.W;
-          const int tmax_vis = p.causal ? p.T - p.W + wi : 0x7fffffff;
-          for (int c0 = 0; c0 < kTok; c0 += 32) {
-            float x[32];
-            tmem_ld32(tm + lane_base + rb * 128 + c0, x);
-            const int t0 = t_begin + i * kTok + c0;
-            float mx = -INFINITY;
+    int tmax_vis[2];
+    for (int rb = 0; rb < 2; ++rb) {
+      const int r = rb * 128 + qd * 32 + lane;  // window row of this thread
+      tmax_vis[rb] = p.causal ? p.T - p.W + r % p.W : 0x7fffffff;
+    }
+    const int t_safe = p.causal ? p.T - p.W : 0x7fffffff;  // tokens every window row sees
+    for (int i = 0; LOGITS && i < n_tiles; ++i) {
+      if (!pwait(&lfull, i & 1, abrt, p.ws, u)) break;
+      tc_fence_after();
+      const int tt0 = t_begin + i * kTok;
+      const bool fast = tt0 + kTok <= t_end && tt0 + kTok - 1 <= t_safe;  // no masking in this tile
+      for (int rb = 0; rb < RWb; ++rb) {
+        for (int c0 = 0; c0 < kTok; c0 += 32) {
+          float x[32];
+          tmem_ld32(tm + lane_base + rb * 128 + c0, x);
+          const int t0 = tt0 + c0;
+          float mx = -INFINITY;
+          if (fast) {
+#pragma unroll
+            for (int jj = 0; jj < 32; ++jj) {
+              x[jj] *= p.qscale;
+              mx = fmaxf(mx, x[jj]);
+            }
+          } else {
 #pragma unroll
             for (int jj = 0; jj < 32; ++jj) {
               const int t = t0 + jj;
-              x[jj] = (t < t_end && t <= tmax_vis) ? x[jj] * p.qscale : -INFINITY;
+              x[jj] = (t < t_end && t <= tmax_vis[rb]) ? x[jj] * p.qscale : -INFINITY;
               mx = fmaxf(mx, x[jj]);
             }
+          }
+          {
             const float mn = fmaxf(m[rb], mx);
             if (mn != -INFINITY) {
               float acc = 0.f;
@@ -283,10 +293,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             }
           }
         }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&lempty);
       }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&lempty);
     }
     if (LOGITS) {
       for (int rb = 0; rb < RWb; ++rb) {
@@ -298,11 +308,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         }
       }
     }
-    sum_k[et] = sk;
-    sum_v[et] = sv;
-    epi_sync();
     const bool got = pwait(&sdone, 0, abrt, p.ws, u);
     tc_fence_after();
+    {
+      float x[32];
+      tmem_ld32(tm + lane_base + 384, x);  // [0]: sum of K's column (this lane), [16]: of V's
+      sum_k[qd * 32 + lane] = x[0];
+      sum_v[qd * 32 + lane] = x[16];
+    }
+    epi_sync();
     const float nc = static_cast<float>(max(0, t_end - t_begin));
     float* rec = p.mrec + ((size_t)u * p.n_chunks + chunk) * rec_floats(p.D);
     const int a = qd * 32 + lane;  // value dim = TMEM lane
@@ -317,9 +331,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         }
       }
     }
-    if (et < p.D) {
-      rec[4 + et] = nc > 0.f ? sum_k[et] / nc : 0.f;
-      rec[4 + p.D + et] = nc > 0.f ? sum_v[et] / nc : 0.f;
+    if (a < p.D) {
+      rec[4 + a] = nc > 0.f ? sum_k[a] / nc : 0.f;
+      rec[4 + p.D + a] = nc > 0.f ? sum_v[a] / nc : 0.f;
     }
     if (et == 0) rec[0] = got ? nc : 0.f;
   }
@@ -342,7 +356,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   __shared__ __align__(8) uint64_t full[kS], empty[kS], lfull[2], lempty[2], qfull;
   __shared__ uint32_t tmem_base;
   __shared__ int abort_flag;
-  __shared__ float s_m[256], s_il[256];
+  __shared__ __align__(16) float s_b[256];  // log2(1 / l_r) - m_r (-inf for padding rows)
+  __shared__ int s_wi[256];                   // window index of row r (r mod W)
 
   const int chunk = blockIdx.x, u = blockIdx.y;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -418,24 +433,34 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             if (rp[0] != -INFINITY) Lsum += rp[1] * fast_exp2(rp[0] - M);
           }
       }
-      s_m[r] = M;
-      s_il[r] = Lsum > 0.f ? 1.f / Lsum : 0.f;
+      s_b[r] = (Lsum > 0.f) ? -log2f(Lsum) - M : -INFINITY;
+      s_wi[r] = r % p.W;
     }
     epi_sync();
+    const int t_safe = p.causal ? p.T - p.W : 0x7fffffff;  // tokens every window row sees
     for (int i = 0; i < n_tiles; ++i) {
       const int b = i & 1;
       if (!pwait(&lfull[b], (i >> 1) & 1, abrt, p.ws, u)) break;
       tc_fence_after();
       const int t = t_begin + i * kTok + qd * 32 + lane;  // token of this thread (TMEM lane)
+      const bool fast = t <= t_safe;  // every window row sees this token
       float acc = 0.f;
       for (int c0 = 0; c0 < RWp; c0 += 32) {
         float x[32];
         tmem_ld32(tm + lane_base + b * 256 + c0, x);
+        if (fast) {  // p = 2^(x qscale + b_r); padding rows have b_r = -inf
 #pragma unroll
-        for (int jj = 0; jj < 32; ++jj) {
-          const int r = c0 + jj;
-          if (r < p.RW && (!p.causal || t <= p.T - p.W + r % p.W))
-            acc += fast_exp2(x[jj] * p.qscale - s_m[r]) * s_il[r];
+          for (int jj = 0; jj < 32; jj += 4) {
+            const float4 b4 = *reinterpret_cast<const float4*>(s_b + c0 + jj);
+            acc += fast_exp2(fmaf(x[jj], p.qscale, b4.x)) + fast_exp2(fmaf(x[jj + 1], p.qscale, b4.y)) +
+                   fast_exp2(fmaf(x[jj + 2], p.qscale, b4.z)) + fast_exp2(fmaf(x[jj + 3], p.qscale, b4.w));
+          }
+        } else {
+#pragma unroll
+          for (int jj = 0; jj < 32; ++jj) {
+            const int r = c0 + jj;
+            if (t <= p.T - p.W + s_wi[r]) acc += fast_exp2(fmaf(x[jj], p.qscale, s_b[r]));
+          }
         }
       }
       tc_fence_before();
@@ -872,7 +897,7 @@ __global__ void __launch_bounds__(256) keep_all_kernel(const CompressArgs a, int
 }
 
 // ------------------------------------------------------------------- host
-constexpr size_t kStatsSmem = 1024 + 2 * 2 * kTileBytes + 2 * 2 * kBoxBytes;  // K, V stages + Q (RWb <= 2)
+constexpr size_t kStatsSmem = 1024 + 2 * 2 * kTileBytes + 2 * 2 * kBoxBytes + 4096;  // K, V stages, Q, ones
 constexpr size_t kScoresSmem = 1024 + 3 * kTileBytes + 2 * 2 * kBoxBytes;
 constexpr size_t kResidualSmem = 1024 + 2 * 2 * kTileBytes + 3 * kTileBytes;
 
