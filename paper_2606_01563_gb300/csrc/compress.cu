@@ -23,9 +23,13 @@
 // warp 1 owns TMEM and issues tcgen05.mma, warps 2-5 run the epilogue; stages
 // hand over through mbarriers whose waits are all bounded.  Head dims below
 // 128 use the same 128-wide MMAs: the missing 64-column box is zero-filled.
+#include <cooperative_groups.h>
+
 #include "common.cuh"
 #include "kernels.h"
 #include "tc.cuh"
+
+namespace cg = cooperative_groups;
 
 namespace mkv {
 
@@ -37,6 +41,7 @@ constexpr int kTileBytes = kTok * kDP * 2;  // one [128 x 128] bf16 tile: 2 boxe
 constexpr int kBoxBytes = kTok * 128;
 constexpr int kTcThreads = 192;  // warp 0 TMA, warp 1 MMA, warps 2..5 epilogue
 constexpr int kSelThreads = 1024;
+constexpr int kPF = 0;  // tiles prefetched into L2 ahead of the one being loaded (0: none)
 constexpr unsigned kFull = 0xffffffffu;
 
 struct Layout {
@@ -46,13 +51,15 @@ struct Layout {
   size_t rec;         // floats per moment record: 4 + 2D + D*D (padded)
   float* rowpart;     // [units][n_chunks][RW][2]  (max in log2 units, sum)
   float* mpart;       // [units][n_chunks][rec]    all-token chunk moments
-  float* rpart;       // [units][rec]              retained-set moments
+  float* rpart;       // [units][n_rchunks][rec]   retained-set chunk moments
+  int n_rchunks;      // chunks of kTok retained rows
   float* s;           // [units][T]
   float* s2;          // [units][T]
   int32_t* idx;       // [units][B]
   __nv_bfloat16* gK;  // [units][B][D] rows of R0
   __nv_bfloat16* gV;
-  float* m0;  // [units][rec] moments of E0
+  float* m0;    // [units][rec] moments of E0
+  float* mall;  // [units][rec] moments of all tokens (the merged chunk records)
 };
 
 __host__ __device__ inline size_t rec_floats(int D) { return align_up(4 + 2 * (size_t)D + (size_t)D * D, 4); }
@@ -74,6 +81,7 @@ Layout make_layout(const mkv_geom& g, int T, int B, int W, int num_sms) {
   L.chunk = static_cast<int>(((tiles + per - 1) / per) * kTok);
   L.n_chunks = (T + L.chunk - 1) / L.chunk;
   L.rec = rec_floats(L.D);
+  L.n_rchunks = (B + kTok - 1) / kTok;
   return L;
 }
 
@@ -88,13 +96,14 @@ size_t carve(Layout& L, void* ws) {
   const size_t U = L.units;
   L.rowpart = reinterpret_cast<float*>(take(U * L.n_chunks * L.RW * 2 * sizeof(float)));
   L.mpart = reinterpret_cast<float*>(take(U * L.n_chunks * L.rec * sizeof(float)));
-  L.rpart = reinterpret_cast<float*>(take(U * L.rec * sizeof(float)));
+  L.rpart = reinterpret_cast<float*>(take(U * L.n_rchunks * L.rec * sizeof(float)));
   L.s = reinterpret_cast<float*>(take(U * (size_t)L.T * sizeof(float)));
   L.s2 = reinterpret_cast<float*>(take(U * (size_t)L.T * sizeof(float)));
   L.idx = reinterpret_cast<int32_t*>(take(U * (size_t)L.B * sizeof(int32_t)));
   L.gK = reinterpret_cast<__nv_bfloat16*>(take(U * (size_t)L.B * L.D * 2));
   L.gV = reinterpret_cast<__nv_bfloat16*>(take(U * (size_t)L.B * L.D * 2));
   L.m0 = reinterpret_cast<float*>(take(U * L.rec * sizeof(float)));
+  L.mall = reinterpret_cast<float*>(take(U * L.rec * sizeof(float)));
   return off;
 }
 
@@ -199,8 +208,18 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         mbar_arrive_expect_tx(&qfull, 2u * RWb * kBoxBytes);
         for (int bx = 0; bx < 2; ++bx) tma_load_3d(sQ + bx * RWb * kBoxBytes, &tmQ, bx * 64, 0, u, &qfull);
       }
+      for (int i = 0; i < min(kPF, n_tiles); ++i)
+        for (int bx = 0; bx < 2; ++bx) {
+          tma_prefetch_3d(&tmK, bx * 64, t_begin + i * kTok, u);
+          tma_prefetch_3d(&tmV, bx * 64, t_begin + i * kTok, u);
+        }
       for (int i = 0; i < n_tiles; ++i) {
         const int s = i % kS, j = i / kS;
+        if (kPF > 0 && i + kPF < n_tiles)
+          for (int bx = 0; bx < 2; ++bx) {
+            tma_prefetch_3d(&tmK, bx * 64, t_begin + (i + kPF) * kTok, u);
+            tma_prefetch_3d(&tmV, bx * 64, t_begin + (i + kPF) * kTok, u);
+          }
         if (j >= 1 && !pwait(&empty[s], (j - 1) & 1, abrt, p.ws, u)) break;
         mbar_arrive_expect_tx(&full[s], 2u * kTileBytes);
         for (int bx = 0; bx < 2; ++bx) {
@@ -390,8 +409,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (lane == 0) {
       mbar_arrive_expect_tx(&qfull, 2u * RWb * kBoxBytes);
       for (int bx = 0; bx < 2; ++bx) tma_load_3d(sQ + bx * RWb * kBoxBytes, &tmQ, bx * 64, 0, u, &qfull);
+      for (int i = kS; i < min(kS + kPF, n_tiles); ++i)
+        for (int bx = 0; bx < 2; ++bx) tma_prefetch_3d(&tmK, bx * 64, t_begin + i * kTok, u);
       for (int i = 0; i < n_tiles; ++i) {
         const int s = i % kS, j = i / kS;
+        if (kPF > 0 && i + kS + kPF < n_tiles)
+          for (int bx = 0; bx < 2; ++bx) tma_prefetch_3d(&tmK, bx * 64, t_begin + (i + kS + kPF) * kTok, u);
         if (j >= 1 && !pwait(&empty[s], (j - 1) & 1, abrt, p.ws, u)) break;
         mbar_arrive_expect_tx(&full[s], kTileBytes);
         for (int bx = 0; bx < 2; ++bx)
@@ -516,6 +539,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     abort_flag = 0;
     mbar_fence_init();
     // the first stages' copies go out while C0' is being prepared
+    for (int i = kS; i < min(kS + kPF, n_tiles); ++i)
+      for (int bx = 0; bx < 2; ++bx) {
+        tma_prefetch_3d(&tmK, bx * 64, t_begin + i * kTok, u);
+        tma_prefetch_3d(&tmV, bx * 64, t_begin + i * kTok, u);
+      }
     for (int i = 0; i < min(kS, n_tiles); ++i) {
       mbar_arrive_expect_tx(&full[i], 2u * kTileBytes);
       for (int bx = 0; bx < 2; ++bx) {
@@ -564,6 +592,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (lane == 0) {
       for (int i = kS; i < n_tiles; ++i) {
         const int s = i % kS, j = i / kS;
+        if (kPF > 0 && i + kPF < n_tiles)
+          for (int bx = 0; bx < 2; ++bx) {
+            tma_prefetch_3d(&tmK, bx * 64, t_begin + (i + kPF) * kTok, u);
+            tma_prefetch_3d(&tmV, bx * 64, t_begin + (i + kPF) * kTok, u);
+          }
         if (!pwait(&empty[s], (j - 1) & 1, abrt, p.ws, u)) break;
         mbar_arrive_expect_tx(&full[s], 2u * kTileBytes);
         for (int bx = 0; bx < 2; ++bx) {
@@ -689,15 +722,24 @@ struct SelectArgs {
   int32_t* dst_seen;
 };
 
-__global__ void __launch_bounds__(kSelThreads) select_kernel(const SelectArgs a) {
-  __shared__ uint32_t hist[256];
-  __shared__ uint32_t whist[8][256];  // private histograms for groups of 4 warps (less contention)
+constexpr int kSelCL = 8;  // CTAs per unit (one cluster), each over a contiguous range of positions
+
+__global__ void __cluster_dims__(kSelCL, 1, 1) __launch_bounds__(kSelThreads) select_kernel(const SelectArgs a) {
+  __shared__ uint32_t hist[2][256];   // this CTA's histogram, double-buffered by pass parity (read remotely)
+  __shared__ uint32_t whist[8][256];  // private histograms for groups of 4 warps (less atomic contention)
+  __shared__ uint32_t ghist[256];     // the cluster's histogram
   __shared__ int wsum[32];
   __shared__ int tot;
   __shared__ uint32_t s_prefix;
   __shared__ int s_need;
-  const int u = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  __shared__ int ex_cnt[2];  // this CTA's ties and certain selections (protected or above the threshold)
+  __shared__ int s_before[2];
+  cg::cluster_group cluster = cg::this_cluster();
+  const int rank = static_cast<int>(cluster.block_rank());
+  const int u = blockIdx.x / kSelCL, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int T = a.T, W = a.W;
+  const int per = (T + kSelCL - 1) / kSelCL;
+  const int r0 = min(T, rank * per), r1 = min(T, r0 + per);
   const float* sc = a.scores + (size_t)u * T;
   const int k = a.B - protected_count(T, W, a.sink, a.keep_window);  // >= 0 (validated), < candidates
 
@@ -709,7 +751,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const SelectArgs a)
       for (int i = tid; i < 8 * 256; i += kSelThreads) (&whist[0][0])[i] = 0;
       __syncthreads();
       uint32_t* wh = whist[warp & 7];
-      for (int t = tid; t < T; t += kSelThreads) {
+      for (int t = r0 + tid; t < r1; t += kSelThreads) {
         if (is_protected(t, T, W, a.sink, a.keep_window)) continue;
         const uint32_t key = float_key(sc[t]);
         if ((key & pmask) == prefix) atomicAdd(&wh[(key >> shift) & 255u], 1u);
@@ -719,14 +761,21 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const SelectArgs a)
         uint32_t c = 0;
 #pragma unroll
         for (int g = 0; g < 8; ++g) c += whist[g][i];
-        hist[i] = c;
+        hist[pass & 1][i] = c;
+      }
+      cluster.sync();  // every CTA's histogram of this pass is complete
+      for (int i = tid; i < 256; i += kSelThreads) {
+        uint32_t c = 0;
+#pragma unroll
+        for (int r = 0; r < kSelCL; ++r) c += cluster.map_shared_rank(&hist[pass & 1][0], r)[i];
+        ghist[i] = c;
       }
       __syncthreads();
       if (warp == 0) {  // the digit where the descending cumulative count reaches `need`
         int cnt[8], tot8 = 0;
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
-          cnt[e] = static_cast<int>(hist[255 - (lane * 8 + e)]);
+          cnt[e] = static_cast<int>(ghist[255 - (lane * 8 + e)]);
           tot8 += cnt[e];
         }
         int incl = tot8;
@@ -750,15 +799,66 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const SelectArgs a)
       need = s_need;
       prefix = s_prefix;
       pmask |= 255u << shift;
-      __syncthreads();
     }
   }
-  int ties_before = 0, sel_before = 0;
+  // counts of this CTA's range, exchanged to place its outputs in ascending order
+  {
+    int n_tie = 0, n_sure = 0;
+    for (int t = r0 + tid; t < r1; t += kSelThreads) {
+      const bool prot = is_protected(t, T, W, a.sink, a.keep_window);
+      if (prot) {
+        ++n_sure;
+      } else if (k > 0) {
+        const uint32_t key = float_key(sc[t]);
+        n_sure += key > prefix;
+        n_tie += key == prefix;
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      n_tie += __shfl_xor_sync(kFull, n_tie, o);
+      n_sure += __shfl_xor_sync(kFull, n_sure, o);
+    }
+    if (lane == 0) {
+      wsum[warp] = n_tie;
+      if (warp == 0) tot = 0;
+    }
+    __syncthreads();
+    if (tid == 0) {
+      int tt = 0;
+      for (int w = 0; w < kSelThreads / 32; ++w) tt += wsum[w];
+      ex_cnt[0] = tt;
+    }
+    __syncthreads();
+    if (lane == 0) wsum[warp] = n_sure;
+    __syncthreads();
+    if (tid == 0) {
+      int ss = 0;
+      for (int w = 0; w < kSelThreads / 32; ++w) ss += wsum[w];
+      ex_cnt[1] = ss;
+    }
+  }
+  cluster.sync();
+  if (tid == 0) {
+    int ties_before = 0, sel_before = 0;
+    for (int r = 0; r < rank; ++r) {
+      const int* rc = cluster.map_shared_rank(ex_cnt, r);
+      const int nt = rc[0], ns = rc[1];
+      const int take = min(max(need - ties_before, 0), nt);  // this rank's ties that are selected
+      sel_before += ns + take;
+      ties_before += nt;
+    }
+    s_before[0] = ties_before;
+    s_before[1] = sel_before;
+  }
+  __syncthreads();
+  int ties_before = s_before[0], sel_before = s_before[1];
+  const int my_first = sel_before;
   int32_t* out = a.idx + (size_t)u * a.B;
-  for (int base = 0; base < T; base += kSelThreads) {
+  for (int base = r0; base < r1; base += kSelThreads) {
     const int t = base + tid;
     bool prot = false, tie = false, gt = false;
-    if (t < T) {
+    if (t < r1) {
       prot = is_protected(t, T, W, a.sink, a.keep_window);
       if (!prot && k > 0) {
         const uint32_t key = float_key(sc[t]);
@@ -782,11 +882,12 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const SelectArgs a)
     sel_before += sel_total;
   }
   __syncthreads();
-  // gather the retained rows (16-byte chunks)
+  // gather the rows this CTA selected (16-byte chunks)
   const int D = a.D;
   const int per_row = D / 8;
-  for (int i = tid; i < a.B * per_row; i += kSelThreads) {
-    const int r = i / per_row, c = i % per_row;
+  const int o0 = min(my_first, a.B), o1 = min(sel_before, a.B);
+  for (int i = tid; i < (o1 - o0) * per_row; i += kSelThreads) {
+    const int r = o0 + i / per_row, c = i % per_row;
     const int t = min(max(out[r], 0), T - 1);  // never read outside the unit's slab
     const size_t src = ((size_t)u * T + t) * D;
     const size_t dst = ((size_t)u * a.dst_cap + r) * D;
@@ -794,30 +895,35 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const SelectArgs a)
     reinterpret_cast<uint4*>(a.dst_V + dst)[c] = reinterpret_cast<const uint4*>(a.V + src)[c];
   }
   if (a.dst_pos)
-    for (int r = tid; r < a.B; r += kSelThreads) a.dst_pos[(size_t)u * a.dst_cap + r] = out[r];
-  if (tid == 0 && a.dst_len) {
+    for (int r = o0 + tid; r < o1; r += kSelThreads) a.dst_pos[(size_t)u * a.dst_cap + r] = out[r];
+  if (rank == 0 && tid == 0 && a.dst_len) {
     a.dst_len[u] = a.B;
     a.dst_seen[u] = T;
   }
+  cluster.sync();  // no CTA leaves while another may still read its shared memory
 }
 
 // --------------------------------------------------------------- finalize
 // Moments of E = all \ R for 8 value dims (rows of C) per CTA: the all-token
 // co-moment is the multi-way Chan merge of the chunk records; R's centred
 // record is removed with the reverse pairwise formula.
+// merge_all = 1: merge the chunk records and keep the result in L.mall;
+// merge_all = 0: start from L.mall (a single record).
 __global__ void __launch_bounds__(256) finalize_kernel(const Layout L, float* out_rec, mkv_moments out_mom,
-                                                       int final_out) {
+                                                       int final_out, int merge_all) {
   constexpr int NT = 256, RB = 8;
   __shared__ float mk[kDP], mv[kDP], mkR[kDP], mvR[kDP];
   __shared__ float s_n;
   const int D = L.D;
   const int rb = blockIdx.x, u = blockIdx.y, tid = threadIdx.x;
   const size_t rf = rec_floats(D);
-  const float* recs = L.mpart + (size_t)u * L.n_chunks * rf;
-  const float* rR = L.rpart + (size_t)u * rf;
+  const int n_rec = merge_all ? L.n_chunks : 1;
+  const float* recs = merge_all ? L.mpart + (size_t)u * L.n_chunks * rf : L.mall + (size_t)u * rf;
+  float* mall = L.mall + (size_t)u * rf;
+  const float* rrecs = L.rpart + (size_t)u * L.n_rchunks * rf;
   if (tid < 2 * D) {
     float num = 0.f, n = 0.f;
-    for (int c = 0; c < L.n_chunks; ++c) {
+    for (int c = 0; c < n_rec; ++c) {
       const float nc = recs[(size_t)c * rf];
       n += nc;
       num += nc * recs[(size_t)c * rf + 4 + tid];
@@ -825,22 +931,41 @@ __global__ void __launch_bounds__(256) finalize_kernel(const Layout L, float* ou
     if (tid < D) mk[tid] = num / n;
     else mv[tid - D] = num / n;
     if (tid == 0) s_n = n;
+    if (merge_all && rb == 0) {
+      mall[4 + tid] = num / n;
+      if (tid == 0) mall[0] = n;
+    }
   }
-  if (tid < D) {
-    mkR[tid] = rR[4 + tid];
-    mvR[tid] = rR[4 + D + tid];
+  __shared__ float s_nR;
+  if (tid < 2 * D) {  // retained set: merge its chunk records' means
+    float num = 0.f, n = 0.f;
+    for (int c = 0; c < L.n_rchunks; ++c) {
+      const float nc = rrecs[(size_t)c * rf];
+      n += nc;
+      num += nc * rrecs[(size_t)c * rf + 4 + tid];
+    }
+    const float mean = n > 0.f ? num / n : 0.f;
+    if (tid < D) mkR[tid] = mean;
+    else mvR[tid - D] = mean;
+    if (tid == 0) s_nR = n;
   }
   __syncthreads();
-  const float n = s_n, nR = rR[0], nE = n - nR;
+  const float n = s_n, nR = s_nR, nE = n - nR;
   for (int e = tid; e < RB * D; e += NT) {
     const int ar = rb * RB + e / D, c = e % D;
     float M = 0.f;
-    for (int ch = 0; ch < L.n_chunks; ++ch) {
+    for (int ch = 0; ch < n_rec; ++ch) {
       const float* r = recs + (size_t)ch * rf;
       const float nc = r[0];
       if (nc > 0.f) M += r[4 + 2 * D + (size_t)ar * D + c] + nc * (r[4 + D + ar] - mv[ar]) * (r[4 + c] - mk[c]);
     }
-    const float MR = rR[4 + 2 * D + (size_t)ar * D + c];
+    if (merge_all) mall[4 + 2 * D + (size_t)ar * D + c] = M;
+    float MR = 0.f;
+    for (int ch = 0; ch < L.n_rchunks; ++ch) {
+      const float* r = rrecs + (size_t)ch * rf;
+      const float nc = r[0];
+      if (nc > 0.f) MR += r[4 + 2 * D + (size_t)ar * D + c] + nc * (r[4 + D + ar] - mvR[ar]) * (r[4 + c] - mkR[c]);
+    }
     float CE = 0.f, mkE_c = 0.f, mvE_a = 0.f;
     if (nE > 0.f) {
       mkE_c = (n * mk[c] - nR * mkR[c]) / nE;
@@ -971,10 +1096,10 @@ cudaError_t run(const CompressArgs& a, const mkv_geom& g, int num_sms, cudaStrea
   sa.K = static_cast<const __nv_bfloat16*>(a.K);
   sa.V = static_cast<const __nv_bfloat16*>(a.V);
   sa.idx = L.idx;
-  TcArgs rset = tp;  // moments of a dense row set: one chunk per unit
+  TcArgs rset = tp;  // moments of a dense row set: chunks of kTok rows
   rset.n_rows = B;
-  rset.chunk = static_cast<int>(align_up(B, kTok));
-  rset.n_chunks = 1;
+  rset.chunk = kTok;
+  rset.n_chunks = L.n_rchunks;
   rset.mrec = L.rpart;
 
   if (a.mi) {
@@ -984,9 +1109,9 @@ cudaError_t run(const CompressArgs& a, const mkv_geom& g, int num_sms, cudaStrea
     s0.dst_K = L.gK;
     s0.dst_V = L.gV;
     s0.dst_cap = B;
-    select_kernel<<<U, kSelThreads, 0, st>>>(s0);
-    stats_tc<0><<<dim3(1, U), kTcThreads, kStatsSmem, st>>>(rset, tmGK, tmGV, tmQ);
-    finalize_kernel<<<dim3(D / 8, U), 256, 0, st>>>(L, L.m0, a.mom, 0);
+    select_kernel<<<U * kSelCL, kSelThreads, 0, st>>>(s0);
+    stats_tc<0><<<dim3(L.n_rchunks, U), kTcThreads, kStatsSmem, st>>>(rset, tmGK, tmGV, tmQ);
+    finalize_kernel<<<dim3(D / 8, U), 256, 0, st>>>(L, L.m0, a.mom, 0, 1);
     TcArgs r = tp;
     r.n_rows = T;
     r.chunk = L.chunk;
@@ -1006,9 +1131,9 @@ cudaError_t run(const CompressArgs& a, const mkv_geom& g, int num_sms, cudaStrea
   s1.dst_pos = a.cache.pos;
   s1.dst_len = a.cache.len;
   s1.dst_seen = a.cache.seen;
-  select_kernel<<<U, kSelThreads, 0, st>>>(s1);
-  stats_tc<0><<<dim3(1, U), kTcThreads, kStatsSmem, st>>>(rset, tmCK, tmCV, tmQ);
-  finalize_kernel<<<dim3(D / 8, U), 256, 0, st>>>(L, nullptr, a.mom, 1);
+  select_kernel<<<U * kSelCL, kSelThreads, 0, st>>>(s1);
+  stats_tc<0><<<dim3(L.n_rchunks, U), kTcThreads, kStatsSmem, st>>>(rset, tmCK, tmCV, tmQ);
+  finalize_kernel<<<dim3(D / 8, U), 256, 0, st>>>(L, nullptr, a.mom, 1, a.mi ? 0 : 1);
   return cudaGetLastError();
 }
 

@@ -16,6 +16,18 @@
 // CTA of a unit to finish (atomic ticket, no waiting) merges the S partial
 // (m, l, o) records with the moment pseudo-partial (log n + scale q.mu_k,
 // f_hat_E) by log-sum-exp and writes the output; it also performs the append.
+//
+// Cluster variant (S <= 16): the S CTAs of a unit form one thread-block
+// cluster.  Partial records and f_hat_E rows go straight into CTA 0's shared
+// memory (distributed shared memory stores), one cluster barrier orders them,
+// and CTA 0 merges: no global partials, no atomics, no second L2 round trip.
+//
+// Both variants are launched as programmatic dependents of the previous
+// kernel in the stream: barrier set-up overlaps its tail, and every global
+// read waits on griddepcontrol.wait (the previous grid complete, its writes
+// visible).
+#include <cooperative_groups.h>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -27,6 +39,23 @@ constexpr int kThreads = 128;  // 4 warps x 16 rows of each 64-row tile
 constexpr int kStages = 3;
 constexpr int kTT = kDecodeTile;
 constexpr unsigned kFull = 0xffffffffu;
+constexpr int kMaxClusterSplits = 16;
+
+namespace cg = cooperative_groups;
+
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_arrive_release() {
+  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait_acquire() {
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
 
 __device__ __forceinline__ void mma_bf16(float (&d)[4], uint32_t a0, uint32_t a2, uint32_t b0, uint32_t b1) {
   // A rows 8..15 are zero (at most 8 query heads per KV head): registers a1, a3 = 0
@@ -122,7 +151,7 @@ __device__ __forceinline__ void process16(WarpState<D>& st, const uint32_t (&qa)
   }
 }
 
-template <int D, int G>
+template <int D, int G, bool CL>
 __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, const __grid_constant__ CUtensorMap tmK,
                                                           const __grid_constant__ CUtensorMap tmV) {
   constexpr int DPL = D / 32;
@@ -143,6 +172,26 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
   const int u = b * a.n_kv + kv;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const float scale = rsqrtf(static_cast<float>(D));
+
+  // cluster variant: CTA 0's receive area [S][G][PS] partials, [G][D] f_hat_E
+  float* sRcv = reinterpret_cast<float*>(dsmem + 2 * kStages * kTileBytes);
+  float* sFr = sRcv + (size_t)a.S * G * PS;
+  float* rcv0 = nullptr;
+  float* fr0 = nullptr;
+  if constexpr (CL) {
+    cluster_arrive_relaxed();  // every CTA of the cluster has started before the first remote store
+    cg::cluster_group cluster = cg::this_cluster();
+    rcv0 = cluster.map_shared_rank(sRcv, 0);
+    fr0 = cluster.map_shared_rank(sFr, 0);
+  }
+  if (tid == 0) {
+    for (int i = 0; i < kStages; ++i) mbar_init(&bars[i], 1);
+    mbar_fence_init();
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
+  }
+  grid_dependency_wait();
+  grid_launch_dependents();
 
   // ---- loads that do not depend on the cache length go out first
   const __nv_bfloat16* qg = reinterpret_cast<const __nv_bfloat16*>(a.q) + ((size_t)u * G) * D;
@@ -213,15 +262,14 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
   };
 
   if (tid == 0) {
-    for (int i = 0; i < kStages; ++i) mbar_init(&bars[i], 1);
-    mbar_fence_init();
     for (int i = 0; i < min(kStages, n_tiles); ++i) issue(i);
   }
   for (int i = tid; i < G * D; i += kThreads) sQ[i] = __bfloat162float(qg[i]) * (scale * kLog2e);
   __syncthreads();
+  if constexpr (CL) cluster_wait_acquire();
 
   if (use_m) {
-    // scale * q . mu_k for every head (every CTA; the last one uses it)
+    // scale * q . mu_k for every head (every CTA; the merging one uses it)
     for (int h = warp; h < G; h += 4) {
       float acc = 0.f;
 #pragma unroll
@@ -261,8 +309,9 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
             acc[h] = warp_sum(acc[h]);
           }
           if (lane == 0) {
+            float* fdst = CL ? fr0 + row : a.fhat + (size_t)u * G * D + row;
 #pragma unroll
-            for (int h = 0; h < G; ++h) a.fhat[((size_t)u * G + h) * D + row] = mvr[k] + acc[h] * (1.f / kLog2e);
+            for (int h = 0; h < G; ++h) fdst[h * D] = mvr[k] + acc[h] * (1.f / kLog2e);
           }
         }
       }
@@ -349,7 +398,7 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
     }
   }
   __syncthreads();
-  float* part = a.partial + ((size_t)u * a.S + s) * G * PS;
+  float* part = CL ? rcv0 + (size_t)s * G * PS : a.partial + ((size_t)u * a.S + s) * G * PS;
   for (int idx = tid; idx < G * D; idx += kThreads) {
     const int h = idx / D, dd = idx % D;
     float M = -INFINITY;
@@ -372,34 +421,51 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
     }
   }
 
-  // ---- ticket: the last CTA of this unit merges everything
-  __threadfence();
-  __syncthreads();
-  if (tid == 0) sTicket = static_cast<int>(atomicAdd(&a.counters[u], 1u));
-  __syncthreads();
-  if (sTicket != a.S - 1) return;
-  __threadfence();
-  if (tid == 0) a.counters[u] = 0u;
-
-  // combine the S partial records: stage them in shared memory with one round
-  // of loads when they fit in the (free) tile ring, else read them in place
-  const float* pu = a.partial + (size_t)u * a.S * G * PS;
   const size_t rec_floats = (size_t)a.S * G * PS;
-  const bool staged = rec_floats * 4 + (2 * a.S * G + G * D) * 4 <= (size_t)kStages * 2 * kTileBytes;
+  bool staged;
+  const float* src;
+  float* sF;  // [G][D] f_hat_E rows (or mu_v for order 0)
   float* sP = reinterpret_cast<float*>(dsmem);
-  const float* src = pu;
-  float* sF = sP;  // [G][D] f_hat_E rows (or mu_v for order 0)
-  if (staged) {
-    sF = sP + rec_floats;
-    for (size_t i = tid; i < rec_floats / 4; i += kThreads)
-      reinterpret_cast<float4*>(sP)[i] = __ldcg(reinterpret_cast<const float4*>(pu) + i);
-    if (use_m) {
+  if constexpr (CL) {
+    // ---- cluster barrier: every partial and f_hat_E row is in CTA 0
+    cluster_arrive_release();
+    cluster_wait_acquire();
+    if (s != 0) return;
+    staged = true;
+    src = sRcv;
+    sF = sFr;
+    if (use_m && a.order != 1)
       for (int i = tid; i < G * D / 4; i += kThreads)
-        reinterpret_cast<float4*>(sF)[i] =
-            (a.order == 1) ? __ldcg(reinterpret_cast<const float4*>(a.fhat + (size_t)u * G * D) + i)
-                           : __ldg(reinterpret_cast<const float4*>(a.mu_v + (size_t)u * D) + (i % (D / 4)));
+        reinterpret_cast<float4*>(sF)[i] = __ldg(reinterpret_cast<const float4*>(a.mu_v + (size_t)u * D) + (i % (D / 4)));
+  } else {
+    // ---- ticket: the last CTA of this unit merges everything
+    __threadfence();
+    __syncthreads();
+    if (tid == 0) sTicket = static_cast<int>(atomicAdd(&a.counters[u], 1u));
+    __syncthreads();
+    if (sTicket != a.S - 1) return;
+    __threadfence();
+    if (tid == 0) a.counters[u] = 0u;
+
+    // combine the S partial records: stage them in shared memory with one
+    // round of loads when they fit in the (free) tile ring, else read them
+    // in place
+    const float* pu = a.partial + (size_t)u * a.S * G * PS;
+    staged = rec_floats * 4 + (2 * a.S * G + G * D) * 4 <= (size_t)kStages * 2 * kTileBytes;
+    src = pu;
+    sF = sP;
+    if (staged) {
+      sF = sP + rec_floats;
+      for (size_t i = tid; i < rec_floats / 4; i += kThreads)
+        reinterpret_cast<float4*>(sP)[i] = __ldcg(reinterpret_cast<const float4*>(pu) + i);
+      if (use_m) {
+        for (int i = tid; i < G * D / 4; i += kThreads)
+          reinterpret_cast<float4*>(sF)[i] =
+              (a.order == 1) ? __ldcg(reinterpret_cast<const float4*>(a.fhat + (size_t)u * G * D) + i)
+                             : __ldg(reinterpret_cast<const float4*>(a.mu_v + (size_t)u * D) + (i % (D / 4)));
+      }
+      src = sP;
     }
-    src = sP;
   }
   float* sW = staged ? sF + G * D : sP;  // [S][G] max, then weight
   float* sLs = sW + a.S * G;             // [S][G] sums
@@ -487,22 +553,80 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
   }
 }
 
+// Whether clusters of S CTAs with `smem` bytes each can be resident (checked
+// once per split count; portable sizes always can).
+template <int D, int G>
+bool cluster_fits(int S, size_t smem) {
+  if (S <= 8) return true;
+  static std::mutex mu;
+  static signed char known[kMaxClusterSplits + 1] = {};
+  std::lock_guard<std::mutex> lock(mu);
+  if (known[S] == 0) {
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(S, 1, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = S;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    int n = 0;
+    const cudaError_t e = cudaOccupancyMaxActiveClusters(&n, decode_kernel<D, G, true>, &cfg);
+    if (e != cudaSuccess) (void)cudaGetLastError();
+    known[S] = (e == cudaSuccess && n > 0) ? 1 : -1;
+  }
+  return known[S] > 0;
+}
+
 template <int D, int G>
 cudaError_t launch_dg(const DecodeArgs& a, cudaStream_t stream) {
-  const size_t smem = (size_t)2 * kStages * kTT * D * 2 + 1024;  // + alignment slack
-  // per-device function attribute; setting it again is harmless
-  cudaError_t e = cudaFuncSetAttribute(decode_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(smem));
+  const size_t ring = (size_t)2 * kStages * kTT * D * 2 + 1024;  // + alignment slack
+  const size_t rcv = ((size_t)a.S * G * (D + 4) + (size_t)G * D + 2 * (size_t)a.S * G) * sizeof(float);
+  const bool cl = a.S <= kMaxClusterSplits;
+  const size_t smem = cl ? ring + rcv : ring;
+  // per-device function attributes; setting them again is harmless
+  cudaError_t e;
+  if (cl) {
+    e = cudaFuncSetAttribute(decode_kernel<D, G, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(smem));
+    if (e == cudaSuccess && a.S > 8)
+      e = cudaFuncSetAttribute(decode_kernel<D, G, true>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  } else {
+    e = cudaFuncSetAttribute(decode_kernel<D, G, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(smem));
+  }
   if (e != cudaSuccess) return e;
+  const bool use_cl = cl && cluster_fits<D, G>(a.S, smem);
   // the cache slabs of all units as one [units * cap][D] matrix
   const uint64_t rows = (uint64_t)a.batch * a.n_kv * a.cap;
   CUtensorMap tmK, tmV;
   if (!encode_tmap_bf16(&tmK, a.K, D, rows, (uint64_t)D * 2, 64, kTT) ||
       !encode_tmap_bf16(&tmV, a.V, D, rows, (uint64_t)D * 2, 64, kTT))
     return cudaErrorInvalidValue;
-  dim3 grid(a.S, a.n_kv, a.batch);
-  decode_kernel<D, G><<<grid, kThreads, smem, stream>>>(a, tmK, tmV);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(a.S, a.n_kv, a.batch);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = use_cl ? smem : ring;
+  cfg.stream = stream;
+  cudaLaunchAttribute at[2];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  at[1].id = cudaLaunchAttributeClusterDimension;
+  at[1].val.clusterDim.x = a.S;
+  at[1].val.clusterDim.y = 1;
+  at[1].val.clusterDim.z = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = use_cl ? 2 : 1;
+  if (use_cl) return cudaLaunchKernelEx(&cfg, decode_kernel<D, G, true>, a, tmK, tmV);
+  if (cl) {  // the cluster did not fit: the ticket variant with the ring only
+    e = cudaFuncSetAttribute(decode_kernel<D, G, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(ring));
+    if (e != cudaSuccess) return e;
+  }
+  return cudaLaunchKernelEx(&cfg, decode_kernel<D, G, false>, a, tmK, tmV);
 }
 
 }  // namespace

@@ -89,6 +89,14 @@ __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, i
       : "memory");
 }
 
+// Prefetch a box of a 3-D tensor into L2 (no shared memory, no completion).
+__device__ __forceinline__ void tma_prefetch_3d(const CUtensorMap* map, int x, int y, int z) {
+  asm volatile("cp.async.bulk.prefetch.tensor.3d.L2.global [%0, {%1, %2, %3}];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(x), "r"(y), "r"(z)
+               : "memory");
+}
+
 // Host: bf16 slabs [units][rows][inner] (unit stride in bytes) as a 3-D
 // tensor map with boxes of box_rows x 64 elements, 128-byte swizzle.  Rows
 // >= `rows` of a unit are outside the tensor and read as zeros.
