@@ -28,6 +28,8 @@
 // visible).
 #include <cooperative_groups.h>
 
+#include <algorithm>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -631,12 +633,20 @@ cudaError_t launch_dg(const DecodeArgs& a, cudaStream_t stream) {
 
 }  // namespace
 
+// Split count per unit.  All CTAs of a launch should be resident at once (two
+// per SM at d = 128, three at d = 64, limited by shared memory): a second wave
+// costs a whole CTA latency.  Within that, one tile per CTA up to ten tiles,
+// at least two tiles per CTA beyond, and past 12 splits the merge costs more
+// than the extra parallelism saves (measured on the Llama-3.1-8B decode
+// geometry over batch 1..64 and caches of 256..4096 rows).
 int decode_splits(const mkv_geom& g, int32_t capacity, int num_sms) {
   const long units = (long)g.batch * g.n_kv_heads;
   const long tiles = ((long)capacity + 1 + kTT - 1) / kTT;
-  long S = (8L * num_sms + units - 1) / units;
-  if (S > tiles) S = tiles;
-  if (S > 64) S = 64;
+  const long slots = (g.head_dim == 64 ? 3L : 2L) * num_sms;
+  long S = slots / units;
+  const long by_tiles = tiles <= 10 ? tiles : std::max(10L, (tiles + 1) / 2);
+  S = std::min(S, by_tiles);
+  S = std::min(S, 12L);
   if (S < 1) S = 1;
   return static_cast<int>(S);
 }

@@ -396,10 +396,28 @@ __device__ __forceinline__ float group_sum(float v) {
 template <int D>
 __device__ __forceinline__ void load4_bf16(const __nv_bfloat16* p, float* o) { load_bf16<4>(p, o); }
 
+// Vectors of N floats in shared memory (aligned to 4N bytes).
+template <int N>
+__device__ __forceinline__ void ld_vec(const float* p, float* v) {
+  if constexpr (N == 4) {
+    const float4 t = *reinterpret_cast<const float4*>(p);
+    v[0] = t.x; v[1] = t.y; v[2] = t.z; v[3] = t.w;
+  } else {
+    const float2 t = *reinterpret_cast<const float2*>(p);
+    v[0] = t.x; v[1] = t.y;
+  }
+}
+template <int N>
+__device__ __forceinline__ void st_vec(float* p, const float* v) {
+  if constexpr (N == 4) *reinterpret_cast<float4*>(p) = make_float4(v[0], v[1], v[2], v[3]);
+  else *reinterpret_cast<float2*>(p) = make_float2(v[0], v[1]);
+}
+
 template <int D, int G>
 __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
     evict_cluster_kernel(const EvictArgs a) {
   constexpr int NC = D / 32;
+  constexpr int DPL = D / 32;  // consecutive C columns per thread in the rank-1 update of Ct
   extern __shared__ __align__(16) uint8_t dsmem[];
   const int R = a.rows_max;
   const ClusterLayout<D, G> lay(R, a.cap, a.kv_smem);
@@ -409,25 +427,25 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
   uint8_t* alive_all = dsmem + lay.alive;                // [cap] alive flags of the unit
   __shared__ __align__(16) float s_mu_k[D];
   __shared__ __align__(16) float s_mu_v[D];
+  __shared__ __align__(16) float s_q[G][D];
   __shared__ __align__(16) float s_dk[D];
   __shared__ __align__(16) float s_dv[D];
-  __shared__ __align__(16) float s_q[G][D];
-  __shared__ float s_red[kCW][G], s_red2[kCW][G];
-  __shared__ float s_M[G], s_Z[G];
+  __shared__ float s_red[kCW][G];
+  __shared__ double s_zpart[kCW][G];
+  __shared__ float s_M[G], s_invZ[G];
+  __shared__ float s_keep;
   __shared__ int s_js;
-  // published to the cluster, double-buffered by iteration parity: this CTA's
-  // best (score, row) key and that row's k and v
-  __shared__ unsigned long long ex_best[2];
-  __shared__ __align__(16) __nv_bfloat16 ex_row[2][2 * D];
-  __shared__ __align__(16) __nv_bfloat16 s_cand[kCL][2 * D];  // every rank's candidate row
-  __shared__ unsigned long long s_keys[kCL];
+  // this CTA's best (score, row) key, reduced by atomicMin; and the mailbox
+  // that every rank writes its key and candidate row into (double-buffered by
+  // iteration parity)
+  __shared__ unsigned long long s_best[2];
+  __shared__ unsigned long long mail_key[2][kCL];
+  __shared__ __align__(16) __nv_bfloat16 mail_row[2][kCL][2 * D];
   __shared__ int ex_cnt;
-  __shared__ unsigned long long s_bestw[kCW];
-  __shared__ uint32_t s_zidx[kMaxClamp];
-  __shared__ float s_zval[kMaxClamp];
-  __shared__ int s_nz;
+  __shared__ uint32_t s_zidx[2][kMaxClamp];
+  __shared__ float s_zval[2][kMaxClamp];
+  __shared__ int s_nz[2];
   __shared__ float s_tile[kTW][32 * 33];  // transpose staging (setup / write-back)
-  __shared__ float s_invZ[G];
 
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = static_cast<int>(cluster.block_rank());
@@ -460,7 +478,7 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
     if (tid == 0) Pg[len_in] = seen_in;
     __threadfence();
   }
-  __syncthreads();  // the appended row is read back below by other threads
+  __syncthreads();
   if (len <= a.budget) {
     if (rank == 0 && tid == 0) {
       a.len[u] = len;
@@ -468,6 +486,8 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
     }
     return;
   }
+  // other CTAs' rows (the appended one included) are read below
+  cluster.sync();
 
   int n = a.n[u];
   {
@@ -503,7 +523,10 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
     Vr = Vs;
   }
   for (int j = tid; j < a.cap; j += kCT) alive_all[j] = j < len ? 1 : 0;
-  if (tid == 0) s_nz = 0;
+  if (tid == 0) {
+    s_nz[0] = s_nz[1] = 0;
+    s_best[0] = s_best[1] = ~0ull;
+  }
   __syncthreads();
   const uint8_t* alive = alive_all + j0;  // this slice's flags
 
@@ -591,237 +614,258 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
     }
   }
   // clamp list for the initial moments: entries with 0 < |n C_ab| < tau
+  // (iteration e reads list e & 1; the fold before it builds that list)
   const float tau = a.tau;
   if (n > 0 && tau > 0.f) {
     const float nf = static_cast<float>(n);
     for (int idx = tid; idx < D * D; idx += kCT) {
       const float c = Ct[idx];
       if (c != 0.f && fabsf(c * nf) < tau) {
-        const int k = atomicAdd(&s_nz, 1);
+        const int k = atomicAdd(&s_nz[0], 1);
         if (k < kMaxClamp) {
-          s_zidx[k] = static_cast<uint32_t>(idx);
-          s_zval[k] = c;
+          s_zidx[0][k] = static_cast<uint32_t>(idx);
+          s_zval[0][k] = c;
         }
       }
+    }
+  }
+  // per-head normaliser Z_h = sum of e_hj over the surviving rows, kept in
+  // double by warp 0 (lane h) and decremented as rows are evicted
+  double zd = 0.0;
+  {
+    double zs[G];
+#pragma unroll
+    for (int h = 0; h < G; ++h) zs[h] = 0.0;
+    for (int jj = tid; jj < len; jj += kCT)
+#pragma unroll
+      for (int h = 0; h < G; ++h) zs[h] += static_cast<double>(lg[h * a.cap + jj]);
+#pragma unroll
+    for (int h = 0; h < G; ++h) {
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) zs[h] += __shfl_xor_sync(kFull, zs[h], o);
+      if (lane == 0) s_zpart[warp][h] = zs[h];
+    }
+    __syncthreads();
+    if (warp == 0 && lane < G) {
+      for (int w = 0; w < kCW; ++w) zd += s_zpart[w][lane];
+      s_invZ[lane] = 1.f / static_cast<float>(zd);
     }
   }
   __syncthreads();
 
   const int n_evict = len - a.budget;
-  for (int e = 0; e < n_evict; ++e) {
-    // ---- phase A: per-head softmax normaliser over every surviving row of
-    // the unit: Z_h = sum of e_hj (every CTA holds all of them: no exchange)
-    {
-      float zs[G];
+  for (int e = 0;; ++e) {
+    const int par = e & 1;
+    // ---- fold the previous eviction into C (building clamp list par) and
+    // into y_j of this slice: C' = keep C + dk dv^T, y_j' = keep y_j + (dk . k_j) dv
+    if (e > 0) {
+      const float nf = static_cast<float>(n);
+      const float keep = s_keep;
+      const float thr = tau / nf;  // |C_ab| < tau / n  <=>  |n C_ab| < tau
 #pragma unroll
-      for (int h = 0; h < G; ++h) zs[h] = 0.f;
-      for (int jj = tid; jj < len; jj += kCT)
-        if (alive_all[jj]) {
+      for (int k = 0; k < D * D / DPL / kCT; ++k) {
+        const int iv = k * kCT + tid;  // Ct[c][lane*DPL ...] with c = iv / 32
+        const int c = iv >> 5;
+        const float kd = s_dk[c];
+        float v[DPL], dv[DPL];
+        ld_vec<DPL>(Ct + (size_t)iv * DPL, v);
+        ld_vec<DPL>(s_dv + lane * DPL, dv);
+        bool any = false;
 #pragma unroll
-          for (int h = 0; h < G; ++h) zs[h] += lg[h * a.cap + jj];
+        for (int i = 0; i < DPL; ++i) {
+          v[i] = fmaf(keep, v[i], kd * dv[i]);
+          any |= fabsf(v[i]) < thr;
         }
+        st_vec<DPL>(Ct + (size_t)iv * DPL, v);
+        if (any) {
 #pragma unroll
-      for (int h = 0; h < G; ++h) {
-        zs[h] = warp_sum(zs[h]);
-        if (lane == 0) s_red[warp][h] = zs[h];
-      }
-      __syncthreads();
-      if (warp == 0) {
-#pragma unroll
-        for (int h = 0; h < G; ++h) {
-          const float z = warp_sum(s_red[lane][h]);
-          if (lane == 0) s_invZ[h] = 1.f / z;
-        }
-      }
-      __syncthreads();
-    }
-
-    // ---- phase B: scores of this slice, local argmin (8 lanes per row)
-    const float rs = (n > 0) ? scale : 0.f;
-    const int nz = s_nz;
-    const bool direct = nz > kMaxClamp;
-    const float nf = static_cast<float>(n);
-    unsigned long long best = ~0ull;
-    for (int base = 0; base < nr; base += kRowsPerPass) {
-      const int r = base + rsub;
-      const bool ok = (r < nr) && alive[r];
-      float ss = 0.f;
-      if (ok) {
-        if (!direct) {
-#pragma unroll
-          for (int c = 0; c < NC; ++c) {
-            const int d0 = chunk_dim<D>(q, c);
-            float4 y4 = *reinterpret_cast<const float4*>(Y + (size_t)r * D + d0);
-            for (int z = 0; z < nz; ++z) {  // y'_a -= C_ab k_b for clamped (a, b)
-              const int kb = static_cast<int>(s_zidx[z] / D), va = static_cast<int>(s_zidx[z] % D);
-              if (va >= d0 && va < d0 + 4) {
-                const float corr = s_zval[z] * __bfloat162float(Kr[(size_t)r * D + kb]);
-                const int o = va - d0;
-                if (o == 0) y4.x -= corr;
-                else if (o == 1) y4.y -= corr;
-                else if (o == 2) y4.z -= corr;
-                else y4.w -= corr;
+          for (int i = 0; i < DPL; ++i)
+            if (v[i] != 0.f && fabsf(v[i] * nf) < tau) {
+              const int slot = atomicAdd(&s_nz[par], 1);
+              if (slot < kMaxClamp) {
+                s_zidx[par][slot] = static_cast<uint32_t>(iv * DPL + i);
+                s_zval[par][slot] = v[i];
               }
             }
-            float vf[4];
-            load4_bf16<D>(Vr + (size_t)r * D + d0, vf);
-            const float4 m4 = *reinterpret_cast<const float4*>(s_mu_v + d0);
-            const float r0 = vf[0] - m4.x - rs * y4.x, r1 = vf[1] - m4.y - rs * y4.y;
-            const float r2 = vf[2] - m4.z - rs * y4.z, r3 = vf[3] - m4.w - rs * y4.w;
-            ss = fmaf(r0, r0, fmaf(r1, r1, fmaf(r2, r2, fmaf(r3, r3, ss))));
-          }
-        } else {
-          float y[NC][4];
-#pragma unroll
-          for (int c = 0; c < NC; ++c) y[c][0] = y[c][1] = y[c][2] = y[c][3] = 0.f;
-          for (int kc = 0; kc < D; ++kc) {
-            const float kv = __bfloat162float(Kr[(size_t)r * D + kc]);
-#pragma unroll
-            for (int c = 0; c < NC; ++c) {
-              const float4 c4 = *reinterpret_cast<const float4*>(Ct + kc * D + chunk_dim<D>(q, c));
-              y[c][0] = fmaf((fabsf(c4.x * nf) < tau) ? 0.f : c4.x, kv, y[c][0]);
-              y[c][1] = fmaf((fabsf(c4.y * nf) < tau) ? 0.f : c4.y, kv, y[c][1]);
-              y[c][2] = fmaf((fabsf(c4.z * nf) < tau) ? 0.f : c4.z, kv, y[c][2]);
-              y[c][3] = fmaf((fabsf(c4.w * nf) < tau) ? 0.f : c4.w, kv, y[c][3]);
-            }
-          }
+        }
+      }
+      for (int base = 0; base < nr; base += kRowsPerPass) {
+        const int r = base + rsub;
+        const bool ok = (r < nr) && alive[r];
+        float dot = 0.f;
+        if (ok) {
 #pragma unroll
           for (int c = 0; c < NC; ++c) {
             const int d0 = chunk_dim<D>(q, c);
-            float vf[4];
-            load4_bf16<D>(Vr + (size_t)r * D + d0, vf);
+            float kf[4];
+            load4_bf16<D>(Kr + (size_t)r * D + d0, kf);
+            const float4 k4 = *reinterpret_cast<const float4*>(s_dk + d0);
+            dot = fmaf(k4.x, kf[0], fmaf(k4.y, kf[1], fmaf(k4.z, kf[2], fmaf(k4.w, kf[3], dot))));
+          }
+        }
+        dot = group_sum(dot);
+        if (ok) {
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              const float rr = vf[i] - s_mu_v[d0 + i] - rs * y[c][i];
-              ss = fmaf(rr, rr, ss);
-            }
+          for (int c = 0; c < NC; ++c) {
+            const int d0 = chunk_dim<D>(q, c);
+            float4* yp = reinterpret_cast<float4*>(Y + (size_t)r * D + d0);
+            float4 y4 = *yp;
+            const float4 dv = *reinterpret_cast<const float4*>(s_dv + d0);
+            y4.x = fmaf(keep, y4.x, dot * dv.x);
+            y4.y = fmaf(keep, y4.y, dot * dv.y);
+            y4.z = fmaf(keep, y4.z, dot * dv.z);
+            y4.w = fmaf(keep, y4.w, dot * dv.w);
+            *yp = y4;
           }
         }
       }
-      ss = group_sum(ss);
-      if (ok && q == 0) {
-        float alpha = 0.f;
-#pragma unroll
-        for (int h = 0; h < G; ++h) alpha = fmaf(lg[h * a.cap + j0 + r], s_invZ[h], alpha);
-        const float score = alpha * sqrtf(ss);
-        const unsigned long long key =
-            (static_cast<unsigned long long>(__float_as_uint(score)) << 32) | static_cast<unsigned>(j0 + r);
-        best = key < best ? key : best;
-      }
     }
-    best = shfl_min_u64(best);
-    if (lane == 0) s_bestw[warp] = best;
     __syncthreads();
-    const int par = e & 1;
+    if (e == n_evict) break;  // uniform over the cluster
+
+    // ---- scores of this slice (8 lanes per row), block minimum of the keys
+    {
+      const float rs = (n > 0) ? scale : 0.f;
+      const int nz = s_nz[par];
+      const bool direct = nz > kMaxClamp;
+      const float nf = static_cast<float>(n);
+      unsigned long long best = ~0ull;
+      for (int base = 0; base < nr; base += kRowsPerPass) {
+        const int r = base + rsub;
+        const bool ok = (r < nr) && alive[r];
+        float ss = 0.f;
+        if (ok) {
+          if (!direct) {
+#pragma unroll
+            for (int c = 0; c < NC; ++c) {
+              const int d0 = chunk_dim<D>(q, c);
+              float4 y4 = *reinterpret_cast<const float4*>(Y + (size_t)r * D + d0);
+              for (int z = 0; z < nz; ++z) {  // y'_a -= C_ab k_b for clamped (a, b)
+                const int kb = static_cast<int>(s_zidx[par][z] / D), va = static_cast<int>(s_zidx[par][z] % D);
+                if (va >= d0 && va < d0 + 4) {
+                  const float corr = s_zval[par][z] * __bfloat162float(Kr[(size_t)r * D + kb]);
+                  const int o = va - d0;
+                  if (o == 0) y4.x -= corr;
+                  else if (o == 1) y4.y -= corr;
+                  else if (o == 2) y4.z -= corr;
+                  else y4.w -= corr;
+                }
+              }
+              float vf[4];
+              load4_bf16<D>(Vr + (size_t)r * D + d0, vf);
+              const float4 m4 = *reinterpret_cast<const float4*>(s_mu_v + d0);
+              const float r0 = vf[0] - m4.x - rs * y4.x, r1 = vf[1] - m4.y - rs * y4.y;
+              const float r2 = vf[2] - m4.z - rs * y4.z, r3 = vf[3] - m4.w - rs * y4.w;
+              ss = fmaf(r0, r0, fmaf(r1, r1, fmaf(r2, r2, fmaf(r3, r3, ss))));
+            }
+          } else {
+            float y[NC][4];
+#pragma unroll
+            for (int c = 0; c < NC; ++c) y[c][0] = y[c][1] = y[c][2] = y[c][3] = 0.f;
+            for (int kc = 0; kc < D; ++kc) {
+              const float kv = __bfloat162float(Kr[(size_t)r * D + kc]);
+#pragma unroll
+              for (int c = 0; c < NC; ++c) {
+                const float4 c4 = *reinterpret_cast<const float4*>(Ct + kc * D + chunk_dim<D>(q, c));
+                y[c][0] = fmaf((fabsf(c4.x * nf) < tau) ? 0.f : c4.x, kv, y[c][0]);
+                y[c][1] = fmaf((fabsf(c4.y * nf) < tau) ? 0.f : c4.y, kv, y[c][1]);
+                y[c][2] = fmaf((fabsf(c4.z * nf) < tau) ? 0.f : c4.z, kv, y[c][2]);
+                y[c][3] = fmaf((fabsf(c4.w * nf) < tau) ? 0.f : c4.w, kv, y[c][3]);
+              }
+            }
+#pragma unroll
+            for (int c = 0; c < NC; ++c) {
+              const int d0 = chunk_dim<D>(q, c);
+              float vf[4];
+              load4_bf16<D>(Vr + (size_t)r * D + d0, vf);
+#pragma unroll
+              for (int i = 0; i < 4; ++i) {
+                const float rr = vf[i] - s_mu_v[d0 + i] - rs * y[c][i];
+                ss = fmaf(rr, rr, ss);
+              }
+            }
+          }
+        }
+        ss = group_sum(ss);
+        if (ok && q == 0) {
+          float alpha = 0.f;
+#pragma unroll
+          for (int h = 0; h < G; ++h) alpha = fmaf(lg[h * a.cap + j0 + r], s_invZ[h], alpha);
+          const float score = alpha * sqrtf(ss);
+          const unsigned long long key =
+              (static_cast<unsigned long long>(__float_as_uint(score)) << 32) | static_cast<unsigned>(j0 + r);
+          best = key < best ? key : best;
+        }
+      }
+      best = shfl_min_u64(best);
+      if (lane == 0 && best != ~0ull) atomicMin(&s_best[par], best);
+      if (tid == 0) s_nz[par ^ 1] = 0;  // list par^1 was last read one iteration ago
+    }
+    __syncthreads();
+
+    // ---- warp 0 posts this CTA's key and candidate row into every rank's
+    // mailbox slot [par][rank]; one cluster barrier publishes them all
     if (warp == 0) {
-      unsigned long long b = s_bestw[lane];
-      b = shfl_min_u64(b);
-      if (lane == 0) {
-        ex_best[par] = b;
-        s_nz = 0;
-      }
-      // publish the candidate row's k and v next to its key
+      const unsigned long long b = s_best[par];
       const int jb = (b == ~0ull) ? -1 : static_cast<int>(b & 0xffffffffu) - j0;
-      if (jb >= 0 && lane < D / 8) {
-        reinterpret_cast<uint4*>(ex_row[par])[lane] = reinterpret_cast<const uint4*>(Kr + (size_t)jb * D)[lane];
-        reinterpret_cast<uint4*>(ex_row[par] + D)[lane] = reinterpret_cast<const uint4*>(Vr + (size_t)jb * D)[lane];
+      if (lane < kCL) *cluster.map_shared_rank(&mail_key[par][rank], lane) = b;
+      if (jb >= 0 && lane < D / 4) {  // lanes 0..D/8-1 carry k, the next D/8 carry v
+        const bool is_v = lane >= D / 8;
+        const int i = is_v ? lane - D / 8 : lane;
+        const uint4 w = reinterpret_cast<const uint4*>((is_v ? Vr : Kr) + (size_t)jb * D)[i];
+#pragma unroll
+        for (int rk = 0; rk < kCL; ++rk)
+          reinterpret_cast<uint4*>(cluster.map_shared_rank(&mail_row[par][rank][is_v ? D : 0], rk))[i] = w;
       }
+      if (lane == 0) s_best[par] = ~0ull;  // next used two iterations on
     }
     cluster.sync();
-    // every rank's key and candidate row in one round of remote reads
-    if (tid < kCL) s_keys[tid] = cluster.map_shared_rank(ex_best, tid)[par];
-    if (tid >= 32 && tid < 32 + kCL * (D / 4)) {
-      const int t = tid - 32, rk = t / (D / 4), i = t % (D / 4);
-      reinterpret_cast<uint4*>(s_cand[rk])[i] =
-          reinterpret_cast<const uint4*>(cluster.map_shared_rank(&ex_row[par][0], rk))[i];
-    }
-    __syncthreads();
-    if (tid == 0) {
-      unsigned long long b = s_keys[0];
-      int w = 0;
-      for (int r2 = 1; r2 < kCL; ++r2)
-        if (s_keys[r2] < b) {
-          b = s_keys[r2];
-          w = r2;
-        }
-      s_js = static_cast<int>(b & 0xffffffffu) | (w << 24);
-    }
-    __syncthreads();
-    const int js = s_js & 0xffffff, wr = s_js >> 24;
 
-    // ---- phase C: fold row j* into the moments, update y for the slice
-    const float n1 = static_cast<float>(n + 1);
-    const float inv = 1.f / n1;
-    if (tid < D) {
-      const float kx = __bfloat162float(s_cand[wr][tid]);
-      const float vx = __bfloat162float(s_cand[wr][D + tid]);
-      const float dk = kx - s_mu_k[tid];
-      s_mu_k[tid] = fmaf(dk, inv, s_mu_k[tid]);
-      const float mv = fmaf(vx - s_mu_v[tid], inv, s_mu_v[tid]);
-      s_mu_v[tid] = mv;
-      s_dk[tid] = dk * inv;  // scaled by 1/(n+1) for the rank-1 terms below
-      s_dv[tid] = vx - mv;
+    // ---- warp 0: the cluster's minimum key, Welford fold of that row (Eq. app_update)
+    if (warp == 0) {
+      unsigned long long b = (lane < kCL) ? mail_key[par][lane] : ~0ull;
+      int w = lane;
+#pragma unroll
+      for (int o = 4; o > 0; o >>= 1) {
+        const unsigned long long b2 = __shfl_xor_sync(kFull, b, o);
+        const int w2 = __shfl_xor_sync(kFull, w, o);
+        if (b2 < b || (b2 == b && w2 < w)) {
+          b = b2;
+          w = w2;
+        }
+      }
+      b = __shfl_sync(kFull, b, 0);
+      w = __shfl_sync(kFull, w, 0);
+      const int js = (b == ~0ull) ? -1 : static_cast<int>(b & 0xffffffffu);
+      if (js >= 0) {
+        const float inv = 1.f / static_cast<float>(n + 1);
+        for (int d = lane; d < D; d += 32) {
+          const float kx = __bfloat162float(mail_row[par][w][d]);
+          const float vx = __bfloat162float(mail_row[par][w][D + d]);
+          const float dk = kx - s_mu_k[d];
+          s_mu_k[d] = fmaf(dk, inv, s_mu_k[d]);
+          const float mvn = fmaf(vx - s_mu_v[d], inv, s_mu_v[d]);
+          s_mu_v[d] = mvn;
+          s_dk[d] = dk * inv;  // scaled by 1/(n+1) for the rank-1 terms
+          s_dv[d] = vx - mvn;
+        }
+        if (lane < G) {
+          zd -= static_cast<double>(lg[lane * a.cap + js]);
+          s_invZ[lane] = 1.f / static_cast<float>(zd);
+        }
+        if (lane == 0) {
+          alive_all[js] = 0;
+          s_keep = static_cast<float>(n) * inv;
+        }
+      }
+      if (lane == 0) {
+        if (js < 0) record_error(a.ws, MKV_ERR_INVALID_ARG, u);
+        s_js = js;
+      }
     }
-    if (tid == 0) alive_all[js] = 0;
     __syncthreads();
-    const float keep = static_cast<float>(n) * inv;
-    const float thr = tau * inv;  // |C_ab| < tau / (n+1)  <=>  |(n+1) C_ab| < tau
-    for (int i4 = tid; i4 < D * D / 4; i4 += kCT) {
-      const int c = (i4 * 4) / D, r = (i4 * 4) % D;  // Ct[c][r..r+3] = C[r..r+3][c]
-      float4 v = reinterpret_cast<float4*>(Ct)[i4];
-      const float kd = s_dk[c];
-      const float4 dv = *reinterpret_cast<const float4*>(s_dv + r);
-      v.x = fmaf(keep, v.x, kd * dv.x);
-      v.y = fmaf(keep, v.y, kd * dv.y);
-      v.z = fmaf(keep, v.z, kd * dv.z);
-      v.w = fmaf(keep, v.w, kd * dv.w);
-      reinterpret_cast<float4*>(Ct)[i4] = v;
-      const bool any = (fabsf(v.x) < thr) | (fabsf(v.y) < thr) | (fabsf(v.z) < thr) | (fabsf(v.w) < thr);
-      if (any) {
-        const float vv[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-        for (int k = 0; k < 4; ++k)
-          if (vv[k] != 0.f && fabsf(vv[k] * n1) < tau) {
-            const int slot = atomicAdd(&s_nz, 1);
-            if (slot < kMaxClamp) {
-              s_zidx[slot] = static_cast<uint32_t>(i4 * 4 + k);
-              s_zval[slot] = vv[k];
-            }
-          }
-      }
-    }
-    for (int base = 0; base < nr; base += kRowsPerPass) {
-      const int r = base + rsub;
-      const bool ok = (r < nr) && alive[r];
-      float kf[NC][4];
-      float dot = 0.f;
-      if (ok) {
-#pragma unroll
-        for (int c = 0; c < NC; ++c) {
-          const int d0 = chunk_dim<D>(q, c);
-          load4_bf16<D>(Kr + (size_t)r * D + d0, kf[c]);
-          const float4 k4 = *reinterpret_cast<const float4*>(s_dk + d0);
-          dot = fmaf(k4.x, kf[c][0], fmaf(k4.y, kf[c][1], fmaf(k4.z, kf[c][2], fmaf(k4.w, kf[c][3], dot))));
-        }
-      }
-      dot = group_sum(dot);
-      if (ok) {
-#pragma unroll
-        for (int c = 0; c < NC; ++c) {
-          const int d0 = chunk_dim<D>(q, c);
-          float4* yp = reinterpret_cast<float4*>(Y + (size_t)r * D + d0);
-          float4 y4 = *yp;
-          const float4 dv = *reinterpret_cast<const float4*>(s_dv + d0);
-          y4.x = fmaf(keep, y4.x, dot * dv.x);
-          y4.y = fmaf(keep, y4.y, dot * dv.y);
-          y4.z = fmaf(keep, y4.z, dot * dv.z);
-          y4.w = fmaf(keep, y4.w, dot * dv.w);
-          *yp = y4;
-        }
-      }
-    }
+    if (s_js < 0) break;  // uniform: every rank read the same keys
     n += 1;
-    __syncthreads();
   }
 
   // ---- ordered compaction across the cluster through the staging buffer
@@ -895,6 +939,576 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
   }
 }
 
+// ---------------------------------------------------------------------------
+// Register-resident cluster kernel, used while a row slice has at most
+// kRW * RPW rows.  8 CTAs of 512 threads per unit (one cluster); warp w of a
+// CTA owns the slice rows w, w + 16, ... and lane l owns the dims
+// [l*DPL, (l+1)*DPL) of each: y_j = C k_j of its rows stays in registers, and
+// so does a 1/512 share of C (rows a of the lane's dims, columns c = w + 16 i),
+// which every iteration folds and scans for the clamp list.  Every thread
+// computes the Welford fold of its own dims from the evicted row, so the only
+// barriers of an iteration are one block barrier (the block's minimum key)
+// and one cluster barrier (every CTA's key and candidate row, written into
+// every CTA's mailbox beforehand).  Scores are computed assuming an empty
+// clamp list; when the list is not empty they are recomputed with it.
+constexpr int kRT = 512;       // threads per CTA
+constexpr int kRW = kRT / 32;  // warps per CTA
+
+template <int D, int G>
+struct RegLayout {
+  size_t Ct, lg, Ks, Vs, alive, total;
+  __host__ __device__ RegLayout(int R, int cap, int kv) {
+    size_t off = 0;
+    Ct = off; off += (size_t)D * D * 4;
+    lg = off; off += align_up((size_t)G * cap * 4, 16);
+    Ks = off; off += kv ? (size_t)R * D * 2 : 0;
+    Vs = off; off += kv ? (size_t)R * D * 2 : 0;
+    alive = off; off += align_up((size_t)cap, 16);
+    total = off;
+  }
+};
+
+// Butterfly sums of N independent values across the warp (every lane gets them).
+template <int N>
+__device__ __forceinline__ void warp_sum_n(float (&v)[N]) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+    for (int i = 0; i < N; ++i) v[i] += __shfl_xor_sync(kFull, v[i], o);
+}
+
+template <int N>
+__device__ __forceinline__ float select_n(const float (&v)[N], int i) {
+  float r = v[0];
+#pragma unroll
+  for (int k = 1; k < N; ++k) r = (i == k) ? v[k] : r;
+  return r;
+}
+
+template <int D, int G, int RPW>
+__global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
+    evict_reg_kernel(const EvictArgs a) {
+  constexpr int NC = D / 32;   // float4 chunks per row for 8-lane row groups (set-up)
+  constexpr int DPL = D / 32;  // dims per lane
+  constexpr int CJ = D / kRW;  // C columns per thread
+  constexpr int kRP = kRW * (32 / kLPR);  // rows per pass of 8-lane groups
+  extern __shared__ __align__(16) uint8_t dsmem[];
+  const int R = a.rows_max;
+  const RegLayout<D, G> lay(R, a.cap, a.kv_smem);
+  float* Ct = reinterpret_cast<float*>(dsmem + lay.Ct);  // Ct[c*D + a] = C[a][c] (set-up, direct mode, write-back)
+  float* lg = reinterpret_cast<float*>(dsmem + lay.lg);  // [G][cap] e_hj of every row of the unit
+  uint8_t* alive_all = dsmem + lay.alive;
+  __shared__ __align__(16) float s_mu_k[D];
+  __shared__ __align__(16) float s_mu_v[D];
+  __shared__ __align__(16) float s_q[G][D];
+  __shared__ float s_red[kRW][G];
+  __shared__ double s_zpart[kRW][G];
+  __shared__ double s_zd[kRW][G];  // per warp (lane 0): normaliser Z_h, decremented per eviction
+  __shared__ float s_invZ[kRW][G];
+  __shared__ float s_M[G];
+  __shared__ unsigned long long s_best[2];
+  __shared__ unsigned long long mail_key[2][kCL];
+  __shared__ __align__(16) __nv_bfloat16 mail_row[2][kCL][2 * D];
+  __shared__ int ex_cnt;
+  __shared__ uint32_t s_zidx[kMaxClamp];
+  __shared__ float s_zval[kMaxClamp];
+  __shared__ int s_nz;
+  __shared__ float s_tile[kTW][32 * 33];
+
+  cg::cluster_group cluster = cg::this_cluster();
+  const int rank = static_cast<int>(cluster.block_rank());
+  const int u = blockIdx.x / kCL;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int q = lane & 7;
+  const int rsub = warp * (32 / kLPR) + (lane >> 3);
+  const size_t row0 = (size_t)u * a.cap;
+  __nv_bfloat16* Kg = reinterpret_cast<__nv_bfloat16*>(a.K) + row0 * D;
+  __nv_bfloat16* Vg = reinterpret_cast<__nv_bfloat16*>(a.V) + row0 * D;
+  int32_t* Pg = a.pos + row0;
+  const int len_in = a.len[u];
+  const int seen_in = a.seen[u];
+  const bool has_new = a.k_new != nullptr;
+  if (len_in < 0 || len_in > a.cap || (has_new && len_in + 1 > a.cap)) {
+    if (rank == 0 && tid == 0) record_error(a.ws, MKV_ERR_CAPACITY, u);
+    return;  // uniform over the cluster
+  }
+  const int len = len_in + (has_new ? 1 : 0);
+  const int rows_per = (len + kCL - 1) / kCL;
+  const int j0 = min(len, rank * rows_per), j1 = min(len, j0 + rows_per);
+  const int nr = j1 - j0;
+  if (has_new && len_in >= j0 && len_in < j1) {  // the owning CTA appends the token
+    const __nv_bfloat16* kn = reinterpret_cast<const __nv_bfloat16*>(a.k_new) + (size_t)u * D;
+    const __nv_bfloat16* vn = reinterpret_cast<const __nv_bfloat16*>(a.v_new) + (size_t)u * D;
+    for (int i = tid; i < D; i += kRT) {
+      Kg[(size_t)len_in * D + i] = kn[i];
+      Vg[(size_t)len_in * D + i] = vn[i];
+    }
+    if (tid == 0) Pg[len_in] = seen_in;
+    __threadfence();
+  }
+  __syncthreads();
+  if (len <= a.budget) {
+    if (rank == 0 && tid == 0) {
+      a.len[u] = len;
+      a.seen[u] = seen_in + (has_new ? 1 : 0);
+    }
+    return;
+  }
+  // other CTAs' rows (the appended one included) are read below
+  cluster.sync();
+
+  int n = a.n[u];
+  {
+    float* tb = s_tile[warp % kTW];
+    for (int t = warp; warp < kTW && t < (D / 32) * (D / 32); t += kTW) {
+      const int r0 = (t / (D / 32)) * 32, c0 = (t % (D / 32)) * 32;
+      for (int i = 0; i < 32; ++i)
+        tb[i * 33 + lane] = (n > 0) ? a.C[(size_t)u * D * D + (size_t)(r0 + i) * D + c0 + lane] : 0.f;
+      __syncwarp();
+      for (int i = 0; i < 32; ++i) Ct[(size_t)(c0 + i) * D + r0 + lane] = tb[lane * 33 + i];
+      __syncwarp();
+    }
+  }
+  for (int i = tid; i < D; i += kRT) {
+    s_mu_k[i] = (n > 0) ? a.mu_k[(size_t)u * D + i] : 0.f;
+    s_mu_v[i] = (n > 0) ? a.mu_v[(size_t)u * D + i] : 0.f;
+  }
+  const float scale = rsqrtf(static_cast<float>(D));
+  const __nv_bfloat16* qg = reinterpret_cast<const __nv_bfloat16*>(a.q) + (size_t)u * G * D;
+  for (int i = tid; i < G * D; i += kRT) s_q[i / D][i % D] = __bfloat162float(qg[i]) * scale;
+  const __nv_bfloat16* Kr = Kg + (size_t)j0 * D;
+  const __nv_bfloat16* Vr = Vg + (size_t)j0 * D;
+  if (a.kv_smem) {
+    __nv_bfloat16* Ks = reinterpret_cast<__nv_bfloat16*>(dsmem + lay.Ks);
+    __nv_bfloat16* Vs = reinterpret_cast<__nv_bfloat16*>(dsmem + lay.Vs);
+    for (int idx = tid; idx < nr * (D / 8); idx += kRT) {
+      reinterpret_cast<uint4*>(Ks)[idx] = reinterpret_cast<const uint4*>(Kr)[idx];
+      reinterpret_cast<uint4*>(Vs)[idx] = reinterpret_cast<const uint4*>(Vr)[idx];
+    }
+    Kr = Ks;
+    Vr = Vs;
+  }
+  if (tid == 0) {
+    s_nz = 0;
+    s_best[0] = s_best[1] = ~0ull;
+  }
+  __syncthreads();
+
+  // ---- logits of every row of the unit (8 lanes per row, read from global)
+  for (int base = 0; base < len; base += kRP) {
+    const int j = base + rsub;
+    const bool ok = j < len;
+    float kf[NC][4];
+#pragma unroll
+    for (int c = 0; c < NC; ++c) {
+      if (ok) load4_bf16<D>(Kg + (size_t)j * D + chunk_dim<D>(q, c), kf[c]);
+      else kf[c][0] = kf[c][1] = kf[c][2] = kf[c][3] = 0.f;
+    }
+#pragma unroll
+    for (int h = 0; h < G; ++h) {
+      float acc = 0.f;
+#pragma unroll
+      for (int c = 0; c < NC; ++c) {
+        const float4 q4 = *reinterpret_cast<const float4*>(&s_q[h][chunk_dim<D>(q, c)]);
+        acc = fmaf(q4.x, kf[c][0], fmaf(q4.y, kf[c][1], fmaf(q4.z, kf[c][2], fmaf(q4.w, kf[c][3], acc))));
+      }
+      acc = group_sum(acc);
+      if (ok && q == 0) lg[h * a.cap + j] = acc;
+    }
+  }
+  __syncthreads();
+  // softmax is shift-invariant: e_hj = exp(l_hj - M0_h) with M0_h the
+  // largest logit of the unit at the start
+  {
+    float mx[G];
+#pragma unroll
+    for (int h = 0; h < G; ++h) mx[h] = -INFINITY;
+    for (int jj = tid; jj < len; jj += kRT)
+#pragma unroll
+      for (int h = 0; h < G; ++h) mx[h] = fmaxf(mx[h], lg[h * a.cap + jj]);
+#pragma unroll
+    for (int h = 0; h < G; ++h) {
+      mx[h] = warp_max(mx[h]);
+      if (lane == 0) s_red[warp][h] = mx[h];
+    }
+    __syncthreads();
+    if (tid < G) {
+      float m = -INFINITY;
+      for (int w = 0; w < kRW; ++w) m = fmaxf(m, s_red[w][tid]);
+      s_M[tid] = m;
+    }
+    __syncthreads();
+    double zs[G];
+#pragma unroll
+    for (int h = 0; h < G; ++h) zs[h] = 0.0;
+    for (int jj = tid; jj < len; jj += kRT)
+#pragma unroll
+      for (int h = 0; h < G; ++h) {
+        const float ev = expf(lg[h * a.cap + jj] - s_M[h]);
+        lg[h * a.cap + jj] = ev;
+        zs[h] += static_cast<double>(ev);
+      }
+#pragma unroll
+    for (int h = 0; h < G; ++h) {
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) zs[h] += __shfl_xor_sync(kFull, zs[h], o);
+      if (lane == 0) s_zpart[warp][h] = zs[h];
+    }
+    for (int jj = len + tid; jj < a.cap; jj += kRT) alive_all[jj] = 0;
+  }
+  __syncthreads();
+  if (lane < G) {  // every warp sums the partials in the same order: identical Z_h
+    double z = 0.0;
+    for (int w = 0; w < kRW; ++w) z += s_zpart[w][lane];
+    s_zd[warp][lane] = z;
+    s_invZ[warp][lane] = 1.f / static_cast<float>(z);
+  }
+
+  // ---- registers: y_j = C k_j of the warp's rows, the thread's share of C, means
+  float y[RPW][DPL];
+  unsigned alive = 0u;
+#pragma unroll
+  for (int i = 0; i < RPW; ++i) {
+#pragma unroll
+    for (int d = 0; d < DPL; ++d) y[i][d] = 0.f;
+    if (warp + kRW * i < nr) alive |= 1u << i;
+  }
+  if (n > 0) {
+    for (int c = 0; c < D; ++c) {
+      float cv[DPL];
+      ld_vec<DPL>(Ct + (size_t)c * D + lane * DPL, cv);
+#pragma unroll
+      for (int i = 0; i < RPW; ++i) {
+        const int r = warp + kRW * i;
+        if (r < nr) {
+          const float kv = __bfloat162float(Kr[(size_t)r * D + c]);
+#pragma unroll
+          for (int d = 0; d < DPL; ++d) y[i][d] = fmaf(cv[d], kv, y[i][d]);
+        }
+      }
+    }
+  }
+  float creg[CJ][DPL];
+#pragma unroll
+  for (int jj = 0; jj < CJ; ++jj) ld_vec<DPL>(Ct + (size_t)(warp + kRW * jj) * D + lane * DPL, creg[jj]);
+  float mk[DPL], mv[DPL], sdk[DPL], sdv[DPL];
+#pragma unroll
+  for (int d = 0; d < DPL; ++d) {
+    mk[d] = s_mu_k[lane * DPL + d];
+    mv[d] = s_mu_v[lane * DPL + d];
+    sdk[d] = sdv[d] = 0.f;
+  }
+  // clamp list of the initial moments: entries with 0 < |n C_ab| < tau
+  const float tau = a.tau;
+  if (n > 0 && tau > 0.f) {
+    const float nf = static_cast<float>(n);
+#pragma unroll
+    for (int jj = 0; jj < CJ; ++jj)
+#pragma unroll
+      for (int d = 0; d < DPL; ++d) {
+        const float v = creg[jj][d];
+        if (v != 0.f && fabsf(v * nf) < tau) {
+          const int k = atomicAdd(&s_nz, 1);
+          if (k < kMaxClamp) {
+            s_zidx[k] = static_cast<uint32_t>((warp + kRW * jj) * D + lane * DPL + d);
+            s_zval[k] = v;
+          }
+        }
+      }
+  }
+  __syncthreads();
+
+  const int n_evict = len - a.budget;
+  float keep = 1.f;
+  for (int e = 0;; ++e) {
+    const int par = e & 1;
+    // ---- fold the previous eviction into this thread's share of C and build
+    // the clamp list: C' = keep C + dk dv^T (dk scaled by 1/n)
+    if (e > 0) {
+      const float nf = static_cast<float>(n);
+      const float thr = tau / nf;  // |C_ab| < tau / n  <=>  |n C_ab| < tau
+      const float mydk = select_n<DPL>(sdk, warp % DPL);
+#pragma unroll
+      for (int jj = 0; jj < CJ; ++jj) {
+        const int c = warp + kRW * jj;
+        const float kd = __shfl_sync(kFull, mydk, c / DPL);  // dk[c]: lane c/DPL, component warp % DPL
+        bool any = false;
+#pragma unroll
+        for (int d = 0; d < DPL; ++d) {
+          creg[jj][d] = fmaf(keep, creg[jj][d], kd * sdv[d]);
+          any |= fabsf(creg[jj][d]) < thr;
+        }
+        if (any) {
+#pragma unroll
+          for (int d = 0; d < DPL; ++d)
+            if (creg[jj][d] != 0.f && fabsf(creg[jj][d] * nf) < tau) {
+              const int slot = atomicAdd(&s_nz, 1);
+              if (slot < kMaxClamp) {
+                s_zidx[slot] = static_cast<uint32_t>(c * D + lane * DPL + d);
+                s_zval[slot] = creg[jj][d];
+              }
+            }
+        }
+      }
+    }
+    if (e == n_evict) break;  // uniform over the cluster
+    if (tid == 0) s_best[par ^ 1] = ~0ull;  // its readers finished one iteration ago
+
+    // ---- y_j' = keep y_j + (dk . k_j) dv, then the residual norms of the warp's rows
+    const float rs = (n > 0) ? scale : 0.f;
+    float part[RPW];
+    if (e > 0) {
+#pragma unroll
+      for (int i = 0; i < RPW; ++i) {
+        part[i] = 0.f;
+        if ((alive >> i) & 1u) {
+          float kf[DPL];
+          load_bf16<DPL>(Kr + (size_t)(warp + kRW * i) * D + lane * DPL, kf);
+#pragma unroll
+          for (int d = 0; d < DPL; ++d) part[i] = fmaf(sdk[d], kf[d], part[i]);
+        }
+      }
+      warp_sum_n<RPW>(part);
+#pragma unroll
+      for (int i = 0; i < RPW; ++i)
+#pragma unroll
+        for (int d = 0; d < DPL; ++d) y[i][d] = fmaf(keep, y[i][d], part[i] * sdv[d]);
+    }
+#pragma unroll
+    for (int i = 0; i < RPW; ++i) {
+      part[i] = 0.f;
+      if ((alive >> i) & 1u) {
+        float vf[DPL];
+        load_bf16<DPL>(Vr + (size_t)(warp + kRW * i) * D + lane * DPL, vf);
+#pragma unroll
+        for (int d = 0; d < DPL; ++d) {
+          const float rr = vf[d] - mv[d] - rs * y[i][d];
+          part[i] = fmaf(rr, rr, part[i]);
+        }
+      }
+    }
+    warp_sum_n<RPW>(part);
+    auto post_keys = [&](const float (&ss)[RPW]) {
+      if (lane == 0) {
+        unsigned long long best = ~0ull;
+#pragma unroll
+        for (int i = 0; i < RPW; ++i)
+          if ((alive >> i) & 1u) {
+            const int r = warp + kRW * i;
+            float alpha = 0.f;
+#pragma unroll
+            for (int h = 0; h < G; ++h) alpha = fmaf(lg[h * a.cap + j0 + r], s_invZ[warp][h], alpha);
+            const float score = alpha * sqrtf(ss[i]);
+            const unsigned long long key =
+                (static_cast<unsigned long long>(__float_as_uint(score)) << 32) | static_cast<unsigned>(j0 + r);
+            best = key < best ? key : best;
+          }
+        if (best != ~0ull) atomicMin(&s_best[par], best);
+      }
+    };
+    post_keys(part);
+    __syncthreads();
+    const int nz = s_nz;
+    if (nz > 0) {  // uniform: clamped entries of C' change y; score again with them
+      const bool direct = nz > kMaxClamp;
+      if (tid == 0) s_best[par] = ~0ull;
+      if (direct) {
+#pragma unroll
+        for (int jj = 0; jj < CJ; ++jj) st_vec<DPL>(Ct + (size_t)(warp + kRW * jj) * D + lane * DPL, creg[jj]);
+      }
+      __syncthreads();
+      const float nf = static_cast<float>(n);
+#pragma unroll
+      for (int i = 0; i < RPW; ++i) {
+        part[i] = 0.f;
+        if ((alive >> i) & 1u) {
+          const int r = warp + kRW * i;
+          float yc[DPL];
+          if (!direct) {
+#pragma unroll
+            for (int d = 0; d < DPL; ++d) yc[d] = y[i][d];
+            for (int z = 0; z < nz; ++z) {  // y'_a -= C_ab k_b for clamped (a, b)
+              const int kb = static_cast<int>(s_zidx[z] / D), va = static_cast<int>(s_zidx[z] % D);
+              if (va / DPL == lane) {
+                const float corr = s_zval[z] * __bfloat162float(Kr[(size_t)r * D + kb]);
+#pragma unroll
+                for (int d = 0; d < DPL; ++d)
+                  if (va % DPL == d) yc[d] -= corr;
+              }
+            }
+          } else {
+#pragma unroll
+            for (int d = 0; d < DPL; ++d) yc[d] = 0.f;
+            for (int c = 0; c < D; ++c) {
+              const float kv = __bfloat162float(Kr[(size_t)r * D + c]);
+              float cv[DPL];
+              ld_vec<DPL>(Ct + (size_t)c * D + lane * DPL, cv);
+#pragma unroll
+              for (int d = 0; d < DPL; ++d) yc[d] = fmaf((fabsf(cv[d] * nf) < tau) ? 0.f : cv[d], kv, yc[d]);
+            }
+          }
+          float vf[DPL];
+          load_bf16<DPL>(Vr + (size_t)r * D + lane * DPL, vf);
+#pragma unroll
+          for (int d = 0; d < DPL; ++d) {
+            const float rr = vf[d] - mv[d] - rs * yc[d];
+            part[i] = fmaf(rr, rr, part[i]);
+          }
+        }
+      }
+      warp_sum_n<RPW>(part);
+      post_keys(part);
+      __syncthreads();
+      if (tid == 0) s_nz = 0;  // every reader of the list is past the barrier above
+    }
+
+    // ---- warp w < 8 posts this CTA's key and candidate row into rank w's mailbox
+    if (warp < kCL) {
+      const unsigned long long b = s_best[par];
+      const int jb = (b == ~0ull) ? -1 : static_cast<int>(b & 0xffffffffu) - j0;
+      if (lane == 0) *cluster.map_shared_rank(&mail_key[par][rank], warp) = b;
+      if (jb >= 0 && lane < D / 4) {  // lanes 0..D/8-1 carry k, the next D/8 carry v
+        const bool is_v = lane >= D / 8;
+        const int i = is_v ? lane - D / 8 : lane;
+        const uint4 w4 = reinterpret_cast<const uint4*>((is_v ? Vr : Kr) + (size_t)jb * D)[i];
+        reinterpret_cast<uint4*>(cluster.map_shared_rank(&mail_row[par][rank][is_v ? D : 0], warp))[i] = w4;
+      }
+    }
+    cluster.sync();
+
+    // ---- every warp: the cluster's minimum key (ties cannot happen: rows differ)
+    unsigned long long b = (lane < kCL) ? mail_key[par][lane] : ~0ull;
+    int src = lane;
+#pragma unroll
+    for (int o = 4; o > 0; o >>= 1) {
+      const unsigned long long b2 = __shfl_xor_sync(kFull, b, o);
+      const int s2 = __shfl_xor_sync(kFull, src, o);
+      if (b2 < b) {
+        b = b2;
+        src = s2;
+      }
+    }
+    b = __shfl_sync(kFull, b, 0);
+    src = __shfl_sync(kFull, src, 0);
+    const int js = (b == ~0ull) ? -1 : static_cast<int>(b & 0xffffffffu);
+    if (js < 0) {  // uniform: every rank read the same keys
+      if (rank == 0 && tid == 0) record_error(a.ws, MKV_ERR_INVALID_ARG, u);
+      break;
+    }
+    // Welford fold of the evicted row for this lane's dims (Eq. app_update)
+    {
+      const float inv = 1.f / static_cast<float>(n + 1);
+      keep = static_cast<float>(n) * inv;
+      float kx[DPL], vx[DPL];
+      load_bf16<DPL>(&mail_row[par][src][lane * DPL], kx);
+      load_bf16<DPL>(&mail_row[par][src][D + lane * DPL], vx);
+#pragma unroll
+      for (int d = 0; d < DPL; ++d) {
+        const float dk = kx[d] - mk[d];
+        mk[d] = fmaf(dk, inv, mk[d]);
+        mv[d] = fmaf(vx[d] - mv[d], inv, mv[d]);
+        sdk[d] = dk * inv;  // scaled by 1/(n+1) for the rank-1 terms
+        sdv[d] = vx[d] - mv[d];
+      }
+      n += 1;
+    }
+    const int jr = js - j0;
+    if (jr >= 0 && jr < nr && jr % kRW == warp) alive &= ~(1u << (jr / kRW));
+    if (lane < G) {
+      const double z = s_zd[warp][lane] - static_cast<double>(lg[lane * a.cap + js]);
+      s_zd[warp][lane] = z;
+      s_invZ[warp][lane] = 1.f / static_cast<float>(z);
+    }
+    __syncwarp();
+  }
+
+  // ---- state back to shared memory: survivors, C (transposed), means
+#pragma unroll
+  for (int i = 0; i < RPW; ++i)
+    if (lane == 0 && warp + kRW * i < nr) alive_all[j0 + warp + kRW * i] = (alive >> i) & 1u;
+#pragma unroll
+  for (int jj = 0; jj < CJ; ++jj) st_vec<DPL>(Ct + (size_t)(warp + kRW * jj) * D + lane * DPL, creg[jj]);
+  if (warp == 0) {
+#pragma unroll
+    for (int d = 0; d < DPL; ++d) {
+      s_mu_k[lane * DPL + d] = mk[d];
+      s_mu_v[lane * DPL + d] = mv[d];
+    }
+  }
+  __syncthreads();
+  const uint8_t* alv = alive_all + j0;
+
+  // ---- ordered compaction across the cluster through the staging buffer
+  {
+    int cnt = 0;
+    for (int r = tid; r < nr; r += kRT) cnt += alv[r];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) cnt += __shfl_xor_sync(kFull, cnt, o);
+    if (lane == 0) s_red[warp][0] = static_cast<float>(cnt);
+    __syncthreads();
+    if (tid == 0) {
+      int c = 0;
+      for (int w = 0; w < kRW; ++w) c += static_cast<int>(s_red[w][0]);
+      ex_cnt = c;
+    }
+  }
+  cluster.sync();
+  int base = 0;
+  for (int r = 0; r < rank; ++r) base += *cluster.map_shared_rank(&ex_cnt, r);
+  const int mine = ex_cnt;
+  uint8_t* st = static_cast<uint8_t*>(a.stage) + (size_t)u * stage_stride(a.cap, D);
+  __nv_bfloat16* SK = reinterpret_cast<__nv_bfloat16*>(st);
+  __nv_bfloat16* SV = SK + (size_t)a.cap * D;
+  int32_t* SP = reinterpret_cast<int32_t*>(SV + (size_t)a.cap * D);
+  for (int c0 = 0; c0 < nr; c0 += 32) {
+    const bool al = (c0 + lane < nr) && alv[c0 + lane];
+    const unsigned m = __ballot_sync(kFull, al);
+    int before = 0;  // survivors in earlier chunks
+    for (int c1 = 0; c1 < c0; c1 += 32) {
+      const bool a1 = (c1 + lane < nr) && alv[c1 + lane];
+      before += __popc(__ballot_sync(kFull, a1));
+    }
+    for (int bit = warp; bit < 32; bit += kRW) {  // warp w moves rows c0 + w, c0 + w + 16
+      if ((m >> bit) & 1u) {
+        const int r = c0 + bit;
+        const int dst = base + before + __popc(m & ((1u << bit) - 1u));
+        for (int i = lane; i < D / 8; i += 32) {
+          reinterpret_cast<uint4*>(SK + (size_t)dst * D)[i] = reinterpret_cast<const uint4*>(Kr + (size_t)r * D)[i];
+          reinterpret_cast<uint4*>(SV + (size_t)dst * D)[i] = reinterpret_cast<const uint4*>(Vr + (size_t)r * D)[i];
+        }
+        if (lane == 0) SP[dst] = Pg[j0 + r];
+      }
+    }
+  }
+  __threadfence();
+  cluster.sync();
+  for (int idx = tid; idx < mine * (D / 8); idx += kRT) {
+    const int row = base + idx / (D / 8), i = idx % (D / 8);
+    reinterpret_cast<uint4*>(Kg + (size_t)row * D)[i] = reinterpret_cast<const uint4*>(SK + (size_t)row * D)[i];
+    reinterpret_cast<uint4*>(Vg + (size_t)row * D)[i] = reinterpret_cast<const uint4*>(SV + (size_t)row * D)[i];
+  }
+  for (int r = tid; r < mine; r += kRT) Pg[base + r] = SP[base + r];
+  if (rank == 0) {
+    float* tb = s_tile[warp % kTW];
+    for (int t = warp; warp < kTW && t < (D / 32) * (D / 32); t += kTW) {
+      const int c0 = (t / (D / 32)) * 32, r0 = (t % (D / 32)) * 32;
+      for (int i = 0; i < 32; ++i) tb[i * 33 + lane] = Ct[(size_t)(c0 + i) * D + r0 + lane];
+      __syncwarp();
+      for (int i = 0; i < 32; ++i) a.C[(size_t)u * D * D + (size_t)(r0 + i) * D + c0 + lane] = tb[lane * 33 + i];
+      __syncwarp();
+    }
+    for (int i = tid; i < D; i += kRT) {
+      a.mu_k[(size_t)u * D + i] = s_mu_k[i];
+      a.mu_v[(size_t)u * D + i] = s_mu_v[i];
+    }
+    if (tid == 0) {
+      a.n[u] = n;
+      a.len[u] = a.budget;
+      a.seen[u] = seen_in + (has_new ? 1 : 0);
+    }
+  }
+}
+
 template <int D, int G>
 size_t cluster_smem(int cap, int* kv) {
   const int R = (cap + kCL - 1) / kCL;
@@ -907,9 +1521,29 @@ size_t cluster_smem(int cap, int* kv) {
   return ClusterLayout<D, G>(R, cap, 0).total;
 }
 
+template <int D, int G, int RPW>
+cudaError_t launch_reg(EvictArgs a, cudaStream_t stream) {
+  a.rows_max = (a.cap + kCL - 1) / kCL;
+  a.kv_smem = 1;
+  size_t smem = RegLayout<D, G>(a.rows_max, a.cap, 1).total;
+  if (smem > kSmemBudget) {
+    a.kv_smem = 0;
+    smem = RegLayout<D, G>(a.rows_max, a.cap, 0).total;
+  }
+  cudaError_t e = cudaFuncSetAttribute(evict_reg_kernel<D, G, RPW>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  evict_reg_kernel<D, G, RPW><<<a.batch * a.n_kv * kCL, kRT, smem, stream>>>(a);
+  return cudaGetLastError();
+}
+
 template <int D, int G>
 cudaError_t launch_dg(const EvictArgs& a0, cudaStream_t stream) {
   EvictArgs a = a0;
+  // rows of one CTA's slice at most; warps of the register kernel hold 5 or 9 each
+  const int slice = (a.cap + kCL - 1) / kCL;
+  if (slice <= kRW * 5) return launch_reg<D, G, 5>(a, stream);
+  if (slice <= kRW * 9) return launch_reg<D, G, 9>(a, stream);
   int kv = 0;
   const size_t csm = cluster_smem<D, G>(a.cap, &kv);
   if (csm <= kSmemBudget) {

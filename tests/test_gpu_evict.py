@@ -138,3 +138,13 @@ def test_evict_budget_zero_and_batch():
     st = setup(rng, 2, 2, 1, 64, [9, 17, 1, 30], 32, [0, 2, 0, 7])
     gpu, refs = run_case(st, 2, 2, 1, 64, 0, False)
     check(gpu, refs, st, 0)
+
+
+@pytest.mark.parametrize("cap", [1000, 1200])
+def test_evict_slice_sizes(cap):
+    """Row slices of 125 rows (register-resident kernel, 9 rows per warp) and
+    150 rows (shared-memory cluster kernel): 30 evictions each."""
+    rng = np.random.default_rng(34 + cap)
+    st = setup(rng, 1, 2, 4, 128, [cap - 11, cap - 20], cap, [300, 0])
+    gpu, refs = run_case(st, 1, 2, 4, 128, cap - 41, True)
+    check(gpu, refs, st, cap - 41)
