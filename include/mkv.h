@@ -194,7 +194,7 @@ MKV_API size_t mkv_decode_workspace_size(mkv_geom geom, int32_t capacity);
  * output is f_hat_E; with neither rows nor moments the kernel records
  * MKV_ERR_INVALID_ARG and writes zeros.  An append past capacity records
  * MKV_ERR_CAPACITY, still attends over the new token, and leaves the cache
- * unchanged.
+ * unchanged.  q, out, k_new and v_new must be 16-byte aligned.
  */
 MKV_API mkv_status mkv_decode_step(mkv_geom geom, const void* q, const void* k_new, const void* v_new,
                            const mkv_cache* cache, const mkv_moments* mom,

@@ -80,6 +80,8 @@ mkv_status mkv_decode_step(mkv_geom geom, const void* q, const void* k_new, cons
   if (!geom_ok(geom)) return (geom.head_dim == 64 || geom.head_dim == 128) ? MKV_ERR_SHAPE : MKV_ERR_UNSUPPORTED;
   if (!q || !out || !p || !cache_ok(cache)) return MKV_ERR_INVALID_ARG;
   if ((k_new == nullptr) != (v_new == nullptr)) return MKV_ERR_INVALID_ARG;
+  if (!aligned(q, 16) || !aligned(out, 16) || (k_new && (!aligned(k_new, 16) || !aligned(v_new, 16))))
+    return MKV_ERR_INVALID_ARG;
   if (p->correction != 0 && p->correction != 1) return MKV_ERR_INVALID_ARG;
   if (p->order != 0 && p->order != 1) return MKV_ERR_INVALID_ARG;
   if (p->correction && !moments_ok(mom)) return MKV_ERR_INVALID_ARG;

@@ -238,15 +238,22 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
     len0 = len0 < 0 ? 0 : a.cap;
   }
   const bool has_new = a.k_new != nullptr;
-  const int L = len0 + (has_new ? 1 : 0);
   const bool use_m = n_e > 0;
-
-  const int tiles_total = (L + kTT - 1) / kTT;
+  // the cached rows are split into whole tiles over the S CTAs; the appended
+  // token is attended to by the last CTA (which holds the fewest rows), whose
+  // threads fetch it now: threads 0..D/8-1 hold 16 bytes of k each, the next
+  // D/8 threads 16 bytes of v
+  const bool own_new = has_new && s == a.S - 1;
+  uint4 new_part = make_uint4(0u, 0u, 0u, 0u);
+  if (own_new && tid < D / 4) {
+    const __nv_bfloat16* src = reinterpret_cast<const __nv_bfloat16*>(tid < D / 8 ? a.k_new : a.v_new) + (size_t)u * D;
+    new_part = reinterpret_cast<const uint4*>(src)[tid % (D / 8)];
+  }
+  const int tiles_total = (len0 + kTT - 1) / kTT;
   const int tiles_per = (tiles_total + a.S - 1) / a.S;
-  const int t_begin = min(L, s * tiles_per * kTT);
-  const int t_end = min(L, t_begin + tiles_per * kTT);
-  const int n_cached = max(0, min(t_end, len0) - t_begin);
-  const bool own_new = has_new && t_begin <= len0 && len0 < t_end;
+  const int t_begin = min(len0, s * tiles_per * kTT);
+  const int t_end = min(len0, t_begin + tiles_per * kTT);
+  const int n_cached = t_end - t_begin;
   const int n_tiles = (n_cached + kTT - 1) / kTT;
 
   // one thread fills a stage: a 64-row box per 64 columns, for K and for V
@@ -266,7 +273,19 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
   if (tid == 0) {
     for (int i = 0; i < min(kStages, n_tiles); ++i) issue(i);
   }
-  for (int i = tid; i < G * D; i += kThreads) sQ[i] = __bfloat162float(qg[i]) * (scale * kLog2e);
+  if (warp == 0 && (lane >> 2) < G) {  // q * scale * log2(e) from the A fragments
+    const int g = lane >> 2, t = lane & 3;
+#pragma unroll
+    for (int kk = 0; kk < D / 16; ++kk) {
+      const __nv_bfloat162 lo = *reinterpret_cast<const __nv_bfloat162*>(&qa[kk][0]);
+      const __nv_bfloat162 hi = *reinterpret_cast<const __nv_bfloat162*>(&qa[kk][1]);
+      float* dq = sQ + g * D + kk * 16 + 2 * t;
+      dq[0] = __low2float(lo) * (scale * kLog2e);
+      dq[1] = __high2float(lo) * (scale * kLog2e);
+      dq[8] = __low2float(hi) * (scale * kLog2e);
+      dq[9] = __high2float(hi) * (scale * kLog2e);
+    }
+  }
   __syncthreads();
   if constexpr (CL) cluster_wait_acquire();
 
@@ -362,22 +381,25 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
     for (int nt = 0; nt < D / 8; ++nt) st.o[nt][0] = st.o[nt][1] = 0.f;
   }
   if (own_new) {  // the appended token: row 0 of stage 0 (free now), rows 1..15 zero
-    const __nv_bfloat16* kn = reinterpret_cast<const __nv_bfloat16*>(a.k_new) + (size_t)u * D;
-    const __nv_bfloat16* vn = reinterpret_cast<const __nv_bfloat16*>(a.v_new) + (size_t)u * D;
-    for (int i = tid; i < 16 * D; i += kThreads) {
-      const int r = i / D, c = i % D;
-      *reinterpret_cast<__nv_bfloat16*>(sK + swz_off(r, c, kTT)) = (r == 0) ? kn[c] : __float2bfloat16_rn(0.f);
-      *reinterpret_cast<__nv_bfloat16*>(sV + swz_off(r, c, kTT)) = (r == 0) ? vn[c] : __float2bfloat16_rn(0.f);
+    // a row is one 128-byte line per 64-column box; the swizzle permutes the
+    // 16-byte chunks within a row, so zero rows are zero in any order
+    for (int i = tid; i < 16 * (D / 8); i += kThreads) {
+      const int r = i / (D / 8), c = (i % (D / 8)) * 8;
+      const uint32_t off = (c >> 6) * kTT * 128 + r * 128 + (((c & 63) >> 3) << 4);
+      *reinterpret_cast<uint4*>(sK + off) = make_uint4(0u, 0u, 0u, 0u);
+      *reinterpret_cast<uint4*>(sV + off) = make_uint4(0u, 0u, 0u, 0u);
+    }
+    __syncthreads();
+    if (tid < D / 4) {
+      const int c = (tid % (D / 8)) * 8;
+      *reinterpret_cast<uint4*>((tid < D / 8 ? sK : sV) + swz_off(0, c, kTT)) = new_part;
     }
     __syncthreads();
     if (warp == 0) process16<D, G>(st, qa, sK, sV, 0, 1, qscale, lane);
-    if (len0 + 1 <= a.cap) {  // nobody reads this cache row during the step
-      __nv_bfloat16* Kd = reinterpret_cast<__nv_bfloat16*>(a.K) + ((size_t)u * a.cap + len0) * D;
-      __nv_bfloat16* Vd = reinterpret_cast<__nv_bfloat16*>(a.V) + ((size_t)u * a.cap + len0) * D;
-      for (int i = tid; i < D; i += kThreads) {
-        Kd[i] = kn[i];
-        Vd[i] = vn[i];
-      }
+    if (len0 + 1 <= a.cap && tid < D / 4) {  // nobody reads this cache row during the step
+      __nv_bfloat16* dst =
+          reinterpret_cast<__nv_bfloat16*>(tid < D / 8 ? a.K : a.V) + ((size_t)u * a.cap + len0) * D;
+      reinterpret_cast<uint4*>(dst)[tid % (D / 8)] = new_part;
     }
   }
 
@@ -433,12 +455,67 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
     cluster_arrive_release();
     cluster_wait_acquire();
     if (s != 0) return;
-    staged = true;
-    src = sRcv;
-    sF = sFr;
-    if (use_m && a.order != 1)
-      for (int i = tid; i < G * D / 4; i += kThreads)
-        reinterpret_cast<float4*>(sF)[i] = __ldg(reinterpret_cast<const float4*>(a.mu_v + (size_t)u * D) + (i % (D / 4)));
+    // warp w merges heads w, w + 4, ...: lane sp < S holds split sp's (m, l);
+    // lane l owns the output dims [l*DPL, (l+1)*DPL).  No block barrier.
+    for (int h = warp; h < G; h += 4) {
+      float m_s = -INFINITY, l_s = 0.f;
+      if (lane < a.S) {
+        m_s = sRcv[((size_t)lane * G + h) * PS + D];
+        l_s = sRcv[((size_t)lane * G + h) * PS + D + 1];
+      }
+      const float Mx = warp_max(l_s > 0.f ? m_s : -INFINITY);
+      const float w_s = (l_s > 0.f && Mx != -INFINITY) ? fast_exp2(m_s - Mx) : 0.f;
+      const float l = warp_sum(l_s * w_s);
+      float acc[DPL];
+#pragma unroll
+      for (int d = 0; d < DPL; ++d) acc[d] = 0.f;
+      for (int sp = 0; sp < a.S; ++sp) {
+        const float wsp = __shfl_sync(kFull, w_s, sp);
+        if (wsp != 0.f) {  // warp-uniform
+          const float* rec = sRcv + ((size_t)sp * G + h) * PS + lane * DPL;
+#pragma unroll
+          for (int d = 0; d < DPL; ++d) acc[d] = fmaf(wsp, rec[d], acc[d]);
+        }
+      }
+      const bool have_r = l > 0.f;
+      const float inv_l = have_r ? 1.f / l : 0.f;
+      float res[DPL], lse = have_r ? Mx * kLn2 + logf(l) : -INFINITY;
+      if (use_m) {
+        const float e = logf(static_cast<float>(n_e)) + sSbar[h];
+        float wR = 0.f;
+        if (have_r) {
+          const float top = fmaxf(lse, e);
+          const float wr = expf(lse - top), we = expf(e - top);
+          wR = wr / (wr + we);
+          lse = top + logf(wr + we);
+        } else {
+          lse = e;
+        }
+#pragma unroll
+        for (int d = 0; d < DPL; ++d) {
+          const float fh = (a.order == 1) ? sFr[h * D + lane * DPL + d] : __ldg(a.mu_v + (size_t)u * D + lane * DPL + d);
+          res[d] = have_r ? wR * (acc[d] * inv_l) + (1.f - wR) * fh : fh;
+        }
+      } else {
+        if (!have_r && lane == 0) record_error(a.ws, MKV_ERR_INVALID_ARG, u);
+#pragma unroll
+        for (int d = 0; d < DPL; ++d) res[d] = acc[d] * inv_l;
+      }
+      float* o = a.out + ((size_t)u * G + h) * D + lane * DPL;
+      if constexpr (DPL == 4) *reinterpret_cast<float4*>(o) = make_float4(res[0], res[1], res[2], res[3]);
+      else *reinterpret_cast<float2*>(o) = make_float2(res[0], res[1]);
+      if (a.lse != nullptr && lane == 0) a.lse[(size_t)u * G + h] = lse;
+    }
+    if (has_new && tid == 0) {  // the row itself was written by the CTA that attended to it
+      if (len0 + 1 > a.cap) {
+        record_error(a.ws, MKV_ERR_CAPACITY, u);
+      } else {
+        a.pos[(size_t)u * a.cap + len0] = a.seen[u];
+        a.seen[u] = a.seen[u] + 1;
+        a.len[u] = len0 + 1;
+      }
+    }
+    return;
   } else {
     // ---- ticket: the last CTA of this unit merges everything
     __threadfence();

@@ -69,6 +69,8 @@ extern "C" MKV_API mkv_status mkv_decode_step_noalloc(mkv_geom geom, const void*
       cache->capacity < 1 || !aligned16(cache->K) || !aligned16(cache->V))
     return MKV_ERR_INVALID_ARG;
   if ((k_new == nullptr) != (v_new == nullptr)) return MKV_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(out) || (k_new && (!aligned16(k_new) || !aligned16(v_new))))
+    return MKV_ERR_INVALID_ARG;
   if ((p->correction != 0 && p->correction != 1) || (p->order != 0 && p->order != 1) || !(p->tau >= 0.f))
     return MKV_ERR_INVALID_ARG;
   if (p->correction && (!mom || !mom->n || !mom->mu_k || !mom->mu_v || !mom->C || !aligned16(mom->C)))
