@@ -8,14 +8,17 @@
 //                            sums -> the chunk's centred moments
 //   scores_tc (chunk, unit)  logits again (token-major) -> s_t = sum over rows
 //                            of exp(l - m_row) / l_row, pooled
-//   select    (unit)         R0 = protected + top-k(s) (radix select, ties to the
-//                            lower position); R0's rows gathered densely
-//   stats_tc  (unit)         moments of the gathered R0 rows (no logits)
-//   finalize  (rows, unit)   M0 = moments(all) - moments(R0) (Chan merges)
+//   select    (8-CTA cluster per unit) R0 = protected + top-k(s): radix select
+//                            with 8-bit digits, histograms summed through
+//                            distributed shared memory, ties to the lower
+//                            position; R0's rows gathered densely
+//   stats_tc  (chunk, unit)  moments of the gathered R0 rows (no logits)
+//   finalize  (rows, unit)   M0 = moments(all) - moments(R0) (Chan merges); the
+//                            all-token record is merged once and kept
 //   residual_tc (chunk, unit) Y = K C0'^T on the tensor cores (C0' split into
 //                            three bf16 parts) -> score2 = s_t ||v - mu_v0 - scale y||
-//   select    (unit)         R = protected + top-k(score2), gathered into the cache
-//   stats_tc  (unit)         moments of the retained rows
+//   select    (cluster, unit) R = protected + top-k(score2), gathered into the cache
+//   stats_tc  (chunk, unit)  moments of the retained rows
 //   finalize  (rows, unit)   moments of E = all \ R -> caller's mkv_moments
 //
 // The tensor-core kernels are warp-specialised: warp 0 issues the TMA copies
