@@ -68,6 +68,23 @@ __device__ __forceinline__ void mma_bf16(float (&d)[4], uint32_t a0, uint32_t a2
       : "r"(a0), "r"(0u), "r"(a2), "r"(0u), "r"(b0), "r"(b1));
 }
 
+__device__ __forceinline__ void mma_bf16_full(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                              uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// (hi, lo) bf16 pair parts of two floats: hi = bf16(x), lo = bf16(x - hi)
+__device__ __forceinline__ void split_bf16x2(float x, float y, uint32_t& hi, uint32_t& lo) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(x, y);
+  const __nv_bfloat162 l = __floats2bfloat162_rn(x - __low2float(h), y - __high2float(h));
+  hi = *reinterpret_cast<const uint32_t*>(&h);
+  lo = *reinterpret_cast<const uint32_t*>(&l);
+}
+
 __device__ __forceinline__ void ldsm_x4_trans(uint32_t (&r)[4], const void* p) {
   asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
                : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
@@ -164,7 +181,7 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
   uint8_t* dsmem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dsmem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sK = dsmem;                          // [stage][box][kTT][128 B]
   uint8_t* sV = dsmem + kStages * kTileBytes;
-  __shared__ float sQ[G * D];  // q * scale * log2(e)
+  __shared__ float sFp[2][4][16][8];  // C'q partial sums: [m16 tile][warp][row][head]
   __shared__ float sSbar[G];
   __shared__ float sM[G], sL[G];
   __shared__ __align__(8) uint64_t bars[kStages];
@@ -207,31 +224,57 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
     }
   }
   const bool corr = a.correction != 0 && a.n != nullptr;
-  constexpr int RB = 4;  // moment rows per warp whose loads are in flight together
+  // Moment rows [r0, r1) of this split: C'q on the tensor cores.  The rows
+  // form m16 tiles (A = C' rows, split into bf16 hi + lo parts: about 16
+  // significant bits); B is q itself, whose fragments are the qa registers
+  // (column n = head).  Up to two tiles (many splits, small batches): warp w
+  // takes the k-steps [w*KPW, (w+1)*KPW) of each tile, its fragments are
+  // loaded now, and the four partial sums meet in shared memory.  More tiles
+  // (few splits, large batches): warp w takes whole tiles w, w + 4, ....
+  constexpr int KPW = D / 64;
   const int rpc = (D + a.S - 1) / a.S;
   const int r0 = s * rpc, r1 = min(D, r0 + rpc);
-  float cv[RB][DPL], mvr[RB], muk[DPL];
+  const int n_mt = (r1 - r0 + 15) / 16;
+  const bool do_c = corr && a.order == 1;
+  const bool split_k = n_mt <= 2;
+  float2 cfr[2][KPW][4];
+  {
+    const int g = lane >> 2, t = lane & 3;
 #pragma unroll
-  for (int k = 0; k < RB; ++k) {
-    const int row = r0 + warp + 4 * k;
-    mvr[k] = 0.f;
+    for (int j = 0; j < 2; ++j) {
+      const int ra = r0 + j * 16 + g, rb = ra + 8;
 #pragma unroll
-    for (int i = 0; i < DPL; ++i) cv[k][i] = 0.f;
-    if (corr && a.order == 1 && row < r1) {
-      const float* Crow = a.C + ((size_t)u * D + row) * D + lane * DPL;
-      if constexpr (DPL == 4) {
-        const float4 t4 = __ldg(reinterpret_cast<const float4*>(Crow));
-        cv[k][0] = t4.x; cv[k][1] = t4.y; cv[k][2] = t4.z; cv[k][3] = t4.w;
-      } else {
-        const float2 t2 = __ldg(reinterpret_cast<const float2*>(Crow));
-        cv[k][0] = t2.x; cv[k][1] = t2.y;
+      for (int kp = 0; kp < KPW; ++kp) {
+        const int c0 = (warp * KPW + kp) * 16 + 2 * t;
+        const float* Ca = a.C + ((size_t)u * D + ra) * D + c0;
+        const float* Cb = a.C + ((size_t)u * D + rb) * D + c0;
+        const bool va = do_c && split_k && ra < r1, vb = do_c && split_k && rb < r1;
+        cfr[j][kp][0] = va ? __ldg(reinterpret_cast<const float2*>(Ca)) : make_float2(0.f, 0.f);
+        cfr[j][kp][1] = vb ? __ldg(reinterpret_cast<const float2*>(Cb)) : make_float2(0.f, 0.f);
+        cfr[j][kp][2] = va ? __ldg(reinterpret_cast<const float2*>(Ca + 8)) : make_float2(0.f, 0.f);
+        cfr[j][kp][3] = vb ? __ldg(reinterpret_cast<const float2*>(Cb + 8)) : make_float2(0.f, 0.f);
       }
-      mvr[k] = __ldg(a.mu_v + (size_t)u * D + row);
     }
   }
+  // mu_v of the (row, head) pairs this thread finishes in the two-tile case
+  constexpr int kPairs = 2 * 16 * 8 / kThreads;  // at most 32 rows x 8 heads
+  float muv_pre[kPairs];
 #pragma unroll
-  for (int i = 0; i < DPL; ++i) muk[i] = corr ? __ldg(a.mu_k + (size_t)u * D + lane * DPL + i) : 0.f;
+  for (int j = 0; j < kPairs; ++j) {
+    const int idx = tid + j * kThreads, row = r0 + idx / G;
+    muv_pre[j] = (do_c && split_k && row < r1) ? __ldg(a.mu_v + (size_t)u * D + row) : 0.f;
+  }
+  // mu_k at this lane's q dims (warp 1 computes scale q . mu_k for its head)
+  float2 mkp[D / 16][2];
+#pragma unroll
+  for (int kk = 0; kk < D / 16; ++kk) {
+    const int t = lane & 3;
+    const bool v = corr && warp == 1 && (lane >> 2) < G;
+    mkp[kk][0] = v ? __ldg(reinterpret_cast<const float2*>(a.mu_k + (size_t)u * D + kk * 16 + 2 * t)) : make_float2(0.f, 0.f);
+    mkp[kk][1] = v ? __ldg(reinterpret_cast<const float2*>(a.mu_k + (size_t)u * D + kk * 16 + 8 + 2 * t)) : make_float2(0.f, 0.f);
+  }
   const int n_e = corr ? a.n[u] : 0;
+  const int seen0 = (CL && s == 0 && tid == 0 && a.k_new != nullptr) ? a.seen[u] : 0;  // for the bookkeeping
   int len0 = a.len[u];
   if (len0 < 0 || len0 > a.cap) {  // corrupt cache state: never read past the slab
     if (tid == 0 && s == 0) record_error(a.ws, MKV_ERR_CAPACITY, u);
@@ -273,67 +316,95 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
   if (tid == 0) {
     for (int i = 0; i < min(kStages, n_tiles); ++i) issue(i);
   }
-  if (warp == 0 && (lane >> 2) < G) {  // q * scale * log2(e) from the A fragments
-    const int g = lane >> 2, t = lane & 3;
+  if (use_m && warp == 1) {  // scale * q . mu_k per head from the qa fragments (lanes 4h..4h+3)
+    const int g = lane >> 2;
+    float acc = 0.f;
 #pragma unroll
     for (int kk = 0; kk < D / 16; ++kk) {
-      const __nv_bfloat162 lo = *reinterpret_cast<const __nv_bfloat162*>(&qa[kk][0]);
-      const __nv_bfloat162 hi = *reinterpret_cast<const __nv_bfloat162*>(&qa[kk][1]);
-      float* dq = sQ + g * D + kk * 16 + 2 * t;
-      dq[0] = __low2float(lo) * (scale * kLog2e);
-      dq[1] = __high2float(lo) * (scale * kLog2e);
-      dq[8] = __low2float(hi) * (scale * kLog2e);
-      dq[9] = __high2float(hi) * (scale * kLog2e);
+      const __nv_bfloat162 q0 = *reinterpret_cast<const __nv_bfloat162*>(&qa[kk][0]);
+      const __nv_bfloat162 q1 = *reinterpret_cast<const __nv_bfloat162*>(&qa[kk][1]);
+      acc = fmaf(__low2float(q0), mkp[kk][0].x, fmaf(__high2float(q0), mkp[kk][0].y, acc));
+      acc = fmaf(__low2float(q1), mkp[kk][1].x, fmaf(__high2float(q1), mkp[kk][1].y, acc));
+    }
+    acc += __shfl_xor_sync(kFull, acc, 1);
+    acc += __shfl_xor_sync(kFull, acc, 2);
+    if ((lane & 3) == 0 && g < G) sSbar[g] = acc * scale;
+  }
+  const float tau = a.tau;
+  const float nf = static_cast<float>(n_e);
+  // one m16 x n8 product over the k-steps [kk0, kk0 + nk) from fragments in
+  // registers (clamp of Eq. fused's C' applied here)
+  auto mma_c = [&](float (&d)[4], const float2 (&f)[4], int kk) {
+    uint32_t hi[4], lo[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float x = (fabsf(f[i].x * nf) < tau) ? 0.f : f[i].x;
+      const float y = (fabsf(f[i].y * nf) < tau) ? 0.f : f[i].y;
+      split_bf16x2(x, y, hi[i], lo[i]);
+    }
+    mma_bf16_full(d, hi[0], hi[1], hi[2], hi[3], qa[kk][0], qa[kk][1]);
+    mma_bf16_full(d, lo[0], lo[1], lo[2], lo[3], qa[kk][0], qa[kk][1]);
+  };
+  if (use_m && do_c && split_k) {
+    const int g = lane >> 2, t = lane & 3;
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      if (j >= n_mt) break;  // warp-uniform
+      float d[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int kp = 0; kp < KPW; ++kp) mma_c(d, cfr[j][kp], warp * KPW + kp);
+      float(*fp)[8] = sFp[j][warp];
+      fp[g][2 * t] = d[0];
+      fp[g][2 * t + 1] = d[1];
+      fp[g + 8][2 * t] = d[2];
+      fp[g + 8][2 * t + 1] = d[3];
     }
   }
   __syncthreads();
   if constexpr (CL) cluster_wait_acquire();
-
-  if (use_m) {
-    // scale * q . mu_k for every head (every CTA; the merging one uses it)
-    for (int h = warp; h < G; h += 4) {
-      float acc = 0.f;
+  // f_hat_E[h][row] = mu_v[row] + scale * (C'q_h)[row]
+  if (use_m && do_c) {
+    float* fdst = CL ? fr0 : a.fhat + (size_t)u * G * D;
+    if (split_k) {
+      const int n_pairs = (r1 - r0) * G;
 #pragma unroll
-      for (int i = 0; i < DPL; ++i) acc = fmaf(sQ[h * D + lane * DPL + i], muk[i], acc);
-      acc = warp_sum(acc);
-      if (lane == 0) sSbar[h] = acc * (1.f / kLog2e);
-    }
-    // moment rows: f_hat_E[h][row] = mu_v[row] + scale * sum_c C'[row][c] q_h[c]
-    if (a.order == 1) {
-      const float tau = a.tau;
-      const float nf = static_cast<float>(n_e);
-      for (int base = r0 + warp; base < r1; base += 4 * RB) {
-        if (base != r0 + warp) {  // rows beyond the first batch (few splits): load now
-#pragma unroll
-          for (int k = 0; k < RB; ++k) {
-            const int row = base + 4 * k;
-            if (row < r1) {
-              const float* Crow = a.C + ((size_t)u * D + row) * D + lane * DPL;
-#pragma unroll
-              for (int i = 0; i < DPL; ++i) cv[k][i] = __ldg(Crow + i);
-              mvr[k] = __ldg(a.mu_v + (size_t)u * D + row);
-            }
-          }
+      for (int j = 0; j < kPairs; ++j) {
+        const int idx = tid + j * kThreads;
+        if (idx < n_pairs) {
+          const int rr = idx / G, h = idx % G;
+          const float* fp = &sFp[rr >> 4][0][rr & 15][h];
+          const float cq = fp[0] + fp[16 * 8] + fp[2 * 16 * 8] + fp[3 * 16 * 8];
+          fdst[h * D + r0 + rr] = muv_pre[j] + scale * cq;
         }
+      }
+    } else {
+      const int g = lane >> 2, t = lane & 3;
+      for (int mt = warp; mt < n_mt; mt += 4) {
+        const int ra = r0 + mt * 16 + g, rb = ra + 8;
+        const bool va = ra < r1, vb = rb < r1;
+        float2 f[D / 16][4];
 #pragma unroll
-        for (int k = 0; k < RB; ++k) {
-          const int row = base + 4 * k;
-          if (row >= r1) break;  // warp-uniform
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const float* Ca = a.C + ((size_t)u * D + ra) * D + kk * 16 + 2 * t;
+          const float* Cb = a.C + ((size_t)u * D + rb) * D + kk * 16 + 2 * t;
+          f[kk][0] = va ? __ldg(reinterpret_cast<const float2*>(Ca)) : make_float2(0.f, 0.f);
+          f[kk][1] = vb ? __ldg(reinterpret_cast<const float2*>(Cb)) : make_float2(0.f, 0.f);
+          f[kk][2] = va ? __ldg(reinterpret_cast<const float2*>(Ca + 8)) : make_float2(0.f, 0.f);
+          f[kk][3] = vb ? __ldg(reinterpret_cast<const float2*>(Cb + 8)) : make_float2(0.f, 0.f);
+        }
+        const float mva = va ? __ldg(a.mu_v + (size_t)u * D + ra) : 0.f;
+        const float mvb = vb ? __ldg(a.mu_v + (size_t)u * D + rb) : 0.f;
+        float d[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-          for (int i = 0; i < DPL; ++i) cv[k][i] = (fabsf(cv[k][i] * nf) < tau) ? 0.f : cv[k][i];
-          float acc[G];
-#pragma unroll
-          for (int h = 0; h < G; ++h) {
-            acc[h] = 0.f;
-#pragma unroll
-            for (int i = 0; i < DPL; ++i) acc[h] = fmaf(cv[k][i], sQ[h * D + lane * DPL + i], acc[h]);
-            acc[h] = warp_sum(acc[h]);
-          }
-          if (lane == 0) {
-            float* fdst = CL ? fr0 + row : a.fhat + (size_t)u * G * D + row;
-#pragma unroll
-            for (int h = 0; h < G; ++h) fdst[h * D] = mvr[k] + acc[h] * (1.f / kLog2e);
-          }
+        for (int kk = 0; kk < D / 16; ++kk) mma_c(d, f[kk], kk);
+        // lane holds rows (g, g + 8) x heads (2t, 2t + 1)
+        if (2 * t < G) {
+          if (va) fdst[(2 * t) * D + ra] = mva + scale * d[0];
+          if (vb) fdst[(2 * t) * D + rb] = mvb + scale * d[2];
+        }
+        if (2 * t + 1 < G) {
+          if (va) fdst[(2 * t + 1) * D + ra] = mva + scale * d[1];
+          if (vb) fdst[(2 * t + 1) * D + rb] = mvb + scale * d[3];
         }
       }
     }
@@ -510,8 +581,8 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
       if (len0 + 1 > a.cap) {
         record_error(a.ws, MKV_ERR_CAPACITY, u);
       } else {
-        a.pos[(size_t)u * a.cap + len0] = a.seen[u];
-        a.seen[u] = a.seen[u] + 1;
+        a.pos[(size_t)u * a.cap + len0] = seen0;
+        a.seen[u] = seen0 + 1;
         a.len[u] = len0 + 1;
       }
     }

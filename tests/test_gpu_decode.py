@@ -70,6 +70,8 @@ CASES = [
     (2, 8, 4, 128, None, 640, None),
     (1, 4, 8, 128, [513, 1, 32, 33], 600, [10, 0, 1, 1000]),
     (3, 2, 1, 64, [31, 64, 65, 200, 7, 129], 256, [0, 5, 9, 100, 2, 40]),
+    # 320 units: one split per unit, so each CTA computes all 64 moment rows
+    (40, 8, 2, 64, None, 96, None),
 ]
 
 
