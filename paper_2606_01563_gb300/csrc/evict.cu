@@ -977,6 +977,34 @@ __device__ __forceinline__ void warp_sum_n(float (&v)[N]) {
     for (int i = 0; i < N; ++i) v[i] += __shfl_xor_sync(kFull, v[i], o);
 }
 
+// One round of a transposing butterfly: lanes with bit o set keep the upper
+// W values, the others the lower W, and each adds its partner's copy.
+template <int W>
+__device__ __forceinline__ void tsum_round(float* v, int lane, int o) {
+  const bool hi = (lane & o) != 0;
+#pragma unroll
+  for (int i = 0; i < W; ++i) {
+    const float send = hi ? v[i] : v[i + W];
+    const float keep = hi ? v[i + W] : v[i];
+    v[i] = keep + __shfl_xor_sync(kFull, send, o);
+  }
+}
+
+// Warp sums of P (8 or 16) values per lane in P - 1 + 5 - log2(P) shuffles:
+// returns, in every lane, the sum over the warp of v[lane >> (5 - log2 P)].
+template <int P>
+__device__ __forceinline__ float transpose_sum(float (&v)[P], int lane) {
+  static_assert(P == 8 || P == 16, "8 or 16 values");
+  if constexpr (P == 16) tsum_round<8>(v, lane, 16);
+  tsum_round<4>(v, lane, P == 16 ? 8 : 16);
+  tsum_round<2>(v, lane, P == 16 ? 4 : 8);
+  tsum_round<1>(v, lane, P == 16 ? 2 : 4);
+  float r = v[0];
+#pragma unroll
+  for (int o = (P == 16 ? 1 : 2); o >= 1; o >>= 1) r += __shfl_xor_sync(kFull, r, o);
+  return r;
+}
+
 template <int N>
 __device__ __forceinline__ float select_n(const float (&v)[N], int i) {
   float r = v[0];
@@ -1003,8 +1031,6 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
   __shared__ __align__(16) float s_q[G][D];
   __shared__ float s_red[kRW][G];
   __shared__ double s_zpart[kRW][G];
-  __shared__ double s_zd[kRW][G];  // per warp (lane 0): normaliser Z_h, decremented per eviction
-  __shared__ float s_invZ[kRW][G];
   __shared__ float s_M[G];
   __shared__ unsigned long long s_best[2];
   __shared__ unsigned long long mail_key[2][kCL];
@@ -1157,11 +1183,25 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
     for (int jj = len + tid; jj < a.cap; jj += kRT) alive_all[jj] = 0;
   }
   __syncthreads();
-  if (lane < G) {  // every warp sums the partials in the same order: identical Z_h
+  // Z_h lives in lane h < G of every warp as a compensated (Kahan) float,
+  // decremented per eviction: value zf - zc.  Every warp sums the partials in
+  // the same order, so all hold identical values.
+  constexpr int P = RPW <= 8 ? 8 : 16;       // padded row count of the transposing sums
+  constexpr int SH = P == 8 ? 2 : 1;         // lane l scores row l >> SH
+  float zf = 1.f, zc = 0.f, zinv = 1.f;
+  if (lane < G) {
     double z = 0.0;
     for (int w = 0; w < kRW; ++w) z += s_zpart[w][lane];
-    s_zd[warp][lane] = z;
-    s_invZ[warp][lane] = 1.f / static_cast<float>(z);
+    zf = static_cast<float>(z);
+    zc = static_cast<float>(static_cast<double>(zf) - z);
+    zinv = 1.f / zf;
+  }
+  // e_hj of the row this lane scores
+  float ereg[G];
+  {
+    const int i = lane >> SH, r = warp + kRW * i;
+#pragma unroll
+    for (int h = 0; h < G; ++h) ereg[h] = (i < RPW && r < nr) ? lg[h * a.cap + j0 + r] : 0.f;
   }
 
   // ---- registers: y_j = C k_j of the warp's rows, the thread's share of C, means
@@ -1268,11 +1308,16 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
           for (int d = 0; d < DPL; ++d) part[i] = fmaf(sdk[d], kf[d], part[i]);
         }
       }
-      warp_sum_n<RPW>(part);
+      float pv[P];
 #pragma unroll
-      for (int i = 0; i < RPW; ++i)
+      for (int i = 0; i < P; ++i) pv[i] = i < RPW ? part[i] : 0.f;
+      const float dsum = transpose_sum<P>(pv, lane);
 #pragma unroll
-        for (int d = 0; d < DPL; ++d) y[i][d] = fmaf(keep, y[i][d], part[i] * sdv[d]);
+      for (int i = 0; i < RPW; ++i) {
+        const float dot = __shfl_sync(kFull, dsum, i << SH);
+#pragma unroll
+        for (int d = 0; d < DPL; ++d) y[i][d] = fmaf(keep, y[i][d], dot * sdv[d]);
+      }
     }
 #pragma unroll
     for (int i = 0; i < RPW; ++i) {
@@ -1287,24 +1332,32 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
         }
       }
     }
-    warp_sum_n<RPW>(part);
+    // residual norms reduced so that lane l holds row l >> SH's; those lanes
+    // score their row, and the warp's minimum key goes to the block minimum
     auto post_keys = [&](const float (&ss)[RPW]) {
-      if (lane == 0) {
-        unsigned long long best = ~0ull;
+      float pv[P];
 #pragma unroll
-        for (int i = 0; i < RPW; ++i)
-          if ((alive >> i) & 1u) {
-            const int r = warp + kRW * i;
-            float alpha = 0.f;
+      for (int i = 0; i < P; ++i) pv[i] = i < RPW ? ss[i] : 0.f;
+      const float sum = transpose_sum<P>(pv, lane);
+      float invz[G];
 #pragma unroll
-            for (int h = 0; h < G; ++h) alpha = fmaf(lg[h * a.cap + j0 + r], s_invZ[warp][h], alpha);
-            const float score = alpha * sqrtf(ss[i]);
-            const unsigned long long key =
-                (static_cast<unsigned long long>(__float_as_uint(score)) << 32) | static_cast<unsigned>(j0 + r);
-            best = key < best ? key : best;
-          }
-        if (best != ~0ull) atomicMin(&s_best[par], best);
+      for (int h = 0; h < G; ++h) invz[h] = __shfl_sync(kFull, zinv, h);
+      const int i = lane >> SH;
+      unsigned long long key = ~0ull;
+      if ((lane & ((1 << SH) - 1)) == 0 && i < RPW && ((alive >> i) & 1u)) {
+        float alpha = 0.f;
+#pragma unroll
+        for (int h = 0; h < G; ++h) alpha = fmaf(ereg[h], invz[h], alpha);
+        const float score = alpha * sqrtf(sum);
+        key = (static_cast<unsigned long long>(__float_as_uint(score)) << 32) |
+              static_cast<unsigned>(j0 + warp + kRW * i);
       }
+#pragma unroll
+      for (int o = 16; o >= (1 << SH); o >>= 1) {
+        const unsigned long long k2 = __shfl_xor_sync(kFull, key, o);
+        key = k2 < key ? k2 : key;
+      }
+      if (lane == 0 && key != ~0ull) atomicMin(&s_best[par], key);
     };
     post_keys(part);
     __syncthreads();
@@ -1356,7 +1409,6 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
           }
         }
       }
-      warp_sum_n<RPW>(part);
       post_keys(part);
       __syncthreads();
       if (tid == 0) s_nz = 0;  // every reader of the list is past the barrier above
@@ -1414,12 +1466,13 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
     }
     const int jr = js - j0;
     if (jr >= 0 && jr < nr && jr % kRW == warp) alive &= ~(1u << (jr / kRW));
-    if (lane < G) {
-      const double z = s_zd[warp][lane] - static_cast<double>(lg[lane * a.cap + js]);
-      s_zd[warp][lane] = z;
-      s_invZ[warp][lane] = 1.f / static_cast<float>(z);
+    if (lane < G) {  // compensated Z_h -= e_h,js
+      const float yk = -lg[lane * a.cap + js] - zc;
+      const float tk = zf + yk;
+      zc = (tk - zf) - yk;
+      zf = tk;
+      zinv = 1.f / zf;
     }
-    __syncwarp();
   }
 
   // ---- state back to shared memory: survivors, C (transposed), means
