@@ -1204,7 +1204,12 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
     for (int h = 0; h < G; ++h) ereg[h] = (i < RPW && r < nr) ? lg[h * a.cap + j0 + r] : 0.f;
   }
 
-  // ---- registers: y_j = C k_j of the warp's rows, the thread's share of C, means
+  // ---- registers, in the raw co-moment form S_tilde = n C (Eq. app_S_tilde):
+  // y_j = S_tilde k_j of the warp's rows, the thread's share of S_tilde, the
+  // means.  A Welford fold then adds (k - mu_k)(v - mu_v')^T to S_tilde and
+  // ((k - mu_k) . k_j)(v - mu_v') to y_j: one FMA per element, and the clamp
+  // test is |S_tilde_ab| < tau with no scaling.
+  const float nf0 = static_cast<float>(n);
   float y[RPW][DPL];
   unsigned alive = 0u;
 #pragma unroll
@@ -1227,10 +1232,18 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
         }
       }
     }
+#pragma unroll
+    for (int i = 0; i < RPW; ++i)
+#pragma unroll
+      for (int d = 0; d < DPL; ++d) y[i][d] *= nf0;
   }
   float creg[CJ][DPL];
 #pragma unroll
-  for (int jj = 0; jj < CJ; ++jj) ld_vec<DPL>(Ct + (size_t)(warp + kRW * jj) * D + lane * DPL, creg[jj]);
+  for (int jj = 0; jj < CJ; ++jj) {
+    ld_vec<DPL>(Ct + (size_t)(warp + kRW * jj) * D + lane * DPL, creg[jj]);
+#pragma unroll
+    for (int d = 0; d < DPL; ++d) creg[jj][d] *= nf0;
+  }
   float mk[DPL], mv[DPL], sdk[DPL], sdv[DPL];
 #pragma unroll
   for (int d = 0; d < DPL; ++d) {
@@ -1238,16 +1251,15 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
     mv[d] = s_mu_v[lane * DPL + d];
     sdk[d] = sdv[d] = 0.f;
   }
-  // clamp list of the initial moments: entries with 0 < |n C_ab| < tau
+  // clamp list of the initial moments: entries with 0 < |S_tilde_ab| < tau
   const float tau = a.tau;
   if (n > 0 && tau > 0.f) {
-    const float nf = static_cast<float>(n);
 #pragma unroll
     for (int jj = 0; jj < CJ; ++jj)
 #pragma unroll
       for (int d = 0; d < DPL; ++d) {
         const float v = creg[jj][d];
-        if (v != 0.f && fabsf(v * nf) < tau) {
+        if (v != 0.f && fabsf(v) < tau) {
           const int k = atomicAdd(&s_nz, 1);
           if (k < kMaxClamp) {
             s_zidx[k] = static_cast<uint32_t>((warp + kRW * jj) * D + lane * DPL + d);
@@ -1259,14 +1271,11 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
   __syncthreads();
 
   const int n_evict = len - a.budget;
-  float keep = 1.f;
   for (int e = 0;; ++e) {
     const int par = e & 1;
-    // ---- fold the previous eviction into this thread's share of C and build
-    // the clamp list: C' = keep C + dk dv^T (dk scaled by 1/n)
+    // ---- fold the previous eviction into this thread's share of S_tilde and
+    // build the clamp list: S_tilde' = S_tilde + dk dv^T
     if (e > 0) {
-      const float nf = static_cast<float>(n);
-      const float thr = tau / nf;  // |C_ab| < tau / n  <=>  |n C_ab| < tau
       const float mydk = select_n<DPL>(sdk, warp % DPL);
 #pragma unroll
       for (int jj = 0; jj < CJ; ++jj) {
@@ -1275,13 +1284,13 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
         bool any = false;
 #pragma unroll
         for (int d = 0; d < DPL; ++d) {
-          creg[jj][d] = fmaf(keep, creg[jj][d], kd * sdv[d]);
-          any |= fabsf(creg[jj][d]) < thr;
+          creg[jj][d] = fmaf(kd, sdv[d], creg[jj][d]);
+          any |= fabsf(creg[jj][d]) < tau;
         }
         if (any) {
 #pragma unroll
           for (int d = 0; d < DPL; ++d)
-            if (creg[jj][d] != 0.f && fabsf(creg[jj][d] * nf) < tau) {
+            if (creg[jj][d] != 0.f && fabsf(creg[jj][d]) < tau) {
               const int slot = atomicAdd(&s_nz, 1);
               if (slot < kMaxClamp) {
                 s_zidx[slot] = static_cast<uint32_t>(c * D + lane * DPL + d);
@@ -1294,8 +1303,9 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
     if (e == n_evict) break;  // uniform over the cluster
     if (tid == 0) s_best[par ^ 1] = ~0ull;  // its readers finished one iteration ago
 
-    // ---- y_j' = keep y_j + (dk . k_j) dv, then the residual norms of the warp's rows
-    const float rs = (n > 0) ? scale : 0.f;
+    // ---- y_j' = y_j + (dk . k_j) dv, then the residual norms of the warp's
+    // rows: r_j = v_j - mu_v - (scale / n) y_j
+    const float rs = (n > 0) ? scale / static_cast<float>(n) : 0.f;
     float part[RPW];
     if (e > 0) {
 #pragma unroll
@@ -1316,7 +1326,7 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
       for (int i = 0; i < RPW; ++i) {
         const float dot = __shfl_sync(kFull, dsum, i << SH);
 #pragma unroll
-        for (int d = 0; d < DPL; ++d) y[i][d] = fmaf(keep, y[i][d], dot * sdv[d]);
+        for (int d = 0; d < DPL; ++d) y[i][d] = fmaf(dot, sdv[d], y[i][d]);
       }
     }
 #pragma unroll
@@ -1370,7 +1380,6 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
         for (int jj = 0; jj < CJ; ++jj) st_vec<DPL>(Ct + (size_t)(warp + kRW * jj) * D + lane * DPL, creg[jj]);
       }
       __syncthreads();
-      const float nf = static_cast<float>(n);
 #pragma unroll
       for (int i = 0; i < RPW; ++i) {
         part[i] = 0.f;
@@ -1380,7 +1389,7 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
           if (!direct) {
 #pragma unroll
             for (int d = 0; d < DPL; ++d) yc[d] = y[i][d];
-            for (int z = 0; z < nz; ++z) {  // y'_a -= C_ab k_b for clamped (a, b)
+            for (int z = 0; z < nz; ++z) {  // y'_a -= S_tilde_ab k_b for clamped (a, b)
               const int kb = static_cast<int>(s_zidx[z] / D), va = static_cast<int>(s_zidx[z] % D);
               if (va / DPL == lane) {
                 const float corr = s_zval[z] * __bfloat162float(Kr[(size_t)r * D + kb]);
@@ -1397,7 +1406,7 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
               float cv[DPL];
               ld_vec<DPL>(Ct + (size_t)c * D + lane * DPL, cv);
 #pragma unroll
-              for (int d = 0; d < DPL; ++d) yc[d] = fmaf((fabsf(cv[d] * nf) < tau) ? 0.f : cv[d], kv, yc[d]);
+              for (int d = 0; d < DPL; ++d) yc[d] = fmaf((fabsf(cv[d]) < tau) ? 0.f : cv[d], kv, yc[d]);
             }
           }
           float vf[DPL];
@@ -1450,7 +1459,6 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
     // Welford fold of the evicted row for this lane's dims (Eq. app_update)
     {
       const float inv = 1.f / static_cast<float>(n + 1);
-      keep = static_cast<float>(n) * inv;
       float kx[DPL], vx[DPL];
       load_bf16<DPL>(&mail_row[par][src][lane * DPL], kx);
       load_bf16<DPL>(&mail_row[par][src][D + lane * DPL], vx);
@@ -1459,7 +1467,7 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
         const float dk = kx[d] - mk[d];
         mk[d] = fmaf(dk, inv, mk[d]);
         mv[d] = fmaf(vx[d] - mv[d], inv, mv[d]);
-        sdk[d] = dk * inv;  // scaled by 1/(n+1) for the rank-1 terms
+        sdk[d] = dk;
         sdv[d] = vx[d] - mv[d];
       }
       n += 1;
@@ -1480,7 +1488,12 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
   for (int i = 0; i < RPW; ++i)
     if (lane == 0 && warp + kRW * i < nr) alive_all[j0 + warp + kRW * i] = (alive >> i) & 1u;
 #pragma unroll
-  for (int jj = 0; jj < CJ; ++jj) st_vec<DPL>(Ct + (size_t)(warp + kRW * jj) * D + lane * DPL, creg[jj]);
+  for (int jj = 0; jj < CJ; ++jj) {
+    float cv[DPL];
+#pragma unroll
+    for (int d = 0; d < DPL; ++d) cv[d] = n > 0 ? creg[jj][d] / static_cast<float>(n) : 0.f;
+    st_vec<DPL>(Ct + (size_t)(warp + kRW * jj) * D + lane * DPL, cv);
+  }
   if (warp == 0) {
 #pragma unroll
     for (int d = 0; d < DPL; ++d) {
