@@ -710,6 +710,34 @@ __device__ __forceinline__ int block_excl_scan(int flag, int* wsum, int* total) 
   return r;
 }
 
+// Exclusive block-wide prefix sum of one int per thread; *total gets the sum.
+__device__ __forceinline__ int block_excl_sum(int v, int* wsum, int* total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(kFull, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) wsum[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    const int w = lane < (int)(blockDim.x >> 5) ? wsum[lane] : 0;
+    int xw = w;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(kFull, xw, o);
+      if (lane >= o) xw += y;
+    }
+    wsum[lane] = xw - w;
+    if (lane == 31) *total = xw;
+  }
+  __syncthreads();
+  const int r = wsum[warp] + x - v;
+  __syncthreads();  // wsum is reused by the next call
+  return r;
+}
+
 struct SelectArgs {
   const float* scores;  // [units][T]
   int T, W, B, sink, keep_window, D;
@@ -723,9 +751,12 @@ struct SelectArgs {
   int32_t* dst_pos;  // optional cache bookkeeping
   int32_t* dst_len;
   int32_t* dst_seen;
+  int smem_keys;  // keys of a CTA's range that the dynamic shared memory holds
 };
 
+constexpr int kFinRB = 2;  // rows of C per finalize CTA
 constexpr int kSelCL = 8;  // CTAs per unit (one cluster), each over a contiguous range of positions
+constexpr int kSelSmemKeys = 24576;  // keys of a CTA's range cached in shared memory (96 KB)
 
 __global__ void __cluster_dims__(kSelCL, 1, 1) __launch_bounds__(kSelThreads) select_kernel(const SelectArgs a) {
   __shared__ uint32_t hist[2][256];   // this CTA's histogram, double-buffered by pass parity (read remotely)
@@ -746,6 +777,27 @@ __global__ void __cluster_dims__(kSelCL, 1, 1) __launch_bounds__(kSelThreads) se
   const float* sc = a.scores + (size_t)u * T;
   const int k = a.B - protected_count(T, W, a.sink, a.keep_window);  // >= 0 (validated), < candidates
 
+  // The CTA's keys are cached in shared memory when they fit (protected
+  // positions hold key 0, which no score maps to: scores are >= 0); larger
+  // ranges are read from global memory on every pass.
+  extern __shared__ uint32_t ks[];
+  const int nk = r1 - r0;
+  const bool cached = nk <= a.smem_keys;
+  auto key_at = [&](int t) -> uint32_t {  // 0 for protected positions
+    if (cached) return ks[t - r0];
+    return is_protected(t, T, W, a.sink, a.keep_window) ? 0u : float_key(sc[t]);
+  };
+  if (cached) {
+    for (int i = tid; i < nk; i += kSelThreads) {
+      const int t = r0 + i;
+      ks[i] = is_protected(t, T, W, a.sink, a.keep_window) ? 0u : float_key(sc[t]);
+    }
+    __syncthreads();
+  }
+  // thread tid owns the contiguous positions [t0, t1) in the ordered passes
+  const int E = (nk + kSelThreads - 1) / kSelThreads;
+  const int t0 = min(r1, r0 + tid * E), t1 = min(r1, t0 + E);
+
   uint32_t prefix = 0, pmask = 0;
   int need = k;
   if (k > 0) {
@@ -754,10 +806,10 @@ __global__ void __cluster_dims__(kSelCL, 1, 1) __launch_bounds__(kSelThreads) se
       for (int i = tid; i < 8 * 256; i += kSelThreads) (&whist[0][0])[i] = 0;
       __syncthreads();
       uint32_t* wh = whist[warp & 7];
-      for (int t = r0 + tid; t < r1; t += kSelThreads) {
-        if (is_protected(t, T, W, a.sink, a.keep_window)) continue;
-        const uint32_t key = float_key(sc[t]);
-        if ((key & pmask) == prefix) atomicAdd(&wh[(key >> shift) & 255u], 1u);
+#pragma unroll 4
+      for (int i = tid; i < nk; i += kSelThreads) {
+        const uint32_t key = key_at(r0 + i);
+        if (key != 0u && (key & pmask) == prefix) atomicAdd(&wh[(key >> shift) & 255u], 1u);
       }
       __syncthreads();
       for (int i = tid; i < 256; i += kSelThreads) {
@@ -804,43 +856,23 @@ __global__ void __cluster_dims__(kSelCL, 1, 1) __launch_bounds__(kSelThreads) se
       pmask |= 255u << shift;
     }
   }
-  // counts of this CTA's range, exchanged to place its outputs in ascending order
-  {
-    int n_tie = 0, n_sure = 0;
-    for (int t = r0 + tid; t < r1; t += kSelThreads) {
-      const bool prot = is_protected(t, T, W, a.sink, a.keep_window);
-      if (prot) {
-        ++n_sure;
-      } else if (k > 0) {
-        const uint32_t key = float_key(sc[t]);
-        n_sure += key > prefix;
-        n_tie += key == prefix;
-      }
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      n_tie += __shfl_xor_sync(kFull, n_tie, o);
-      n_sure += __shfl_xor_sync(kFull, n_sure, o);
-    }
-    if (lane == 0) {
-      wsum[warp] = n_tie;
-      if (warp == 0) tot = 0;
-    }
-    __syncthreads();
-    if (tid == 0) {
-      int tt = 0;
-      for (int w = 0; w < kSelThreads / 32; ++w) tt += wsum[w];
-      ex_cnt[0] = tt;
-    }
-    __syncthreads();
-    if (lane == 0) wsum[warp] = n_sure;
-    __syncthreads();
-    if (tid == 0) {
-      int ss = 0;
-      for (int w = 0; w < kSelThreads / 32; ++w) ss += wsum[w];
-      ex_cnt[1] = ss;
+  // per-thread counts: protected or above the threshold key (certain), and
+  // ties with it; scanned over the block, then over the cluster's ranks
+  int n_tie = 0, n_sure = 0;
+  for (int t = t0; t < t1; ++t) {
+    const uint32_t key = key_at(t);
+    if (key == 0u) {
+      ++n_sure;  // protected
+    } else if (k > 0) {
+      n_sure += key > prefix ? 1 : 0;
+      n_tie += key == prefix ? 1 : 0;
     }
   }
+  const int tie_excl = block_excl_sum(n_tie, wsum, &tot);
+  if (tid == 0) ex_cnt[0] = tot;
+  const int sure_excl = block_excl_sum(n_sure, wsum, &tot);
+  if (tid == 0) ex_cnt[1] = tot;
+  (void)sure_excl;
   cluster.sync();
   if (tid == 0) {
     int ties_before = 0, sel_before = 0;
@@ -855,35 +887,31 @@ __global__ void __cluster_dims__(kSelCL, 1, 1) __launch_bounds__(kSelThreads) se
     s_before[1] = sel_before;
   }
   __syncthreads();
-  int ties_before = s_before[0], sel_before = s_before[1];
-  const int my_first = sel_before;
+  const int cta_ties_before = s_before[0], cta_sel_before = s_before[1];
+  // this thread's selections: its certain ones and the ties that still fit
+  int tb = cta_ties_before + tie_excl;
+  const int my_sel = n_sure + min(max(need - tb, 0), n_tie);
+  const int sel_excl = block_excl_sum(my_sel, wsum, &tot);
+  const int my_first = cta_sel_before;
+  int o = cta_sel_before + sel_excl;
   int32_t* out = a.idx + (size_t)u * a.B;
-  for (int base = r0; base < r1; base += kSelThreads) {
-    const int t = base + tid;
-    bool prot = false, tie = false, gt = false;
-    if (t < r1) {
-      prot = is_protected(t, T, W, a.sink, a.keep_window);
-      if (!prot && k > 0) {
-        const uint32_t key = float_key(sc[t]);
-        gt = key > prefix;
-        tie = key == prefix;
-      }
+  for (int t = t0; t < t1; ++t) {
+    const uint32_t key = key_at(t);
+    bool sel = true;  // protected
+    if (key != 0u) {
+      const bool tie = k > 0 && key == prefix;
+      sel = (k > 0 && key > prefix) || (tie && tb < need);
+      tb += tie ? 1 : 0;
     }
-    const int tr = block_excl_scan(tie ? 1 : 0, wsum, &tot);
-    const int tie_total = tot;
-    const bool sel = prot || gt || (tie && ties_before + tr < need);
-    const int sr = block_excl_scan(sel ? 1 : 0, wsum, &tot);
-    const int sel_total = tot;
     if (sel) {
-      const int o = sel_before + sr;
       if (o < a.B) {
         out[o] = t;
         if (a.diag_idx) a.diag_idx[(size_t)u * a.B + o] = t;
       }
+      ++o;
     }
-    ties_before += tie_total;
-    sel_before += sel_total;
   }
+  const int sel_before = cta_sel_before + tot;  // this CTA's selections end here
   __syncthreads();
   // gather the rows this CTA selected (16-byte chunks)
   const int D = a.D;
@@ -907,89 +935,102 @@ __global__ void __cluster_dims__(kSelCL, 1, 1) __launch_bounds__(kSelThreads) se
 }
 
 // --------------------------------------------------------------- finalize
-// Moments of E = all \ R for 8 value dims (rows of C) per CTA: the all-token
-// co-moment is the multi-way Chan merge of the chunk records; R's centred
-// record is removed with the reverse pairwise formula.
-// merge_all = 1: merge the chunk records and keep the result in L.mall;
-// merge_all = 0: start from L.mall (a single record).
+// Moments of E = all \ R for kFinRB value dims (rows of C) per CTA.  Each
+// set's co-moment is the multi-way Chan merge of its chunk records, taken
+// about the first chunk's means x0 so that no global mean is needed first:
+//   M = sum_ch [M_ch + n_ch d_ch d_ch^T] - n dbar dbar^T,  d_ch = mu_ch - x0,
+//   dbar = sum_ch n_ch d_ch / n,  mu = x0 + dbar.
+// R's centred record is then removed with the reverse pairwise formula.
+// merge_all = 1: the all-token set is the chunk records (its merge is kept
+// in L.mall); merge_all = 0: it is L.mall itself.
 __global__ void __launch_bounds__(256) finalize_kernel(const Layout L, float* out_rec, mkv_moments out_mom,
                                                        int final_out, int merge_all) {
-  constexpr int NT = 256, RB = 8;
-  __shared__ float mk[kDP], mv[kDP], mkR[kDP], mvR[kDP];
-  __shared__ float s_n;
+  constexpr int NT = 256, RB = kFinRB, CHB = 32;
+  __shared__ float s_nc[CHB], s_dv[CHB][RB], s_dk[CHB][kDP];
+  __shared__ float s_x0v[RB], s_x0k[kDP];
   const int D = L.D;
   const int rb = blockIdx.x, u = blockIdx.y, tid = threadIdx.x;
   const size_t rf = rec_floats(D);
+  const int ar = tid / D, c = tid % D;  // this thread's element (row rb*RB + ar, column c)
+  const bool act = tid < RB * D;
+  const int row = rb * RB + ar;
+
+  struct Set {
+    float n, sv, sk, M;
+  };
+  // merge n_ch records starting at rbase for this thread's element
+  auto merge = [&](const float* rbase, int n_ch, float& x0v, float& x0k) -> Set {
+    Set st{0.f, 0.f, 0.f, 0.f};
+    __syncthreads();
+    if (tid < RB) s_x0v[tid] = rbase[4 + D + rb * RB + tid];
+    for (int i = tid; i < D; i += NT) s_x0k[i] = rbase[4 + i];
+    __syncthreads();
+    x0v = act ? s_x0v[ar] : 0.f;
+    x0k = s_x0k[act ? c : 0];
+    for (int g0 = 0; g0 < n_ch; g0 += CHB) {
+      const int nb = min(CHB, n_ch - g0);
+      if (g0 > 0) __syncthreads();
+      for (int i = tid; i < nb * (1 + RB + D); i += NT) {
+        const int ch = i / (1 + RB + D), j = i % (1 + RB + D);
+        const float* r = rbase + (size_t)(g0 + ch) * rf;
+        if (j == 0) s_nc[ch] = r[0];
+        else if (j <= RB) s_dv[ch][j - 1] = r[4 + D + rb * RB + j - 1] - s_x0v[j - 1];
+        else s_dk[ch][j - 1 - RB] = r[4 + (j - 1 - RB)] - s_x0k[j - 1 - RB];
+      }
+      __syncthreads();
+      if (act) {
+#pragma unroll 8
+        for (int ch = 0; ch < nb; ++ch) {
+          const float nc = s_nc[ch];
+          const float m = rbase[(size_t)(g0 + ch) * rf + 4 + 2 * D + (size_t)row * D + c];
+          if (nc > 0.f) {
+            const float dv = s_dv[ch][ar], dk = s_dk[ch][c];
+            st.n += nc;
+            st.sv = fmaf(nc, dv, st.sv);
+            st.sk = fmaf(nc, dk, st.sk);
+            st.M += m + nc * dv * dk;
+          }
+        }
+      }
+    }
+    return st;
+  };
   const int n_rec = merge_all ? L.n_chunks : 1;
   const float* recs = merge_all ? L.mpart + (size_t)u * L.n_chunks * rf : L.mall + (size_t)u * rf;
-  float* mall = L.mall + (size_t)u * rf;
-  const float* rrecs = L.rpart + (size_t)u * L.n_rchunks * rf;
-  if (tid < 2 * D) {
-    float num = 0.f, n = 0.f;
-    for (int c = 0; c < n_rec; ++c) {
-      const float nc = recs[(size_t)c * rf];
-      n += nc;
-      num += nc * recs[(size_t)c * rf + 4 + tid];
-    }
-    if (tid < D) mk[tid] = num / n;
-    else mv[tid - D] = num / n;
-    if (tid == 0) s_n = n;
-    if (merge_all && rb == 0) {
-      mall[4 + tid] = num / n;
-      if (tid == 0) mall[0] = n;
-    }
+  float x0v, x0k, x0vR, x0kR;
+  const Set A = merge(recs, n_rec, x0v, x0k);
+  const Set R = merge(L.rpart + (size_t)u * L.n_rchunks * rf, L.n_rchunks, x0vR, x0kR);
+  if (!act) return;
+  const float n = A.n, nR = R.n, nE = n - nR;
+  const float mv = x0v + A.sv / n, mk = x0k + A.sk / n;
+  const float M = A.M - A.sv * A.sk / n;
+  const float mvR = nR > 0.f ? x0vR + R.sv / nR : 0.f, mkR = nR > 0.f ? x0kR + R.sk / nR : 0.f;
+  const float MR = nR > 0.f ? R.M - R.sv * R.sk / nR : 0.f;
+  if (merge_all) {
+    float* mall = L.mall + (size_t)u * rf;
+    mall[4 + 2 * D + (size_t)row * D + c] = M;
+    if (rb == 0 && ar == 0) mall[4 + c] = mk;
+    if (c == 0) mall[4 + D + row] = mv;
+    if (rb == 0 && tid == 0) mall[0] = n;
   }
-  __shared__ float s_nR;
-  if (tid < 2 * D) {  // retained set: merge its chunk records' means
-    float num = 0.f, n = 0.f;
-    for (int c = 0; c < L.n_rchunks; ++c) {
-      const float nc = rrecs[(size_t)c * rf];
-      n += nc;
-      num += nc * rrecs[(size_t)c * rf + 4 + tid];
-    }
-    const float mean = n > 0.f ? num / n : 0.f;
-    if (tid < D) mkR[tid] = mean;
-    else mvR[tid - D] = mean;
-    if (tid == 0) s_nR = n;
+  float CE = 0.f, mkE = 0.f, mvE = 0.f;
+  if (nE > 0.f) {
+    mkE = (n * mk - nR * mkR) / nE;
+    mvE = (n * mv - nR * mvR) / nE;
+    const float ME = M - MR - (nE * nR / n) * (mvR - mvE) * (mkR - mkE);
+    CE = ME / nE;
   }
-  __syncthreads();
-  const float n = s_n, nR = s_nR, nE = n - nR;
-  for (int e = tid; e < RB * D; e += NT) {
-    const int ar = rb * RB + e / D, c = e % D;
-    float M = 0.f;
-    for (int ch = 0; ch < n_rec; ++ch) {
-      const float* r = recs + (size_t)ch * rf;
-      const float nc = r[0];
-      if (nc > 0.f) M += r[4 + 2 * D + (size_t)ar * D + c] + nc * (r[4 + D + ar] - mv[ar]) * (r[4 + c] - mk[c]);
-    }
-    if (merge_all) mall[4 + 2 * D + (size_t)ar * D + c] = M;
-    float MR = 0.f;
-    for (int ch = 0; ch < L.n_rchunks; ++ch) {
-      const float* r = rrecs + (size_t)ch * rf;
-      const float nc = r[0];
-      if (nc > 0.f) MR += r[4 + 2 * D + (size_t)ar * D + c] + nc * (r[4 + D + ar] - mvR[ar]) * (r[4 + c] - mkR[c]);
-    }
-    float CE = 0.f, mkE_c = 0.f, mvE_a = 0.f;
-    if (nE > 0.f) {
-      mkE_c = (n * mk[c] - nR * mkR[c]) / nE;
-      mvE_a = (n * mv[ar] - nR * mvR[ar]) / nE;
-      const float ME = M - MR - (nE * nR / n) * (mvR[ar] - mvE_a) * (mkR[c] - mkE_c);
-      CE = ME / nE;
-    }
-    if (final_out) {
-      out_mom.C[((size_t)u * D + ar) * D + c] = CE;
-      if (c == 0) out_mom.mu_v[(size_t)u * D + ar] = mvE_a;
-      if (rb == 0 && e < D) out_mom.mu_k[(size_t)u * D + c] = mkE_c;
-    } else {
-      float* o = out_rec + (size_t)u * rf;
-      o[4 + 2 * D + (size_t)ar * D + c] = CE;
-      if (c == 0) o[4 + D + ar] = mvE_a;
-      if (rb == 0 && e < D) o[4 + c] = mkE_c;
-    }
-  }
-  if (rb == 0 && tid == 0) {
-    if (final_out) out_mom.n[u] = static_cast<int32_t>(nE);
-    else out_rec[(size_t)u * rf] = nE;
+  if (final_out) {
+    out_mom.C[((size_t)u * D + row) * D + c] = CE;
+    if (c == 0) out_mom.mu_v[(size_t)u * D + row] = mvE;
+    if (rb == 0 && ar == 0) out_mom.mu_k[(size_t)u * D + c] = mkE;
+    if (rb == 0 && tid == 0) out_mom.n[u] = static_cast<int32_t>(nE);
+  } else {
+    float* o = out_rec + (size_t)u * rf;
+    o[4 + 2 * D + (size_t)row * D + c] = CE;
+    if (c == 0) o[4 + D + row] = mvE;
+    if (rb == 0 && ar == 0) o[4 + c] = mkE;
+    if (rb == 0 && tid == 0) o[0] = nE;
   }
 }
 
@@ -1090,6 +1131,10 @@ cudaError_t run(const CompressArgs& a, const mkv_geom& g, int num_sms, cudaStrea
   }
 
   SelectArgs sa{};
+  const int sel_per = (T + kSelCL - 1) / kSelCL;
+  sa.smem_keys = sel_per <= kSelSmemKeys ? sel_per : 0;
+  const size_t sel_smem = (size_t)sa.smem_keys * sizeof(uint32_t);
+  if ((e = attr((const void*)select_kernel, sel_smem)) != cudaSuccess) return e;
   sa.T = T;
   sa.W = a.window;
   sa.B = B;
@@ -1112,9 +1157,9 @@ cudaError_t run(const CompressArgs& a, const mkv_geom& g, int num_sms, cudaStrea
     s0.dst_K = L.gK;
     s0.dst_V = L.gV;
     s0.dst_cap = B;
-    select_kernel<<<U * kSelCL, kSelThreads, 0, st>>>(s0);
+    select_kernel<<<U * kSelCL, kSelThreads, sel_smem, st>>>(s0);
     stats_tc<0><<<dim3(L.n_rchunks, U), kTcThreads, kStatsSmem, st>>>(rset, tmGK, tmGV, tmQ);
-    finalize_kernel<<<dim3(D / 8, U), 256, 0, st>>>(L, L.m0, a.mom, 0, 1);
+    finalize_kernel<<<dim3(D / kFinRB, U), 256, 0, st>>>(L, L.m0, a.mom, 0, 1);
     TcArgs r = tp;
     r.n_rows = T;
     r.chunk = L.chunk;
@@ -1134,9 +1179,9 @@ cudaError_t run(const CompressArgs& a, const mkv_geom& g, int num_sms, cudaStrea
   s1.dst_pos = a.cache.pos;
   s1.dst_len = a.cache.len;
   s1.dst_seen = a.cache.seen;
-  select_kernel<<<U * kSelCL, kSelThreads, 0, st>>>(s1);
+  select_kernel<<<U * kSelCL, kSelThreads, sel_smem, st>>>(s1);
   stats_tc<0><<<dim3(L.n_rchunks, U), kTcThreads, kStatsSmem, st>>>(rset, tmCK, tmCV, tmQ);
-  finalize_kernel<<<dim3(D / 8, U), 256, 0, st>>>(L, nullptr, a.mom, 1, a.mi ? 0 : 1);
+  finalize_kernel<<<dim3(D / kFinRB, U), 256, 0, st>>>(L, nullptr, a.mom, 1, a.mi ? 0 : 1);
   return cudaGetLastError();
 }
 
