@@ -46,7 +46,7 @@ EVICT_EVERY = 64
 # dram__bytes_read.sum + dram__bytes_write.sum per launch from one ncu capture
 # of the bench workload (profiles/decode_kernel_llama8b_layer_t8k.md), valid
 # while the kernel source is byte-identical to what was captured
-NCU_TRAFFIC = {"decode": {"bytes": 2960000, "sha": "9fb88b5b9a60089926a38c7edacc56759fb7b7cf27a265b397a7c2a005ea476e"}}
+NCU_TRAFFIC = {"decode": {"bytes": 2956544, "sha": "96f534fad4c4b86f72c6ca4e256ae141cb86bdc91bda7cf9bb256cb93069d783"}}
 
 
 def parse():
