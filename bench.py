@@ -395,7 +395,9 @@ def run_gpu(args):
 
 def decode_sweep(torch, mkv, dev, flush, hbm):
     """Decode throughput cells: batch x budget on the Llama geometry, dense fp32 C,
-    correction on/off; every launch timed alone with L2 flushed before it."""
+    correction on/off.  Each cell is timed two ways: one launch alone with L2
+    flushed before it (graph launch included), and the steady state over many
+    layers' caches (decode_layers)."""
     res = []
     H, G, D = 8, 4, 128
     gen = torch.Generator(device=dev)
@@ -444,8 +446,66 @@ def decode_sweep(torch, mkv, dev, flush, hbm):
                              "frac": round(byt / t / 1e6 / hbm, 4), "tokens_per_s": round(b / (t / 1e3), 1)}
             code, _ = mkv.mkv_get_device_error(ws, st)
             cell["ok"] = code == 0
-            res.append(cell)
             del cache, mom, ws
+            cell.update(decode_layers(torch, mkv, dev, flush, hbm, b, B, gen, st))
+            res.append(cell)
+    return res
+
+
+def decode_layers(torch, mkv, dev, flush, hbm, b, B, gen, st):
+    """Steady-state decode as in a model: one launch per layer, each layer with
+    its own cache and moments, the layers' bytes together at least twice the
+    L2 (so every launch reads HBM), back to back in one CUDA graph; L2 flushed
+    before every replay.  Per-launch time = replay time / layers."""
+    H, G, D = 8, 4, 128
+    g = mkv.geom(b, H, G, D)
+    units = b * H
+    per_layer = units * (B * D * 4 + D * D * 4 + 2 * D * 4 + 4) + b * H * G * D * (2 + 4)
+    layers = int(min(256, max(4, -(-2 * 129 * 2 ** 20 // per_layer))))
+    Kall = torch.randn(layers, b, H, B, D, device=dev, generator=gen).bfloat16()
+    Vall = torch.randn(layers, b, H, B, D, device=dev, generator=gen).bfloat16()
+    Call = 0.05 * torch.randn(layers, b, H, D, D, device=dev, generator=gen)
+    mk = 0.05 * torch.randn(layers, b, H, D, device=dev, generator=gen)
+    mv = 0.05 * torch.randn(layers, b, H, D, device=dev, generator=gen)
+    n = torch.full((layers, b, H), 8192, dtype=torch.int32, device=dev)
+    pos = torch.zeros(b, H, B, dtype=torch.int32, device=dev)
+    lens = torch.full((b, H), B, dtype=torch.int32, device=dev)
+    seen = torch.full((b, H), B, dtype=torch.int32, device=dev)
+    q = torch.randn(b, H * G, D, device=dev, generator=gen).bfloat16()
+    out = torch.empty(b, H * G, D, device=dev)
+    ws = mkv.alloc_workspace(mkv.mkv_decode_workspace_size(g, B), dev)
+    caches = [mkv.Cache(Kall[l], Vall[l], pos, lens, seen) for l in range(layers)]
+    moms = [mkv.Moments(n[l], mk[l], mv[l], Call[l]) for l in range(layers)]
+    res = {}
+    for corr in (1, 0):
+        p = mkv.mkv_decode_params(corr, 1, 1e-6)
+        with torch.cuda.stream(st):
+            for l in range(layers):
+                mkv.mkv_decode_step(g, q, None, None, caches[l], moms[l], p, out, None, ws, st)
+            gr = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gr, stream=st, capture_error_mode="relaxed"):
+            for l in range(layers):
+                mkv.mkv_decode_step(g, q, None, None, caches[l], moms[l], p, out, None, ws, st)
+        times = []
+        for it in range(6):
+            with torch.cuda.stream(st):
+                flush.zero_()
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(st)
+                gr.replay()
+                e1.record(st)
+            st.synchronize()
+            if it >= 2:
+                times.append(e0.elapsed_time(e1) / layers)
+        t = float(np.median(times))
+        byt = units * (B * D * 4 + (D * D * 4 + 2 * D * 4 + 4 if corr else 0)) + b * H * G * D * (2 + 4)
+        res[("corr" if corr else "plain") + "_layers"] = {
+            "us": round(t * 1e3, 2), "gbs": round(byt / t / 1e6, 1), "frac": round(byt / t / 1e6 / hbm, 4),
+            "tokens_per_s": round(b / (t / 1e3), 1), "layers": layers}
+        del gr
+    code, _ = mkv.mkv_get_device_error(ws, st)
+    res["ok_layers"] = code == 0
+    del Kall, Vall, Call, caches, moms
     return res
 
 
