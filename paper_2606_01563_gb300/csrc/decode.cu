@@ -256,6 +256,11 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
       }
     }
   }
+  if (do_c && !split_k && tid == 0 && r1 > r0) {  // whole-tile case: the rows are read after the tiles
+    const float* base = a.C + ((size_t)u * D + r0) * D;
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base), "r"((uint32_t)((r1 - r0) * D * 4))
+                 : "memory");
+  }
   // mu_v of the (row, head) pairs this thread finishes in the two-tile case
   constexpr int kPairs = 2 * 16 * 8 / kThreads;  // at most 32 rows x 8 heads
   float muv_pre[kPairs];
