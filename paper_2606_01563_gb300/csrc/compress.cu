@@ -43,6 +43,9 @@ constexpr int kDP = 128;                    // padded head dim of every MMA
 constexpr int kTileBytes = kTok * kDP * 2;  // one [128 x 128] bf16 tile: 2 boxes of 16 KB
 constexpr int kBoxBytes = kTok * 128;
 constexpr int kTcThreads = 192;  // warp 0 TMA, warp 1 MMA, warps 2..5 epilogue
+// stats_tc: two epilogue groups of 4 warps (2..5 and 6..9), each taking half
+// of a tile's tokens, so that two warps per scheduler share the softmax work
+constexpr int kStatsThreads = 320;
 constexpr int kSelThreads = 1024;
 constexpr int kPF = 0;  // tiles prefetched into L2 ahead of the one being loaded (0: none)
 constexpr unsigned kFull = 0xffffffffu;
@@ -159,7 +162,7 @@ struct TcArgs {
 // LOGITS = 1: window-row statistics and chunk moments of the prompt;
 // LOGITS = 0: moments only (a dense row set).
 template <int LOGITS>
-__global__ void __launch_bounds__(kTcThreads, 1)
+__global__ void __launch_bounds__(kStatsThreads, 1)
     stats_tc(const TcArgs p, const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
              const __grid_constant__ CUtensorMap tmQ) {
   constexpr int kS = 2;
@@ -173,6 +176,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   __shared__ uint32_t tmem_base;
   __shared__ int abort_flag;
   __shared__ float sum_k[kDP], sum_v[kDP];
+  __shared__ float s_m1[2][128], s_l1[2][128];  // the second epilogue group's row stats
 
   const int chunk = blockIdx.x, u = blockIdx.y;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -188,14 +192,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       mbar_init(&empty[i], 1);  // the stage is free once its MMAs have completed
     }
     mbar_init(&lfull, 1);
-    mbar_init(&lempty, 4);
+    mbar_init(&lempty, 8);
     mbar_init(&qfull, 1);
     mbar_init(&sdone, 1);
     abort_flag = 0;
     mbar_fence_init();
   }
   if (warp == 1) tmem_alloc(&tmem_base, 512);
-  if (warp >= 2) {  // the ones operand of the column sums K^T 1 and V^T 1
+  if (warp >= 2 && warp < 6) {  // the ones operand of the column sums K^T 1 and V^T 1
     for (int i = tid - 64; i < 2 * 16 * 128 / 16; i += 128)
       reinterpret_cast<uint4*>(sOnes)[i] = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u);
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -269,8 +273,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       umma_commit(&sdone);
     }
   } else {
-    // ---- epilogue: warps 2..5; TMEM lane quarter qd = warp % 4
-    const int et = tid - 64, qd = warp & 3;
+    // ---- epilogue: group 0 = warps 2..5 (tokens 0..63 of a tile), group 1 =
+    // warps 6..9 (tokens 64..127); TMEM lane quarter qd = warp % 4
+    const int grp = (warp - 2) >> 2;
+    const int et = tid - 64 - grp * 128, qd = warp & 3;
     const uint32_t lane_base = static_cast<uint32_t>(qd * 32) << 16;
     float m[2] = {-INFINITY, -INFINITY}, l[2] = {0.f, 0.f};
     int tmax_vis[2];
@@ -285,7 +291,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       const int tt0 = t_begin + i * kTok;
       const bool fast = tt0 + kTok <= t_end && tt0 + kTok - 1 <= t_safe;  // no masking in this tile
       for (int rb = 0; rb < RWb; ++rb) {
-        for (int c0 = 0; c0 < kTok; c0 += 32) {
+        for (int c0 = grp * 64; c0 < grp * 64 + 64; c0 += 32) {
           float x[32];
           tmem_ld32(tm + lane_base + rb * 128 + c0, x);
           const int t0 = tt0 + c0;
@@ -320,16 +326,31 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(&lempty);
     }
-    if (LOGITS) {
-      for (int rb = 0; rb < RWb; ++rb) {
-        const int r = rb * 128 + qd * 32 + lane;
-        if (r < p.RW) {
-          float* rp = p.rowpart + (((size_t)u * p.n_chunks + chunk) * p.RW + r) * 2;
-          rp[0] = m[rb];
-          rp[1] = l[rb];
+    if (LOGITS) {  // merge the two groups' (max, sum) of each row
+      if (grp == 1)
+        for (int rb = 0; rb < RWb; ++rb) {
+          s_m1[rb][qd * 32 + lane] = m[rb];
+          s_l1[rb][qd * 32 + lane] = l[rb];
         }
-      }
+      asm volatile("bar.sync 2, 256;" ::: "memory");
+      if (grp == 0)
+        for (int rb = 0; rb < RWb; ++rb) {
+          const int r = rb * 128 + qd * 32 + lane;
+          const float m1 = s_m1[rb][qd * 32 + lane], l1 = s_l1[rb][qd * 32 + lane];
+          const float M = fmaxf(m[rb], m1);
+          float L = 0.f;
+          if (M != -INFINITY) {
+            if (m[rb] != -INFINITY) L += l[rb] * fast_exp2(m[rb] - M);
+            if (m1 != -INFINITY) L += l1 * fast_exp2(m1 - M);
+          }
+          if (r < p.RW) {
+            float* rp = p.rowpart + (((size_t)u * p.n_chunks + chunk) * p.RW + r) * 2;
+            rp[0] = M;
+            rp[1] = L;
+          }
+        }
     }
+    if (grp == 0) {
     const bool got = pwait(&sdone, 0, abrt, p.ws, u);
     tc_fence_after();
     {
@@ -358,6 +379,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       rec[4 + p.D + a] = nc > 0.f ? sum_v[a] / nc : 0.f;
     }
     if (et == 0) rec[0] = got ? nc : 0.f;
+    }
   }
   tc_fence_before();
   __syncthreads();
@@ -1118,7 +1140,7 @@ cudaError_t run(const CompressArgs& a, const mkv_geom& g, int num_sms, cudaStrea
     p1.n_chunks = L.n_chunks;
     p1.rowpart = L.rowpart;
     p1.mrec = L.mpart;
-    stats_tc<1><<<cg, kTcThreads, kStatsSmem, st>>>(p1, tmK, tmV, tmQ);
+    stats_tc<1><<<cg, kStatsThreads, kStatsSmem, st>>>(p1, tmK, tmV, tmQ);
     TcArgs p2 = p1;
     p2.s_out = L.s;
     p2.diag = a.diag_scores;
@@ -1158,7 +1180,7 @@ cudaError_t run(const CompressArgs& a, const mkv_geom& g, int num_sms, cudaStrea
     s0.dst_V = L.gV;
     s0.dst_cap = B;
     select_kernel<<<U * kSelCL, kSelThreads, sel_smem, st>>>(s0);
-    stats_tc<0><<<dim3(L.n_rchunks, U), kTcThreads, kStatsSmem, st>>>(rset, tmGK, tmGV, tmQ);
+    stats_tc<0><<<dim3(L.n_rchunks, U), kStatsThreads, kStatsSmem, st>>>(rset, tmGK, tmGV, tmQ);
     finalize_kernel<<<dim3(D / kFinRB, U), 256, 0, st>>>(L, L.m0, a.mom, 0, 1);
     TcArgs r = tp;
     r.n_rows = T;
@@ -1180,7 +1202,7 @@ cudaError_t run(const CompressArgs& a, const mkv_geom& g, int num_sms, cudaStrea
   s1.dst_len = a.cache.len;
   s1.dst_seen = a.cache.seen;
   select_kernel<<<U * kSelCL, kSelThreads, sel_smem, st>>>(s1);
-  stats_tc<0><<<dim3(L.n_rchunks, U), kTcThreads, kStatsSmem, st>>>(rset, tmCK, tmCV, tmQ);
+  stats_tc<0><<<dim3(L.n_rchunks, U), kStatsThreads, kStatsSmem, st>>>(rset, tmCK, tmCV, tmQ);
   finalize_kernel<<<dim3(D / kFinRB, U), 256, 0, st>>>(L, nullptr, a.mom, 1, a.mi ? 0 : 1);
   return cudaGetLastError();
 }
