@@ -390,7 +390,7 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
 }
 
 // -------------------------------------------------------------- scores_tc
-__global__ void __launch_bounds__(kTcThreads, 1)
+__global__ void __launch_bounds__(kStatsThreads, 1)
     scores_tc(const TcArgs p, const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmQ) {
   constexpr int kS = 3;
   extern __shared__ __align__(1024) uint8_t smraw[];
@@ -467,10 +467,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       }
     }
   } else {
-    const int et = tid - 64, qd = warp & 3;
+    // two epilogue groups (warps 2..5 and 6..9) take alternate tiles; group g
+    // always reads TMEM buffer g
+    const int grp = (warp - 2) >> 2, qd = warp & 3;
     const uint32_t lane_base = static_cast<uint32_t>(qd * 32) << 16;
     // merged row statistics of every window row
-    for (int r = et; r < RWp; r += 128) {
+    for (int r = tid - 64; r < RWp; r += 256) {
       float M = -INFINITY, Lsum = 0.f;
       if (r < p.RW) {
         for (int c = 0; c < p.n_chunks; ++c)
@@ -484,9 +486,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       s_b[r] = (Lsum > 0.f) ? -log2f(Lsum) - M : -INFINITY;
       s_wi[r] = r % p.W;
     }
-    epi_sync();
+    asm volatile("bar.sync 1, 256;" ::: "memory");
     const int t_safe = p.causal ? p.T - p.W : 0x7fffffff;  // tokens every window row sees
-    for (int i = 0; i < n_tiles; ++i) {
+    for (int i = grp; i < n_tiles; i += 2) {
       const int b = i & 1;
       if (!pwait(&lfull[b], (i >> 1) & 1, abrt, p.ws, u)) break;
       tc_fence_after();
@@ -1144,7 +1146,7 @@ cudaError_t run(const CompressArgs& a, const mkv_geom& g, int num_sms, cudaStrea
     TcArgs p2 = p1;
     p2.s_out = L.s;
     p2.diag = a.diag_scores;
-    scores_tc<<<cg, kTcThreads, kScoresSmem, st>>>(p2, tmK, tmQ);
+    scores_tc<<<cg, kStatsThreads, kScoresSmem, st>>>(p2, tmK, tmQ);
   }
   if (keep_all) {
     if (D == 128) keep_all_kernel<128><<<dim3((T + 7) / 8, U), 256, 0, st>>>(a, T);
