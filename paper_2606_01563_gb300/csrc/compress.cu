@@ -532,7 +532,7 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
 }
 
 // ------------------------------------------------------------ residual_tc
-__global__ void __launch_bounds__(kTcThreads, 1)
+__global__ void __launch_bounds__(kStatsThreads, 1)
     residual_tc(const TcArgs p, const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV) {
   constexpr int kS = 2;
   extern __shared__ __align__(1024) uint8_t smraw[];
@@ -580,7 +580,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
   }
   if (warp == 1) tmem_alloc(&tmem_base, 256);
-  if (warp >= 2) {
+  if (warp >= 2 && warp < 6) {
     // C0' (clamped where |n0 C0| < tau) as three bf16 parts in the K-major
     // swizzled layout: row a = value dim (N), 128-byte rows over key dims (K)
     const int a = tid - 64;
@@ -654,10 +654,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       }
     }
   } else {
-    const int qd = warp & 3;
+    // two epilogue groups (warps 2..5 and 6..9) take alternate tiles; group g
+    // always reads TMEM buffer g
+    const int grp = (warp - 2) >> 2, qd = warp & 3;
     const uint32_t lane_base = static_cast<uint32_t>(qd * 32) << 16;
     const int row = qd * 32 + lane;  // token within the tile = TMEM lane
-    for (int i = 0; i < n_tiles; ++i) {
+    for (int i = grp; i < n_tiles; i += 2) {
       const int s = i % kS, j = i / kS, b = i & 1;
       if (!pwait(&yfull[b], (i >> 1) & 1, abrt, p.ws, u)) break;
       if (!pwait(&full[s], j & 1, abrt, p.ws, u)) break;
@@ -1192,7 +1194,7 @@ cudaError_t run(const CompressArgs& a, const mkv_geom& g, int num_sms, cudaStrea
     r.s_in = L.s;
     r.s_out = L.s2;
     r.diag = a.diag_score2;
-    residual_tc<<<cg, kTcThreads, kResidualSmem, st>>>(r, tmK, tmV);
+    residual_tc<<<cg, kStatsThreads, kResidualSmem, st>>>(r, tmK, tmV);
   }
   SelectArgs s1 = sa;
   s1.scores = a.mi ? L.s2 : L.s;
