@@ -165,13 +165,17 @@ template <int LOGITS>
 __global__ void __launch_bounds__(kStatsThreads, 1)
     stats_tc(const TcArgs p, const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
              const __grid_constant__ CUtensorMap tmQ) {
-  constexpr int kS = 2;
+  // without logits (moments of a gathered row set, one tile per CTA): one
+  // stage, no Q, and half the TMEM, so that several CTAs share an SM
+  constexpr int kS = LOGITS ? 2 : 1;
+  constexpr uint32_t kTmemCols = LOGITS ? 512 : 256;
+  constexpr int cS = LOGITS ? 256 : 0, cSum = LOGITS ? 384 : 128;  // TMEM columns of V^T K and the sums
   extern __shared__ __align__(1024) uint8_t smraw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
   uint8_t* sK = sm;                        // [kS][128 x 128]
   uint8_t* sV = sm + kS * kTileBytes;      // [kS][128 x 128]
   uint8_t* sQ = sm + 2 * kS * kTileBytes;  // [2 boxes][RWb*128 rows][128 B]
-  uint8_t* sOnes = sQ + 2 * 2 * kBoxBytes;  // [2 boxes][16 rows][128 B] of bf16 1.0
+  uint8_t* sOnes = sQ + (LOGITS ? 2 * 2 * kBoxBytes : 0);  // [2 boxes][16 rows][128 B] of bf16 1.0
   __shared__ __align__(8) uint64_t full[kS], empty[kS], lfull, lempty, qfull, sdone;
   __shared__ uint32_t tmem_base;
   __shared__ int abort_flag;
@@ -198,7 +202,7 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
     abort_flag = 0;
     mbar_fence_init();
   }
-  if (warp == 1) tmem_alloc(&tmem_base, 512);
+  if (warp == 1) tmem_alloc(&tmem_base, kTmemCols);
   if (warp >= 2 && warp < 6) {  // the ones operand of the column sums K^T 1 and V^T 1
     for (int i = tid - 64; i < 2 * 16 * 128 / 16; i += 128)
       reinterpret_cast<uint4*>(sOnes)[i] = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u);
@@ -264,9 +268,9 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
           const uint64_t dk = sdesc_sw128(aK + kk * 2048, kBoxBytes, 1024);
           const uint64_t d1 = sdesc_sw128(a1 + (kk >> 2) * 2048 + (kk & 3) * 32, 16, 1024);
           const uint32_t acc = (i > 0 || kk > 0) ? 1u : 0u;
-          umma_bf16(tm + 256, dv, dk, idS, acc);
-          umma_bf16(tm + 384, dk, d1, id1, acc);  // column sums of K (lane = key dim)
-          umma_bf16(tm + 400, dv, d1, id1, acc);  // column sums of V (lane = value dim)
+          umma_bf16(tm + cS, dv, dk, idS, acc);
+          umma_bf16(tm + cSum, dk, d1, id1, acc);       // column sums of K (lane = key dim)
+          umma_bf16(tm + cSum + 16, dv, d1, id1, acc);  // column sums of V (lane = value dim)
         }
         umma_commit(&empty[s]);
       }
@@ -355,24 +359,30 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
     tc_fence_after();
     {
       float x[32];
-      tmem_ld32(tm + lane_base + 384, x);  // [0]: sum of K's column (this lane), [16]: of V's
+      tmem_ld32(tm + lane_base + cSum, x);  // [0]: sum of K's column (this lane), [16]: of V's
       sum_k[qd * 32 + lane] = x[0];
       sum_v[qd * 32 + lane] = x[16];
     }
     epi_sync();
     const float nc = static_cast<float>(max(0, t_end - t_begin));
+    const float inv_nc = nc > 0.f ? 1.f / nc : 0.f;
     float* rec = p.mrec + ((size_t)u * p.n_chunks + chunk) * rec_floats(p.D);
     const int a = qd * 32 + lane;  // value dim = TMEM lane
+    // centred co-moment rows staged 32 columns at a time through the (now
+    // free) K stage, so that the record is written in coalesced rows
+    float* stg = reinterpret_cast<float*>(sK);  // [128][33]
     for (int c0 = 0; c0 < kDP; c0 += 32) {
       float srow[32];
-      tmem_ld32(tm + lane_base + 256 + c0, srow);
-      if (a < p.D && nc > 0.f) {
+      tmem_ld32(tm + lane_base + cS + c0, srow);
 #pragma unroll
-        for (int jj = 0; jj < 32; ++jj) {
-          const int c = c0 + jj;
-          if (c < p.D) rec[4 + 2 * p.D + (size_t)a * p.D + c] = srow[jj] - sum_v[a] * sum_k[c] / nc;
+      for (int jj = 0; jj < 32; ++jj) stg[a * 33 + jj] = srow[jj] - sum_v[a] * sum_k[c0 + jj] * inv_nc;
+      epi_sync();
+      if (nc > 0.f)
+        for (int idx = et; idx < 128 * 32; idx += 128) {
+          const int r = idx >> 5, c = c0 + (idx & 31);
+          if (r < p.D && c < p.D) rec[4 + 2 * p.D + (size_t)r * p.D + c] = stg[r * 33 + (idx & 31)];
         }
-      }
+      epi_sync();
     }
     if (a < p.D) {
       rec[4 + a] = nc > 0.f ? sum_k[a] / nc : 0.f;
@@ -385,7 +395,7 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tm, 512);
+    tmem_dealloc(tm, kTmemCols);
   }
 }
 
@@ -1093,6 +1103,7 @@ __global__ void __launch_bounds__(256) keep_all_kernel(const CompressArgs a, int
 
 // ------------------------------------------------------------------- host
 constexpr size_t kStatsSmem = 1024 + 2 * 2 * kTileBytes + 2 * 2 * kBoxBytes + 4096;  // K, V stages, Q, ones
+constexpr size_t kStats0Smem = 1024 + 2 * kTileBytes + 4096;                            // one K, V stage, ones
 constexpr size_t kScoresSmem = 1024 + 3 * kTileBytes + 2 * 2 * kBoxBytes;
 constexpr size_t kResidualSmem = 1024 + 2 * 2 * kTileBytes + 3 * kTileBytes;
 
@@ -1106,7 +1117,7 @@ cudaError_t run(const CompressArgs& a, const mkv_geom& g, int num_sms, cudaStrea
     return cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes));
   };
   if ((e = attr((const void*)stats_tc<1>, kStatsSmem)) != cudaSuccess) return e;
-  if ((e = attr((const void*)stats_tc<0>, kStatsSmem)) != cudaSuccess) return e;
+  if ((e = attr((const void*)stats_tc<0>, kStats0Smem)) != cudaSuccess) return e;
   if ((e = attr((const void*)scores_tc, kScoresSmem)) != cudaSuccess) return e;
   if ((e = attr((const void*)residual_tc, kResidualSmem)) != cudaSuccess) return e;
 
@@ -1184,7 +1195,7 @@ cudaError_t run(const CompressArgs& a, const mkv_geom& g, int num_sms, cudaStrea
     s0.dst_V = L.gV;
     s0.dst_cap = B;
     select_kernel<<<U * kSelCL, kSelThreads, sel_smem, st>>>(s0);
-    stats_tc<0><<<dim3(L.n_rchunks, U), kStatsThreads, kStatsSmem, st>>>(rset, tmGK, tmGV, tmQ);
+    stats_tc<0><<<dim3(L.n_rchunks, U), kStatsThreads, kStats0Smem, st>>>(rset, tmGK, tmGV, tmQ);
     finalize_kernel<<<dim3(D / kFinRB, U), 256, 0, st>>>(L, L.m0, a.mom, 0, 1);
     TcArgs r = tp;
     r.n_rows = T;
@@ -1206,7 +1217,7 @@ cudaError_t run(const CompressArgs& a, const mkv_geom& g, int num_sms, cudaStrea
   s1.dst_len = a.cache.len;
   s1.dst_seen = a.cache.seen;
   select_kernel<<<U * kSelCL, kSelThreads, sel_smem, st>>>(s1);
-  stats_tc<0><<<dim3(L.n_rchunks, U), kStatsThreads, kStatsSmem, st>>>(rset, tmCK, tmCV, tmQ);
+  stats_tc<0><<<dim3(L.n_rchunks, U), kStatsThreads, kStats0Smem, st>>>(rset, tmCK, tmCV, tmQ);
   finalize_kernel<<<dim3(D / kFinRB, U), 256, 0, st>>>(L, nullptr, a.mom, 1, a.mi ? 0 : 1);
   return cudaGetLastError();
 }
