@@ -1437,21 +1437,14 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
     }
     cluster.sync();
 
-    // ---- every warp: the cluster's minimum key (ties cannot happen: rows differ)
-    unsigned long long b = (lane < kCL) ? mail_key[par][lane] : ~0ull;
-    int src = lane;
-#pragma unroll
-    for (int o = 4; o > 0; o >>= 1) {
-      const unsigned long long b2 = __shfl_xor_sync(kFull, b, o);
-      const int s2 = __shfl_xor_sync(kFull, src, o);
-      if (b2 < b) {
-        b = b2;
-        src = s2;
-      }
-    }
-    b = __shfl_sync(kFull, b, 0);
-    src = __shfl_sync(kFull, src, 0);
-    const int js = (b == ~0ull) ? -1 : static_cast<int>(b & 0xffffffffu);
+    // ---- every warp: the cluster's minimum key (ties cannot happen: rows
+    // differ), by two warp-wide minimum reductions (score bits, then row)
+    const unsigned long long bk = (lane < kCL) ? mail_key[par][lane] : ~0ull;
+    const unsigned khi = static_cast<unsigned>(bk >> 32), klo = static_cast<unsigned>(bk);
+    const unsigned mhi = __reduce_min_sync(kFull, khi);
+    const unsigned mlo = __reduce_min_sync(kFull, khi == mhi ? klo : 0xffffffffu);
+    const int src = __ffs(__ballot_sync(kFull, khi == mhi && klo == mlo)) - 1;
+    const int js = (mhi == 0xffffffffu && mlo == 0xffffffffu) ? -1 : static_cast<int>(mlo);
     if (js < 0) {  // uniform: every rank read the same keys
       if (rank == 0 && tid == 0) record_error(a.ws, MKV_ERR_INVALID_ARG, u);
       break;
