@@ -476,16 +476,23 @@ def decode_layers(torch, mkv, dev, flush, hbm, b, B, gen, st):
     ws = mkv.alloc_workspace(mkv.mkv_decode_workspace_size(g, B), dev)
     caches = [mkv.Cache(Kall[l], Vall[l], pos, lens, seen) for l in range(layers)]
     moms = [mkv.Moments(n[l], mk[l], mv[l], Call[l]) for l in range(layers)]
+    # the 16-bit moment storage of Sec. C.2: a bf16 copy of every layer's C
+    C16 = torch.empty(layers, b, H, D, D, dtype=torch.bfloat16, device=dev)
+    for l in range(layers):
+        mkv.mkv_moments_pack_bf16(g, moms[l], C16[l])
     res = {}
-    for corr in (1, 0):
-        p = mkv.mkv_decode_params(corr, 1, 1e-6)
+    for corr in (1, 0, 2):
+        p = mkv.mkv_decode_params(min(corr, 1), 1, 1e-6)
+        ps = [p] * layers
+        if corr == 2:
+            ps = [mkv.mkv_decode_params(1, 1, 1e-6, C16[l].data_ptr()) for l in range(layers)]
         with torch.cuda.stream(st):
             for l in range(layers):
-                mkv.mkv_decode_step(g, q, None, None, caches[l], moms[l], p, out, None, ws, st)
+                mkv.mkv_decode_step(g, q, None, None, caches[l], moms[l], ps[l], out, None, ws, st)
             gr = torch.cuda.CUDAGraph()
         with torch.cuda.graph(gr, stream=st, capture_error_mode="relaxed"):
             for l in range(layers):
-                mkv.mkv_decode_step(g, q, None, None, caches[l], moms[l], p, out, None, ws, st)
+                mkv.mkv_decode_step(g, q, None, None, caches[l], moms[l], ps[l], out, None, ws, st)
         times = []
         for it in range(6):
             with torch.cuda.stream(st):
@@ -498,14 +505,15 @@ def decode_layers(torch, mkv, dev, flush, hbm, b, B, gen, st):
             if it >= 2:
                 times.append(e0.elapsed_time(e1) / layers)
         t = float(np.median(times))
-        byt = units * (B * D * 4 + (D * D * 4 + 2 * D * 4 + 4 if corr else 0)) + b * H * G * D * (2 + 4)
-        res[("corr" if corr else "plain") + "_layers"] = {
+        cbytes = {0: 0, 1: D * D * 4 + 2 * D * 4 + 4, 2: D * D * 2 + 2 * D * 4 + 4}[corr]
+        byt = units * (B * D * 4 + cbytes) + b * H * G * D * (2 + 4)
+        res[{0: "plain", 1: "corr", 2: "corr_c16"}[corr] + "_layers"] = {
             "us": round(t * 1e3, 2), "gbs": round(byt / t / 1e6, 1), "frac": round(byt / t / 1e6 / hbm, 4),
             "tokens_per_s": round(b / (t / 1e3), 1), "layers": layers}
         del gr
     code, _ = mkv.mkv_get_device_error(ws, st)
     res["ok_layers"] = code == 0
-    del Kall, Vall, Call, caches, moms
+    del Kall, Vall, Call, C16, caches, moms
     return res
 
 

@@ -128,7 +128,20 @@ typedef struct {
   int32_t correction; /* 1: merge the moment term; 0: plain attention over R   */
   int32_t order;      /* 1: f_hat_E = v_bar + S_tilde q/(n sqrt d); 0: v_bar only */
   float tau;          /* clamp |S_tilde_ab| < tau to 0 before S_tilde q         */
+  const void* C16;    /* optional bf16 [b, h_kv, d, d] copy of the moments' C   */
+                      /* (16-bit moment storage, Sec. C.2; mkv_moments_pack_bf16): */
+                      /* when set, the order-1 term reads C from it (half the  */
+                      /* bytes) instead of mkv_moments.C; 16-byte aligned.     */
 } mkv_decode_params;
+
+/*
+ * 16-bit moment storage (Sec. C.2 keeps the moments in 16 bits): writes
+ * C16[u] = bf16(mom->C[u]) (round to nearest even) for every unit, one launch
+ * on `stream`.  C16 is caller-owned device memory of b * h_kv * d * d bf16,
+ * 16-byte aligned; pass it as mkv_decode_params.C16.  Returns
+ * MKV_ERR_INVALID_ARG on null or misaligned pointers.
+ */
+MKV_API mkv_status mkv_moments_pack_bf16(mkv_geom geom, const mkv_moments* mom, void* C16, void* stream);
 
 /* Human-readable name of a status code (static string). */
 MKV_API const char* mkv_status_str(mkv_status s);

@@ -86,6 +86,7 @@ mkv_status mkv_decode_step(mkv_geom geom, const void* q, const void* k_new, cons
   if (p->order != 0 && p->order != 1) return MKV_ERR_INVALID_ARG;
   if (p->correction && !moments_ok(mom)) return MKV_ERR_INVALID_ARG;
   if (!(p->tau >= 0.f)) return MKV_ERR_INVALID_ARG;
+  if (p->C16 && !aligned(p->C16, 16)) return MKV_ERR_INVALID_ARG;
   const int sms = num_sms_current();
   const size_t need = decode_workspace_bytes(geom, cache->capacity, sms);
   if (!workspace || workspace_bytes < need || !aligned(workspace, 256)) return MKV_ERR_WORKSPACE;
@@ -103,6 +104,7 @@ mkv_status mkv_decode_step(mkv_geom geom, const void* q, const void* k_new, cons
   a.mu_k = p->correction ? mom->mu_k : nullptr;
   a.mu_v = p->correction ? mom->mu_v : nullptr;
   a.C = p->correction ? mom->C : nullptr;
+  a.C16 = p->correction ? static_cast<const __nv_bfloat16*>(p->C16) : nullptr;
   a.correction = p->correction;
   a.order = p->order;
   a.tau = p->tau;
@@ -112,6 +114,13 @@ mkv_status mkv_decode_step(mkv_geom geom, const void* q, const void* k_new, cons
   a.n_kv = geom.n_kv_heads;
   decode_carve(a, geom, cache->capacity, sms, workspace);
   return cuda_status(launch_decode(a, geom.head_dim, geom.group, static_cast<cudaStream_t>(stream)));
+}
+
+mkv_status mkv_moments_pack_bf16(mkv_geom geom, const mkv_moments* mom, void* C16, void* stream) {
+  if (!geom_ok(geom)) return (geom.head_dim == 64 || geom.head_dim == 128) ? MKV_ERR_SHAPE : MKV_ERR_UNSUPPORTED;
+  if (!moments_ok(mom) || !C16 || !aligned(C16, 16)) return MKV_ERR_INVALID_ARG;
+  const size_t n = (size_t)geom.batch * geom.n_kv_heads * geom.head_dim * geom.head_dim;
+  return cuda_status(launch_pack_bf16(mom->C, static_cast<__nv_bfloat16*>(C16), n, static_cast<cudaStream_t>(stream)));
 }
 
 // ------------------------------------------------------------------- evict

@@ -170,7 +170,7 @@ __device__ __forceinline__ void process16(WarpState<D>& st, const uint32_t (&qa)
   }
 }
 
-template <int D, int G, bool CL>
+template <int D, int G, bool CL, bool C16>
 __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, const __grid_constant__ CUtensorMap tmK,
                                                           const __grid_constant__ CUtensorMap tmV) {
   constexpr int DPL = D / 32;
@@ -237,28 +237,46 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
   const int n_mt = (r1 - r0 + 15) / 16;
   const bool do_c = corr && a.order == 1;
   const bool split_k = n_mt <= 2;
+  // C[row][c0], C[row][c0 + 1] as float2, from C or from its bf16 copy
+  constexpr bool c16 = C16;  // moment rows read from the bf16 copy of C
+  auto ld_c2 = [&](int row, int c0) -> float2 {
+    const size_t off = ((size_t)u * D + row) * D + c0;
+    if constexpr (c16) return __bfloat1622float2(__ldg(reinterpret_cast<const __nv_bfloat162*>(a.C16 + off)));
+    else return __ldg(reinterpret_cast<const float2*>(a.C + off));
+  };
   float2 cfr[2][KPW][4];
   {
     const int g = lane >> 2, t = lane & 3;
+    auto load_frags = [&](auto ld) {
 #pragma unroll
-    for (int j = 0; j < 2; ++j) {
-      const int ra = r0 + j * 16 + g, rb = ra + 8;
+      for (int j = 0; j < 2; ++j) {
+        const int ra = r0 + j * 16 + g, rb = ra + 8;
 #pragma unroll
-      for (int kp = 0; kp < KPW; ++kp) {
-        const int c0 = (warp * KPW + kp) * 16 + 2 * t;
-        const float* Ca = a.C + ((size_t)u * D + ra) * D + c0;
-        const float* Cb = a.C + ((size_t)u * D + rb) * D + c0;
-        const bool va = do_c && split_k && ra < r1, vb = do_c && split_k && rb < r1;
-        cfr[j][kp][0] = va ? __ldg(reinterpret_cast<const float2*>(Ca)) : make_float2(0.f, 0.f);
-        cfr[j][kp][1] = vb ? __ldg(reinterpret_cast<const float2*>(Cb)) : make_float2(0.f, 0.f);
-        cfr[j][kp][2] = va ? __ldg(reinterpret_cast<const float2*>(Ca + 8)) : make_float2(0.f, 0.f);
-        cfr[j][kp][3] = vb ? __ldg(reinterpret_cast<const float2*>(Cb + 8)) : make_float2(0.f, 0.f);
+        for (int kp = 0; kp < KPW; ++kp) {
+          const int c0 = (warp * KPW + kp) * 16 + 2 * t;
+          const bool va = do_c && split_k && ra < r1, vb = do_c && split_k && rb < r1;
+          cfr[j][kp][0] = va ? ld(ra, c0) : make_float2(0.f, 0.f);
+          cfr[j][kp][1] = vb ? ld(rb, c0) : make_float2(0.f, 0.f);
+          cfr[j][kp][2] = va ? ld(ra, c0 + 8) : make_float2(0.f, 0.f);
+          cfr[j][kp][3] = vb ? ld(rb, c0 + 8) : make_float2(0.f, 0.f);
+        }
       }
-    }
+    };
+    if constexpr (c16)
+      load_frags([&](int row, int c0) {
+        return __bfloat1622float2(
+            __ldg(reinterpret_cast<const __nv_bfloat162*>(a.C16 + ((size_t)u * D + row) * D + c0)));
+      });
+    else
+      load_frags([&](int row, int c0) {
+        return __ldg(reinterpret_cast<const float2*>(a.C + ((size_t)u * D + row) * D + c0));
+      });
   }
   if (do_c && !split_k && tid == 0 && r1 > r0) {  // whole-tile case: the rows are read after the tiles
-    const float* base = a.C + ((size_t)u * D + r0) * D;
-    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base), "r"((uint32_t)((r1 - r0) * D * 4))
+    const void* base = c16 ? static_cast<const void*>(a.C16 + ((size_t)u * D + r0) * D)
+                           : static_cast<const void*>(a.C + ((size_t)u * D + r0) * D);
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base),
+                 "r"((uint32_t)((r1 - r0) * D * (c16 ? 2 : 4)))
                  : "memory");
   }
   // mu_v of the (row, head) pairs this thread finishes in the two-tile case
@@ -348,7 +366,7 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
       split_bf16x2(x, y, hi[i], lo[i]);
     }
     mma_bf16_full(d, hi[0], hi[1], hi[2], hi[3], qa[kk][0], qa[kk][1]);
-    mma_bf16_full(d, lo[0], lo[1], lo[2], lo[3], qa[kk][0], qa[kk][1]);
+    mma_bf16_full(d, lo[0], lo[1], lo[2], lo[3], qa[kk][0], qa[kk][1]);  // zero for a bf16 copy of C
   };
   if (use_m && do_c && split_k) {
     const int g = lane >> 2, t = lane & 3;
@@ -390,12 +408,11 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
         float2 f[D / 16][4];
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
-          const float* Ca = a.C + ((size_t)u * D + ra) * D + kk * 16 + 2 * t;
-          const float* Cb = a.C + ((size_t)u * D + rb) * D + kk * 16 + 2 * t;
-          f[kk][0] = va ? __ldg(reinterpret_cast<const float2*>(Ca)) : make_float2(0.f, 0.f);
-          f[kk][1] = vb ? __ldg(reinterpret_cast<const float2*>(Cb)) : make_float2(0.f, 0.f);
-          f[kk][2] = va ? __ldg(reinterpret_cast<const float2*>(Ca + 8)) : make_float2(0.f, 0.f);
-          f[kk][3] = vb ? __ldg(reinterpret_cast<const float2*>(Cb + 8)) : make_float2(0.f, 0.f);
+          const int c0 = kk * 16 + 2 * t;
+          f[kk][0] = va ? ld_c2(ra, c0) : make_float2(0.f, 0.f);
+          f[kk][1] = vb ? ld_c2(rb, c0) : make_float2(0.f, 0.f);
+          f[kk][2] = va ? ld_c2(ra, c0 + 8) : make_float2(0.f, 0.f);
+          f[kk][3] = vb ? ld_c2(rb, c0 + 8) : make_float2(0.f, 0.f);
         }
         const float mva = va ? __ldg(a.mu_v + (size_t)u * D + ra) : 0.f;
         const float mvb = vb ? __ldg(a.mu_v + (size_t)u * D + rb) : 0.f;
@@ -522,9 +539,9 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
   }
 
   const size_t rec_floats = (size_t)a.S * G * PS;
-  bool staged;
-  const float* src;
-  float* sF;  // [G][D] f_hat_E rows (or mu_v for order 0)
+  bool staged = false;
+  const float* src = nullptr;
+  float* sF = nullptr;  // [G][D] f_hat_E rows (or mu_v for order 0)
   float* sP = reinterpret_cast<float*>(dsmem);
   if constexpr (CL) {
     // ---- cluster barrier: every partial and f_hat_E row is in CTA 0
@@ -710,7 +727,7 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
 
 // Whether clusters of S CTAs with `smem` bytes each can be resident (checked
 // once per split count; portable sizes always can).
-template <int D, int G>
+template <int D, int G, bool C16>
 bool cluster_fits(int S, size_t smem) {
   if (S <= 8) return true;
   static std::mutex mu;
@@ -729,15 +746,15 @@ bool cluster_fits(int S, size_t smem) {
     cfg.attrs = at;
     cfg.numAttrs = 1;
     int n = 0;
-    const cudaError_t e = cudaOccupancyMaxActiveClusters(&n, decode_kernel<D, G, true>, &cfg);
+    const cudaError_t e = cudaOccupancyMaxActiveClusters(&n, decode_kernel<D, G, true, C16>, &cfg);
     if (e != cudaSuccess) (void)cudaGetLastError();
     known[S] = (e == cudaSuccess && n > 0) ? 1 : -1;
   }
   return known[S] > 0;
 }
 
-template <int D, int G>
-cudaError_t launch_dg(const DecodeArgs& a, cudaStream_t stream) {
+template <int D, int G, bool C16>
+cudaError_t launch_dgc(const DecodeArgs& a, cudaStream_t stream) {
   const size_t ring = (size_t)2 * kStages * kTT * D * 2 + 1024;  // + alignment slack
   const size_t rcv = ((size_t)a.S * G * (D + 4) + (size_t)G * D + 2 * (size_t)a.S * G) * sizeof(float);
   const bool cl = a.S <= kMaxClusterSplits;
@@ -745,16 +762,16 @@ cudaError_t launch_dg(const DecodeArgs& a, cudaStream_t stream) {
   // per-device function attributes; setting them again is harmless
   cudaError_t e;
   if (cl) {
-    e = cudaFuncSetAttribute(decode_kernel<D, G, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    e = cudaFuncSetAttribute(decode_kernel<D, G, true, C16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(smem));
     if (e == cudaSuccess && a.S > 8)
-      e = cudaFuncSetAttribute(decode_kernel<D, G, true>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+      e = cudaFuncSetAttribute(decode_kernel<D, G, true, C16>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   } else {
-    e = cudaFuncSetAttribute(decode_kernel<D, G, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    e = cudaFuncSetAttribute(decode_kernel<D, G, false, C16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(smem));
   }
   if (e != cudaSuccess) return e;
-  const bool use_cl = cl && cluster_fits<D, G>(a.S, smem);
+  const bool use_cl = cl && cluster_fits<D, G, C16>(a.S, smem);
   // the cache slabs of all units as one [units * cap][D] matrix
   const uint64_t rows = (uint64_t)a.batch * a.n_kv * a.cap;
   CUtensorMap tmK, tmV;
@@ -775,13 +792,18 @@ cudaError_t launch_dg(const DecodeArgs& a, cudaStream_t stream) {
   at[1].val.clusterDim.z = 1;
   cfg.attrs = at;
   cfg.numAttrs = use_cl ? 2 : 1;
-  if (use_cl) return cudaLaunchKernelEx(&cfg, decode_kernel<D, G, true>, a, tmK, tmV);
+  if (use_cl) return cudaLaunchKernelEx(&cfg, decode_kernel<D, G, true, C16>, a, tmK, tmV);
   if (cl) {  // the cluster did not fit: the ticket variant with the ring only
-    e = cudaFuncSetAttribute(decode_kernel<D, G, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    e = cudaFuncSetAttribute(decode_kernel<D, G, false, C16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(ring));
     if (e != cudaSuccess) return e;
   }
-  return cudaLaunchKernelEx(&cfg, decode_kernel<D, G, false>, a, tmK, tmV);
+  return cudaLaunchKernelEx(&cfg, decode_kernel<D, G, false, C16>, a, tmK, tmV);
+}
+
+template <int D, int G>
+cudaError_t launch_dg(const DecodeArgs& a, cudaStream_t stream) {
+  return a.C16 != nullptr ? launch_dgc<D, G, true>(a, stream) : launch_dgc<D, G, false>(a, stream);
 }
 
 }  // namespace
@@ -792,6 +814,27 @@ cudaError_t launch_dg(const DecodeArgs& a, cudaStream_t stream) {
 // at least two tiles per CTA beyond, and past 12 splits the merge costs more
 // than the extra parallelism saves (measured on the Llama-3.1-8B decode
 // geometry over batch 1..64 and caches of 256..4096 rows).
+namespace {
+__global__ void __launch_bounds__(256) pack_bf16_kernel(const float* __restrict__ C, __nv_bfloat16* __restrict__ C16,
+                                                        size_t n4) {
+  for (size_t i = (size_t)blockIdx.x * 256 + threadIdx.x; i < n4; i += (size_t)gridDim.x * 256) {
+    const float4 v = reinterpret_cast<const float4*>(C)[i];
+    __nv_bfloat162 lo = __floats2bfloat162_rn(v.x, v.y), hi = __floats2bfloat162_rn(v.z, v.w);
+    uint2 w;
+    w.x = *reinterpret_cast<uint32_t*>(&lo);
+    w.y = *reinterpret_cast<uint32_t*>(&hi);
+    reinterpret_cast<uint2*>(C16)[i] = w;
+  }
+}
+}  // namespace
+
+cudaError_t launch_pack_bf16(const float* C, __nv_bfloat16* C16, size_t n, cudaStream_t stream) {
+  const size_t n4 = n / 4;  // d * d is a multiple of 4
+  const int blocks = static_cast<int>(std::min<size_t>((n4 + 255) / 256, 65535));
+  if (n4 > 0) pack_bf16_kernel<<<blocks, 256, 0, stream>>>(C, C16, n4);
+  return cudaGetLastError();
+}
+
 int decode_splits(const mkv_geom& g, int32_t capacity, int num_sms) {
   const long units = (long)g.batch * g.n_kv_heads;
   const long tiles = ((long)capacity + 1 + kTT - 1) / kTT;

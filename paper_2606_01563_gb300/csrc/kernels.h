@@ -1,6 +1,7 @@
 // Internal launcher interface between the C-ABI layer (api.cu) and the kernels.
 #pragma once
 
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stddef.h>
 #include <stdint.h>
@@ -24,6 +25,7 @@ struct DecodeArgs {
   const float* mu_k;
   const float* mu_v;
   const float* C;
+  const __nv_bfloat16* C16;  // optional bf16 copy of C (read instead of C when set)
   int32_t correction;
   int32_t order;
   float tau;
@@ -45,6 +47,7 @@ size_t decode_workspace_bytes(const mkv_geom& g, int32_t capacity, int num_sms);
 // Carves the workspace and fills the ws/counters/partial/fhat fields.
 void decode_carve(DecodeArgs& a, const mkv_geom& g, int32_t capacity, int num_sms, void* ws);
 cudaError_t launch_decode(const DecodeArgs& a, int head_dim, int group, cudaStream_t stream);
+cudaError_t launch_pack_bf16(const float* C, __nv_bfloat16* C16, size_t n, cudaStream_t stream);
 // The same carving for an explicit split count S (used by the entry point
 // whose scratch has a fixed maximum size).
 size_t decode_workspace_bytes_splits(const mkv_geom& g, int S);

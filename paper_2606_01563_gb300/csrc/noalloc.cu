@@ -75,6 +75,7 @@ extern "C" MKV_API mkv_status mkv_decode_step_noalloc(mkv_geom geom, const void*
     return MKV_ERR_INVALID_ARG;
   if (p->correction && (!mom || !mom->n || !mom->mu_k || !mom->mu_v || !mom->C || !aligned16(mom->C)))
     return MKV_ERR_INVALID_ARG;
+  if (p->C16 && !aligned16(p->C16)) return MKV_ERR_INVALID_ARG;
   // The smallest split count needs one partial record per query head: reject
   // geometries whose scratch would exceed the fixed array before any set-up.
   if (decode_workspace_bytes_splits(geom, 1) > kNoAllocScratchBytes) return MKV_ERR_WORKSPACE;
@@ -100,6 +101,7 @@ extern "C" MKV_API mkv_status mkv_decode_step_noalloc(mkv_geom geom, const void*
   a.mu_k = p->correction ? mom->mu_k : nullptr;
   a.mu_v = p->correction ? mom->mu_v : nullptr;
   a.C = p->correction ? mom->C : nullptr;
+  a.C16 = p->correction ? static_cast<const __nv_bfloat16*>(p->C16) : nullptr;
   a.correction = p->correction;
   a.order = p->order;
   a.tau = p->tau;

@@ -43,7 +43,7 @@ class mkv_compress_diag(ctypes.Structure):
 
 
 class mkv_decode_params(ctypes.Structure):
-    _fields_ = [("correction", c_i32), ("order", c_i32), ("tau", ctypes.c_float)]
+    _fields_ = [("correction", c_i32), ("order", c_i32), ("tau", ctypes.c_float), ("C16", c_vp)]
 
 
 STATUS = {0: "MKV_OK", 1: "MKV_ERR_INVALID_ARG", 2: "MKV_ERR_SHAPE", 3: "MKV_ERR_CAPACITY",
@@ -51,7 +51,7 @@ STATUS = {0: "MKV_OK", 1: "MKV_ERR_INVALID_ARG", 2: "MKV_ERR_SHAPE", 3: "MKV_ERR
 
 EXPORTS = ("mkv_status_str", "mkv_version", "mkv_compress_workspace_size", "mkv_compress",
            "mkv_decode_workspace_size", "mkv_decode_step", "mkv_evict_workspace_size",
-           "mkv_evict_append", "mkv_get_device_error", "mkv_decode_step_noalloc")
+           "mkv_evict_append", "mkv_get_device_error", "mkv_decode_step_noalloc", "mkv_moments_pack_bf16")
 
 
 class MKVError(RuntimeError):
@@ -95,6 +95,8 @@ def lib():
         L.mkv_evict_append.restype = c_i32
         L.mkv_evict_append.argtypes = [mkv_geom, c_vp, c_vp, c_vp, c_i32, ctypes.POINTER(mkv_cache),
                                        ctypes.POINTER(mkv_moments), ctypes.c_float, c_vp, ctypes.c_size_t, c_vp]
+        L.mkv_moments_pack_bf16.restype = c_i32
+        L.mkv_moments_pack_bf16.argtypes = [mkv_geom, ctypes.POINTER(mkv_moments), c_vp, c_vp]
         L.mkv_get_device_error.restype = c_i32
         L.mkv_get_device_error.argtypes = [c_vp, c_vp, ctypes.POINTER(c_i32)]
         _lib = L
@@ -231,6 +233,12 @@ def mkv_evict_append(g, q, k_new, v_new, budget, cache: Cache, mom: Moments, tau
     code = lib().mkv_evict_append(g, _ptr(q), _ptr(k_new), _ptr(v_new), budget, ctypes.byref(c),
                                   ctypes.byref(m), tau, _ptr(ws), ws.numel(), _stream(stream))
     _check(code, "mkv_evict_append")
+
+
+def mkv_moments_pack_bf16(g, mom: Moments, C16, stream=None):
+    """C16 (bf16 [b, h_kv, d, d]) = bf16(mom.C): the 16-bit copy mkv_decode_params.C16 points at."""
+    m = mom.c()
+    _check(lib().mkv_moments_pack_bf16(g, ctypes.byref(m), _ptr(C16), _stream(stream)), "mkv_moments_pack_bf16")
 
 
 def mkv_get_device_error(ws, stream=None):

@@ -179,3 +179,38 @@ def test_decode_sweep_full_size(batch, budget):
     assert code == 0
     assert_output_close(out, ref, "sweep")
     np.testing.assert_allclose(lse, ref_lse, rtol=0, atol=1e-3)
+
+
+@pytest.mark.parametrize("case", [1, 4])
+@pytest.mark.parametrize("order", [1, 0])
+def test_decode_bf16_moment_storage(case, order):
+    """16-bit moment storage: mkv_moments_pack_bf16 rounds C to bf16 exactly as
+    torch does, and decode reading that copy matches the oracle run on the
+    bf16-rounded C (order 0 ignores C)."""
+    b, H, G, D, lens, cap, n_list = CASES[case]
+    rng = np.random.default_rng(300 + case)
+    if lens is None:
+        lens = rng.integers(1, cap - 1, b * H)
+    if n_list is None:
+        n_list = rng.integers(0, 5000, b * H)
+    st = make_state(rng, b, H, G, D, lens, cap, n_list)
+    g = mkv.geom(b, H, G, D)
+    mom = mkv.Moments(i32(st["n"]), f32(st["mu_k"]), f32(st["mu_v"]), f32(st["C"]))
+    C16 = torch.empty(b, H, D, D, dtype=torch.bfloat16, device="cuda")
+    mkv.mkv_moments_pack_bf16(g, mom, C16)
+    ref16 = torch.from_numpy(st["C"]).to(torch.bfloat16)
+    assert torch.equal(C16.cpu().view(torch.int16), ref16.view(torch.int16))
+    cache = mkv.Cache(bf16(st["K"]), bf16(st["V"]),
+                      i32(np.broadcast_to(np.arange(st["cap"]), (b, H, st["cap"]))),
+                      i32(st["lens"]), i32(st["lens"] + 1000))
+    out = torch.empty(b, H * G, D, device="cuda")
+    lse = torch.empty(b, H * G, device="cuda")
+    ws = mkv.alloc_workspace(mkv.mkv_decode_workspace_size(g, st["cap"]))
+    p = mkv.mkv_decode_params(1, order, 1e-6, C16.data_ptr())
+    mkv.mkv_decode_step(g, bf16(st["q"]), bf16(st["kn"]), bf16(st["vn"]), cache, mom, p, out, lse, ws)
+    code, _ = mkv.mkv_get_device_error(ws)
+    assert code == 0
+    st16 = dict(st, C=ref16.float().numpy())
+    ref, ref_lse = run_oracle(st16, b, H, G, D, True, 1, order, 1e-6)
+    assert_output_close(host(out), ref, "decode out (bf16 C)")
+    np.testing.assert_allclose(host(lse), ref_lse, rtol=0, atol=1e-4 * np.maximum(1, np.abs(ref_lse)).max())

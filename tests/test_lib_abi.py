@@ -27,7 +27,7 @@ def declared_functions():
 
 def test_every_declared_symbol_is_exported(L):
     names = declared_functions()
-    assert len(names) == 10, names
+    assert len(names) == 11, names
     assert set(names) == set(mkv.EXPORTS)
     for n in names:
         assert hasattr(L, n), n
@@ -74,6 +74,17 @@ def test_decode_validation(L):
     assert decode(L, g, ws=None) == 7
     assert decode(L, g, wsb=16) == 7
     assert decode(L, g, ws=FAKE + 8) == 7                    # misaligned workspace
+    assert decode(L, g, p=mkv.mkv_decode_params(1, 1, 0.0, FAKE + 8)) == 1  # misaligned bf16 C copy
+    assert decode(L, g, q=FAKE + 4) == 1                     # misaligned q
+
+
+def test_pack_bf16_validation(L):
+    g = mkv.geom(1, 2, 4, 128)
+    m = mkv.mkv_moments(FAKE, FAKE, FAKE, FAKE)
+    assert L.mkv_moments_pack_bf16(g, ctypes.byref(m), None, None) == 1
+    assert L.mkv_moments_pack_bf16(g, ctypes.byref(m), FAKE + 8, None) == 1
+    assert L.mkv_moments_pack_bf16(g, None, FAKE, None) == 1
+    assert L.mkv_moments_pack_bf16(mkv.geom(1, 2, 4, 96), ctypes.byref(m), FAKE, None) == 6
 
 
 def test_workspace_sizes(L):
