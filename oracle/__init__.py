@@ -22,7 +22,13 @@ Parity status of each function (what pins it, in tests/test_oracle_pins.py):
       reading itself is the library's definition (parity unpinned by the paper
       beyond its parts: the paper does not say how the moment filter enters
       the prefill)
+  select_topk_joint -- exhaustive check over all subsets of (head, position)
+      pairs on tiny inputs; one head reduces to select_topk
+  compress_adaptive -- one head equals `compress`; stage-by-stage brute force
+      on tiny inputs; the joint allocation across heads is the library's
+      reading of the paper's Ada-KV protocol (Sec. 5.1), pinned only by its
+      definition beyond those reductions
   storage_bytes -- Table 5 figures
 """
 from .momentkv import *  # noqa: F401,F403
-from .momentkv import Moments, CompressResult, EvictResult  # noqa: F401
+from .momentkv import Moments, CompressResult, CompressAdaptiveResult, EvictResult  # noqa: F401

@@ -513,6 +513,85 @@ def compress(K, V, Q_obs, budget, window, sink=1, keep_window=True, pool=1,
     return CompressResult(R, moments_of(K[~keep], V[~keep]), s, R0, score2, gap1, gap2)
 
 
+def select_topk_joint(scores, k, protected):
+    """Adaptive budget across heads (Ada-KV allocation, Sec. 5.1): R_h =
+    protected_h u the k highest-scoring unprotected (head, position) pairs of
+    all heads together.
+
+    scores, protected: [H, T].  Order: higher score first, equal scores ->
+    lower head, then lower position first.  Returns (list of sorted R_h, gap
+    at the joint boundary as in select_topk).
+    """
+    scores = np.asarray(scores, F64)
+    H, T = scores.shape
+    cand = [(h, t) for h in range(H) for t in range(T) if not protected[h, t]]
+    order = sorted(cand, key=lambda ht: (-scores[ht], ht[0], ht[1]))
+    chosen = order[:k]
+    gap = math.inf
+    if 0 < k < len(order):
+        a, b = scores[order[k - 1]], scores[order[k]]
+        gap = (a - b) / abs(a) if a != 0 else (0.0 if b == a else math.inf)
+    keep = np.asarray(protected, bool).copy()
+    for h, t in chosen:
+        keep[h, t] = True
+    return [np.nonzero(keep[h])[0].astype(np.int64) for h in range(H)], gap
+
+
+@dataclass
+class CompressAdaptiveResult:
+    idx: list                # per head: retained positions, ascending
+    moments: list            # per head: Moments of E_h = all \ R_h
+    scores: np.ndarray       # [H, T] stage-1 (pooled) window scores
+    idx_stage1: list         # per head: R0_h
+    score2: np.ndarray | None
+    gap1: float
+    gap2: float | None
+
+
+def compress_adaptive(K, V, Q_obs, budget, window, sink=1, keep_window=True, pool=1,
+                      mi=True, tau=0.0, causal=True):
+    """Prefill compression of the H KV heads of one layer with the budget
+    allocated across heads (the paper's protocol builds on Ada-KV: the layer's
+    budget H * budget is shared by the heads according to their attention
+    mass, Sec. 5.1).
+
+    K, V: [H, T, d]; Q_obs: [H, g, w, d].  Reading: both selection stages of
+    `compress` become joint top-k over the heads' unprotected positions, with
+    k = H * budget - sum_h |protected_h| (select_topk_joint); every head keeps
+    its own protected set; M0_h and the output moments are per head.  With
+    T <= budget every head keeps everything.
+    """
+    K = np.asarray(K, F64)
+    V = np.asarray(V, F64)
+    H, T, d = K.shape
+    s = np.stack([pool_scores(window_scores(Q_obs[h], K[h], causal), pool) for h in range(H)])
+    if T <= budget:
+        all_idx = [np.arange(T) for _ in range(H)]
+        return CompressAdaptiveResult(all_idx, [Moments.zeros(d) for _ in range(H)], s, all_idx, None,
+                                      math.inf, None)
+    prot = np.stack([protected_mask(T, window, sink, keep_window) for _ in range(H)])
+    k = H * budget - int(prot.sum())
+    if k < 0:
+        raise ValueError("budget smaller than the protected set")
+    R0, gap1 = select_topk_joint(s, k, prot)
+    R, score2, gap2 = R0, None, None
+    if mi:
+        score2 = np.zeros((H, T))
+        for h in range(H):
+            keep0 = np.zeros(T, bool)
+            keep0[R0[h]] = True
+            M0 = moments_of(K[h][~keep0], V[h][~keep0])
+            r = residual(K[h], V[h], M0, tau)
+            score2[h] = s[h] * np.sqrt((r * r).sum(axis=1))
+        R, gap2 = select_topk_joint(score2, k, prot)
+    moms = []
+    for h in range(H):
+        keep = np.zeros(T, bool)
+        keep[R[h]] = True
+        moms.append(moments_of(K[h][~keep], V[h][~keep]))
+    return CompressAdaptiveResult(R, moms, s, R0, score2, gap1, gap2)
+
+
 # ---------------------------------------------------------------------------
 # Diagnostics used by the pins (Sec. 3; Appendix A.2, B)
 # ---------------------------------------------------------------------------

@@ -42,6 +42,10 @@ MUTATIONS = {
                               "out[c0:c0 + pool] = s[c0:c0 + pool].max()"),
     "raw-sum conversion sign": ("S = n * np.asarray(m.C, F64) + np.outer(s_v, s_k) / n",
                                 "S = n * np.asarray(m.C, F64) - np.outer(s_v, s_k) / n"),
+    "joint top-k ties to the higher head": ("key=lambda ht: (-scores[ht], ht[0], ht[1])",
+                                           "key=lambda ht: (-scores[ht], -ht[0], ht[1])"),
+    "adaptive budget without the protected rows": ("k = H * budget - int(prot.sum())",
+                                                   "k = H * budget"),
     "clamp applied to C instead of S_tilde": (
         "S_tilde = clamp_s_tilde(m.n * np.asarray(m.C, F64), tau)\n    return",
         "S_tilde = m.n * clamp_s_tilde(np.asarray(m.C, F64), tau)\n    return"),

@@ -464,6 +464,84 @@ def test_compress_stagewise_brute_force():
     assert full.idx.tolist() == list(range(T)) and full.moments.n == 0
 
 
+def test_select_topk_joint_exhaustive():
+    """Joint selection over heads: the unique k-subset of unprotected (head,
+    position) pairs whose members all precede every rejected pair in (higher
+    score, lower head, lower position) order; one head is select_topk."""
+    r = rng(19)
+    for trial in range(20):
+        H, T = 2, 6
+        s = r.integers(0, 3, (H, T)).astype(float)
+        prot = np.zeros((H, T), bool)
+        prot[:, 0] = True
+        cand = [(h, t) for h in range(H) for t in range(T) if not prot[h, t]]
+        k = int(r.integers(0, len(cand) + 1))
+        found = []
+        for sub in itertools.combinations(cand, k):
+            rest = [c for c in cand if c not in sub]
+            if all((s[a] > s[b]) or (s[a] == s[b] and a < b) for a in sub for b in rest):
+                found.append(sub)
+        assert len(found) == 1
+        R, _ = O.select_topk_joint(s, k, prot)
+        for h in range(H):
+            want = sorted([t for (hh, t) in found[0] if hh == h] + np.nonzero(prot[h])[0].tolist())
+            assert R[h].tolist() == want
+    s1 = r.standard_normal((1, 12))
+    p1 = np.zeros((1, 12), bool); p1[0, :2] = True
+    R, _ = O.select_topk_joint(s1, 5, p1)
+    assert R[0].tolist() == O.select_topk(s1[0], 5, p1[0])[0].tolist()
+
+
+def test_compress_adaptive_reductions_and_stages():
+    """Adaptive allocation: one head is `compress`; with several heads the
+    stages are recomputed from library attention, explicit evicted rows and
+    an independent joint sort; the layer keeps H * budget rows in total."""
+    r = rng(20)
+    T, d, g, w, B, H = 36, 5, 2, 4, 12, 3
+    K = r.standard_normal((H, T, d)) * np.array([0.5, 1.5, 3.0])[:, None, None]
+    V = r.standard_normal((H, T, d))
+    Q = r.standard_normal((H, g, w, d)) * 2
+    one = O.compress_adaptive(K[:1], V[:1], Q[:1], B, w, mi=True)
+    ref = O.compress(K[0], V[0], Q[0], B, w, mi=True)
+    assert one.idx[0].tolist() == ref.idx.tolist()
+    np.testing.assert_allclose(one.moments[0].C, ref.moments.C, atol=1e-12)
+    res = O.compress_adaptive(K, V, Q, B, w, mi=True)
+    mask = np.zeros((w, T), bool)
+    for i in range(w):
+        mask[i, :T - w + i + 1] = True
+    s = np.stack([sum(attn_weights(Q[h, j], K[h], mask).sum(axis=0) for j in range(g)) for h in range(H)])
+    np.testing.assert_allclose(res.scores, s, atol=1e-12)
+    prot = np.zeros((H, T), bool); prot[:, 0] = True; prot[:, T - w:] = True
+    k = H * B - int(prot.sum())
+
+    def top(x):
+        cand = [(h, t) for h in range(H) for t in range(T) if not prot[h, t]]
+        order = sorted(cand, key=lambda c: (-x[c], c[0], c[1]))[:k]
+        return [sorted([t for (hh, t) in order if hh == h] + np.nonzero(prot[h])[0].tolist()) for h in range(H)]
+
+    R0 = top(s)
+    assert [x.tolist() for x in res.idx_stage1] == R0
+    score2 = np.zeros((H, T))
+    for h in range(H):
+        E0 = np.setdiff1d(np.arange(T), R0[h])
+        f0 = sdpa(np.zeros(d), K[h][E0], V[h][E0])[0]
+        J = fd_jacobian_at_zero(K[h][E0], V[h][E0])
+        score2[h] = s[h] * np.linalg.norm(V[h] - f0 - K[h] @ J.T, axis=1)
+    np.testing.assert_allclose(res.score2, score2, rtol=1e-6, atol=1e-9)
+    R = top(score2)
+    assert [x.tolist() for x in res.idx] == R
+    assert sum(len(x) for x in R) == H * B
+    assert len({len(x) for x in R}) > 1  # the budget moved between heads
+    for h in range(H):
+        E = np.setdiff1d(np.arange(T), R[h])
+        sums = (0, np.zeros(d), np.zeros(d), np.zeros((d, d)))
+        for t in E:
+            sums = O.add_token_sums(sums, K[h][t], V[h][t])
+        mm = O.from_sums(*sums)
+        assert res.moments[h].n == len(E)
+        np.testing.assert_allclose(res.moments[h].C, mm.C, atol=1e-12)
+
+
 # --------------------------------------------------------------------------
 # Phase 1 (Algorithm 1)
 # --------------------------------------------------------------------------
