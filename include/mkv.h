@@ -114,13 +114,18 @@ typedef struct {
   int32_t mi;          /* 1: moment-informed second stage; 0: window scores only */
   int32_t causal;      /* 1: window query i (position T-w+i) sees keys t <= T-w+i */
   float tau;           /* clamp |S_tilde_ab| < tau to 0 in the residual (App. C.2) */
+  int32_t adaptive;    /* 1: the layer's budget h_kv * budget is shared by the KV */
+                       /* heads of each batch item (Ada-KV allocation, Sec. 5.1): */
+                       /* both selections take the top of all heads' unprotected  */
+                       /* (head, position) pairs together; 0: budget per unit    */
 } mkv_compress_params;
 
 /* Optional outputs of mkv_compress for inspection; any field may be NULL. */
 typedef struct {
   float* scores;       /* fp32 [b, h_kv, T] pooled window scores s_t               */
   float* score2;       /* fp32 [b, h_kv, T] s_t * ||r_t|| (mi=1); protected rows 0 */
-  int32_t* idx_stage1; /* int32 [b, h_kv, budget] first-stage retained positions    */
+  int32_t* idx_stage1; /* int32 [b, h_kv, budget] first-stage retained positions;   */
+                       /* with adaptive, [b, h_kv * budget] of h * T + t, ascending */
 } mkv_compress_diag;
 
 /* Decode parameters (Algorithm 1 Phase 2, Table 4, App. C.2). */
@@ -173,8 +178,15 @@ MKV_API size_t mkv_compress_workspace_size(mkv_geom geom, int32_t T, const mkv_c
  *   4. writes the retained rows of R to out_cache in ascending position
  *      (K, V, pos), len = |R|, seen = T, and the moments of E = all \ R to
  *      out_mom (overwritten).  If T <= budget every token is kept and n = 0.
+ * With adaptive = 1 (T > budget), steps 2 and 3 select jointly over the h_kv
+ * heads of a batch item: R_h = protected_h plus head h's share of the top
+ * h_kv * (budget - |protected|) unprotected (head, position) pairs; ties keep
+ * the lower head, then the lower position.  len then differs per head and
+ * sums to h_kv * budget over a batch item; rows of out_cache from len up to
+ * the next multiple of 128 (below capacity) are overwritten with zeros.
  * Requirements: budget >= sink + (keep_window ? w : 0), 1 <= w <= T,
- * out_cache->capacity >= min(T, budget), T <= 1,048,576.
+ * out_cache->capacity >= min(T, budget) (adaptive: >= min(T, h_kv * budget -
+ * (h_kv - 1) * |protected|), h_kv <= 64, h_kv * T <= 2^28), T <= 1,048,576.
  */
 MKV_API mkv_status mkv_compress(mkv_geom geom, int32_t T, const void* K, const void* V, const void* Q_obs,
                         const mkv_compress_params* p, const mkv_cache* out_cache,

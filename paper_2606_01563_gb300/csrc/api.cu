@@ -66,7 +66,7 @@ const char* mkv_status_str(mkv_status s) {
   return "unknown status";
 }
 
-int32_t mkv_version(void) { return 100; }
+int32_t mkv_version(void) { return 200; }
 
 // ------------------------------------------------------------------ decode
 size_t mkv_decode_workspace_size(mkv_geom geom, int32_t capacity) {
@@ -173,7 +173,18 @@ static mkv_status compress_params_ok(const mkv_geom& geom, int32_t T, const mkv_
   if ((long)geom.group * p->window > 1024) return MKV_ERR_SHAPE;
   if (T > p->budget && protected_count_host(T, p->window, p->sink, p->keep_window) > p->budget)
     return MKV_ERR_INVALID_ARG;
+  if (p->adaptive != 0 && p->adaptive != 1) return MKV_ERR_INVALID_ARG;
+  if (p->adaptive && (geom.n_kv_heads > 64 || (long)geom.n_kv_heads * T > (1L << 28))) return MKV_ERR_SHAPE;
   return MKV_OK;
+}
+
+// rows one unit may retain: min(T, budget), or with the adaptive allocation
+// the unit's protected rows plus every joint selection of its batch item
+static long max_retained(const mkv_geom& geom, int32_t T, const mkv_compress_params* p) {
+  if (T <= p->budget || !p->adaptive) return T < p->budget ? T : p->budget;
+  const long prot = protected_count_host(T, p->window, p->sink, p->keep_window);
+  const long m = (long)geom.n_kv_heads * (p->budget - prot) + prot;
+  return m < T ? m : T;
 }
 
 size_t mkv_compress_workspace_size(mkv_geom geom, int32_t T, const mkv_compress_params* p) {
@@ -188,8 +199,7 @@ mkv_status mkv_compress(mkv_geom geom, int32_t T, const void* K, const void* V, 
   if (st != MKV_OK) return st;
   if (!K || !V || !Q_obs || !cache_ok(out_cache) || !moments_ok(out_mom)) return MKV_ERR_INVALID_ARG;
   if (!aligned(K, 16) || !aligned(V, 16) || !aligned(Q_obs, 16)) return MKV_ERR_INVALID_ARG;
-  const int32_t keep = T < p->budget ? T : p->budget;
-  if (out_cache->capacity < keep) return MKV_ERR_CAPACITY;
+  if (out_cache->capacity < max_retained(geom, T, p)) return MKV_ERR_CAPACITY;
   const int sms = num_sms_current();
   const size_t need = compress_workspace_bytes(geom, T, *p, sms);
   if (!workspace || workspace_bytes < need || !aligned(workspace, 256)) return MKV_ERR_WORKSPACE;
@@ -206,6 +216,7 @@ mkv_status mkv_compress(mkv_geom geom, int32_t T, const void* K, const void* V, 
   a.mi = p->mi;
   a.causal = p->causal;
   a.tau = p->tau;
+  a.adaptive = p->adaptive;
   a.cache = *out_cache;
   a.mom = *out_mom;
   a.diag_scores = diag ? diag->scores : nullptr;

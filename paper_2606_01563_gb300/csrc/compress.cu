@@ -26,6 +26,7 @@
 // warp 1 owns TMEM and issues tcgen05.mma, warps 2-5 run the epilogue; stages
 // hand over through mbarriers whose waits are all bounded.  Head dims below
 // 128 use the same 128-wide MMAs: the missing 64-column box is zero-filled.
+#include <algorithm>
 #include <cooperative_groups.h>
 
 #include "common.cuh"
@@ -53,6 +54,8 @@ constexpr unsigned kFull = 0xffffffffu;
 struct Layout {
   int D, G, W, RW, RWb;  // head dim, group, window, window rows = G*W, 128-row blocks of them
   int T, B;
+  int hs;    // units per selection group: 1, or the KV heads of a batch item (adaptive budget)
+  int Bcap;  // rows of each unit's gathered slab: B, or the adaptive maximum rounded up to kTok
   int units, n_chunks, chunk;
   size_t rec;         // floats per moment record: 4 + 2D + D*D (padded)
   float* rowpart;     // [units][n_chunks][RW][2]  (max in log2 units, sum)
@@ -61,8 +64,9 @@ struct Layout {
   int n_rchunks;      // chunks of kTok retained rows
   float* s;           // [units][T]
   float* s2;          // [units][T]
-  int32_t* idx;       // [units][B]
-  __nv_bfloat16* gK;  // [units][B][D] rows of R0
+  int32_t* idx;       // [units / hs][hs * B] selection lists (h * T + t), ascending
+  int32_t* cnt;       // [units] rows each unit retains
+  __nv_bfloat16* gK;  // [units][Bcap][D] rows of R0
   __nv_bfloat16* gV;
   float* m0;    // [units][rec] moments of E0
   float* mall;  // [units][rec] moments of all tokens (the merged chunk records)
@@ -70,8 +74,24 @@ struct Layout {
 
 __host__ __device__ inline size_t rec_floats(int D) { return align_up(4 + 2 * (size_t)D + (size_t)D * D, 4); }
 
-Layout make_layout(const mkv_geom& g, int T, int B, int W, int num_sms) {
+__host__ __device__ __forceinline__ int protected_count(int T, int W, int sink, int keep_window) {
+  const int s = sink < T ? sink : T;
+  const int w = keep_window ? (W < T ? W : T) : 0;
+  const int overlap = s - (T - w) > 0 ? s - (T - w) : 0;
+  return s + w - overlap;
+}
+
+Layout make_layout(const mkv_geom& g, int T, int B, int W, int sink, int keep_window, int adaptive,
+                   int num_sms) {
   Layout L{};
+  L.hs = 1;
+  L.Bcap = B;
+  if (adaptive && T > B) {  // a unit keeps its protected rows plus up to every joint selection
+    const long prot = protected_count(T, W, sink, keep_window);
+    const long most = std::min<long>(T, (long)g.n_kv_heads * (B - prot) + prot);
+    L.hs = g.n_kv_heads;
+    L.Bcap = static_cast<int>((most + kTok - 1) / kTok * kTok);
+  }
   L.D = g.head_dim;
   L.G = g.group;
   L.W = W;
@@ -87,7 +107,7 @@ Layout make_layout(const mkv_geom& g, int T, int B, int W, int num_sms) {
   L.chunk = static_cast<int>(((tiles + per - 1) / per) * kTok);
   L.n_chunks = (T + L.chunk - 1) / L.chunk;
   L.rec = rec_floats(L.D);
-  L.n_rchunks = (B + kTok - 1) / kTok;
+  L.n_rchunks = (L.Bcap + kTok - 1) / kTok;
   return L;
 }
 
@@ -106,8 +126,9 @@ size_t carve(Layout& L, void* ws) {
   L.s = reinterpret_cast<float*>(take(U * (size_t)L.T * sizeof(float)));
   L.s2 = reinterpret_cast<float*>(take(U * (size_t)L.T * sizeof(float)));
   L.idx = reinterpret_cast<int32_t*>(take(U * (size_t)L.B * sizeof(int32_t)));
-  L.gK = reinterpret_cast<__nv_bfloat16*>(take(U * (size_t)L.B * L.D * 2));
-  L.gV = reinterpret_cast<__nv_bfloat16*>(take(U * (size_t)L.B * L.D * 2));
+  L.cnt = reinterpret_cast<int32_t*>(take(U * sizeof(int32_t)));
+  L.gK = reinterpret_cast<__nv_bfloat16*>(take(U * (size_t)L.Bcap * L.D * 2));
+  L.gV = reinterpret_cast<__nv_bfloat16*>(take(U * (size_t)L.Bcap * L.D * 2));
   L.m0 = reinterpret_cast<float*>(take(U * L.rec * sizeof(float)));
   L.mall = reinterpret_cast<float*>(take(U * L.rec * sizeof(float)));
   return off;
@@ -115,13 +136,6 @@ size_t carve(Layout& L, void* ws) {
 
 __device__ __forceinline__ bool is_protected(int t, int T, int W, int sink, int keep_window) {
   return t < sink || (keep_window && t >= T - W);
-}
-
-__host__ __device__ __forceinline__ int protected_count(int T, int W, int sink, int keep_window) {
-  const int s = sink < T ? sink : T;
-  const int w = keep_window ? (W < T ? W : T) : 0;
-  const int overlap = s - (T - w) > 0 ? s - (T - w) : 0;
-  return s + w - overlap;
 }
 
 // bf16 element (r, c) of a [128 x 128] tile held as two 64-column boxes with
@@ -144,6 +158,7 @@ __device__ __forceinline__ bool pwait(uint64_t* bar, uint32_t parity, volatile i
 
 struct TcArgs {
   int n_rows;  // rows of each unit's slab that take part
+  const int32_t* rows_u;  // optional per-unit row counts (<= n_rows) that replace n_rows
   int chunk;   // rows per CTA (multiple of kTok)
   int n_chunks;
   int D, RW, RWb, W, T, causal, sink, keep_window, pool;
@@ -185,10 +200,16 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
   const int chunk = blockIdx.x, u = blockIdx.y;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int t_begin = chunk * p.chunk;
-  const int t_end = min(p.n_rows, t_begin + p.chunk);
+  const int n_rows = (!LOGITS && p.rows_u != nullptr) ? p.rows_u[u] : p.n_rows;
+  const int t_end = min(n_rows, t_begin + p.chunk);
   const int n_tiles = (max(0, t_end - t_begin) + kTok - 1) / kTok;
   const int RWb = p.RWb;
   volatile int* abrt = &abort_flag;
+  if (!LOGITS && n_tiles == 0) {  // a chunk past this unit's rows: an empty record (n = 0, zero means)
+    float* rec = p.mrec + ((size_t)u * p.n_chunks + chunk) * rec_floats(p.D);
+    for (int i = tid; i < 4 + 2 * p.D; i += kStatsThreads) rec[i] = 0.f;
+    return;
+  }
 
   if (tid == 0) {
     for (int i = 0; i < kS; ++i) {
@@ -719,8 +740,10 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
 }
 
 // ----------------------------------------------------------------- select
-// One CTA (1024 threads) per unit: R = protected + the k highest keys among
-// the other positions (ties to the lower position), written ascending; the
+// One cluster of kSelCL CTAs per selection group -- a unit, or with the
+// adaptive budget the hs KV heads of a batch item, whose (head, position)
+// pairs f = h * T + t are ranked together.  R = protected + the k highest
+// keys among the other pairs (ties to the lower f), written ascending; the
 // rows of R are gathered into dst_K/dst_V [unit][dst_cap][D] (with positions,
 // length and tokens seen when the destination is a cache).
 __device__ __forceinline__ int block_excl_scan(int flag, int* wsum, int* total) {
@@ -788,11 +811,15 @@ struct SelectArgs {
   int32_t* dst_len;
   int32_t* dst_seen;
   int smem_keys;  // keys of a CTA's range that the dynamic shared memory holds
+  int hs;         // units per selection group (1: one unit; > 1: the KV heads of a batch item)
+  int32_t* cnt;   // [units] rows retained per unit (read by the moments of the gathered set)
+  int zero_pad;   // 1: zero the slab rows from cnt up to the next multiple of kTok (below dst_cap)
 };
 
 constexpr int kFinRB = 2;  // rows of C per finalize CTA
-constexpr int kSelCL = 8;  // CTAs per unit (one cluster), each over a contiguous range of positions
-constexpr int kSelSmemKeys = 24576;  // keys of a CTA's range cached in shared memory (96 KB)
+constexpr int kSelCL = 8;  // CTAs per selection group (one cluster), each over a contiguous range of pairs
+constexpr int kSelSmemKeys = 49152;  // keys of a CTA's range cached in shared memory (192 KB)
+constexpr int kMaxHs = 64;           // KV heads of a batch item with the adaptive budget
 
 __global__ void __cluster_dims__(kSelCL, 1, 1) __launch_bounds__(kSelThreads) select_kernel(const SelectArgs a) {
   __shared__ uint32_t hist[2][256];   // this CTA's histogram, double-buffered by pass parity (read remotely)
@@ -804,14 +831,17 @@ __global__ void __cluster_dims__(kSelCL, 1, 1) __launch_bounds__(kSelThreads) se
   __shared__ int s_need;
   __shared__ int ex_cnt[2];  // this CTA's ties and certain selections (protected or above the threshold)
   __shared__ int s_before[2];
+  __shared__ int s_hstart[kMaxHs + 1];  // first slot of each head in the group's selection list
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = static_cast<int>(cluster.block_rank());
-  const int u = blockIdx.x / kSelCL, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int T = a.T, W = a.W;
-  const int per = (T + kSelCL - 1) / kSelCL;
-  const int r0 = min(T, rank * per), r1 = min(T, r0 + per);
-  const float* sc = a.scores + (size_t)u * T;
-  const int k = a.B - protected_count(T, W, a.sink, a.keep_window);  // >= 0 (validated), < candidates
+  const int grp = blockIdx.x / kSelCL, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int T = a.T, W = a.W, hs = a.hs;
+  const int N = hs * T;  // pairs of the group
+  const int per = (N + kSelCL - 1) / kSelCL;
+  const int r0 = min(N, rank * per), r1 = min(N, r0 + per);
+  const float* sc = a.scores + (size_t)grp * N;  // the group's units are consecutive
+  // >= 0 (validated), < candidates
+  const int k = hs * (a.B - protected_count(T, W, a.sink, a.keep_window));
 
   // The CTA's keys are cached in shared memory when they fit (protected
   // positions hold key 0, which no score maps to: scores are >= 0); larger
@@ -819,15 +849,15 @@ __global__ void __cluster_dims__(kSelCL, 1, 1) __launch_bounds__(kSelThreads) se
   extern __shared__ uint32_t ks[];
   const int nk = r1 - r0;
   const bool cached = nk <= a.smem_keys;
-  auto key_at = [&](int t) -> uint32_t {  // 0 for protected positions
-    if (cached) return ks[t - r0];
-    return is_protected(t, T, W, a.sink, a.keep_window) ? 0u : float_key(sc[t]);
+  auto key_of = [&](int f) -> uint32_t {
+    const int t = hs == 1 ? f : f % T;
+    return is_protected(t, T, W, a.sink, a.keep_window) ? 0u : float_key(sc[f]);
+  };
+  auto key_at = [&](int f) -> uint32_t {  // 0 for protected positions
+    return cached ? ks[f - r0] : key_of(f);
   };
   if (cached) {
-    for (int i = tid; i < nk; i += kSelThreads) {
-      const int t = r0 + i;
-      ks[i] = is_protected(t, T, W, a.sink, a.keep_window) ? 0u : float_key(sc[t]);
-    }
+    for (int i = tid; i < nk; i += kSelThreads) ks[i] = key_of(r0 + i);
     __syncthreads();
   }
   // thread tid owns the contiguous positions [t0, t1) in the ordered passes
@@ -930,7 +960,8 @@ __global__ void __cluster_dims__(kSelCL, 1, 1) __launch_bounds__(kSelThreads) se
   const int sel_excl = block_excl_sum(my_sel, wsum, &tot);
   const int my_first = cta_sel_before;
   int o = cta_sel_before + sel_excl;
-  int32_t* out = a.idx + (size_t)u * a.B;
+  const int n_sel = hs * a.B;  // the group's selections (protected included)
+  int32_t* out = a.idx + (size_t)grp * n_sel;
   for (int t = t0; t < t1; ++t) {
     const uint32_t key = key_at(t);
     bool sel = true;  // protected
@@ -940,33 +971,74 @@ __global__ void __cluster_dims__(kSelCL, 1, 1) __launch_bounds__(kSelThreads) se
       tb += tie ? 1 : 0;
     }
     if (sel) {
-      if (o < a.B) {
+      if (o < n_sel) {
         out[o] = t;
-        if (a.diag_idx) a.diag_idx[(size_t)u * a.B + o] = t;
+        if (a.diag_idx) a.diag_idx[(size_t)grp * n_sel + o] = t;
       }
       ++o;
     }
   }
   const int sel_before = cta_sel_before + tot;  // this CTA's selections end here
+  if (hs > 1) {
+    // each head's slots are a contiguous run of the ascending list: its
+    // first slot is the first entry >= h * T (a search of the whole list,
+    // which the cluster barrier makes visible)
+    cluster.sync();
+    if (tid <= hs) {
+      int lo = 0, hi = n_sel;
+      while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (__ldcg(out + mid) < tid * T) lo = mid + 1;
+        else hi = mid;
+      }
+      s_hstart[tid] = lo;
+    }
+  } else if (tid == 0) {
+    s_hstart[0] = 0;
+    s_hstart[1] = a.B;
+  }
   __syncthreads();
   // gather the rows this CTA selected (16-byte chunks)
   const int D = a.D;
   const int per_row = D / 8;
-  const int o0 = min(my_first, a.B), o1 = min(sel_before, a.B);
+  const int o0 = min(my_first, n_sel), o1 = min(sel_before, n_sel);
   for (int i = tid; i < (o1 - o0) * per_row; i += kSelThreads) {
-    const int r = o0 + i / per_row, c = i % per_row;
-    const int t = min(max(out[r], 0), T - 1);  // never read outside the unit's slab
-    const size_t src = ((size_t)u * T + t) * D;
-    const size_t dst = ((size_t)u * a.dst_cap + r) * D;
+    const int o_ = o0 + i / per_row, c = i % per_row;
+    const int f = min(max(out[o_], 0), N - 1);  // never read outside the group's slabs
+    const int h = hs == 1 ? 0 : f / T;
+    const int r = o_ - s_hstart[h];
+    if (r >= a.dst_cap) continue;  // capacity is validated on the host
+    const size_t u = (size_t)grp * hs + h;
+    const size_t src = ((size_t)grp * N + f) * D;
+    const size_t dst = (u * a.dst_cap + r) * D;
     reinterpret_cast<uint4*>(a.dst_K + dst)[c] = reinterpret_cast<const uint4*>(a.K + src)[c];
     reinterpret_cast<uint4*>(a.dst_V + dst)[c] = reinterpret_cast<const uint4*>(a.V + src)[c];
   }
   if (a.dst_pos)
-    for (int r = o0 + tid; r < o1; r += kSelThreads) a.dst_pos[(size_t)u * a.dst_cap + r] = out[r];
-  if (rank == 0 && tid == 0 && a.dst_len) {
-    a.dst_len[u] = a.B;
-    a.dst_seen[u] = T;
+    for (int o_ = o0 + tid; o_ < o1; o_ += kSelThreads) {
+      const int f = out[o_], h = hs == 1 ? 0 : f / T;
+      const int r = o_ - s_hstart[h];
+      if (r < a.dst_cap) a.dst_pos[((size_t)grp * hs + h) * a.dst_cap + r] = f - h * T;
+    }
+  if (rank == 0 && tid < hs) {
+    const int u = grp * hs + tid, c = s_hstart[tid + 1] - s_hstart[tid];
+    if (a.cnt) a.cnt[u] = c;
+    if (a.dst_len) {
+      a.dst_len[u] = c;
+      a.dst_seen[u] = T;
+    }
   }
+  if (a.zero_pad)  // rows [c, next multiple of kTok) of each unit: the moments of the slab read whole tiles
+    for (int h = rank; h < hs; h += kSelCL) {
+      const int c = s_hstart[h + 1] - s_hstart[h];
+      const int r1z = min(a.dst_cap, (c + kTok - 1) / kTok * kTok);
+      const size_t base = ((size_t)grp * hs + h) * a.dst_cap;
+      for (int i = tid; i < max(0, r1z - c) * per_row; i += kSelThreads) {
+        const size_t dst = (base + c + i / per_row) * D;
+        reinterpret_cast<uint4*>(a.dst_K + dst)[i % per_row] = make_uint4(0u, 0u, 0u, 0u);
+        reinterpret_cast<uint4*>(a.dst_V + dst)[i % per_row] = make_uint4(0u, 0u, 0u, 0u);
+      }
+    }
   cluster.sync();  // no CTA leaves while another may still read its shared memory
 }
 
@@ -1018,8 +1090,8 @@ __global__ void __launch_bounds__(256) finalize_kernel(const Layout L, float* ou
 #pragma unroll 8
         for (int ch = 0; ch < nb; ++ch) {
           const float nc = s_nc[ch];
-          const float m = rbase[(size_t)(g0 + ch) * rf + 4 + 2 * D + (size_t)row * D + c];
-          if (nc > 0.f) {
+          if (nc > 0.f) {  // an empty record's co-moment is never written
+            const float m = rbase[(size_t)(g0 + ch) * rf + 4 + 2 * D + (size_t)row * D + c];
             const float dv = s_dv[ch][ar], dk = s_dk[ch][c];
             st.n += nc;
             st.sv = fmaf(nc, dv, st.sv);
@@ -1108,9 +1180,10 @@ constexpr size_t kScoresSmem = 1024 + 3 * kTileBytes + 2 * 2 * kBoxBytes;
 constexpr size_t kResidualSmem = 1024 + 2 * 2 * kTileBytes + 3 * kTileBytes;
 
 cudaError_t run(const CompressArgs& a, const mkv_geom& g, int num_sms, cudaStream_t st) {
-  Layout L = make_layout(g, a.T, a.budget, a.window, num_sms);
+  Layout L = make_layout(g, a.T, a.budget, a.window, a.sink, a.keep_window, a.adaptive, num_sms);
   carve(L, a.ws);
-  const int D = g.head_dim, T = a.T, B = a.budget, U = L.units;
+  const int D = g.head_dim, T = a.T, B = a.budget, U = L.units, Bc = L.Bcap;
+  const bool joint = L.hs > 1;
   const bool keep_all = T <= B;
   cudaError_t e = cudaSuccess;
   auto attr = [](const void* f, size_t bytes) {
@@ -1126,11 +1199,14 @@ cudaError_t run(const CompressArgs& a, const mkv_geom& g, int num_sms, cudaStrea
   bool ok = encode_tmap_bf16_3d(&tmK, a.K, D, T, U, rs, (uint64_t)T * rs, kTok) &&
             encode_tmap_bf16_3d(&tmV, a.V, D, T, U, rs, (uint64_t)T * rs, kTok) &&
             encode_tmap_bf16_3d(&tmQ, a.Q, D, L.RW, U, rs, (uint64_t)L.RW * rs, L.RWb * 128);
+  // the retained rows: B per unit, or (joint) up to the capacity with the
+  // rows past each unit's count zero up to the tile (or outside the map)
+  const int cache_rows = joint ? a.cache.capacity : B;
   if (!keep_all)
-    ok = ok && encode_tmap_bf16_3d(&tmGK, L.gK, D, B, U, rs, (uint64_t)B * rs, kTok) &&
-         encode_tmap_bf16_3d(&tmGV, L.gV, D, B, U, rs, (uint64_t)B * rs, kTok) &&
-         encode_tmap_bf16_3d(&tmCK, a.cache.K, D, B, U, rs, (uint64_t)a.cache.capacity * rs, kTok) &&
-         encode_tmap_bf16_3d(&tmCV, a.cache.V, D, B, U, rs, (uint64_t)a.cache.capacity * rs, kTok);
+    ok = ok && encode_tmap_bf16_3d(&tmGK, L.gK, D, Bc, U, rs, (uint64_t)Bc * rs, kTok) &&
+         encode_tmap_bf16_3d(&tmGV, L.gV, D, Bc, U, rs, (uint64_t)Bc * rs, kTok) &&
+         encode_tmap_bf16_3d(&tmCK, a.cache.K, D, cache_rows, U, rs, (uint64_t)a.cache.capacity * rs, kTok) &&
+         encode_tmap_bf16_3d(&tmCV, a.cache.V, D, cache_rows, U, rs, (uint64_t)a.cache.capacity * rs, kTok);
   if (!ok) return cudaErrorInvalidValue;
 
   TcArgs tp{};
@@ -1168,7 +1244,8 @@ cudaError_t run(const CompressArgs& a, const mkv_geom& g, int num_sms, cudaStrea
   }
 
   SelectArgs sa{};
-  const int sel_per = (T + kSelCL - 1) / kSelCL;
+  const int n_groups = U / L.hs;
+  const int sel_per = (L.hs * T + kSelCL - 1) / kSelCL;
   sa.smem_keys = sel_per <= kSelSmemKeys ? sel_per : 0;
   const size_t sel_smem = (size_t)sa.smem_keys * sizeof(uint32_t);
   if ((e = attr((const void*)select_kernel, sel_smem)) != cudaSuccess) return e;
@@ -1181,8 +1258,12 @@ cudaError_t run(const CompressArgs& a, const mkv_geom& g, int num_sms, cudaStrea
   sa.K = static_cast<const __nv_bfloat16*>(a.K);
   sa.V = static_cast<const __nv_bfloat16*>(a.V);
   sa.idx = L.idx;
+  sa.hs = L.hs;
+  sa.cnt = L.cnt;
+  sa.zero_pad = joint ? 1 : 0;
   TcArgs rset = tp;  // moments of a dense row set: chunks of kTok rows
-  rset.n_rows = B;
+  rset.n_rows = Bc;
+  rset.rows_u = joint ? L.cnt : nullptr;
   rset.chunk = kTok;
   rset.n_chunks = L.n_rchunks;
   rset.mrec = L.rpart;
@@ -1193,8 +1274,8 @@ cudaError_t run(const CompressArgs& a, const mkv_geom& g, int num_sms, cudaStrea
     s0.diag_idx = a.diag_idx1;
     s0.dst_K = L.gK;
     s0.dst_V = L.gV;
-    s0.dst_cap = B;
-    select_kernel<<<U * kSelCL, kSelThreads, sel_smem, st>>>(s0);
+    s0.dst_cap = Bc;
+    select_kernel<<<n_groups * kSelCL, kSelThreads, sel_smem, st>>>(s0);
     stats_tc<0><<<dim3(L.n_rchunks, U), kStatsThreads, kStats0Smem, st>>>(rset, tmGK, tmGV, tmQ);
     finalize_kernel<<<dim3(D / kFinRB, U), 256, 0, st>>>(L, L.m0, a.mom, 0, 1);
     TcArgs r = tp;
@@ -1216,7 +1297,7 @@ cudaError_t run(const CompressArgs& a, const mkv_geom& g, int num_sms, cudaStrea
   s1.dst_pos = a.cache.pos;
   s1.dst_len = a.cache.len;
   s1.dst_seen = a.cache.seen;
-  select_kernel<<<U * kSelCL, kSelThreads, sel_smem, st>>>(s1);
+  select_kernel<<<n_groups * kSelCL, kSelThreads, sel_smem, st>>>(s1);
   stats_tc<0><<<dim3(L.n_rchunks, U), kStatsThreads, kStats0Smem, st>>>(rset, tmCK, tmCV, tmQ);
   finalize_kernel<<<dim3(D / kFinRB, U), 256, 0, st>>>(L, nullptr, a.mom, 1, a.mi ? 0 : 1);
   return cudaGetLastError();
@@ -1225,7 +1306,7 @@ cudaError_t run(const CompressArgs& a, const mkv_geom& g, int num_sms, cudaStrea
 }  // namespace
 
 size_t compress_workspace_bytes(const mkv_geom& g, int32_t T, const mkv_compress_params& p, int num_sms) {
-  Layout L = make_layout(g, T, p.budget, p.window, num_sms);
+  Layout L = make_layout(g, T, p.budget, p.window, p.sink, p.keep_window, p.adaptive, num_sms);
   return carve(L, nullptr);
 }
 

@@ -97,6 +97,7 @@ struct CompressArgs {
   int32_t mi;
   int32_t causal;
   float tau;
+  int32_t adaptive;   // 1: joint selection over the KV heads of each batch item
   mkv_cache cache;
   mkv_moments mom;
   float* diag_scores;

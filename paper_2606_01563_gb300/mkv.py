@@ -35,7 +35,7 @@ class mkv_cache(ctypes.Structure):
 
 class mkv_compress_params(ctypes.Structure):
     _fields_ = [("budget", c_i32), ("window", c_i32), ("sink", c_i32), ("keep_window", c_i32),
-                ("pool", c_i32), ("mi", c_i32), ("causal", c_i32), ("tau", ctypes.c_float)]
+                ("pool", c_i32), ("mi", c_i32), ("causal", c_i32), ("tau", ctypes.c_float), ("adaptive", c_i32)]
 
 
 class mkv_compress_diag(ctypes.Structure):

@@ -34,7 +34,7 @@ def test_every_declared_symbol_is_exported(L):
 
 
 def test_version_and_status_strings(L):
-    assert mkv.mkv_version() == 100
+    assert mkv.mkv_version() == 200
     for code in range(8):
         assert mkv.mkv_status_str(code)
     assert mkv.mkv_status_str(99) == "unknown status"
@@ -120,6 +120,15 @@ def test_compress_validation(L):
     assert compress(L, g, 1024, P(), K=None) == 1
     assert compress(L, g, 1024, P(), wsb=1024) == 7
     assert compress(L, mkv.geom(1, 2, 2, 100), 1024, P()) == 6
+    # adaptive budget: a head may keep 17 protected rows plus all 2 * 111 joint selections
+    assert compress(L, g, 1024, P(adaptive=2)) == 1
+    assert compress(L, g, 1024, P(adaptive=1), cache=fake_cache(238)) == 3
+    assert compress(L, g, 1024, P(adaptive=1), cache=fake_cache(239), wsb=1024) == 7
+    assert compress(L, g, 200, P(adaptive=1), cache=fake_cache(199), wsb=1024) == 3   # min(T, ...) = T
+    assert compress(L, mkv.geom(1, 65, 2, 64), 1024, P(adaptive=1)) == 2
+    ws0 = L.mkv_compress_workspace_size(g, 1024, ctypes.byref(P()))
+    ws1 = L.mkv_compress_workspace_size(g, 1024, ctypes.byref(P(adaptive=1)))
+    assert ws1 > ws0 > 0
 
 
 def test_evict_validation(L):
