@@ -519,7 +519,9 @@ def decode_layers(torch, mkv, dev, flush, hbm, b, B, gen, st):
 
 def compress_long(torch, mkv, inputs, dev, flush, hbm):
     """Compress throughput at 32K (Qwen3-4B geometry, batch 4, budget 1024) and 128K
-    (Llama-3.1-8B geometry, batch 1, budget 128, window 64) context, one layer."""
+    (Llama-3.1-8B geometry, batch 1, budget 128, window 64) context, one layer;
+    ms_adaptive is the same compression with the budget shared by the KV heads
+    of each batch item."""
     res = {}
     st = torch.cuda.Stream(dev)
     for name in ("qwen4b_t32k", "llama8b_t128k"):
@@ -530,29 +532,37 @@ def compress_long(torch, mkv, inputs, dev, flush, hbm):
         K, V, Q = gen.prefill()
         tb = inputs.to_bf16_tensor
         K, V, Q = tb(K).to(dev), tb(V).to(dev), tb(Q).to(dev)
-        p = mkv.mkv_compress_params(wl.budget, wl.window, 1, 1, 1, 1, 1, 1e-6)
-        cache, mom = mkv.alloc_cache(g, wl.budget + EVICT_EVERY, dev), mkv.alloc_moments(g, dev)
-        ws = mkv.alloc_workspace(mkv.mkv_compress_workspace_size(g, wl.T, p), dev)
-        times = []
-        for it in range(5):
-            with torch.cuda.stream(st):
-                flush.zero_()
-                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-                e0.record(st)
-                mkv.mkv_compress(g, wl.T, K, V, Q, p, cache, mom, ws, stream=st)
-                e1.record(st)
-            st.synchronize()
-            if it >= 1:
-                times.append(e0.elapsed_time(e1))
-        code, _ = mkv.mkv_get_device_error(ws, st)
-        t = float(np.median(times))
-        units = G.batch * G.n_kv_heads
-        byt = units * 2 * wl.T * G.head_dim * 2
-        flops = units * (2 * G.group * wl.window * wl.T * G.head_dim + 4 * wl.T * G.head_dim ** 2)
-        res[name] = {"T": wl.T, "batch": G.batch, "budget": wl.budget, "ms": round(t, 3),
-                     "gbs": round(byt / t / 1e6, 1), "frac_hbm": round(byt / t / 1e6 / hbm, 4),
-                     "tflops": round(flops / t / 1e9, 2), "ok": code == 0}
-        del K, V, Q, cache, mom, ws
+        prot = 1 + wl.window
+        for adaptive in (0, 1):
+            p = mkv.mkv_compress_params(wl.budget, wl.window, 1, 1, 1, 1, 1, 1e-6, adaptive)
+            cap = min(wl.T, G.n_kv_heads * (wl.budget - prot) + prot) if adaptive else wl.budget + EVICT_EVERY
+            cache, mom = mkv.alloc_cache(g, cap, dev), mkv.alloc_moments(g, dev)
+            ws = mkv.alloc_workspace(mkv.mkv_compress_workspace_size(g, wl.T, p), dev)
+            times = []
+            for it in range(5):
+                with torch.cuda.stream(st):
+                    flush.zero_()
+                    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                    e0.record(st)
+                    mkv.mkv_compress(g, wl.T, K, V, Q, p, cache, mom, ws, stream=st)
+                    e1.record(st)
+                st.synchronize()
+                if it >= 1:
+                    times.append(e0.elapsed_time(e1))
+            code, _ = mkv.mkv_get_device_error(ws, st)
+            t = float(np.median(times))
+            if adaptive:  # the budget shared by the KV heads of each batch item
+                res[name]["ms_adaptive"] = round(t, 3)
+                res[name]["ok"] = res[name]["ok"] and code == 0
+            else:
+                units = G.batch * G.n_kv_heads
+                byt = units * 2 * wl.T * G.head_dim * 2
+                flops = units * (2 * G.group * wl.window * wl.T * G.head_dim + 4 * wl.T * G.head_dim ** 2)
+                res[name] = {"T": wl.T, "batch": G.batch, "budget": wl.budget, "ms": round(t, 3),
+                             "gbs": round(byt / t / 1e6, 1), "frac_hbm": round(byt / t / 1e6 / hbm, 4),
+                             "tflops": round(flops / t / 1e9, 2), "ok": code == 0}
+            del cache, mom, ws
+        del K, V, Q
         torch.cuda.empty_cache()
     return res
 

@@ -56,6 +56,7 @@ struct Layout {
   int T, B;
   int hs;    // units per selection group: 1, or the KV heads of a batch item (adaptive budget)
   int Bcap;  // rows of each unit's gathered slab: B, or the adaptive maximum rounded up to kTok
+  int Tc;    // joint selection entries per unit: T, or the length of its candidate list
   int units, n_chunks, chunk;
   size_t rec;         // floats per moment record: 4 + 2D + D*D (padded)
   float* rowpart;     // [units][n_chunks][RW][2]  (max in log2 units, sum)
@@ -66,6 +67,10 @@ struct Layout {
   float* s2;          // [units][T]
   int32_t* idx;       // [units / hs][hs * B] selection lists (h * T + t), ascending
   int32_t* cnt;       // [units] rows each unit retains
+  int32_t* cand;      // [units][Tc] per-unit candidates of a joint selection (when Tc < T)
+  int32_t* hbeg;      // [units] first slot of each unit in idx
+  int32_t* tile0;     // [units / hs][hs + 1] first retained-row tile of each unit in its group (joint)
+  int gtiles;         // bound on a group's retained-row tiles (joint)
   __nv_bfloat16* gK;  // [units][Bcap][D] rows of R0
   __nv_bfloat16* gV;
   float* m0;    // [units][rec] moments of E0
@@ -86,11 +91,18 @@ Layout make_layout(const mkv_geom& g, int T, int B, int W, int sink, int keep_wi
   Layout L{};
   L.hs = 1;
   L.Bcap = B;
+  L.Tc = T;
   if (adaptive && T > B) {  // a unit keeps its protected rows plus up to every joint selection
     const long prot = protected_count(T, W, sink, keep_window);
     const long most = std::min<long>(T, (long)g.n_kv_heads * (B - prot) + prot);
     L.hs = g.n_kv_heads;
     L.Bcap = static_cast<int>((most + kTok - 1) / kTok * kTok);
+    // every pair of the joint top k is in its own head's top k, so a first
+    // per-unit selection of those (`most` rows with the protected ones)
+    // leaves the joint one fewer entries when they are well below T
+    if (2 * most <= T) L.Tc = static_cast<int>(most);
+    // sum_h ceil(c_h / kTok) with sum_h c_h = hs * B
+    L.gtiles = static_cast<int>(((long)L.hs * B + (long)L.hs * (kTok - 1)) / kTok);
   }
   L.D = g.head_dim;
   L.G = g.group;
@@ -127,6 +139,9 @@ size_t carve(Layout& L, void* ws) {
   L.s2 = reinterpret_cast<float*>(take(U * (size_t)L.T * sizeof(float)));
   L.idx = reinterpret_cast<int32_t*>(take(U * (size_t)L.B * sizeof(int32_t)));
   L.cnt = reinterpret_cast<int32_t*>(take(U * sizeof(int32_t)));
+  L.cand = L.Tc < L.T ? reinterpret_cast<int32_t*>(take(U * (size_t)L.Tc * sizeof(int32_t))) : nullptr;
+  L.hbeg = reinterpret_cast<int32_t*>(take(U * sizeof(int32_t)));
+  L.tile0 = reinterpret_cast<int32_t*>(take((U / L.hs) * (size_t)(L.hs + 1) * sizeof(int32_t)));
   L.gK = reinterpret_cast<__nv_bfloat16*>(take(U * (size_t)L.Bcap * L.D * 2));
   L.gV = reinterpret_cast<__nv_bfloat16*>(take(U * (size_t)L.Bcap * L.D * 2));
   L.m0 = reinterpret_cast<float*>(take(U * L.rec * sizeof(float)));
@@ -159,6 +174,8 @@ __device__ __forceinline__ bool pwait(uint64_t* bar, uint32_t parity, volatile i
 struct TcArgs {
   int n_rows;  // rows of each unit's slab that take part
   const int32_t* rows_u;  // optional per-unit row counts (<= n_rows) that replace n_rows
+  const int32_t* tile0;   // optional [groups][hs + 1]: grid (tiles of a group, groups), as in gather_kernel
+  int hs;
   int chunk;   // rows per CTA (multiple of kTok)
   int n_chunks;
   int D, RW, RWb, W, T, causal, sink, keep_window, pool;
@@ -197,7 +214,15 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
   __shared__ float sum_k[kDP], sum_v[kDP];
   __shared__ float s_m1[2][128], s_l1[2][128];  // the second epilogue group's row stats
 
-  const int chunk = blockIdx.x, u = blockIdx.y;
+  int chunk = blockIdx.x, u = blockIdx.y;
+  if (!LOGITS && p.tile0 != nullptr) {  // the group's tiles, unit by unit
+    const int32_t* t0 = p.tile0 + (size_t)blockIdx.y * (p.hs + 1);
+    if (chunk >= t0[p.hs]) return;
+    int h = 0;
+    while (h + 1 < p.hs && t0[h + 1] <= chunk) ++h;
+    u = blockIdx.y * p.hs + h;
+    chunk -= t0[h];
+  }
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int t_begin = chunk * p.chunk;
   const int n_rows = (!LOGITS && p.rows_u != nullptr) ? p.rows_u[u] : p.n_rows;
@@ -802,18 +827,21 @@ struct SelectArgs {
   int T, W, B, sink, keep_window, D;
   const __nv_bfloat16* K;  // prompt [units][T][D]
   const __nv_bfloat16* V;
-  int32_t* idx;          // [units][B] retained positions (workspace)
+  int32_t* idx;          // [groups][hs * B] selection lists, h * T + position, ascending (workspace)
   int32_t* diag_idx;     // optional copy
-  __nv_bfloat16* dst_K;  // [units][dst_cap][D]
+  __nv_bfloat16* dst_K;  // optional (one unit per group): the rows are gathered here, [units][dst_cap][D]
   __nv_bfloat16* dst_V;
   int dst_cap;
-  int32_t* dst_pos;  // optional cache bookkeeping
+  int32_t* dst_pos;      // optional cache bookkeeping
   int32_t* dst_len;
   int32_t* dst_seen;
   int smem_keys;  // keys of a CTA's range that the dynamic shared memory holds
   int hs;         // units per selection group (1: one unit; > 1: the KV heads of a batch item)
-  int32_t* cnt;   // [units] rows retained per unit (read by the moments of the gathered set)
-  int zero_pad;   // 1: zero the slab rows from cnt up to the next multiple of kTok (below dst_cap)
+  const int32_t* cand;  // optional [units][Tc] ascending candidate positions per unit (null: all T)
+  int Tc;               // entries per unit taking part: T, or the candidate lists' length
+  int32_t* cnt;    // optional [units] rows retained per unit
+  int32_t* hbeg;   // optional [units] the unit's first slot in idx
+  int32_t* tile0;  // optional [groups][hs + 1] first kTok-row tile of each unit within its group, and the total
 };
 
 constexpr int kFinRB = 2;  // rows of C per finalize CTA
@@ -821,7 +849,7 @@ constexpr int kSelCL = 8;  // CTAs per selection group (one cluster), each over 
 constexpr int kSelSmemKeys = 49152;  // keys of a CTA's range cached in shared memory (192 KB)
 constexpr int kMaxHs = 64;           // KV heads of a batch item with the adaptive budget
 
-__global__ void __cluster_dims__(kSelCL, 1, 1) __launch_bounds__(kSelThreads) select_kernel(const SelectArgs a) {
+__global__ void __cluster_dims__(kSelCL, 1, 1) __launch_bounds__(kSelThreads, 2) select_kernel(const SelectArgs a) {
   __shared__ uint32_t hist[2][256];   // this CTA's histogram, double-buffered by pass parity (read remotely)
   __shared__ uint32_t whist[8][256];  // private histograms for groups of 4 warps (less atomic contention)
   __shared__ uint32_t ghist[256];     // the cluster's histogram
@@ -832,14 +860,24 @@ __global__ void __cluster_dims__(kSelCL, 1, 1) __launch_bounds__(kSelThreads) se
   __shared__ int ex_cnt[2];  // this CTA's ties and certain selections (protected or above the threshold)
   __shared__ int s_before[2];
   __shared__ int s_hstart[kMaxHs + 1];  // first slot of each head in the group's selection list
+  __shared__ int s_hcnt[kMaxHs];        // this CTA's selections per head (read remotely)
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = static_cast<int>(cluster.block_rank());
   const int grp = blockIdx.x / kSelCL, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int T = a.T, W = a.W, hs = a.hs;
-  const int N = hs * T;  // pairs of the group
+  // entries f = h * Tc + j of the group stand for (head h, position t), t = j
+  // or the candidate cand[h][j]; either way f ascending is (h, t) ascending
+  const int Tc = a.Tc;
+  const int N = hs * Tc;
   const int per = (N + kSelCL - 1) / kSelCL;
   const int r0 = min(N, rank * per), r1 = min(N, r0 + per);
-  const float* sc = a.scores + (size_t)grp * N;  // the group's units are consecutive
+  const float* sc = a.scores + (size_t)grp * hs * T;  // the group's units are consecutive
+  const int32_t* cand = a.cand ? a.cand + (size_t)grp * N : nullptr;
+  auto pos_of = [&](int f, int& h) -> int {  // (head, position) of entry f
+    h = hs == 1 ? 0 : f / Tc;
+    const int j = f - h * Tc;
+    return cand ? cand[f] : j;
+  };
   // >= 0 (validated), < candidates
   const int k = hs * (a.B - protected_count(T, W, a.sink, a.keep_window));
 
@@ -850,16 +888,17 @@ __global__ void __cluster_dims__(kSelCL, 1, 1) __launch_bounds__(kSelThreads) se
   const int nk = r1 - r0;
   const bool cached = nk <= a.smem_keys;
   auto key_of = [&](int f) -> uint32_t {
-    const int t = hs == 1 ? f : f % T;
-    return is_protected(t, T, W, a.sink, a.keep_window) ? 0u : float_key(sc[f]);
+    int h;
+    const int t = pos_of(f, h);
+    return is_protected(t, T, W, a.sink, a.keep_window) ? 0u : float_key(sc[(size_t)h * T + t]);
   };
   auto key_at = [&](int f) -> uint32_t {  // 0 for protected positions
     return cached ? ks[f - r0] : key_of(f);
   };
-  if (cached) {
+  for (int h = tid; h < hs; h += kSelThreads) s_hcnt[h] = 0;
+  if (cached)
     for (int i = tid; i < nk; i += kSelThreads) ks[i] = key_of(r0 + i);
-    __syncthreads();
-  }
+  __syncthreads();
   // thread tid owns the contiguous positions [t0, t1) in the ordered passes
   const int E = (nk + kSelThreads - 1) / kSelThreads;
   const int t0 = min(r1, r0 + tid * E), t1 = min(r1, t0 + E);
@@ -962,6 +1001,7 @@ __global__ void __cluster_dims__(kSelCL, 1, 1) __launch_bounds__(kSelThreads) se
   int o = cta_sel_before + sel_excl;
   const int n_sel = hs * a.B;  // the group's selections (protected included)
   int32_t* out = a.idx + (size_t)grp * n_sel;
+  int cur_h = 0, cur_n = 0;  // this thread's run of selections in one head (ranges rarely span two)
   for (int t = t0; t < t1; ++t) {
     const uint32_t key = key_at(t);
     bool sel = true;  // protected
@@ -971,75 +1011,144 @@ __global__ void __cluster_dims__(kSelCL, 1, 1) __launch_bounds__(kSelThreads) se
       tb += tie ? 1 : 0;
     }
     if (sel) {
-      if (o < n_sel) {
-        out[o] = t;
-        if (a.diag_idx) a.diag_idx[(size_t)grp * n_sel + o] = t;
+      if (o < n_sel) {  // stored as h * T + position
+        int h;
+        const int pt = pos_of(t, h);
+        out[o] = h * T + pt;
+        if (a.diag_idx) a.diag_idx[(size_t)grp * n_sel + o] = h * T + pt;
+        if (h != cur_h) {
+          if (cur_n) atomicAdd(&s_hcnt[cur_h], cur_n);
+          cur_h = h;
+          cur_n = 0;
+        }
+        ++cur_n;
       }
       ++o;
     }
   }
-  const int sel_before = cta_sel_before + tot;  // this CTA's selections end here
   if (hs > 1) {
-    // each head's slots are a contiguous run of the ascending list: its
-    // first slot is the first entry >= h * T (a search of the whole list,
-    // which the cluster barrier makes visible)
+    // each head's slots are a contiguous run of the ascending list, as long
+    // as the head's selections in all CTAs of the cluster
+    if (cur_n) atomicAdd(&s_hcnt[cur_h], cur_n);
     cluster.sync();
-    if (tid <= hs) {
-      int lo = 0, hi = n_sel;
-      while (lo < hi) {
-        const int mid = (lo + hi) >> 1;
-        if (__ldcg(out + mid) < tid * T) lo = mid + 1;
-        else hi = mid;
-      }
-      s_hstart[tid] = lo;
+    if (tid < hs) {
+      int c = 0;
+#pragma unroll
+      for (int r = 0; r < kSelCL; ++r) c += cluster.map_shared_rank(s_hcnt, r)[tid];
+      s_hstart[tid + 1] = c;
+    }
+    __syncthreads();
+    if (tid == 0) {
+      s_hstart[0] = 0;
+      for (int h = 0; h < hs; ++h) s_hstart[h + 1] += s_hstart[h];
     }
   } else if (tid == 0) {
     s_hstart[0] = 0;
     s_hstart[1] = a.B;
   }
   __syncthreads();
-  // gather the rows this CTA selected (16-byte chunks)
-  const int D = a.D;
-  const int per_row = D / 8;
-  const int o0 = min(my_first, n_sel), o1 = min(sel_before, n_sel);
-  for (int i = tid; i < (o1 - o0) * per_row; i += kSelThreads) {
-    const int o_ = o0 + i / per_row, c = i % per_row;
-    const int f = min(max(out[o_], 0), N - 1);  // never read outside the group's slabs
-    const int h = hs == 1 ? 0 : f / T;
-    const int r = o_ - s_hstart[h];
-    if (r >= a.dst_cap) continue;  // capacity is validated on the host
-    const size_t u = (size_t)grp * hs + h;
-    const size_t src = ((size_t)grp * N + f) * D;
-    const size_t dst = (u * a.dst_cap + r) * D;
-    reinterpret_cast<uint4*>(a.dst_K + dst)[c] = reinterpret_cast<const uint4*>(a.K + src)[c];
-    reinterpret_cast<uint4*>(a.dst_V + dst)[c] = reinterpret_cast<const uint4*>(a.V + src)[c];
-  }
-  if (a.dst_pos)
-    for (int o_ = o0 + tid; o_ < o1; o_ += kSelThreads) {
-      const int f = out[o_], h = hs == 1 ? 0 : f / T;
-      const int r = o_ - s_hstart[h];
-      if (r < a.dst_cap) a.dst_pos[((size_t)grp * hs + h) * a.dst_cap + r] = f - h * T;
+  if (hs == 1 && a.dst_K) {
+    // gather the rows this CTA selected (16-byte chunks); a joint selection's
+    // rows are gathered by gather_kernel over the whole GPU instead
+    const int D = a.D, per_row = D / 8, u = grp;
+    const int o0 = min(my_first, n_sel), o1 = min(my_first + tot, n_sel);
+    for (int i = tid; i < (o1 - o0) * per_row; i += kSelThreads) {
+      const int r = o0 + i / per_row, c = i % per_row;
+      const int t = min(max(out[r], 0), T - 1);  // never read outside the unit's slab
+      const size_t src = ((size_t)u * T + t) * D;
+      const size_t dst = ((size_t)u * a.dst_cap + r) * D;
+      reinterpret_cast<uint4*>(a.dst_K + dst)[c] = reinterpret_cast<const uint4*>(a.K + src)[c];
+      reinterpret_cast<uint4*>(a.dst_V + dst)[c] = reinterpret_cast<const uint4*>(a.V + src)[c];
     }
+    if (a.dst_pos)
+      for (int r = o0 + tid; r < o1; r += kSelThreads) a.dst_pos[(size_t)u * a.dst_cap + r] = out[r];
+  }
   if (rank == 0 && tid < hs) {
     const int u = grp * hs + tid, c = s_hstart[tid + 1] - s_hstart[tid];
     if (a.cnt) a.cnt[u] = c;
+    if (a.hbeg) a.hbeg[u] = grp * n_sel + s_hstart[tid];
     if (a.dst_len) {
       a.dst_len[u] = c;
       a.dst_seen[u] = T;
     }
   }
-  if (a.zero_pad)  // rows [c, next multiple of kTok) of each unit: the moments of the slab read whole tiles
-    for (int h = rank; h < hs; h += kSelCL) {
-      const int c = s_hstart[h + 1] - s_hstart[h];
-      const int r1z = min(a.dst_cap, (c + kTok - 1) / kTok * kTok);
-      const size_t base = ((size_t)grp * hs + h) * a.dst_cap;
-      for (int i = tid; i < max(0, r1z - c) * per_row; i += kSelThreads) {
-        const size_t dst = (base + c + i / per_row) * D;
-        reinterpret_cast<uint4*>(a.dst_K + dst)[i % per_row] = make_uint4(0u, 0u, 0u, 0u);
-        reinterpret_cast<uint4*>(a.dst_V + dst)[i % per_row] = make_uint4(0u, 0u, 0u, 0u);
+  if (rank == 0 && tid == 0 && a.tile0) {
+    int acc = 0;
+    for (int h = 0; h < hs; ++h) {
+      a.tile0[grp * (hs + 1) + h] = acc;
+      acc += (s_hstart[h + 1] - s_hstart[h] + kTok - 1) / kTok;
+    }
+    a.tile0[grp * (hs + 1) + hs] = acc;
+  }
+  cluster.sync();  // no CTA leaves while another may still read its shared memory
+}
+
+// ----------------------------------------------------------------- gather
+// Copies each unit's retained rows (in list order) into dst_K/dst_V
+// [unit][dst_cap][D], one kTok-row tile per CTA, with the positions when the
+// destination is a cache.  With zero_pad the tile's rows past the unit's count
+// are written as zeros (the moments of the slab read whole tiles).  With tile0
+// the grid is (tiles of a group, groups) and each CTA finds its unit there.
+struct GatherArgs {
+  const int32_t* idx;    // selection lists, h * T + position
+  const int32_t* hbeg;   // [units] the unit's first slot in idx
+  const int32_t* cnt;    // [units] its rows
+  const int32_t* tile0;  // optional [groups][hs + 1]
+  int hs, T, D;
+  const __nv_bfloat16* K;  // prompt [units][T][D]
+  const __nv_bfloat16* V;
+  __nv_bfloat16* dst_K;
+  __nv_bfloat16* dst_V;
+  int dst_cap;
+  int32_t* dst_pos;  // optional
+  int zero_pad;
+};
+
+constexpr int kGatherThreads = 512;
+
+__global__ void __launch_bounds__(kGatherThreads) gather_kernel(const GatherArgs a) {
+  int u = blockIdx.y, tile = blockIdx.x, h = 0;
+  if (a.tile0) {
+    const int32_t* t0 = a.tile0 + (size_t)blockIdx.y * (a.hs + 1);
+    if (tile >= t0[a.hs]) return;
+    while (h + 1 < a.hs && t0[h + 1] <= tile) ++h;
+    u = blockIdx.y * a.hs + h;
+    tile -= t0[h];
+  }
+  const int c = a.cnt[u];
+  const int r0 = tile * kTok;
+  const int r1 = min(a.zero_pad ? a.dst_cap : c, r0 + kTok);
+  const int per_row = a.D / 8, per2 = 2 * per_row;  // 16-byte chunks of a row of K and V
+  const int n_items = max(0, r1 - r0) * per2;
+  const int32_t* lst = a.idx + a.hbeg[u];
+  const int hT = h * a.T;
+  constexpr int UG = 4;  // chunks in flight per thread
+  for (int base = threadIdx.x; base < n_items; base += kGatherThreads * UG) {
+    uint4 v[UG];
+    size_t dst[UG];
+    bool isV[UG];
+#pragma unroll
+    for (int q = 0; q < UG; ++q) {
+      const int i = base + q * kGatherThreads;
+      const int r = r0 + i / per2, cc = i % per2;
+      isV[q] = cc >= per_row;
+      const int ch = isV[q] ? cc - per_row : cc;
+      dst[q] = ((size_t)u * a.dst_cap + r) * a.D + ch * 8;
+      v[q] = make_uint4(0u, 0u, 0u, 0u);
+      if (i < n_items && r < c) {
+        const int t = min(max(lst[r] - hT, 0), a.T - 1);  // never read outside the unit's slab
+        const __nv_bfloat16* src = (isV[q] ? a.V : a.K) + ((size_t)u * a.T + t) * a.D + ch * 8;
+        v[q] = *reinterpret_cast<const uint4*>(src);
       }
     }
-  cluster.sync();  // no CTA leaves while another may still read its shared memory
+#pragma unroll
+    for (int q = 0; q < UG; ++q)
+      if (base + q * kGatherThreads < n_items)
+        *reinterpret_cast<uint4*>((isV[q] ? a.dst_V : a.dst_K) + dst[q]) = v[q];
+  }
+  if (a.dst_pos)
+    for (int r = r0 + threadIdx.x; r < min(c, r0 + kTok); r += kGatherThreads)
+      a.dst_pos[(size_t)u * a.dst_cap + r] = lst[r] - hT;
 }
 
 // --------------------------------------------------------------- finalize
@@ -1070,8 +1179,8 @@ __global__ void __launch_bounds__(256) finalize_kernel(const Layout L, float* ou
   auto merge = [&](const float* rbase, int n_ch, float& x0v, float& x0k) -> Set {
     Set st{0.f, 0.f, 0.f, 0.f};
     __syncthreads();
-    if (tid < RB) s_x0v[tid] = rbase[4 + D + rb * RB + tid];
-    for (int i = tid; i < D; i += NT) s_x0k[i] = rbase[4 + i];
+    if (tid < RB) s_x0v[tid] = n_ch > 0 ? rbase[4 + D + rb * RB + tid] : 0.f;
+    for (int i = tid; i < D; i += NT) s_x0k[i] = n_ch > 0 ? rbase[4 + i] : 0.f;
     __syncthreads();
     x0v = act ? s_x0v[ar] : 0.f;
     x0k = s_x0k[act ? c : 0];
@@ -1105,9 +1214,11 @@ __global__ void __launch_bounds__(256) finalize_kernel(const Layout L, float* ou
   };
   const int n_rec = merge_all ? L.n_chunks : 1;
   const float* recs = merge_all ? L.mpart + (size_t)u * L.n_chunks * rf : L.mall + (size_t)u * rf;
+  // a joint selection leaves the unit's rows in its first ceil(cnt / kTok) records
+  const int n_rrec = L.hs > 1 ? min(L.n_rchunks, (L.cnt[u] + kTok - 1) / kTok) : L.n_rchunks;
   float x0v, x0k, x0vR, x0kR;
   const Set A = merge(recs, n_rec, x0v, x0k);
-  const Set R = merge(L.rpart + (size_t)u * L.n_rchunks * rf, L.n_rchunks, x0vR, x0kR);
+  const Set R = merge(L.rpart + (size_t)u * L.n_rchunks * rf, n_rrec, x0vR, x0kR);
   if (!act) return;
   const float n = A.n, nR = R.n, nE = n - nR;
   const float mv = x0v + A.sv / n, mk = x0k + A.sk / n;
@@ -1245,11 +1356,16 @@ cudaError_t run(const CompressArgs& a, const mkv_geom& g, int num_sms, cudaStrea
 
   SelectArgs sa{};
   const int n_groups = U / L.hs;
-  const int sel_per = (L.hs * T + kSelCL - 1) / kSelCL;
-  sa.smem_keys = sel_per <= kSelSmemKeys ? sel_per : 0;
-  const size_t sel_smem = (size_t)sa.smem_keys * sizeof(uint32_t);
-  if ((e = attr((const void*)select_kernel, sel_smem)) != cudaSuccess) return e;
+  const bool prefilter = L.cand != nullptr;
+  // keys a CTA caches when its range fits, for the joint (or per-unit) selection and the prefilter
+  auto cached_keys = [](long per) { return per <= kSelSmemKeys ? static_cast<int>(per) : 0; };
+  sa.smem_keys = cached_keys((L.hs * (long)L.Tc + kSelCL - 1) / kSelCL);
+  const int pf_keys = cached_keys((T + kSelCL - 1) / kSelCL);
+  const size_t sel_smem = (size_t)sa.smem_keys * sizeof(uint32_t), pf_smem = (size_t)pf_keys * sizeof(uint32_t);
+  if ((e = attr((const void*)select_kernel, std::max(sel_smem, pf_smem))) != cudaSuccess) return e;
   sa.T = T;
+  sa.Tc = L.Tc;
+  sa.cand = L.cand;
   sa.W = a.window;
   sa.B = B;
   sa.sink = a.sink;
@@ -1260,10 +1376,43 @@ cudaError_t run(const CompressArgs& a, const mkv_geom& g, int num_sms, cudaStrea
   sa.idx = L.idx;
   sa.hs = L.hs;
   sa.cnt = L.cnt;
-  sa.zero_pad = joint ? 1 : 0;
+  sa.hbeg = L.hbeg;
+  sa.tile0 = joint ? L.tile0 : nullptr;
+  // the candidates of a joint selection over `scores`: each unit's protected
+  // rows and its top Tc - |protected| (a per-unit selection)
+  auto prefilter_launch = [&](const float* scores) {
+    if (!prefilter) return;
+    SelectArgs pf = sa;
+    pf.scores = scores;
+    pf.hs = 1;
+    pf.Tc = T;
+    pf.cand = nullptr;
+    pf.B = L.Tc;
+    pf.idx = L.cand;
+    pf.smem_keys = pf_keys;
+    pf.cnt = nullptr;
+    pf.hbeg = nullptr;
+    pf.tile0 = nullptr;
+    select_kernel<<<U * kSelCL, kSelThreads, pf_smem, st>>>(pf);
+  };
+  // the retained rows' tiles: (chunks, units), or (a group's tiles, groups)
+  const dim3 tiles = joint ? dim3(L.gtiles, n_groups) : dim3(L.n_rchunks, U);
+  GatherArgs ga{};
+  ga.idx = L.idx;
+  ga.hbeg = L.hbeg;
+  ga.cnt = L.cnt;
+  ga.tile0 = sa.tile0;
+  ga.hs = L.hs;
+  ga.T = T;
+  ga.D = D;
+  ga.K = sa.K;
+  ga.V = sa.V;
+  ga.zero_pad = joint ? 1 : 0;
   TcArgs rset = tp;  // moments of a dense row set: chunks of kTok rows
   rset.n_rows = Bc;
   rset.rows_u = joint ? L.cnt : nullptr;
+  rset.tile0 = sa.tile0;
+  rset.hs = L.hs;
   rset.chunk = kTok;
   rset.n_chunks = L.n_rchunks;
   rset.mrec = L.rpart;
@@ -1272,11 +1421,19 @@ cudaError_t run(const CompressArgs& a, const mkv_geom& g, int num_sms, cudaStrea
     SelectArgs s0 = sa;
     s0.scores = L.s;
     s0.diag_idx = a.diag_idx1;
-    s0.dst_K = L.gK;
-    s0.dst_V = L.gV;
-    s0.dst_cap = Bc;
+    GatherArgs g0 = ga;
+    g0.dst_K = L.gK;
+    g0.dst_V = L.gV;
+    g0.dst_cap = Bc;
+    if (!joint) {
+      s0.dst_K = g0.dst_K;
+      s0.dst_V = g0.dst_V;
+      s0.dst_cap = g0.dst_cap;
+    }
+    prefilter_launch(L.s);
     select_kernel<<<n_groups * kSelCL, kSelThreads, sel_smem, st>>>(s0);
-    stats_tc<0><<<dim3(L.n_rchunks, U), kStatsThreads, kStats0Smem, st>>>(rset, tmGK, tmGV, tmQ);
+    if (joint) gather_kernel<<<tiles, kGatherThreads, 0, st>>>(g0);
+    stats_tc<0><<<tiles, kStatsThreads, kStats0Smem, st>>>(rset, tmGK, tmGV, tmQ);
     finalize_kernel<<<dim3(D / kFinRB, U), 256, 0, st>>>(L, L.m0, a.mom, 0, 1);
     TcArgs r = tp;
     r.n_rows = T;
@@ -1291,14 +1448,23 @@ cudaError_t run(const CompressArgs& a, const mkv_geom& g, int num_sms, cudaStrea
   SelectArgs s1 = sa;
   s1.scores = a.mi ? L.s2 : L.s;
   s1.diag_idx = a.mi ? nullptr : a.diag_idx1;
-  s1.dst_K = static_cast<__nv_bfloat16*>(a.cache.K);
-  s1.dst_V = static_cast<__nv_bfloat16*>(a.cache.V);
-  s1.dst_cap = a.cache.capacity;
-  s1.dst_pos = a.cache.pos;
   s1.dst_len = a.cache.len;
   s1.dst_seen = a.cache.seen;
+  GatherArgs g1 = ga;
+  g1.dst_K = static_cast<__nv_bfloat16*>(a.cache.K);
+  g1.dst_V = static_cast<__nv_bfloat16*>(a.cache.V);
+  g1.dst_cap = a.cache.capacity;
+  g1.dst_pos = a.cache.pos;
+  if (!joint) {
+    s1.dst_K = g1.dst_K;
+    s1.dst_V = g1.dst_V;
+    s1.dst_cap = g1.dst_cap;
+    s1.dst_pos = g1.dst_pos;
+  }
+  prefilter_launch(s1.scores);
   select_kernel<<<n_groups * kSelCL, kSelThreads, sel_smem, st>>>(s1);
-  stats_tc<0><<<dim3(L.n_rchunks, U), kStatsThreads, kStats0Smem, st>>>(rset, tmCK, tmCV, tmQ);
+  if (joint) gather_kernel<<<tiles, kGatherThreads, 0, st>>>(g1);
+  stats_tc<0><<<tiles, kStatsThreads, kStats0Smem, st>>>(rset, tmCK, tmCV, tmQ);
   finalize_kernel<<<dim3(D / kFinRB, U), 256, 0, st>>>(L, nullptr, a.mom, 1, a.mi ? 0 : 1);
   return cudaGetLastError();
 }

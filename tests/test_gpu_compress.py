@@ -213,10 +213,57 @@ def test_adaptive_budget_covers_prompt():
 
 
 def test_adaptive_uncached_select_keys():
-    # 8 heads x 60000 positions: each select CTA's range exceeds its shared-memory key cache
-    wl = Workload("a-long", Geometry(1, 8, 1, 64), 60000, 640, 16, "logscale")
+    # 8 heads x 60000 positions and a budget that leaves no per-head prefilter:
+    # each select CTA's range of the joint list exceeds its shared-memory key cache
+    wl = Workload("a-long", Geometry(1, 8, 1, 64), 60000, 4000, 16, "logscale")
     run_adaptive(wl, seed=14)
+
+
+def test_adaptive_dense_joint_selection():
+    # a unit may keep up to 1549 of its 2000 rows: the joint selection ranks every pair
+    wl = Workload("a-dense", Geometry(1, 4, 2, 64), 2000, 400, 16, "outlier")
+    out, n = run_adaptive(wl, seed=15, cap_extra=3)
+    assert n == 1
 
 
 def test_adaptive_llama_layer_full_size():
     run_adaptive(WORKLOADS["llama8b_layer_t8k"])
+
+
+def test_adaptive_then_decode():
+    """A decode step over the unequal per-head caches that the adaptive
+    compression leaves, against the oracle's decode over its own sets."""
+    from gpu_util import assert_output_close
+    wl = Workload("a4d", Geometry(1, 4, 4, 128), 3001, 200, 32, "logscale")
+    gen = Generator(wl, seed=21)
+    K, V, Q = gen.prefill()
+    G_, T, B = wl.geom, wl.T, wl.budget
+    H, G, D = G_.n_kv_heads, G_.group, G_.head_dim
+    g = mkv.geom(1, H, G, D)
+    prot = 1 + wl.window
+    cap = min(T, H * (B - prot) + prot) + 1
+    cache, mom = mkv.alloc_cache(g, cap), mkv.alloc_moments(g)
+    p = mkv.mkv_compress_params(B, wl.window, 1, 1, 1, 1, 1, 1e-6, 1)
+    ws = mkv.alloc_workspace(mkv.mkv_compress_workspace_size(g, T, p))
+    mkv.mkv_compress(g, T, bf16(K), bf16(V), bf16(Q), p, cache, mom, ws)
+    ref = O.compress_adaptive(K[0], V[0], Q[0], B, wl.window, 1, True, 1, True, 1e-6)
+    assert ref.gap1 > GAP_EXACT and ref.gap2 > GAP_EXACT
+    rng = np.random.default_rng(5)
+    q = (rng.standard_normal((1, H * G, D)) * 0.5).astype(np.float32)
+    kn = rng.standard_normal((1, H, D)).astype(np.float32)
+    vn = rng.standard_normal((1, H, D)).astype(np.float32)
+    q, kn, vn = (host(bf16(x)) for x in (q, kn, vn))  # the bf16 values the kernel reads
+    out = torch.empty(1, H * G, D, device="cuda")
+    dws = mkv.alloc_workspace(mkv.mkv_decode_workspace_size(g, cap))
+    mkv.mkv_decode_step(g, bf16(q), bf16(kn), bf16(vn), cache, mom, mkv.mkv_decode_params(1, 1, 1e-6), out, None,
+                        dws)
+    code, _ = mkv.mkv_get_device_error(dws)
+    assert code == 0
+    want = np.zeros((H * G, D))
+    for h in range(H):
+        idx = ref.idx[h]
+        o, _, _, _ = O.decode_step(q[0, h * G:(h + 1) * G], K[0, h][idx], V[0, h][idx], ref.moments[h],
+                                   kn[0, h], vn[0, h], True, 1, 1e-6)
+        want[h * G:(h + 1) * G] = o
+    assert_output_close(host(out)[0], want, "decode after adaptive compress")
+    assert len(np.unique(host(cache.len))) > 1
