@@ -46,7 +46,7 @@ EVICT_EVERY = 64
 # dram__bytes_read.sum + dram__bytes_write.sum per launch from one ncu capture
 # of the bench workload (profiles/decode_kernel_llama8b_layer_t8k.md), valid
 # while the kernel source is byte-identical to what was captured
-NCU_TRAFFIC = {"decode": {"bytes": 2956544, "sha": "96f534fad4c4b86f72c6ca4e256ae141cb86bdc91bda7cf9bb256cb93069d783"}}
+NCU_TRAFFIC = {"decode": {"bytes": 2957824, "sha": "cae859a97e7522f4734a03b06acc930e0c955429058da8ae3e193e7a3cd1da6f"}}
 
 
 def parse():
