@@ -14,8 +14,9 @@ value      generated decode tokens per second of whole-step time (device-timed,
 e2e        the same with the step's inputs copied from pinned host memory and
            the decode outputs copied back inside the timed region.
 roofline   the dominant kernel against the measured HBM copy bandwidth.
-extra keys the decode sweep cells (batch x budget, correction on/off), and
-           compress throughput at 32K and 128K context.
+extra keys the decode sweep cells (batch x budget, correction on/off),
+           compress throughput at 32K and 128K context, and the continuous
+           eviction mode (one Algorithm 1 step per token at the budget).
 
 --impl reference times the fp64 oracle on the host cores instead (a bounded
 sample: one KV-head unit of the same workload per step, scaled to the whole).
@@ -384,6 +385,7 @@ def run_gpu(args):
     if rank == 0 and not args.no_extras:
         line["decode_sweep"] = decode_sweep(torch, mkv, dev, flush, hbm)
         line["compress_long"] = compress_long(torch, mkv, inputs, dev, flush, hbm)
+        line["continuous_eviction"] = continuous_eviction(torch, mkv, dev)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline()
     if dist:
@@ -514,6 +516,66 @@ def decode_layers(torch, mkv, dev, flush, hbm, b, B, gen, st):
     code, _ = mkv.mkv_get_device_error(ws, st)
     res["ok_layers"] = code == 0
     del Kall, Vall, Call, C16, caches, moms
+    return res
+
+
+def continuous_eviction(torch, mkv, dev, steps=64):
+    """Algorithm 1 once per generated token with the cache at its budget (one
+    append and one eviction per step, Llama-3.1-8B geometry, budget 512):
+    mkv_decode_evict_step against the two calls it replaces
+    (mkv_evict_append, then mkv_decode_step), each as a graph of `steps` steps."""
+    res = []
+    for b in (1, 8):
+        H, G, D, B, cap = 8, 4, 128, 512, 576
+        g = mkv.geom(b, H, G, D)
+        gen = torch.Generator(device=dev).manual_seed(3)
+        rnd = lambda *shape: torch.randn(*shape, device=dev, generator=gen)
+        K0, V0 = rnd(b, H, cap, D).bfloat16(), rnd(b, H, cap, D).bfloat16()
+        qs, kn, vn = rnd(steps, b, H * G, D).bfloat16(), rnd(steps, b, H, D).bfloat16(), rnd(steps, b, H, D).bfloat16()
+        mom0 = (0.05 * rnd(b, H, D), 0.05 * rnd(b, H, D), 0.01 * rnd(b, H, D, D))
+        out = torch.empty(b, H * G, D, device=dev)
+        p = mkv.mkv_decode_params(1, 1, 1e-6)
+        st = torch.cuda.Stream(dev)
+        cell = {"batch": b, "budget": B}
+        for mode in ("fused", "two_calls"):
+            cache = mkv.Cache(K0.clone(), V0.clone(),
+                              torch.arange(cap, dtype=torch.int32, device=dev).expand(b, H, cap).contiguous(),
+                              torch.full((b, H), B, dtype=torch.int32, device=dev),
+                              torch.full((b, H), 10 ** 4, dtype=torch.int32, device=dev))
+            mom = mkv.Moments(torch.full((b, H), 7000, dtype=torch.int32, device=dev), *(x.clone() for x in mom0))
+            wsf = mkv.alloc_workspace(mkv.mkv_decode_evict_workspace_size(g, cap), dev)
+            wse = mkv.alloc_workspace(mkv.mkv_evict_workspace_size(g, cap), dev)
+            wsd = mkv.alloc_workspace(mkv.mkv_decode_workspace_size(g, cap), dev)
+
+            def body():
+                for i in range(steps):
+                    if mode == "fused":
+                        mkv.mkv_decode_evict_step(g, qs[i], kn[i], vn[i], B, cache, mom, p, out, None, wsf, st)
+                    else:
+                        mkv.mkv_evict_append(g, qs[i], kn[i], vn[i], B, cache, mom, 1e-6, wse, st)
+                        mkv.mkv_decode_step(g, qs[i], None, None, cache, mom, p, out, None, wsd, st)
+            with torch.cuda.stream(st):
+                body()
+                st.synchronize()
+                gr = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gr, stream=st, capture_error_mode="relaxed"):
+                body()
+            times = []
+            for it in range(4):
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                with torch.cuda.stream(st):
+                    e0.record(st)
+                    gr.replay()
+                    e1.record(st)
+                st.synchronize()
+                if it >= 1:
+                    times.append(e0.elapsed_time(e1) * 1e3 / steps)
+            ok = all(mkv.mkv_get_device_error(w, st)[0] == 0 for w in (wsf, wse, wsd))
+            cell[mode] = {"us_per_step": round(float(np.median(times)), 2),
+                          "tokens_per_s": round(b * 1e6 / float(np.median(times)), 1), "ok": ok}
+            del gr, cache, mom, wsf, wse, wsd
+        res.append(cell)
+        torch.cuda.empty_cache()
     return res
 
 

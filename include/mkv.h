@@ -14,6 +14,9 @@
  *                     moment term in one normaliser     (Algorithm 1 Phase 2)
  *   mkv_evict_append  append a token and evict one at a time down to the
  *                     budget by the moment-informed score (Algorithm 1 Phase 1)
+ *   mkv_decode_evict_step  the whole of Algorithm 1 for one generated token:
+ *                     append, Phase 1 down to the budget, Phase 2 (continuous
+ *                     per-token eviction)
  *
  * Conventions shared by every call
  *  - Pointers are DEVICE pointers unless a comment says otherwise; the
@@ -280,6 +283,39 @@ MKV_API size_t mkv_evict_workspace_size(mkv_geom geom, int32_t capacity);
 MKV_API mkv_status mkv_evict_append(mkv_geom geom, const void* q, const void* k_new, const void* v_new,
                             int32_t budget, const mkv_cache* cache, const mkv_moments* mom,
                             float tau, void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * Bytes of device workspace mkv_decode_evict_step needs for this geometry and
+ * cache capacity on the current device.  Returns 0 if the arguments are
+ * invalid.  The workspace must be zero-filled before its first use; every
+ * call leaves it ready for the next one.
+ */
+MKV_API size_t mkv_decode_evict_workspace_size(mkv_geom geom, int32_t capacity);
+
+/*
+ * One decoding step of Algorithm 1 for every unit: append (k_new, v_new) at
+ * row len with position seen, run Phase 1 while len > budget (exactly as
+ * mkv_evict_append with tau = p->tau), then Phase 2 over the surviving rows
+ * and the updated moments (exactly as mkv_decode_step without a new token:
+ * out, lse and p->correction, p->order, p->tau as documented there).  With a
+ * budget at or above the new length nothing is evicted, so one call per
+ * generated token keeps the cache at the budget once it is reached: the
+ * paper's continuous eviction mode.  Where a unit's rows fit the register
+ * eviction kernel (capacity <= 8 * 144) both phases run in one launch;
+ * larger capacities run the eviction and the decode kernels back to back.
+ *   q             bf16 [b, g*h_kv, d]   this step's queries (score the rows
+ *                                       in Phase 1 and attend in Phase 2)
+ *   k_new, v_new  bf16 [b, h_kv, d]     the token appended (both required)
+ *   out           fp32 [b, g*h_kv, d]   corrected output
+ *   lse           fp32 [b, g*h_kv]      optional, as in mkv_decode_step
+ * Requirements: as mkv_evict_append and mkv_decode_step; p->C16 must be NULL
+ * (the moments change inside the call).  q, out, k_new and v_new must be
+ * 16-byte aligned.
+ */
+MKV_API mkv_status mkv_decode_evict_step(mkv_geom geom, const void* q, const void* k_new, const void* v_new,
+                                 int32_t budget, const mkv_cache* cache, const mkv_moments* mom,
+                                 const mkv_decode_params* p, float* out, float* lse,
+                                 void* workspace, size_t workspace_bytes, void* stream);
 
 /*
  * Synchronises `stream`, returns the first error a kernel recorded in this

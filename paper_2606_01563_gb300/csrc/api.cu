@@ -160,6 +160,87 @@ mkv_status mkv_evict_append(mkv_geom geom, const void* q, const void* k_new, con
   return cuda_status(launch_evict(a, geom.head_dim, geom.group, static_cast<cudaStream_t>(stream)));
 }
 
+// ---------------------------------------------------------- decode + evict
+// One workspace for both phases: [error header][eviction scratch][decode
+// scratch], the decode part carved after the eviction part and both
+// reporting into the common header.
+static size_t decode_evict_bytes(const mkv_geom& geom, int32_t capacity, int sms) {
+  return evict_workspace_bytes(geom, capacity) + decode_workspace_bytes(geom, capacity, sms) - kHeaderBytes;
+}
+
+size_t mkv_decode_evict_workspace_size(mkv_geom geom, int32_t capacity) {
+  if (!geom_ok(geom) || capacity < 1 || capacity > 65536) return 0;
+  return decode_evict_bytes(geom, capacity, num_sms_current());
+}
+
+mkv_status mkv_decode_evict_step(mkv_geom geom, const void* q, const void* k_new, const void* v_new, int32_t budget,
+                                 const mkv_cache* cache, const mkv_moments* mom, const mkv_decode_params* p,
+                                 float* out, float* lse, void* workspace, size_t workspace_bytes, void* stream) {
+  if (!geom_ok(geom)) return (geom.head_dim == 64 || geom.head_dim == 128) ? MKV_ERR_SHAPE : MKV_ERR_UNSUPPORTED;
+  if (!q || !k_new || !v_new || !out || !p || !cache_ok(cache) || !moments_ok(mom) || budget < 0)
+    return MKV_ERR_INVALID_ARG;
+  if (!aligned(q, 16) || !aligned(out, 16) || !aligned(k_new, 16) || !aligned(v_new, 16)) return MKV_ERR_INVALID_ARG;
+  if ((p->correction != 0 && p->correction != 1) || (p->order != 0 && p->order != 1) || !(p->tau >= 0.f) ||
+      p->C16 != nullptr)
+    return MKV_ERR_INVALID_ARG;
+  if (cache->capacity > 65536) return MKV_ERR_SHAPE;
+  const int sms = num_sms_current();
+  const size_t need = decode_evict_bytes(geom, cache->capacity, sms);
+  if (!workspace || workspace_bytes < need || !aligned(workspace, 256)) return MKV_ERR_WORKSPACE;
+  EvictArgs e{};
+  e.q = q;
+  e.k_new = k_new;
+  e.v_new = v_new;
+  e.K = cache->K;
+  e.V = cache->V;
+  e.pos = cache->pos;
+  e.len = cache->len;
+  e.seen = cache->seen;
+  e.cap = cache->capacity;
+  e.n = mom->n;
+  e.mu_k = mom->mu_k;
+  e.mu_v = mom->mu_v;
+  e.C = mom->C;
+  e.budget = budget;
+  e.tau = p->tau;
+  e.batch = geom.batch;
+  e.n_kv = geom.n_kv_heads;
+  evict_carve(e, geom, cache->capacity, workspace);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (evict_fuses_output(cache->capacity)) {  // Phase 2 in the eviction kernel's epilogue
+    e.out = out;
+    e.lse = lse;
+    e.correction = p->correction;
+    e.order = p->order;
+    return cuda_status(launch_evict(e, geom.head_dim, geom.group, st));
+  }
+  cudaError_t ce = launch_evict(e, geom.head_dim, geom.group, st);
+  if (ce != cudaSuccess) return cuda_status(ce);
+  DecodeArgs a{};
+  a.q = q;
+  a.K = cache->K;
+  a.V = cache->V;
+  a.pos = cache->pos;
+  a.len = cache->len;
+  a.seen = cache->seen;
+  a.cap = cache->capacity;
+  a.n = p->correction ? mom->n : nullptr;
+  a.mu_k = p->correction ? mom->mu_k : nullptr;
+  a.mu_v = p->correction ? mom->mu_v : nullptr;
+  a.C = p->correction ? mom->C : nullptr;
+  a.correction = p->correction;
+  a.order = p->order;
+  a.tau = p->tau;
+  a.out = out;
+  a.lse = lse;
+  a.batch = geom.batch;
+  a.n_kv = geom.n_kv_heads;
+  uint8_t* w = static_cast<uint8_t*>(workspace);
+  decode_carve(a, geom, cache->capacity, sms, w + evict_workspace_bytes(geom, cache->capacity) - kHeaderBytes);
+  a.ws = workspace;
+  return cuda_status(launch_decode(a, geom.head_dim, geom.group, st));
+}
+
 // ---------------------------------------------------------------- compress
 static mkv_status compress_params_ok(const mkv_geom& geom, int32_t T, const mkv_compress_params* p) {
   if (!geom_ok(geom)) return (geom.head_dim == 64 || geom.head_dim == 128) ? MKV_ERR_SHAPE : MKV_ERR_UNSUPPORTED;

@@ -1040,6 +1040,7 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
   __shared__ float s_zval[kMaxClamp];
   __shared__ int s_nz;
   __shared__ float s_tile[kTW][32 * 33];
+  __shared__ float s_p2[G][D + 1];  // Phase 2: this CTA's sums of e_hj v_j and e_hj over its survivors
 
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = static_cast<int>(cluster.block_rank());
@@ -1073,7 +1074,8 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
     __threadfence();
   }
   __syncthreads();
-  if (len <= a.budget) {
+  const bool fused = a.out != nullptr;  // Phase 2 follows the evictions in this kernel
+  if (len <= a.budget && !fused) {
     if (rank == 0 && tid == 0) {
       a.len[u] = len;
       a.seen[u] = seen_in + (has_new ? 1 : 0);
@@ -1099,6 +1101,7 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
     s_mu_k[i] = (n > 0) ? a.mu_k[(size_t)u * D + i] : 0.f;
     s_mu_v[i] = (n > 0) ? a.mu_v[(size_t)u * D + i] : 0.f;
   }
+  for (int i = tid; fused && i < G * (D + 1); i += kRT) (&s_p2[0][0])[i] = 0.f;
   const float scale = rsqrtf(static_cast<float>(D));
   const __nv_bfloat16* qg = reinterpret_cast<const __nv_bfloat16*>(a.q) + (size_t)u * G * D;
   for (int i = tid; i < G * D; i += kRT) s_q[i / D][i % D] = __bfloat162float(qg[i]) * scale;
@@ -1270,7 +1273,7 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
   }
   __syncthreads();
 
-  const int n_evict = len - a.budget;
+  const int n_evict = max(0, len - a.budget);
   for (int e = 0;; ++e) {
     const int par = e & 1;
     // ---- fold the previous eviction into this thread's share of S_tilde and
@@ -1497,6 +1500,120 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
   __syncthreads();
   const uint8_t* alv = alive_all + j0;
 
+  // ---- Phase 2 (fused): this CTA's sums over its survivors of e_hj v_j and
+  // e_hj (e_hj = exp(l_hj - M0_h)); rank 0 combines the cluster's sums after
+  // the next cluster barrier
+  if (fused) {
+    float acc[G][DPL], zp[G];
+#pragma unroll
+    for (int h = 0; h < G; ++h) {
+      zp[h] = 0.f;
+#pragma unroll
+      for (int d = 0; d < DPL; ++d) acc[h][d] = 0.f;
+    }
+#pragma unroll
+    for (int i = 0; i < RPW; ++i)
+      if ((alive >> i) & 1u) {
+        const int r = warp + kRW * i;
+        float vf[DPL];
+        load_bf16<DPL>(Vr + (size_t)r * D + lane * DPL, vf);
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+          const float ev = lg[h * a.cap + j0 + r];
+          zp[h] += ev;
+#pragma unroll
+          for (int d = 0; d < DPL; ++d) acc[h][d] = fmaf(ev, vf[d], acc[h][d]);
+        }
+      }
+#pragma unroll
+    for (int h = 0; h < G; ++h) {
+#pragma unroll
+      for (int d = 0; d < DPL; ++d) atomicAdd(&s_p2[h][lane * DPL + d], acc[h][d]);
+      if (lane == 0) atomicAdd(&s_p2[h][D], zp[h]);
+    }
+  }
+  // rank 0: S_tilde' q_h (clamped entries zeroed) from its share of S_tilde,
+  // and log Z_hat_E = ln n + q_h . mu_k (q is held pre-scaled)
+  float* s_fe = &s_tile[0][0];       // [G][D]
+  float* s_lze = &s_tile[2][0];      // [G]
+  float* s_fr = &s_tile[2][0] + 32;  // [G][D + 1] the cluster's sums
+  if (fused && rank == 0) {
+    for (int i = tid; i < G * D; i += kRT) s_fe[i] = 0.f;
+    __syncthreads();
+    if (a.order && n > 0) {
+#pragma unroll
+      for (int h = 0; h < G; ++h) {
+        float pq[DPL];
+#pragma unroll
+        for (int d = 0; d < DPL; ++d) pq[d] = 0.f;
+#pragma unroll
+        for (int jj = 0; jj < CJ; ++jj) {
+          const float qc = s_q[h][warp + kRW * jj];
+#pragma unroll
+          for (int d = 0; d < DPL; ++d) pq[d] = fmaf(fabsf(creg[jj][d]) < tau ? 0.f : creg[jj][d], qc, pq[d]);
+        }
+#pragma unroll
+        for (int d = 0; d < DPL; ++d) atomicAdd(&s_fe[h * D + lane * DPL + d], pq[d]);
+      }
+    }
+    if (warp < G) {
+      float dq = 0.f;
+#pragma unroll
+      for (int d = 0; d < DPL; ++d) dq = fmaf(s_q[warp][lane * DPL + d], s_mu_k[lane * DPL + d], dq);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) dq += __shfl_xor_sync(kFull, dq, o);
+      if (lane == 0) s_lze[warp] = n > 0 ? logf(static_cast<float>(n)) + dq : -INFINITY;
+    }
+  }
+  // rank 0 writes the output once the cluster's sums are final (the caller
+  // places this between two cluster barriers, so that no CTA has left)
+  auto phase2_out = [&]() {
+    if (!fused || rank != 0) return;
+    for (int i = tid; i < G * (D + 1); i += kRT) {
+      float v = 0.f;
+#pragma unroll
+      for (int r = 0; r < kCL; ++r) v += cluster.map_shared_rank(&s_p2[0][0], r)[i];
+      s_fr[i] = v;
+    }
+    __syncthreads();
+    const bool use_m = a.correction && n > 0;
+    const bool empty = len - n_evict == 0;
+    if (empty && !use_m && tid == 0) record_error(a.ws, MKV_ERR_INVALID_ARG, u);
+    for (int i = tid; i < G * D; i += kRT) {
+      const int h = i / D, c = i % D;
+      const float zr = s_fr[h * (D + 1) + D];
+      const float lzr = s_M[h] + logf(zr);
+      const float fr = zr > 0.f ? s_fr[h * (D + 1) + c] / zr : 0.f;
+      const float fe = s_mu_v[c] + (n > 0 ? s_fe[h * D + c] / static_cast<float>(n) : 0.f);
+      float o, l;
+      if (empty) {
+        o = use_m ? fe : 0.f;
+        l = use_m ? s_lze[h] : -INFINITY;
+      } else if (!use_m) {
+        o = fr;
+        l = lzr;
+      } else {
+        const float lze = s_lze[h];
+        const float top = fmaxf(lzr, lze);
+        l = top + logf(expf(lzr - top) + expf(lze - top));
+        const float wr = expf(lzr - l);
+        o = wr * fr + (1.f - wr) * fe;
+      }
+      a.out[((size_t)u * G + h) * D + c] = o;
+      if (a.lse && c == 0) a.lse[(size_t)u * G + h] = l;
+    }
+  };
+  if (fused && n_evict == 0) {  // nothing evicted: the cache keeps its rows in place
+    cluster.sync();
+    phase2_out();
+    if (rank == 0 && tid == 0) {
+      a.len[u] = len;
+      a.seen[u] = seen_in + (has_new ? 1 : 0);
+    }
+    cluster.sync();  // no CTA leaves while rank 0 may still read its sums
+    return;
+  }
+
   // ---- ordered compaction across the cluster through the staging buffer
   {
     int cnt = 0;
@@ -1512,6 +1629,7 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
     }
   }
   cluster.sync();
+  phase2_out();
   int base = 0;
   for (int r = 0; r < rank; ++r) base += *cluster.map_shared_rank(&ex_cnt, r);
   const int mine = ex_cnt;
@@ -1637,6 +1755,8 @@ void evict_carve(EvictArgs& a, const mkv_geom& g, int32_t capacity, void* ws) {
   a.scratch = reinterpret_cast<float*>(p + kHeaderBytes);
   a.stage = p + kHeaderBytes + align_up(units * g.group * (size_t)capacity * sizeof(float), 256);
 }
+
+bool evict_fuses_output(int32_t capacity) { return (capacity + kCL - 1) / kCL <= kRW * 9; }
 
 cudaError_t launch_evict(const EvictArgs& a, int head_dim, int group, cudaStream_t stream) {
 #define MKV_EVICT_CASE(D, G) \

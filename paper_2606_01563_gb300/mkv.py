@@ -51,7 +51,8 @@ STATUS = {0: "MKV_OK", 1: "MKV_ERR_INVALID_ARG", 2: "MKV_ERR_SHAPE", 3: "MKV_ERR
 
 EXPORTS = ("mkv_status_str", "mkv_version", "mkv_compress_workspace_size", "mkv_compress",
            "mkv_decode_workspace_size", "mkv_decode_step", "mkv_evict_workspace_size",
-           "mkv_evict_append", "mkv_get_device_error", "mkv_decode_step_noalloc", "mkv_moments_pack_bf16")
+           "mkv_evict_append", "mkv_get_device_error", "mkv_decode_step_noalloc", "mkv_moments_pack_bf16",
+           "mkv_decode_evict_workspace_size", "mkv_decode_evict_step")
 
 
 class MKVError(RuntimeError):
@@ -95,6 +96,12 @@ def lib():
         L.mkv_evict_append.restype = c_i32
         L.mkv_evict_append.argtypes = [mkv_geom, c_vp, c_vp, c_vp, c_i32, ctypes.POINTER(mkv_cache),
                                        ctypes.POINTER(mkv_moments), ctypes.c_float, c_vp, ctypes.c_size_t, c_vp]
+        L.mkv_decode_evict_workspace_size.restype = ctypes.c_size_t
+        L.mkv_decode_evict_workspace_size.argtypes = [mkv_geom, c_i32]
+        L.mkv_decode_evict_step.restype = c_i32
+        L.mkv_decode_evict_step.argtypes = [mkv_geom, c_vp, c_vp, c_vp, c_i32, ctypes.POINTER(mkv_cache),
+                                            ctypes.POINTER(mkv_moments), ctypes.POINTER(mkv_decode_params),
+                                            c_vp, c_vp, c_vp, ctypes.c_size_t, c_vp]
         L.mkv_moments_pack_bf16.restype = c_i32
         L.mkv_moments_pack_bf16.argtypes = [mkv_geom, ctypes.POINTER(mkv_moments), c_vp, c_vp]
         L.mkv_get_device_error.restype = c_i32
@@ -233,6 +240,20 @@ def mkv_evict_append(g, q, k_new, v_new, budget, cache: Cache, mom: Moments, tau
     code = lib().mkv_evict_append(g, _ptr(q), _ptr(k_new), _ptr(v_new), budget, ctypes.byref(c),
                                   ctypes.byref(m), tau, _ptr(ws), ws.numel(), _stream(stream))
     _check(code, "mkv_evict_append")
+
+
+def mkv_decode_evict_workspace_size(g, capacity):
+    return lib().mkv_decode_evict_workspace_size(g, capacity)
+
+
+def mkv_decode_evict_step(g, q, k_new, v_new, budget, cache: Cache, mom: Moments, p: mkv_decode_params, out, lse,
+                          ws, stream=None):
+    """Algorithm 1 for one generated token: append, evict down to `budget`, corrected output."""
+    c, m = cache.c(), mom.c()
+    code = lib().mkv_decode_evict_step(g, _ptr(q), _ptr(k_new), _ptr(v_new), budget, ctypes.byref(c),
+                                       ctypes.byref(m), ctypes.byref(p), _ptr(out), _ptr(lse), _ptr(ws), ws.numel(),
+                                       _stream(stream))
+    _check(code, "mkv_decode_evict_step")
 
 
 def mkv_moments_pack_bf16(g, mom: Moments, C16, stream=None):

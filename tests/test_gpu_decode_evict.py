@@ -1,0 +1,118 @@
+"""One decoding step of Algorithm 1 (append, Phase 1 down to the budget,
+Phase 2) on the GPU against the fp64 oracle's evict_append followed by its
+decode_step, through the C ABI: the corrected output and its log-normaliser
+(2e-3 of the output's max-abs), the surviving rows (exact), and the updated
+moments (1e-4 relative).  Covers the one-launch path (Phase 2 in the
+eviction kernel), the two-launch path for large caches, steps with nothing
+to evict, eviction down to an empty cache, and several continuous steps."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2606_01563_gb300 import mkv
+from paper_2606_01563_gb300.inputs import bf16_round
+from gpu_util import GAP_EXACT, assert_moment_close, assert_output_close, bf16, f32, host, i32
+from test_gpu_evict import setup
+
+pytestmark = pytest.mark.gpu
+
+
+def oracle_step(st, bi, h, G, budget, tau, correction, order, K, V, pos, m, kn, vn, pos_new):
+    q = st["q"][bi, h * G:(h + 1) * G]
+    r = O.evict_append(q, K, V, pos, m, budget, tau, kn, vn, pos_new)
+    o, lse, _, _ = O.decode_step(q, r.K, r.V, r.moments, None, None, bool(correction), order, tau)
+    return r, o, lse
+
+
+def run_steps(st, b, H, G, D, budget, steps=1, correction=1, order=1, tau=1e-6, seed=0):
+    """`steps` calls of mkv_decode_evict_step, each with fresh queries and a
+    new token, against the oracle carrying its own state."""
+    rng = np.random.default_rng(seed)
+    g = mkv.geom(b, H, G, D)
+    cap = st["cap"]
+    pos0 = np.broadcast_to(np.arange(cap, dtype=np.int32) * 3, (b, H, cap)).copy()
+    seen0 = 10 ** 6
+    cache = mkv.Cache(bf16(st["K"]), bf16(st["V"]), i32(pos0), i32(st["lens"]), i32(np.full((b, H), seen0)))
+    mom = mkv.Moments(i32(st["n"]), f32(st["mu_k"]), f32(st["mu_v"]), f32(st["C"]))
+    ws = mkv.alloc_workspace(mkv.mkv_decode_evict_workspace_size(g, cap))
+    p = mkv.mkv_decode_params(correction, order, tau)
+    ref = {}
+    for bi in range(b):
+        for h in range(H):
+            L = st["lens"][bi, h]
+            ref[bi, h] = dict(K=st["K"][bi, h, :L], V=st["V"][bi, h, :L], pos=pos0[bi, h, :L],
+                              m=O.Moments(int(st["n"][bi, h]), st["mu_k"][bi, h], st["mu_v"][bi, h], st["C"][bi, h]))
+    for step in range(steps):
+        if step > 0:
+            st = dict(st, q=bf16_round(2.0 * rng.standard_normal((b, H * G, D))),
+                      kn=bf16_round(1.5 * rng.standard_normal((b, H, D))),
+                      vn=bf16_round(rng.standard_normal((b, H, D))))
+        out = torch.full((b, H * G, D), float("nan"), device="cuda")
+        lse = torch.full((b, H * G), float("nan"), device="cuda")
+        mkv.mkv_decode_evict_step(g, bf16(st["q"]), bf16(st["kn"]), bf16(st["vn"]), budget, cache, mom, p, out, lse,
+                                  ws)
+        code, info = mkv.mkv_get_device_error(ws)
+        assert code == 0, (code, info)
+        got = dict(out=host(out), lse=host(lse), K=host(cache.K), V=host(cache.V), pos=host(cache.pos),
+                   len=host(cache.len), seen=host(cache.seen), n=host(mom.n), mu_k=host(mom.mu_k),
+                   mu_v=host(mom.mu_v), C=host(mom.C))
+        for (bi, h), s in ref.items():
+            r, o, l = oracle_step(st, bi, h, G, budget, tau, correction, order, s["K"], s["V"], s["pos"], s["m"],
+                                  st["kn"][bi, h], st["vn"][bi, h], seen0 + step)
+            if r.gaps:
+                assert min(r.gaps) > GAP_EXACT, "fixture has a near-tie; pick another seed"
+            n_r = len(r.pos)
+            assert got["len"][bi, h] == n_r and got["seen"][bi, h] == seen0 + step + 1
+            np.testing.assert_array_equal(got["pos"][bi, h, :n_r], r.pos)
+            if n_r:
+                np.testing.assert_array_equal(got["K"][bi, h, :n_r], r.K)
+                np.testing.assert_array_equal(got["V"][bi, h, :n_r], r.V)
+            assert got["n"][bi, h] == r.moments.n
+            if r.moments.n:
+                assert_moment_close(got["mu_k"][bi, h], r.moments.mu_k, "mu_k")
+                assert_moment_close(got["mu_v"][bi, h], r.moments.mu_v, "mu_v")
+                assert_moment_close(got["C"][bi, h], r.moments.C, "C")
+            assert_output_close(got["out"][bi, h * G:(h + 1) * G], o, f"out step {step} unit {(bi, h)}")
+            np.testing.assert_allclose(got["lse"][bi, h * G:(h + 1) * G], l, rtol=1e-4, atol=1e-4)
+            s.update(K=r.K, V=r.V, pos=r.pos, m=r.moments)
+    return got
+
+
+def test_tiny_several_evictions_in_one_step():
+    rng = np.random.default_rng(31)
+    st = setup(rng, 1, 2, 2, 64, [40, 33], 48, [0, 25])
+    run_steps(st, 1, 2, 2, 64, 24)
+
+
+@pytest.mark.parametrize("correction,order", [(1, 1), (1, 0), (0, 1)])
+def test_llama_continuous_one_eviction_per_step(correction, order):
+    """Cache at the budget (512 of 576 rows): every step appends and evicts one."""
+    rng = np.random.default_rng(32)
+    st = setup(rng, 1, 8, 4, 128, [512] * 8, 576, [3000] * 4 + [0] * 4)
+    run_steps(st, 1, 8, 4, 128, 512, steps=3, correction=correction, order=order, seed=5)
+
+
+def test_below_budget_nothing_evicted():
+    rng = np.random.default_rng(33)
+    st = setup(rng, 2, 2, 2, 64, [10, 3, 0, 7], 16, [0, 1, 2, 3])
+    run_steps(st, 2, 2, 2, 64, 12)
+
+
+def test_evict_to_empty_cache_gives_moment_term():
+    rng = np.random.default_rng(34)
+    st = setup(rng, 1, 2, 4, 64, [5, 2], 8, [7, 1])
+    run_steps(st, 1, 2, 4, 64, 0)
+
+
+def test_two_launch_path_large_cache():
+    """Capacity 1300 (> 8 x 144 rows): eviction kernel, then the decode kernel."""
+    rng = np.random.default_rng(35)
+    st = setup(rng, 1, 2, 2, 128, [1200, 1100], 1300, [500, 0])
+    run_steps(st, 1, 2, 2, 128, 1150, steps=2, seed=6)
+
+
+def test_group_8_d64_batch():
+    rng = np.random.default_rng(36)
+    st = setup(rng, 2, 2, 8, 64, [100, 64, 65, 99], 128, [10, 0, 200, 3])
+    run_steps(st, 2, 2, 8, 64, 64, steps=2, seed=7)

@@ -27,7 +27,7 @@ def declared_functions():
 
 def test_every_declared_symbol_is_exported(L):
     names = declared_functions()
-    assert len(names) == 11, names
+    assert len(names) == 13, names
     assert set(names) == set(mkv.EXPORTS)
     for n in names:
         assert hasattr(L, n), n
@@ -129,6 +129,29 @@ def test_compress_validation(L):
     ws0 = L.mkv_compress_workspace_size(g, 1024, ctypes.byref(P()))
     ws1 = L.mkv_compress_workspace_size(g, 1024, ctypes.byref(P(adaptive=1)))
     assert ws1 > ws0 > 0
+
+
+def test_decode_evict_validation(L):
+    g = mkv.geom(1, 2, 2, 64)
+    c, m = fake_cache(), fake_moments()
+    P = lambda **kw: mkv.mkv_decode_params(**{**dict(correction=1, order=1, tau=1e-6, C16=None), **kw})
+
+    def run(**kw):
+        p = kw.get("p", P())
+        return L.mkv_decode_evict_step(kw.get("g", g), kw.get("q", FAKE), kw.get("kn", FAKE), FAKE,
+                                       kw.get("budget", 8), ctypes.byref(c), ctypes.byref(m), ctypes.byref(p),
+                                       kw.get("out", FAKE), None, kw.get("ws", FAKE), kw.get("wsb", 1 << 30), None)
+    assert run(budget=-1) == 1
+    assert run(q=None) == 1
+    assert run(kn=None) == 1                      # the token to append is required
+    assert run(out=FAKE + 8) == 1                 # misaligned output
+    assert run(p=P(order=2)) == 1
+    assert run(p=P(C16=FAKE)) == 1                # a 16-bit copy of C would be stale
+    assert run(wsb=8) == 7
+    assert run(g=mkv.geom(1, 2, 5, 64)) == 2
+    n = L.mkv_decode_evict_workspace_size(g, 64)
+    assert n >= L.mkv_evict_workspace_size(g, 64) and n >= L.mkv_decode_workspace_size(g, 64)
+    assert L.mkv_decode_evict_workspace_size(g, 0) == 0
 
 
 def test_evict_validation(L):
