@@ -522,8 +522,8 @@ def decode_layers(torch, mkv, dev, flush, hbm, b, B, gen, st):
 def continuous_eviction(torch, mkv, dev, steps=64):
     """Algorithm 1 once per generated token with the cache at its budget (one
     append and one eviction per step, Llama-3.1-8B geometry, budget 512):
-    mkv_decode_evict_step against the two calls it replaces
-    (mkv_evict_append, then mkv_decode_step), each as a graph of `steps` steps."""
+    mkv_decode_evict_step, and the two calls it stands for (mkv_evict_append,
+    then mkv_decode_step), each as a graph of `steps` steps."""
     res = []
     for b in (1, 8):
         H, G, D, B, cap = 8, 4, 128, 512, 576
@@ -537,7 +537,7 @@ def continuous_eviction(torch, mkv, dev, steps=64):
         p = mkv.mkv_decode_params(1, 1, 1e-6)
         st = torch.cuda.Stream(dev)
         cell = {"batch": b, "budget": B}
-        for mode in ("fused", "two_calls"):
+        for mode in ("one_call", "two_calls"):
             cache = mkv.Cache(K0.clone(), V0.clone(),
                               torch.arange(cap, dtype=torch.int32, device=dev).expand(b, H, cap).contiguous(),
                               torch.full((b, H), B, dtype=torch.int32, device=dev),
@@ -549,7 +549,7 @@ def continuous_eviction(torch, mkv, dev, steps=64):
 
             def body():
                 for i in range(steps):
-                    if mode == "fused":
+                    if mode == "one_call":
                         mkv.mkv_decode_evict_step(g, qs[i], kn[i], vn[i], B, cache, mom, p, out, None, wsf, st)
                     else:
                         mkv.mkv_evict_append(g, qs[i], kn[i], vn[i], B, cache, mom, 1e-6, wse, st)

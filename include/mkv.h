@@ -300,9 +300,8 @@ MKV_API size_t mkv_decode_evict_workspace_size(mkv_geom geom, int32_t capacity);
  * out, lse and p->correction, p->order, p->tau as documented there).  With a
  * budget at or above the new length nothing is evicted, so one call per
  * generated token keeps the cache at the budget once it is reached: the
- * paper's continuous eviction mode.  Where a unit's rows fit the register
- * eviction kernel (capacity <= 8 * 144) both phases run in one launch;
- * larger capacities run the eviction and the decode kernels back to back.
+ * paper's continuous eviction mode.  The eviction and the decode kernels
+ * run back to back on `stream` (two launches, one workspace).
  *   q             bf16 [b, g*h_kv, d]   this step's queries (score the rows
  *                                       in Phase 1 and attend in Phase 2)
  *   k_new, v_new  bf16 [b, h_kv, d]     the token appended (both required)

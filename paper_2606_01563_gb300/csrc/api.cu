@@ -206,14 +206,9 @@ mkv_status mkv_decode_evict_step(mkv_geom geom, const void* q, const void* k_new
   e.batch = geom.batch;
   e.n_kv = geom.n_kv_heads;
   evict_carve(e, geom, cache->capacity, workspace);
+  // Phase 1 by the eviction kernel, then Phase 2 by the decode kernel (whose
+  // set-up overlaps the eviction's tail through programmatic dependent launch)
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  if (evict_fuses_output(cache->capacity)) {  // Phase 2 in the eviction kernel's epilogue
-    e.out = out;
-    e.lse = lse;
-    e.correction = p->correction;
-    e.order = p->order;
-    return cuda_status(launch_evict(e, geom.head_dim, geom.group, st));
-  }
   cudaError_t ce = launch_evict(e, geom.head_dim, geom.group, st);
   if (ce != cudaSuccess) return cuda_status(ce);
   DecodeArgs a{};

@@ -355,6 +355,7 @@ constexpr int kRPW = 32 / kLPR;  // rows per warp per pass
 constexpr int kRowsPerPass = kCW * kRPW;
 constexpr int kMaxClamp = 64;    // clamped entries corrected incrementally
 constexpr int kTW = 4;           // warps that run the 32x32 tile transposes
+constexpr int kTWR = 8;          // the same in the register kernel
 // dynamic shared memory available next to the kernel's ~30 KB of static arrays
 constexpr size_t kSmemBudget = 192 * 1024;
 
@@ -960,7 +961,7 @@ struct RegLayout {
   __host__ __device__ RegLayout(int R, int cap, int kv) {
     size_t off = 0;
     Ct = off; off += (size_t)D * D * 4;
-    lg = off; off += align_up((size_t)G * cap * 4, 16);
+    lg = off; off += align_up((size_t)G * R * 4, 16);
     Ks = off; off += kv ? (size_t)R * D * 2 : 0;
     Vs = off; off += kv ? (size_t)R * D * 2 : 0;
     alive = off; off += align_up((size_t)cap, 16);
@@ -1024,14 +1025,16 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
   const int R = a.rows_max;
   const RegLayout<D, G> lay(R, a.cap, a.kv_smem);
   float* Ct = reinterpret_cast<float*>(dsmem + lay.Ct);  // Ct[c*D + a] = C[a][c] (set-up, direct mode, write-back)
-  float* lg = reinterpret_cast<float*>(dsmem + lay.lg);  // [G][cap] e_hj of every row of the unit
+  float* lg = reinterpret_cast<float*>(dsmem + lay.lg);  // [G][R] e_hj of this CTA's rows
   uint8_t* alive_all = dsmem + lay.alive;
   __shared__ __align__(16) float s_mu_k[D];
   __shared__ __align__(16) float s_mu_v[D];
   __shared__ __align__(16) float s_q[G][D];
   __shared__ float s_red[kRW][G];
-  __shared__ double s_zpart[kRW][G];
-  __shared__ float s_M[G];
+  __shared__ float s_zpart[kRW][G];
+  __shared__ float s_M[G];        // this CTA's largest logit per head (read remotely), then the unit's
+  __shared__ float s_Z[G];        // this CTA's sum of exp(l - s_M) per head (read remotely)
+  __shared__ float mail_e[2][kCL][G];  // e_h of each CTA's candidate row
   __shared__ unsigned long long s_best[2];
   __shared__ unsigned long long mail_key[2][kCL];
   __shared__ __align__(16) __nv_bfloat16 mail_row[2][kCL][2 * D];
@@ -1039,8 +1042,7 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
   __shared__ uint32_t s_zidx[kMaxClamp];
   __shared__ float s_zval[kMaxClamp];
   __shared__ int s_nz;
-  __shared__ float s_tile[kTW][32 * 33];
-  __shared__ float s_p2[G][D + 1];  // Phase 2: this CTA's sums of e_hj v_j and e_hj over its survivors
+  __shared__ float s_tile[kTWR][32 * 33];
 
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = static_cast<int>(cluster.block_rank());
@@ -1074,8 +1076,7 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
     __threadfence();
   }
   __syncthreads();
-  const bool fused = a.out != nullptr;  // Phase 2 follows the evictions in this kernel
-  if (len <= a.budget && !fused) {
+  if (len <= a.budget) {
     if (rank == 0 && tid == 0) {
       a.len[u] = len;
       a.seen[u] = seen_in + (has_new ? 1 : 0);
@@ -1087,8 +1088,8 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
 
   int n = a.n[u];
   {
-    float* tb = s_tile[warp % kTW];
-    for (int t = warp; warp < kTW && t < (D / 32) * (D / 32); t += kTW) {
+    float* tb = s_tile[warp % kTWR];
+    for (int t = warp; warp < kTWR && t < (D / 32) * (D / 32); t += kTWR) {
       const int r0 = (t / (D / 32)) * 32, c0 = (t % (D / 32)) * 32;
       for (int i = 0; i < 32; ++i)
         tb[i * 33 + lane] = (n > 0) ? a.C[(size_t)u * D * D + (size_t)(r0 + i) * D + c0 + lane] : 0.f;
@@ -1101,7 +1102,6 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
     s_mu_k[i] = (n > 0) ? a.mu_k[(size_t)u * D + i] : 0.f;
     s_mu_v[i] = (n > 0) ? a.mu_v[(size_t)u * D + i] : 0.f;
   }
-  for (int i = tid; fused && i < G * (D + 1); i += kRT) (&s_p2[0][0])[i] = 0.f;
   const float scale = rsqrtf(static_cast<float>(D));
   const __nv_bfloat16* qg = reinterpret_cast<const __nv_bfloat16*>(a.q) + (size_t)u * G * D;
   for (int i = tid; i < G * D; i += kRT) s_q[i / D][i % D] = __bfloat162float(qg[i]) * scale;
@@ -1123,14 +1123,14 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
   }
   __syncthreads();
 
-  // ---- logits of every row of the unit (8 lanes per row, read from global)
-  for (int base = 0; base < len; base += kRP) {
+  // ---- logits of this CTA's rows (8 lanes per row)
+  for (int base = 0; base < nr; base += kRP) {
     const int j = base + rsub;
-    const bool ok = j < len;
+    const bool ok = j < nr;
     float kf[NC][4];
 #pragma unroll
     for (int c = 0; c < NC; ++c) {
-      if (ok) load4_bf16<D>(Kg + (size_t)j * D + chunk_dim<D>(q, c), kf[c]);
+      if (ok) load4_bf16<D>(Kr + (size_t)j * D + chunk_dim<D>(q, c), kf[c]);
       else kf[c][0] = kf[c][1] = kf[c][2] = kf[c][3] = 0.f;
     }
 #pragma unroll
@@ -1142,19 +1142,21 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
         acc = fmaf(q4.x, kf[c][0], fmaf(q4.y, kf[c][1], fmaf(q4.z, kf[c][2], fmaf(q4.w, kf[c][3], acc))));
       }
       acc = group_sum(acc);
-      if (ok && q == 0) lg[h * a.cap + j] = acc;
+      if (ok && q == 0) lg[h * R + j] = acc;
     }
   }
   __syncthreads();
   // softmax is shift-invariant: e_hj = exp(l_hj - M0_h) with M0_h the
-  // largest logit of the unit at the start
+  // unit's largest logit at the start.  Each CTA takes (max, sum) over its
+  // rows; one cluster exchange gives M0_h and Z_h, and the CTA rescales its
+  // e_hj by exp(m_h - M0_h).
   {
     float mx[G];
 #pragma unroll
     for (int h = 0; h < G; ++h) mx[h] = -INFINITY;
-    for (int jj = tid; jj < len; jj += kRT)
+    for (int jj = tid; jj < nr; jj += kRT)
 #pragma unroll
-      for (int h = 0; h < G; ++h) mx[h] = fmaxf(mx[h], lg[h * a.cap + jj]);
+      for (int h = 0; h < G; ++h) mx[h] = fmaxf(mx[h], lg[h * R + jj]);
 #pragma unroll
     for (int h = 0; h < G; ++h) {
       mx[h] = warp_max(mx[h]);
@@ -1167,16 +1169,12 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
       s_M[tid] = m;
     }
     __syncthreads();
-    double zs[G];
+    float zs[G];
 #pragma unroll
-    for (int h = 0; h < G; ++h) zs[h] = 0.0;
-    for (int jj = tid; jj < len; jj += kRT)
+    for (int h = 0; h < G; ++h) zs[h] = 0.f;
+    for (int jj = tid; jj < nr; jj += kRT)
 #pragma unroll
-      for (int h = 0; h < G; ++h) {
-        const float ev = expf(lg[h * a.cap + jj] - s_M[h]);
-        lg[h * a.cap + jj] = ev;
-        zs[h] += static_cast<double>(ev);
-      }
+      for (int h = 0; h < G; ++h) zs[h] += expf(lg[h * R + jj] - s_M[h]);
 #pragma unroll
     for (int h = 0; h < G; ++h) {
 #pragma unroll
@@ -1184,27 +1182,59 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
       if (lane == 0) s_zpart[warp][h] = zs[h];
     }
     for (int jj = len + tid; jj < a.cap; jj += kRT) alive_all[jj] = 0;
+    __syncthreads();
+    if (tid < G) {
+      float z = 0.f;
+      for (int w = 0; w < kRW; ++w) z += s_zpart[w][tid];
+      s_Z[tid] = z;
+    }
   }
-  __syncthreads();
-  // Z_h lives in lane h < G of every warp as a compensated (Kahan) float,
-  // decremented per eviction: value zf - zc.  Every warp sums the partials in
-  // the same order, so all hold identical values.
+  cluster.sync();  // every CTA's (max, sum) is published
   constexpr int P = RPW <= 8 ? 8 : 16;       // padded row count of the transposing sums
   constexpr int SH = P == 8 ? 2 : 1;         // lane l scores row l >> SH
+  // Z_h lives in lane h < G of every warp as a compensated (Kahan) float,
+  // decremented per eviction: value zf - zc.  Every CTA combines the
+  // published partials in the same order, so all hold identical values.
   float zf = 1.f, zc = 0.f, zinv = 1.f;
-  if (lane < G) {
-    double z = 0.0;
-    for (int w = 0; w < kRW; ++w) z += s_zpart[w][lane];
-    zf = static_cast<float>(z);
-    zc = static_cast<float>(static_cast<double>(zf) - z);
-    zinv = 1.f / zf;
+  {
+    __shared__ float s_Mg[G], s_Zg[G];
+    if (tid < G) {  // thread h: the unit's maximum and normaliser of head h
+      float mr[kCL], m = -INFINITY;
+#pragma unroll
+      for (int r = 0; r < kCL; ++r) {
+        mr[r] = cluster.map_shared_rank(s_M, r)[tid];
+        m = fmaxf(m, mr[r]);
+      }
+      float z = 0.f;
+#pragma unroll
+      for (int r = 0; r < kCL; ++r)
+        if (mr[r] != -INFINITY) z += cluster.map_shared_rank(s_Z, r)[tid] * expf(mr[r] - m);
+      s_Mg[tid] = m;
+      s_Zg[tid] = z;
+    }
+    __syncthreads();
+    float f[G];  // this CTA's rescale to the unit's maximum
+#pragma unroll
+    for (int h = 0; h < G; ++h) f[h] = s_M[h] != -INFINITY ? expf(s_M[h] - s_Mg[h]) : 0.f;
+    for (int jj = tid; jj < nr; jj += kRT)
+#pragma unroll
+      for (int h = 0; h < G; ++h) lg[h * R + jj] = expf(lg[h * R + jj] - s_M[h]) * f[h];
+    if (lane < G) {
+      zf = s_Zg[lane];
+      zinv = 1.f / zf;
+    }
+    // once no CTA reads this one's partials any more, the unit's maxima
+    // replace its own (Phase 2 reads them)
+    cluster.sync();
+    if (tid < G) s_M[tid] = s_Mg[tid];
   }
+  __syncthreads();
   // e_hj of the row this lane scores
   float ereg[G];
   {
     const int i = lane >> SH, r = warp + kRW * i;
 #pragma unroll
-    for (int h = 0; h < G; ++h) ereg[h] = (i < RPW && r < nr) ? lg[h * a.cap + j0 + r] : 0.f;
+    for (int h = 0; h < G; ++h) ereg[h] = (i < RPW && r < nr) ? lg[h * R + r] : 0.f;
   }
 
   // ---- registers, in the raw co-moment form S_tilde = n C (Eq. app_S_tilde):
@@ -1431,6 +1461,7 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
       const unsigned long long b = s_best[par];
       const int jb = (b == ~0ull) ? -1 : static_cast<int>(b & 0xffffffffu) - j0;
       if (lane == 0) *cluster.map_shared_rank(&mail_key[par][rank], warp) = b;
+      if (jb >= 0 && lane < G) *cluster.map_shared_rank(&mail_e[par][rank][lane], warp) = lg[lane * R + jb];
       if (jb >= 0 && lane < D / 4) {  // lanes 0..D/8-1 carry k, the next D/8 carry v
         const bool is_v = lane >= D / 8;
         const int i = is_v ? lane - D / 8 : lane;
@@ -1471,7 +1502,7 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
     const int jr = js - j0;
     if (jr >= 0 && jr < nr && jr % kRW == warp) alive &= ~(1u << (jr / kRW));
     if (lane < G) {  // compensated Z_h -= e_h,js
-      const float yk = -lg[lane * a.cap + js] - zc;
+      const float yk = -mail_e[par][src][lane] - zc;
       const float tk = zf + yk;
       zc = (tk - zf) - yk;
       zf = tk;
@@ -1500,120 +1531,6 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
   __syncthreads();
   const uint8_t* alv = alive_all + j0;
 
-  // ---- Phase 2 (fused): this CTA's sums over its survivors of e_hj v_j and
-  // e_hj (e_hj = exp(l_hj - M0_h)); rank 0 combines the cluster's sums after
-  // the next cluster barrier
-  if (fused) {
-    float acc[G][DPL], zp[G];
-#pragma unroll
-    for (int h = 0; h < G; ++h) {
-      zp[h] = 0.f;
-#pragma unroll
-      for (int d = 0; d < DPL; ++d) acc[h][d] = 0.f;
-    }
-#pragma unroll
-    for (int i = 0; i < RPW; ++i)
-      if ((alive >> i) & 1u) {
-        const int r = warp + kRW * i;
-        float vf[DPL];
-        load_bf16<DPL>(Vr + (size_t)r * D + lane * DPL, vf);
-#pragma unroll
-        for (int h = 0; h < G; ++h) {
-          const float ev = lg[h * a.cap + j0 + r];
-          zp[h] += ev;
-#pragma unroll
-          for (int d = 0; d < DPL; ++d) acc[h][d] = fmaf(ev, vf[d], acc[h][d]);
-        }
-      }
-#pragma unroll
-    for (int h = 0; h < G; ++h) {
-#pragma unroll
-      for (int d = 0; d < DPL; ++d) atomicAdd(&s_p2[h][lane * DPL + d], acc[h][d]);
-      if (lane == 0) atomicAdd(&s_p2[h][D], zp[h]);
-    }
-  }
-  // rank 0: S_tilde' q_h (clamped entries zeroed) from its share of S_tilde,
-  // and log Z_hat_E = ln n + q_h . mu_k (q is held pre-scaled)
-  float* s_fe = &s_tile[0][0];       // [G][D]
-  float* s_lze = &s_tile[2][0];      // [G]
-  float* s_fr = &s_tile[2][0] + 32;  // [G][D + 1] the cluster's sums
-  if (fused && rank == 0) {
-    for (int i = tid; i < G * D; i += kRT) s_fe[i] = 0.f;
-    __syncthreads();
-    if (a.order && n > 0) {
-#pragma unroll
-      for (int h = 0; h < G; ++h) {
-        float pq[DPL];
-#pragma unroll
-        for (int d = 0; d < DPL; ++d) pq[d] = 0.f;
-#pragma unroll
-        for (int jj = 0; jj < CJ; ++jj) {
-          const float qc = s_q[h][warp + kRW * jj];
-#pragma unroll
-          for (int d = 0; d < DPL; ++d) pq[d] = fmaf(fabsf(creg[jj][d]) < tau ? 0.f : creg[jj][d], qc, pq[d]);
-        }
-#pragma unroll
-        for (int d = 0; d < DPL; ++d) atomicAdd(&s_fe[h * D + lane * DPL + d], pq[d]);
-      }
-    }
-    if (warp < G) {
-      float dq = 0.f;
-#pragma unroll
-      for (int d = 0; d < DPL; ++d) dq = fmaf(s_q[warp][lane * DPL + d], s_mu_k[lane * DPL + d], dq);
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) dq += __shfl_xor_sync(kFull, dq, o);
-      if (lane == 0) s_lze[warp] = n > 0 ? logf(static_cast<float>(n)) + dq : -INFINITY;
-    }
-  }
-  // rank 0 writes the output once the cluster's sums are final (the caller
-  // places this between two cluster barriers, so that no CTA has left)
-  auto phase2_out = [&]() {
-    if (!fused || rank != 0) return;
-    for (int i = tid; i < G * (D + 1); i += kRT) {
-      float v = 0.f;
-#pragma unroll
-      for (int r = 0; r < kCL; ++r) v += cluster.map_shared_rank(&s_p2[0][0], r)[i];
-      s_fr[i] = v;
-    }
-    __syncthreads();
-    const bool use_m = a.correction && n > 0;
-    const bool empty = len - n_evict == 0;
-    if (empty && !use_m && tid == 0) record_error(a.ws, MKV_ERR_INVALID_ARG, u);
-    for (int i = tid; i < G * D; i += kRT) {
-      const int h = i / D, c = i % D;
-      const float zr = s_fr[h * (D + 1) + D];
-      const float lzr = s_M[h] + logf(zr);
-      const float fr = zr > 0.f ? s_fr[h * (D + 1) + c] / zr : 0.f;
-      const float fe = s_mu_v[c] + (n > 0 ? s_fe[h * D + c] / static_cast<float>(n) : 0.f);
-      float o, l;
-      if (empty) {
-        o = use_m ? fe : 0.f;
-        l = use_m ? s_lze[h] : -INFINITY;
-      } else if (!use_m) {
-        o = fr;
-        l = lzr;
-      } else {
-        const float lze = s_lze[h];
-        const float top = fmaxf(lzr, lze);
-        l = top + logf(expf(lzr - top) + expf(lze - top));
-        const float wr = expf(lzr - l);
-        o = wr * fr + (1.f - wr) * fe;
-      }
-      a.out[((size_t)u * G + h) * D + c] = o;
-      if (a.lse && c == 0) a.lse[(size_t)u * G + h] = l;
-    }
-  };
-  if (fused && n_evict == 0) {  // nothing evicted: the cache keeps its rows in place
-    cluster.sync();
-    phase2_out();
-    if (rank == 0 && tid == 0) {
-      a.len[u] = len;
-      a.seen[u] = seen_in + (has_new ? 1 : 0);
-    }
-    cluster.sync();  // no CTA leaves while rank 0 may still read its sums
-    return;
-  }
-
   // ---- ordered compaction across the cluster through the staging buffer
   {
     int cnt = 0;
@@ -1629,7 +1546,6 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
     }
   }
   cluster.sync();
-  phase2_out();
   int base = 0;
   for (int r = 0; r < rank; ++r) base += *cluster.map_shared_rank(&ex_cnt, r);
   const int mine = ex_cnt;
@@ -1665,15 +1581,17 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
     reinterpret_cast<uint4*>(Vg + (size_t)row * D)[i] = reinterpret_cast<const uint4*>(SV + (size_t)row * D)[i];
   }
   for (int r = tid; r < mine; r += kRT) Pg[base + r] = SP[base + r];
-  if (rank == 0) {
-    float* tb = s_tile[warp % kTW];
-    for (int t = warp; warp < kTW && t < (D / 32) * (D / 32); t += kTW) {
+  {  // C back to global, its 32 x 32 tiles shared out over the cluster's CTAs
+    float* tb = s_tile[warp % kTWR];
+    for (int t = rank + kCL * warp; warp < kTWR && t < (D / 32) * (D / 32); t += kCL * kTWR) {
       const int c0 = (t / (D / 32)) * 32, r0 = (t % (D / 32)) * 32;
       for (int i = 0; i < 32; ++i) tb[i * 33 + lane] = Ct[(size_t)(c0 + i) * D + r0 + lane];
       __syncwarp();
       for (int i = 0; i < 32; ++i) a.C[(size_t)u * D * D + (size_t)(r0 + i) * D + c0 + lane] = tb[lane * 33 + i];
       __syncwarp();
     }
+  }
+  if (rank == 0) {
     for (int i = tid; i < D; i += kRT) {
       a.mu_k[(size_t)u * D + i] = s_mu_k[i];
       a.mu_v[(size_t)u * D + i] = s_mu_v[i];
@@ -1755,8 +1673,6 @@ void evict_carve(EvictArgs& a, const mkv_geom& g, int32_t capacity, void* ws) {
   a.scratch = reinterpret_cast<float*>(p + kHeaderBytes);
   a.stage = p + kHeaderBytes + align_up(units * g.group * (size_t)capacity * sizeof(float), 256);
 }
-
-bool evict_fuses_output(int32_t capacity) { return (capacity + kCL - 1) / kCL <= kRW * 9; }
 
 cudaError_t launch_evict(const EvictArgs& a, int head_dim, int group, cudaStream_t stream) {
 #define MKV_EVICT_CASE(D, G) \

@@ -77,20 +77,11 @@ struct EvictArgs {
   int32_t kv_smem;   // cluster kernel: the slice's K/V rows are cached in shared memory
   int32_t batch;
   int32_t n_kv;
-  // Phase 2 fused into the eviction (register kernel only): when out is set,
-  // the kernel also writes the corrected output over the survivors
-  float* out;  // fp32 [b, Hkv*G, D]
-  float* lse;  // fp32 [b, Hkv*G] or null
-  int32_t correction;
-  int32_t order;
 };
 
 size_t evict_workspace_bytes(const mkv_geom& g, int32_t capacity);
 void evict_carve(EvictArgs& a, const mkv_geom& g, int32_t capacity, void* ws);
 cudaError_t launch_evict(const EvictArgs& a, int head_dim, int group, cudaStream_t stream);
-// true when launch_evict runs the register kernel for this capacity, which
-// can fuse Phase 2 (EvictArgs::out)
-bool evict_fuses_output(int32_t capacity);
 
 // ---------------------------------------------------------------- compress
 struct CompressArgs {

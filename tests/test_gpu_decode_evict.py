@@ -2,8 +2,8 @@
 Phase 2) on the GPU against the fp64 oracle's evict_append followed by its
 decode_step, through the C ABI: the corrected output and its log-normaliser
 (2e-3 of the output's max-abs), the surviving rows (exact), and the updated
-moments (1e-4 relative).  Covers the one-launch path (Phase 2 in the
-eviction kernel), the two-launch path for large caches, steps with nothing
+moments (1e-4 relative).  Covers the register eviction kernel and the
+larger-cache eviction kernels ahead of the decode kernel, steps with nothing
 to evict, eviction down to an empty cache, and several continuous steps."""
 import numpy as np
 import pytest
@@ -105,8 +105,8 @@ def test_evict_to_empty_cache_gives_moment_term():
     run_steps(st, 1, 2, 4, 64, 0)
 
 
-def test_two_launch_path_large_cache():
-    """Capacity 1300 (> 8 x 144 rows): eviction kernel, then the decode kernel."""
+def test_large_cache_eviction_kernel():
+    """Capacity 1300 (> 8 x 144 rows): the shared-memory cluster eviction kernel."""
     rng = np.random.default_rng(35)
     st = setup(rng, 1, 2, 2, 128, [1200, 1100], 1300, [500, 0])
     run_steps(st, 1, 2, 2, 128, 1150, steps=2, seed=6)
