@@ -1310,29 +1310,27 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
     // build the clamp list: S_tilde' = S_tilde + dk dv^T
     if (e > 0) {
       const float mydk = select_n<DPL>(sdk, warp % DPL);
-      float kd[CJ];  // dk[c], c = warp + kRW jj: lane c/DPL, component warp % DPL
 #pragma unroll
-      for (int jj = 0; jj < CJ; ++jj) kd[jj] = __shfl_sync(kFull, mydk, (warp + kRW * jj) / DPL);
-      bool any = false;  // one test over the whole share; the list is built only when it fires
-#pragma unroll
-      for (int jj = 0; jj < CJ; ++jj)
+      for (int jj = 0; jj < CJ; ++jj) {
+        const int c = warp + kRW * jj;
+        const float kd = __shfl_sync(kFull, mydk, c / DPL);  // dk[c]: lane c/DPL, component warp % DPL
+        bool any = false;
 #pragma unroll
         for (int d = 0; d < DPL; ++d) {
-          creg[jj][d] = fmaf(kd[jj], sdv[d], creg[jj][d]);
-          any |= (creg[jj][d] != 0.f) & (fabsf(creg[jj][d]) < tau);
+          creg[jj][d] = fmaf(kd, sdv[d], creg[jj][d]);
+          any |= fabsf(creg[jj][d]) < tau;
         }
-      if (any) {
-#pragma unroll
-        for (int jj = 0; jj < CJ; ++jj)
+        if (any) {
 #pragma unroll
           for (int d = 0; d < DPL; ++d)
             if (creg[jj][d] != 0.f && fabsf(creg[jj][d]) < tau) {
               const int slot = atomicAdd(&s_nz, 1);
               if (slot < kMaxClamp) {
-                s_zidx[slot] = static_cast<uint32_t>((warp + kRW * jj) * D + lane * DPL + d);
+                s_zidx[slot] = static_cast<uint32_t>(c * D + lane * DPL + d);
                 s_zval[slot] = creg[jj][d];
               }
             }
+        }
       }
     }
     if (e == n_evict) break;  // uniform over the cluster
