@@ -267,3 +267,40 @@ def test_adaptive_then_decode():
         want[h * G:(h + 1) * G] = o
     assert_output_close(host(out)[0], want, "decode after adaptive compress")
     assert len(np.unique(host(cache.len))) > 1
+
+
+def test_adaptive_head_with_no_retained_rows():
+    """No protected rows and one free slot per head: head 0's window queries
+    point at two of its keys, head 1's keys are near zero (flat attention), so
+    the joint top 2 are both head 0's and head 1 keeps nothing (len 0; its
+    moments cover all T rows)."""
+    from paper_2606_01563_gb300.inputs import bf16_round
+    rng = np.random.default_rng(41)
+    T, d, g_, w = 256, 64, 2, 8
+    K = np.empty((1, 2, T, d))
+    K[0, 0] = rng.standard_normal((T, d))
+    K[0, 1] = 0.01 * rng.standard_normal((T, d))
+    V = rng.standard_normal((1, 2, T, d))
+    Q = np.empty((1, 2, g_, w, d))
+    for gi in range(g_):
+        for i in range(w):
+            tgt = K[0, 0, 10] if (gi + i) % 2 == 0 else K[0, 0, 200]
+            Q[0, 0, gi, i] = 3.0 * tgt
+    Q[0, 1] = rng.standard_normal((g_, w, d))
+    K, V, Q = bf16_round(K), bf16_round(V), bf16_round(Q)
+    g = mkv.geom(1, 2, g_, d)
+    p = mkv.mkv_compress_params(1, w, 0, 0, 1, 1, 1, 1e-6, 1)
+    cache, mom = mkv.alloc_cache(g, 2), mkv.alloc_moments(g)
+    ws = mkv.alloc_workspace(mkv.mkv_compress_workspace_size(g, T, p))
+    mkv.mkv_compress(g, T, bf16(K), bf16(V), bf16(Q), p, cache, mom, ws)
+    assert mkv.mkv_get_device_error(ws)[0] == 0
+    ref = O.compress_adaptive(K[0], V[0], Q[0], 1, w, 0, False, 1, True, 1e-6)
+    assert [len(r) for r in ref.idx] == [2, 0]
+    np.testing.assert_array_equal(host(cache.len)[0], [2, 0])
+    np.testing.assert_array_equal(host(cache.pos)[0, 0], ref.idx[0])
+    for h in range(2):
+        m = ref.moments[h]
+        assert host(mom.n)[0, h] == m.n
+        assert_moment_close(host(mom.mu_k)[0, h], m.mu_k, "mu_k")
+        assert_moment_close(host(mom.mu_v)[0, h], m.mu_v, "mu_v")
+        assert_moment_close(host(mom.C)[0, h], m.C, "C")
