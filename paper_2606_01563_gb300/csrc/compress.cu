@@ -43,7 +43,6 @@ constexpr int kTok = 128;                   // tokens per tile
 constexpr int kDP = 128;                    // padded head dim of every MMA
 constexpr int kTileBytes = kTok * kDP * 2;  // one [128 x 128] bf16 tile: 2 boxes of 16 KB
 constexpr int kBoxBytes = kTok * 128;
-constexpr int kTcThreads = 192;  // warp 0 TMA, warp 1 MMA, warps 2..5 epilogue
 // stats_tc: two epilogue groups of 4 warps (2..5 and 6..9), each taking half
 // of a tile's tokens, so that two warps per scheduler share the softmax work
 constexpr int kStatsThreads = 320;
@@ -151,12 +150,6 @@ size_t carve(Layout& L, void* ws) {
 
 __device__ __forceinline__ bool is_protected(int t, int T, int W, int sink, int keep_window) {
   return t < sink || (keep_window && t >= T - W);
-}
-
-// bf16 element (r, c) of a [128 x 128] tile held as two 64-column boxes with
-// the 128-byte swizzle (the TMA layout).
-__device__ __forceinline__ float tile_at(const uint8_t* tile, int r, int c) {
-  return __bfloat162float(*reinterpret_cast<const __nv_bfloat16*>(tile + swz_off(r, c, kTok)));
 }
 
 __device__ __forceinline__ void epi_sync() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
@@ -768,32 +761,11 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
 // One cluster of kSelCL CTAs per selection group -- a unit, or with the
 // adaptive budget the hs KV heads of a batch item, whose (head, position)
 // pairs f = h * T + t are ranked together.  R = protected + the k highest
-// keys among the other pairs (ties to the lower f), written ascending; the
-// rows of R are gathered into dst_K/dst_V [unit][dst_cap][D] (with positions,
-// length and tokens seen when the destination is a cache).
-__device__ __forceinline__ int block_excl_scan(int flag, int* wsum, int* total) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const unsigned m = __ballot_sync(kFull, flag);
-  const int in_warp = __popc(m & ((1u << lane) - 1u));
-  if (lane == 0) wsum[warp] = __popc(m);
-  __syncthreads();
-  if (warp == 0) {
-    const int v = wsum[lane];
-    int x = v;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int y = __shfl_up_sync(kFull, x, o);
-      if (lane >= o) x += y;
-    }
-    wsum[lane] = x - v;
-    if (lane == 31) *total = x;
-  }
-  __syncthreads();
-  const int r = wsum[warp] + in_warp;
-  __syncthreads();
-  return r;
-}
-
+// keys among the other pairs (ties to the lower f), written ascending, with
+// each unit's count and first slot.  For one unit per group the kernel also
+// gathers R's rows into dst_K/dst_V [unit][dst_cap][D] (with positions when
+// the destination is a cache); a joint selection's rows are gathered by
+// gather_kernel.
 // Exclusive block-wide prefix sum of one int per thread; *total gets the sum.
 __device__ __forceinline__ int block_excl_sum(int v, int* wsum, int* total) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
