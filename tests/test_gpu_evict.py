@@ -148,3 +148,12 @@ def test_evict_slice_sizes(cap):
     st = setup(rng, 1, 2, 4, 128, [cap - 11, cap - 20], cap, [300, 0])
     gpu, refs = run_case(st, 1, 2, 4, 128, cap - 41, True)
     check(gpu, refs, st, cap - 41)
+
+
+def test_evict_many_units():
+    """24 units at capacity 200: three waves of 8-CTA clusters of the register
+    kernel (5 rows per warp)."""
+    rng = np.random.default_rng(27)
+    st = setup(rng, 3, 8, 2, 128, [190] * 24, 200, [400, 0] * 12)
+    gpu, refs = run_case(st, 3, 8, 2, 128, 140, True)
+    check(gpu, refs, st, 140)
