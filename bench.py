@@ -15,8 +15,9 @@ e2e        the same with the step's inputs copied from pinned host memory and
            the decode outputs copied back inside the timed region.
 roofline   the dominant kernel against the measured HBM copy bandwidth.
 extra keys the decode sweep cells (batch x budget, correction on/off),
-           compress throughput at 32K and 128K context, and the continuous
-           eviction mode (one Algorithm 1 step per token at the budget).
+           compress throughput at 32K and 128K context, the continuous
+           eviction mode (one Algorithm 1 step per token at the budget), and
+           32 layers' decode in one launch against one launch per layer.
 
 --impl reference times the fp64 oracle on the host cores instead (a bounded
 sample: one KV-head unit of the same workload per step, scaled to the whole).
@@ -386,6 +387,7 @@ def run_gpu(args):
         line["decode_sweep"] = decode_sweep(torch, mkv, dev, flush, hbm)
         line["compress_long"] = compress_long(torch, mkv, inputs, dev, flush, hbm)
         line["continuous_eviction"] = continuous_eviction(torch, mkv, dev)
+        line["layers_one_launch"] = layers_one_launch(torch, mkv, dev, flush, hbm)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline()
     if dist:
@@ -516,6 +518,64 @@ def decode_layers(torch, mkv, dev, flush, hbm, b, B, gen, st):
     code, _ = mkv.mkv_get_device_error(ws, st)
     res["ok_layers"] = code == 0
     del Kall, Vall, Call, C16, caches, moms
+    return res
+
+
+def layers_one_launch(torch, mkv, dev, flush, hbm, layers=32, B=512):
+    """Decode for all 32 layers of the Llama-3.1-8B geometry at batch 1 (budget
+    512, correction on), two ways: the layers' caches, moments and queries
+    stacked on the batch dimension and decoded by one launch, and one launch
+    per layer back to back in a graph.  The single launch applies where the
+    layers' queries are available together (independent per-layer state, no
+    cross-layer dependency inside the step)."""
+    H, G, D = 8, 4, 128
+    gen = torch.Generator(device=dev).manual_seed(9)
+    rnd = lambda *shape: torch.randn(*shape, device=dev, generator=gen)
+    K, V = rnd(layers, H, B, D).bfloat16(), rnd(layers, H, B, D).bfloat16()
+    C, mk, mv = 0.05 * rnd(layers, H, D, D), 0.05 * rnd(layers, H, D), 0.05 * rnd(layers, H, D)
+    n = torch.full((layers, H), 8192, dtype=torch.int32, device=dev)
+    pos = torch.zeros(layers, H, B, dtype=torch.int32, device=dev)
+    lens = torch.full((layers, H), B, dtype=torch.int32, device=dev)
+    q = rnd(layers, H * G, D).bfloat16()
+    out = torch.empty(layers, H * G, D, device=dev)
+    p = mkv.mkv_decode_params(1, 1, 1e-6)
+    st = torch.cuda.Stream(dev)
+    gall, g1 = mkv.geom(layers, H, G, D), mkv.geom(1, H, G, D)
+    ws_all = mkv.alloc_workspace(mkv.mkv_decode_workspace_size(gall, B), dev)
+    ws_1 = mkv.alloc_workspace(mkv.mkv_decode_workspace_size(g1, B), dev)
+    stacked = (mkv.Cache(K, V, pos, lens, lens.clone()), mkv.Moments(n, mk, mv, C))
+    per = [(mkv.Cache(K[l:l + 1], V[l:l + 1], pos[l:l + 1], lens[l:l + 1], lens[l:l + 1].clone()),
+            mkv.Moments(n[l:l + 1], mk[l:l + 1], mv[l:l + 1], C[l:l + 1])) for l in range(layers)]
+    res = {"layers": layers, "batch": 1, "budget": B}
+    for mode in ("one_launch", "per_layer"):
+        def body():
+            if mode == "one_launch":
+                mkv.mkv_decode_step(gall, q, None, None, stacked[0], stacked[1], p, out, None, ws_all, st)
+            else:
+                for l in range(layers):
+                    mkv.mkv_decode_step(g1, q[l:l + 1], None, None, per[l][0], per[l][1], p, out[l:l + 1], None,
+                                        ws_1, st)
+        with torch.cuda.stream(st):
+            body()
+            gr = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gr, stream=st, capture_error_mode="relaxed"):
+            body()
+        times = []
+        for it in range(10):
+            with torch.cuda.stream(st):
+                flush.zero_()
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(st)
+                gr.replay()
+                e1.record(st)
+            st.synchronize()
+            if it >= 2:
+                times.append(e0.elapsed_time(e1))
+        t = float(np.median(times))
+        byt = layers * H * (B * D * 4 + D * D * 4 + 2 * D * 4 + 4) + layers * H * G * D * (2 + 4)
+        res[mode] = {"us": round(t * 1e3, 2), "gbs": round(byt / t / 1e6, 1), "frac": round(byt / t / 1e6 / hbm, 4)}
+        del gr
+    res["ok"] = all(mkv.mkv_get_device_error(w, st)[0] == 0 for w in (ws_all, ws_1))
     return res
 
 
