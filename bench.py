@@ -62,6 +62,21 @@ def parse():
     return ap.parse_args()
 
 
+def job_throughput(total_ms, steps, tokens_per_rank, dist=None, device=None):
+    """Whole-job timing of `steps` timed steps over the ranks (one replica per
+    GPU): the slowest rank's total time, and the tokens all ranks processed in
+    it.  Returns (ms per step, tokens/s)."""
+    world = 1
+    if dist is not None:
+        import torch
+        t = torch.tensor([total_ms], dtype=torch.float64, device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+        world = dist.get_world_size()
+    ms_per_step = total_ms / steps
+    return ms_per_step, tokens_per_rank * world / (ms_per_step / 1e3)
+
+
 def dist_env():
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -307,14 +322,7 @@ def run_gpu(args):
     compress_ms = seg[:, 0]
     decode_ms = seg[:, 1::2].sum(axis=1)
     evict_ms = seg[:, 2::2].sum(axis=1)
-    total_ms = float(step_ms.sum())
-    if dist:
-        t = torch.tensor([total_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
-    ms_per_step = total_ms / args.steps
-    tokens = step.G.batch * step.S * world
-    value = tokens / (ms_per_step / 1e3)
+    ms_per_step, value = job_throughput(float(step_ms.sum()), args.steps, step.G.batch * step.S, dist, dev)
 
     # ---- end to end: host inputs in, decode outputs back, inside the timed region
     e2e_ms = []
@@ -334,8 +342,7 @@ def run_gpu(args):
             e1.record(st)
         st.synchronize()
         e2e_ms.append(e0.elapsed_time(e1))
-    e2e_step = float(np.mean(e2e_ms))
-    e2e_value = tokens / (e2e_step / 1e3)
+    e2e_step, e2e_value = job_throughput(float(np.sum(e2e_ms)), len(e2e_ms), step.G.batch * step.S, dist, dev)
 
     # ---- roofline of the dominant kernel
     hbm, peak_kind = peaks()
