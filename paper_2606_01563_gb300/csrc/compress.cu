@@ -21,11 +21,21 @@
 //   stats_tc  (chunk, unit)  moments of the retained rows
 //   finalize  (rows, unit)   moments of E = all \ R -> caller's mkv_moments
 //
+// With the budget shared by the KV heads of a batch item (adaptive), each
+// select ranks the (head, position) pairs of the batch item together: a
+// per-unit select first keeps each head's own top k as candidates (the joint
+// top k lies among them) when that prunes at least half the pairs, then one
+// cluster per batch item ranks the candidates.  gather_kernel copies the
+// unequal per-head row sets, and stats_tc / gather_kernel take a grid over
+// each batch item's actual 128-row tiles.
+//
 // The tensor-core kernels are warp-specialised: warp 0 issues the TMA copies
 // (3-D tensor maps over per-unit slabs: rows past a unit's end read as zeros),
-// warp 1 owns TMEM and issues tcgen05.mma, warps 2-5 run the epilogue; stages
-// hand over through mbarriers whose waits are all bounded.  Head dims below
-// 128 use the same 128-wide MMAs: the missing 64-column box is zero-filled.
+// warp 1 owns TMEM and issues tcgen05.mma, and the other warps run the
+// epilogue (two groups of four in stats_tc, scores_tc and residual_tc);
+// stages hand over through mbarriers whose waits are all bounded.  Head dims
+// below 128 use the same 128-wide MMAs: the missing 64-column box is
+// zero-filled.
 #include <algorithm>
 #include <cooperative_groups.h>
 

@@ -11,11 +11,14 @@
 // (mma.m16n8k16, bf16 in, fp32 accumulate) with the G query heads as the M
 // rows; P is split into bf16 hi + lo parts so the mixing weights keep ~16
 // bits.  The moment term S_tilde q / (n sqrt d) is spread over the same CTAs:
-// CTA s computes rows [s*D/S, ...) of C'q for all G heads, so C (64 KB fp32
-// at d=128) is read once per unit, concurrently with the K/V stream.  The last
-// CTA of a unit to finish (atomic ticket, no waiting) merges the S partial
-// (m, l, o) records with the moment pseudo-partial (log n + scale q.mu_k,
-// f_hat_E) by log-sum-exp and writes the output; it also performs the append.
+// CTA s computes rows [s*D/S, ...) of C'q for all G heads on the tensor cores
+// (C' rows split into bf16 hi + lo parts as the A operand, the q fragments as
+// B), so C (64 KB fp32 at d=128, or its bf16 copy in the C16 variant) is read
+// once per unit, concurrently with the K/V stream.  The appended token is
+// attended to by the last split, which also writes its row.  The last CTA of
+// a unit to finish (atomic ticket, no waiting) merges the S partial (m, l, o)
+// records with the moment pseudo-partial (log n + scale q.mu_k, f_hat_E) by
+// log-sum-exp, writes the output and updates the length.
 //
 // Cluster variant (S <= 16): the S CTAs of a unit form one thread-block
 // cluster.  Partial records and f_hat_E rows go straight into CTA 0's shared

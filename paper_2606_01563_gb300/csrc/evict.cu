@@ -11,8 +11,11 @@
 // consecutive output dims of one column: conflict-free 128-bit loads while
 // the key element is a broadcast.  Rows are compacted in order at the end.
 //
-// Two kernels compute the same thing:
-//  - evict_cluster_kernel (used whenever a row slice fits in shared memory):
+// Three kernels compute the same thing, chosen by the capacity:
+//  - evict_reg_kernel (row slices of up to 144 rows; described before it):
+//    the state of the loop in registers, one block and one cluster barrier
+//    per eviction;
+//  - evict_cluster_kernel (larger slices that fit shared memory):
 //    a thread-block cluster of 8 CTAs per unit, each owning a contiguous slice
 //    of the rows.  Per iteration the CTAs exchange per-head (max, sum) and
 //    their local argmin through distributed shared memory (two cluster
@@ -944,14 +947,17 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
 // Register-resident cluster kernel, used while a row slice has at most
 // kRW * RPW rows.  8 CTAs of 512 threads per unit (one cluster); warp w of a
 // CTA owns the slice rows w, w + 16, ... and lane l owns the dims
-// [l*DPL, (l+1)*DPL) of each: y_j = C k_j of its rows stays in registers, and
-// so does a 1/512 share of C (rows a of the lane's dims, columns c = w + 16 i),
-// which every iteration folds and scans for the clamp list.  Every thread
-// computes the Welford fold of its own dims from the evicted row, so the only
-// barriers of an iteration are one block barrier (the block's minimum key)
-// and one cluster barrier (every CTA's key and candidate row, written into
-// every CTA's mailbox beforehand).  Scores are computed assuming an empty
-// clamp list; when the list is not empty they are recomputed with it.
+// [l*DPL, (l+1)*DPL) of each.  State in the raw co-moment form S_tilde = n C:
+// y_j = S_tilde k_j of the warp's rows stays in registers, and so does a
+// 1/512 share of S_tilde (rows a of the lane's dims, columns c = w + 16 i),
+// which every iteration folds and scans for the clamp list.  Set-up: each CTA
+// takes the logits and softmax (max, sum) of its own rows, and one cluster
+// exchange gives the unit's maximum and normaliser.  Every thread computes the
+// Welford fold of its own dims from the evicted row, so the only barriers of
+// an iteration are one block barrier (the block's minimum key) and one
+// cluster barrier (every CTA's key, candidate row and its softmax terms,
+// written into every CTA's mailbox beforehand).  Scores are computed assuming
+// an empty clamp list; when the list is not empty they are recomputed with it.
 constexpr int kRT = 512;       // threads per CTA
 constexpr int kRW = kRT / 32;  // warps per CTA
 
