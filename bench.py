@@ -287,7 +287,7 @@ class Step:
             if code != 0:
                 raise RuntimeError(f"device error {code} (unit {info})")
 
-    # algorithmic bytes (SURVEY-style accounting: every input read once, every output written once)
+    # algorithmic bytes: every input read once, every output written once
     def decode_bytes_total(self):
         G, d = self.G, self.G.head_dim
         units = G.batch * G.n_kv_heads
