@@ -60,6 +60,8 @@ def parse():
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--no-extras", action="store_true", help="skip the decode sweep and long-context compress")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--only", choices=["decode_sweep", "compress_long", "continuous_eviction", "layers_one_launch"],
+                    help="run one extra leg alone and print its result (for profiling that leg)")
     return ap.parse_args()
 
 
@@ -324,6 +326,15 @@ def run_gpu(args):
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=dev)
     mkv.lib()
+    if args.only:
+        hbm, _ = peaks()
+        flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=dev)
+        legs = {"decode_sweep": lambda: decode_sweep(torch, mkv, dev, flush, hbm),
+                "compress_long": lambda: compress_long(torch, mkv, inputs, dev, flush, hbm),
+                "continuous_eviction": lambda: continuous_eviction(torch, mkv, dev),
+                "layers_one_launch": lambda: layers_one_launch(torch, mkv, dev, flush, hbm)}
+        print(json.dumps({"only": args.only, args.only: legs[args.only]()}), flush=True)
+        return
     step = Step(torch, mkv, inputs, seed=1000 * rank, dev=dev)
     step.capture()
     flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=dev)

@@ -188,6 +188,7 @@ MKV_API size_t mkv_compress_workspace_size(mkv_geom geom, int32_t T, const mkv_c
  * sums to h_kv * budget over a batch item; rows of out_cache from len up to
  * the next multiple of 128 (below capacity) are overwritten with zeros.
  * Requirements: budget >= sink + (keep_window ? w : 0), 1 <= w <= T,
+ * g * w <= 256 window rows (else MKV_ERR_SHAPE),
  * out_cache->capacity >= min(T, budget) (adaptive: >= min(T, h_kv * budget -
  * (h_kv - 1) * |protected|), h_kv <= 64, h_kv * T <= 2^28), T <= 1,048,576.
  */

@@ -246,7 +246,9 @@ static mkv_status compress_params_ok(const mkv_geom& geom, int32_t T, const mkv_
     return MKV_ERR_INVALID_ARG;
   if (!(p->pool == 1 || p->pool == 2 || p->pool == 4 || p->pool == 8 || p->pool == 16 || p->pool == 32))
     return MKV_ERR_INVALID_ARG;
-  if ((long)geom.group * p->window > 1024) return MKV_ERR_SHAPE;
+  // the g * w window rows fill at most two 128-row blocks: the Q stage in
+  // shared memory, the logits columns in TMEM and one Q tensor-map box
+  if ((long)geom.group * p->window > 256) return MKV_ERR_SHAPE;
   if (T > p->budget && protected_count_host(T, p->window, p->sink, p->keep_window) > p->budget)
     return MKV_ERR_INVALID_ARG;
   if (p->adaptive != 0 && p->adaptive != 1) return MKV_ERR_INVALID_ARG;

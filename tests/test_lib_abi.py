@@ -113,6 +113,7 @@ def test_compress_validation(L):
     assert compress(L, g, 1024, P(budget=10)) == 1            # budget below sink + window
     assert compress(L, g, 1024, P(window=0)) == 1
     assert compress(L, g, 8, P(window=16)) == 1               # window longer than the prompt
+    assert compress(L, mkv.geom(1, 2, 4, 64), 1024, P(budget=200, window=65)) == 2  # 260 window rows
     assert compress(L, g, 1024, P(pool=3)) == 1
     assert compress(L, g, 1024, P(mi=2)) == 1
     assert compress(L, g, 0, P()) == 1
