@@ -62,7 +62,10 @@ typedef enum {
   MKV_ERR_WORKSPACE = 7    /* workspace missing, too small or misaligned    */
 } mkv_status;
 
-/* Attention geometry of one layer.  head_dim in {64, 128}; group in {1,2,4,8}. */
+/* Attention geometry of one layer.  head_dim in {64, 128}; group in {1,2,4,8};
+ * 1 <= batch <= 65535 and 1 <= n_kv_heads <= 65535 (grid dimensions of the
+ * kernels), batch * n_kv_heads <= 65535 * 64, and for mkv_compress
+ * batch * n_kv_heads <= 65535.  Others return MKV_ERR_SHAPE. */
 typedef struct {
   int32_t batch;
   int32_t n_kv_heads;

@@ -21,9 +21,11 @@ int num_sms_current() {
   return n;
 }
 
+// batch and KV heads are grid dimensions of the decode launch (z and y), so
+// each stays within 65535
 bool geom_ok(const mkv_geom& g) {
-  return g.batch >= 1 && g.n_kv_heads >= 1 && (g.head_dim == 64 || g.head_dim == 128) &&
-         (g.group == 1 || g.group == 2 || g.group == 4 || g.group == 8) &&
+  return g.batch >= 1 && g.n_kv_heads >= 1 && g.batch <= 65535 && g.n_kv_heads <= 65535 &&
+         (g.head_dim == 64 || g.head_dim == 128) && (g.group == 1 || g.group == 2 || g.group == 4 || g.group == 8) &&
          (long)g.batch * g.n_kv_heads <= 65535L * 64;
 }
 
@@ -249,6 +251,8 @@ static mkv_status compress_params_ok(const mkv_geom& geom, int32_t T, const mkv_
   // the g * w window rows fill at most two 128-row blocks: the Q stage in
   // shared memory, the logits columns in TMEM and one Q tensor-map box
   if ((long)geom.group * p->window > 256) return MKV_ERR_SHAPE;
+  // the compress kernels take one grid row (y) per unit
+  if ((long)geom.batch * geom.n_kv_heads > 65535) return MKV_ERR_SHAPE;
   if (T > p->budget && protected_count_host(T, p->window, p->sink, p->keep_window) > p->budget)
     return MKV_ERR_INVALID_ARG;
   if (p->adaptive != 0 && p->adaptive != 1) return MKV_ERR_INVALID_ARG;

@@ -64,6 +64,8 @@ def test_decode_validation(L):
     assert decode(L, mkv.geom(1, 2, 4, 96)) == 6            # head_dim unsupported
     assert decode(L, mkv.geom(1, 2, 3, 128)) == 2           # group unsupported
     assert decode(L, mkv.geom(0, 2, 4, 128)) == 2           # empty batch
+    assert decode(L, mkv.geom(65536, 1, 4, 128)) == 2       # batch past the grid's z limit
+    assert decode(L, mkv.geom(1, 65536, 4, 128)) == 2       # KV heads past the grid's y limit
     assert decode(L, g, q=None) == 1
     assert decode(L, g, out=None) == 1
     assert decode(L, g, kn=FAKE) == 1                        # k_new without v_new
@@ -114,6 +116,7 @@ def test_compress_validation(L):
     assert compress(L, g, 1024, P(window=0)) == 1
     assert compress(L, g, 8, P(window=16)) == 1               # window longer than the prompt
     assert compress(L, mkv.geom(1, 2, 4, 64), 1024, P(budget=200, window=65)) == 2  # 260 window rows
+    assert compress(L, mkv.geom(256, 256, 2, 64), 1024, P()) == 2   # 65536 units: one grid row each
     assert compress(L, g, 1024, P(pool=3)) == 1
     assert compress(L, g, 1024, P(mi=2)) == 1
     assert compress(L, g, 0, P()) == 1
