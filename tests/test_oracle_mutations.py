@@ -49,6 +49,42 @@ MUTATIONS = {
     "clamp applied to C instead of S_tilde": (
         "S_tilde = clamp_s_tilde(m.n * np.asarray(m.C, F64), tau)\n    return",
         "S_tilde = m.n * clamp_s_tilde(np.asarray(m.C, F64), tau)\n    return"),
+    "co-moment without the key mean": ("S_tilde += np.outer(V_E[i], K_E[i] - k_bar)",
+                                       "S_tilde += np.outer(V_E[i], K_E[i])"),
+    "window scores not normalised per row": ("s[:visible] += np.exp(lg - log_partition(lg))",
+                                             "s[:visible] += np.exp(lg)"),
+    "causal mask dropped": ("visible = T - w + i + 1 if causal else T", "visible = T"),
+    "protected window one short": ("m[max(0, T - window):] = True", "m[max(0, T - window + 1):] = True"),
+    "one sink too many": ("m[:min(sink, T)] = True", "m[:min(sink + 1, T)] = True"),
+    "residual without the value mean": ("r[j] = V[j] - m.mu_v - S_tilde @ K[j]", "r[j] = V[j] - S_tilde @ K[j]"),
+    "residual with a centred key": ("r[j] = V[j] - m.mu_v - S_tilde @ K[j]",
+                                    "r[j] = V[j] - m.mu_v - S_tilde @ (K[j] - m.mu_k)"),
+    "Jensen logit sign": ("return math.log(m.n) + float(np.asarray(q, F64) @ m.mu_k)",
+                          "return math.log(m.n) - float(np.asarray(q, F64) @ m.mu_k)"),
+    "f_hat_E without 1/sqrt(d)": ("S_tilde @ np.asarray(q, F64) / (m.n * math.sqrt(d))",
+                                  "S_tilde @ np.asarray(q, F64) / m.n"),
+    "order 0 keeps the covariance term": ("if order == 0:\n        return np.array(m.mu_v, F64)",
+                                          "if order == -1:\n        return np.array(m.mu_v, F64)"),
+    "log-sum-exp without its shift": ("lse = top + math.log(", "lse = math.log("),
+    "decode does not append": (
+        "        K_R = np.vstack([K_R, np.asarray(k_new, F64)[None]])\n"
+        "        V_R = np.vstack([V_R, np.asarray(v_new, F64)[None]])",
+        "        pass"),
+    "recovery identity sign": ("S_tilde = S - np.outer(s_v, s_k) / n\n    return k_bar",
+                               "S_tilde = S + np.outer(s_v, s_k) / n\n    return k_bar"),
+    "Welford key-mean step": ("mu_k = m.mu_k + dk / n1", "mu_k = m.mu_k + dk / (n1 + 1)"),
+    "Chan mean weighted by the wrong count": ("mu_k = a.mu_k + dk * (b.n / n)", "mu_k = a.mu_k + dk * (a.n / n)"),
+    "alpha from the first query head only": (
+        "    for h in range(q.shape[0]):\n        s = logits(q[h], K_R)",
+        "    for h in range(1):\n        s = logits(q[h], K_R)"),
+    "eviction ties to the higher position": ("j_star = int(np.argmin(scores))",
+                                             "j_star = len(scores) - 1 - int(np.argmin(scores[::-1]))"),
+    "evicted token not added to the sums": ("sums = add_token_sums(sums, K[j_star], V[j_star])", "sums = sums"),
+    "M0 from the retained set": ("M0 = moments_of(K[~keep0], V[~keep0])", "M0 = moments_of(K[keep0], V[keep0])"),
+    "output moments from the retained set": ("return CompressResult(R, moments_of(K[~keep], V[~keep])",
+                                             "return CompressResult(R, moments_of(K[keep], V[keep])"),
+    "adaptive M0 from the retained set": ("M0 = moments_of(K[h][~keep0], V[h][~keep0])",
+                                          "M0 = moments_of(K[h][keep0], V[h][keep0])"),
 }
 
 
