@@ -6,7 +6,7 @@
  * mean mu_v and value-key cross-covariance C -- and uses it twice: to choose
  * which tokens to evict (moment residual, Eq. residual) and to add back a
  * closed-form first-order estimate of the evicted tokens' attention output
- * (Eqs. fhat, jensen, fused).  Three calls cover the data-parallel path:
+ * (Eqs. fhat, jensen, fused).  Four calls cover the data-parallel path:
  *
  *   mkv_compress      prefill: window scores, budget top-k, moment filter,
  *                     evicted-set moments                    (Sec. 5.1, 4.2)
@@ -116,7 +116,7 @@ typedef struct {
   int32_t window;      /* w: observation window = the last w positions        */
   int32_t sink;        /* leading positions always kept (the paper keeps 1)   */
   int32_t keep_window; /* 1: the w window positions are always kept           */
-  int32_t pool;        /* adjacent-token chunk size for scores, 1 = off (Sec. 5.1 uses 4) */
+  int32_t pool;        /* adjacent-token chunk size for scores: 1 (off), 2, 4, 8, 16 or 32 (Sec. 5.1 uses 4) */
   int32_t mi;          /* 1: moment-informed second stage; 0: window scores only */
   int32_t causal;      /* 1: window query i (position T-w+i) sees keys t <= T-w+i */
   float tau;           /* clamp |S_tilde_ab| < tau to 0 in the residual (App. C.2) */
@@ -281,8 +281,9 @@ MKV_API size_t mkv_evict_workspace_size(mkv_geom geom, int32_t capacity);
  * the smallest score (ties: the lower position), fold it into the moments
  * (n+1; the equivalent of Eq. app_update on (n, mu_k, mu_v, C)) and remove
  * it.  Surviving rows keep their ascending position order.
- * Requirements: 0 <= budget, len + (k_new ? 1 : 0) <= capacity (else the
- * kernel records MKV_ERR_CAPACITY and leaves the unit unchanged).
+ * Requirements: 0 <= budget, capacity <= 65536 (else MKV_ERR_SHAPE),
+ * len + (k_new ? 1 : 0) <= capacity (else the kernel records
+ * MKV_ERR_CAPACITY and leaves the unit unchanged).
  */
 MKV_API mkv_status mkv_evict_append(mkv_geom geom, const void* q, const void* k_new, const void* v_new,
                             int32_t budget, const mkv_cache* cache, const mkv_moments* mom,
