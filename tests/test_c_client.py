@@ -133,3 +133,14 @@ def test_header_compiles_as_cpp(tmp_path):
     r = subprocess.run([cxx, "-std=c++17", "-Wall", "-Wextra", "-Werror", "-fsyntax-only", "-I", INCLUDE, str(src)],
                        capture_output=True, text=True)
     assert r.returncode == 0, r.stderr
+
+
+def test_binding_structs_match_the_c_layout():
+    import ctypes
+    assert ctypes.sizeof(mkv.mkv_geom) == 16
+    assert ctypes.sizeof(mkv.mkv_moments) == 32
+    assert ctypes.sizeof(mkv.mkv_cache) == 48 and mkv.mkv_cache.capacity.offset == 40
+    assert ctypes.sizeof(mkv.mkv_compress_params) == 36
+    assert mkv.mkv_compress_params.tau.offset == 28 and mkv.mkv_compress_params.adaptive.offset == 32
+    assert ctypes.sizeof(mkv.mkv_decode_params) == 24 and mkv.mkv_decode_params.C16.offset == 16
+    assert ctypes.sizeof(mkv.mkv_compress_diag) == 24
