@@ -787,7 +787,7 @@ def cpu_baseline():
     return {"value": round(tokens / est, 3), "unit": "tokens/s", "cores": max(1, round(cpu / wall)),
             "kind": "oracle", "sample": f"{n} of {units} KV-head units of the full step (compress T=8192, "
             f"256 decode steps, 4 evictions), fp64 numpy, scaled by {units}/{n}; "
-            f"{wall:.1f} s wall, host nproc={os.cpu_count()}"}
+            f"{wall:.1f} s wall, host nproc={os.cpu_count()}; cores = CPU time / wall time (numpy's BLAS threads)"}
 
 
 def run_reference(args):
@@ -810,7 +810,7 @@ def run_reference(args):
     value = tokens / (est_ms / 1e3)
     cores = max(1, round(cpu / wall))
     sample = (f"each step: one of {units} KV-head units of the full step (compress T=8192, 256 decode steps, "
-              f"4 evictions) through the fp64 oracle, scaled by {units}")
+              f"4 evictions) through the fp64 oracle, scaled by {units}; cores = CPU time / wall time")
     print(json.dumps({"impl": "reference", "metric": METRIC, "value": round(value, 3), "unit": "tokens/s",
                       "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(est_ms, 2),
                       "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
