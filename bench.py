@@ -21,6 +21,8 @@ extra keys the decode sweep cells (batch x budget, correction on/off),
 
 --impl reference times the fp64 oracle on the host cores instead (a bounded
 sample: one KV-head unit of the same workload per step, scaled to the whole).
+--only LEG runs one of the extra legs alone and prints its result, so that a
+profiler can capture that leg without the step's decode launches.
 """
 from __future__ import annotations
 
