@@ -83,6 +83,9 @@ typedef struct {
  *                                 row a indexes value dims, column c key dims.
  * n = 0 means "no evicted token" (the other fields are then ignored); a
  * zero-filled struct is the state at the start of a generation (Sec. 5.1).
+ * Alignment: mu_k 8 bytes, mu_v and C 16 bytes (the kernels read them with
+ * vector loads); a misaligned pointer is rejected with MKV_ERR_INVALID_ARG
+ * before anything is launched.
  */
 typedef struct {
   int32_t* n;
@@ -255,8 +258,12 @@ MKV_API mkv_status mkv_decode_step(mkv_geom geom, const void* q, const void* k_n
  *  - Every call shares the array: calls that overlap on the GPU (e.g. on two
  *    streams) race and give wrong results.  Serialise them.
  *  - Errors the kernel detects are recorded in the array's error word, which
- *    this call does not expose; the outputs in those cases are as described
- *    for mkv_decode_step.
+ *    this call does not expose and never clears: the first recorded error
+ *    stays set until the process exits.  The outputs in those cases are as
+ *    described for mkv_decode_step.
+ *  - The array's address is looked up on every call; if it changed (the
+ *    library's device code was loaded again, e.g. after cudaDeviceReset) the
+ *    set-up above runs again.
  */
 MKV_API mkv_status mkv_decode_step_noalloc(mkv_geom geom, const void* q, const void* k_new, const void* v_new,
                                            const mkv_cache* cache, const mkv_moments* mom,

@@ -5,6 +5,7 @@
 
 #include "common.cuh"
 #include "kernels.h"
+#include "validate.h"
 
 using namespace mkv;
 
@@ -19,26 +20,6 @@ int num_sms_current() {
   if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
   if (dev >= 0 && dev < 64) cache[dev] = n;
   return n;
-}
-
-// batch and KV heads are grid dimensions of the decode launch (z and y), so
-// each stays within 65535
-bool geom_ok(const mkv_geom& g) {
-  return g.batch >= 1 && g.n_kv_heads >= 1 && g.batch <= 65535 && g.n_kv_heads <= 65535 &&
-         (g.head_dim == 64 || g.head_dim == 128) && (g.group == 1 || g.group == 2 || g.group == 4 || g.group == 8) &&
-         (long)g.batch * g.n_kv_heads <= 65535L * 64;
-}
-
-bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
-
-bool cache_ok(const mkv_cache* c) {
-  return c && c->K && c->V && c->pos && c->len && c->seen && c->capacity >= 1 && aligned(c->K, 16) &&
-         aligned(c->V, 16);
-}
-
-bool moments_ok(const mkv_moments* m) {
-  return m && m->n && m->mu_k && m->mu_v && m->C && aligned(m->C, 16) && aligned(m->mu_k, 4) &&
-         aligned(m->mu_v, 4);
 }
 
 int protected_count_host(int T, int W, int sink, int keep_window) {
@@ -79,16 +60,8 @@ size_t mkv_decode_workspace_size(mkv_geom geom, int32_t capacity) {
 mkv_status mkv_decode_step(mkv_geom geom, const void* q, const void* k_new, const void* v_new,
                            const mkv_cache* cache, const mkv_moments* mom, const mkv_decode_params* p,
                            float* out, float* lse, void* workspace, size_t workspace_bytes, void* stream) {
-  if (!geom_ok(geom)) return (geom.head_dim == 64 || geom.head_dim == 128) ? MKV_ERR_SHAPE : MKV_ERR_UNSUPPORTED;
-  if (!q || !out || !p || !cache_ok(cache)) return MKV_ERR_INVALID_ARG;
-  if ((k_new == nullptr) != (v_new == nullptr)) return MKV_ERR_INVALID_ARG;
-  if (!aligned(q, 16) || !aligned(out, 16) || (k_new && (!aligned(k_new, 16) || !aligned(v_new, 16))))
-    return MKV_ERR_INVALID_ARG;
-  if (p->correction != 0 && p->correction != 1) return MKV_ERR_INVALID_ARG;
-  if (p->order != 0 && p->order != 1) return MKV_ERR_INVALID_ARG;
-  if (p->correction && !moments_ok(mom)) return MKV_ERR_INVALID_ARG;
-  if (!(p->tau >= 0.f)) return MKV_ERR_INVALID_ARG;
-  if (p->C16 && !aligned(p->C16, 16)) return MKV_ERR_INVALID_ARG;
+  const mkv_status chk = decode_args_status(geom, q, k_new, v_new, cache, mom, p, out);
+  if (chk != MKV_OK) return chk;
   const int sms = num_sms_current();
   const size_t need = decode_workspace_bytes(geom, cache->capacity, sms);
   if (!workspace || workspace_bytes < need || !aligned(workspace, 256)) return MKV_ERR_WORKSPACE;
@@ -119,7 +92,7 @@ mkv_status mkv_decode_step(mkv_geom geom, const void* q, const void* k_new, cons
 }
 
 mkv_status mkv_moments_pack_bf16(mkv_geom geom, const mkv_moments* mom, void* C16, void* stream) {
-  if (!geom_ok(geom)) return (geom.head_dim == 64 || geom.head_dim == 128) ? MKV_ERR_SHAPE : MKV_ERR_UNSUPPORTED;
+  if (!geom_ok(geom)) return geom_status(geom);
   if (!moments_ok(mom) || !C16 || !aligned(C16, 16)) return MKV_ERR_INVALID_ARG;
   const size_t n = (size_t)geom.batch * geom.n_kv_heads * geom.head_dim * geom.head_dim;
   return cuda_status(launch_pack_bf16(mom->C, static_cast<__nv_bfloat16*>(C16), n, static_cast<cudaStream_t>(stream)));
@@ -134,7 +107,7 @@ size_t mkv_evict_workspace_size(mkv_geom geom, int32_t capacity) {
 mkv_status mkv_evict_append(mkv_geom geom, const void* q, const void* k_new, const void* v_new, int32_t budget,
                             const mkv_cache* cache, const mkv_moments* mom, float tau, void* workspace,
                             size_t workspace_bytes, void* stream) {
-  if (!geom_ok(geom)) return (geom.head_dim == 64 || geom.head_dim == 128) ? MKV_ERR_SHAPE : MKV_ERR_UNSUPPORTED;
+  if (!geom_ok(geom)) return geom_status(geom);
   if (!q || !cache_ok(cache) || !moments_ok(mom) || budget < 0 || !(tau >= 0.f)) return MKV_ERR_INVALID_ARG;
   if ((k_new == nullptr) != (v_new == nullptr)) return MKV_ERR_INVALID_ARG;
   if (cache->capacity > 65536) return MKV_ERR_SHAPE;
@@ -178,7 +151,7 @@ size_t mkv_decode_evict_workspace_size(mkv_geom geom, int32_t capacity) {
 mkv_status mkv_decode_evict_step(mkv_geom geom, const void* q, const void* k_new, const void* v_new, int32_t budget,
                                  const mkv_cache* cache, const mkv_moments* mom, const mkv_decode_params* p,
                                  float* out, float* lse, void* workspace, size_t workspace_bytes, void* stream) {
-  if (!geom_ok(geom)) return (geom.head_dim == 64 || geom.head_dim == 128) ? MKV_ERR_SHAPE : MKV_ERR_UNSUPPORTED;
+  if (!geom_ok(geom)) return geom_status(geom);
   if (!q || !k_new || !v_new || !out || !p || !cache_ok(cache) || !moments_ok(mom) || budget < 0)
     return MKV_ERR_INVALID_ARG;
   if (!aligned(q, 16) || !aligned(out, 16) || !aligned(k_new, 16) || !aligned(v_new, 16)) return MKV_ERR_INVALID_ARG;
@@ -240,7 +213,7 @@ mkv_status mkv_decode_evict_step(mkv_geom geom, const void* q, const void* k_new
 
 // ---------------------------------------------------------------- compress
 static mkv_status compress_params_ok(const mkv_geom& geom, int32_t T, const mkv_compress_params* p) {
-  if (!geom_ok(geom)) return (geom.head_dim == 64 || geom.head_dim == 128) ? MKV_ERR_SHAPE : MKV_ERR_UNSUPPORTED;
+  if (!geom_ok(geom)) return geom_status(geom);
   if (!p || T < 1 || T > (1 << 20) || p->budget < 1 || p->window < 1 || p->window > T || p->sink < 0)
     return MKV_ERR_INVALID_ARG;
   if ((p->keep_window != 0 && p->keep_window != 1) || (p->mi != 0 && p->mi != 1) ||

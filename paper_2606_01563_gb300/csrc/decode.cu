@@ -874,28 +874,6 @@ void decode_carve(DecodeArgs& a, const mkv_geom& g, int32_t capacity, int num_sm
   a.S = S;
 }
 
-size_t decode_workspace_bytes_splits(const mkv_geom& g, int S) {
-  const size_t units = (size_t)g.batch * g.n_kv_heads;
-  size_t off = kHeaderBytes;
-  off += align_up(units * sizeof(uint32_t), 256);
-  off += align_up(units * S * g.group * (g.head_dim + 4) * sizeof(float), 256);
-  off += align_up(units * g.group * g.head_dim * sizeof(float), 256);
-  return off;
-}
-
-void decode_carve_splits(DecodeArgs& a, const mkv_geom& g, int S, void* ws) {
-  const size_t units = (size_t)g.batch * g.n_kv_heads;
-  uint8_t* p = static_cast<uint8_t*>(ws);
-  a.ws = ws;
-  size_t off = kHeaderBytes;
-  a.counters = reinterpret_cast<uint32_t*>(p + off);
-  off += align_up(units * sizeof(uint32_t), 256);
-  a.partial = reinterpret_cast<float*>(p + off);
-  off += align_up(units * S * g.group * (g.head_dim + 4) * sizeof(float), 256);
-  a.fhat = reinterpret_cast<float*>(p + off);
-  a.S = S;
-}
-
 cudaError_t launch_decode(const DecodeArgs& a, int head_dim, int group, cudaStream_t stream) {
 #define MKV_DECODE_CASE(D, G) \
   if (head_dim == D && group == G) return launch_dg<D, G>(a, stream);

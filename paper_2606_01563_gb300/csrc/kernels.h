@@ -48,10 +48,6 @@ size_t decode_workspace_bytes(const mkv_geom& g, int32_t capacity, int num_sms);
 void decode_carve(DecodeArgs& a, const mkv_geom& g, int32_t capacity, int num_sms, void* ws);
 cudaError_t launch_decode(const DecodeArgs& a, int head_dim, int group, cudaStream_t stream);
 cudaError_t launch_pack_bf16(const float* C, __nv_bfloat16* C16, size_t n, cudaStream_t stream);
-// The same carving for an explicit split count S (used by the entry point
-// whose scratch has a fixed maximum size).
-size_t decode_workspace_bytes_splits(const mkv_geom& g, int S);
-void decode_carve_splits(DecodeArgs& a, const mkv_geom& g, int S, void* ws);
 
 // ------------------------------------------------------------------- evict
 struct EvictArgs {

@@ -78,6 +78,40 @@ def test_decode_validation(L):
     assert decode(L, g, ws=FAKE + 8) == 7                    # misaligned workspace
     assert decode(L, g, p=mkv.mkv_decode_params(1, 1, 0.0, FAKE + 8)) == 1  # misaligned bf16 C copy
     assert decode(L, g, q=FAKE + 4) == 1                     # misaligned q
+    # mu_k is read as float2 and mu_v as float4: 4-byte alignment is not enough
+    assert decode(L, g, mom=mkv.mkv_moments(FAKE, FAKE + 4, FAKE, FAKE)) == 1
+    assert decode(L, g, mom=mkv.mkv_moments(FAKE, FAKE, FAKE + 8, FAKE)) == 1
+    assert decode(L, g, mom=mkv.mkv_moments(FAKE, FAKE, FAKE, FAKE + 8)) == 1
+    # without the correction the moments are not read, so they are not checked
+    assert decode(L, g, mom=mkv.mkv_moments(FAKE, FAKE + 4, FAKE, FAKE), p=mkv.mkv_decode_params(0, 1, 0.0),
+                  wsb=16) == 7
+
+
+def noalloc(L, g, q=FAKE, cache=None, mom=None, p=None, out=FAKE):
+    cache = cache or fake_cache()
+    mom = mom or fake_moments()
+    p = p or mkv.mkv_decode_params(1, 1, 1e-6)
+    return L.mkv_decode_step_noalloc(g, q, None, None, ctypes.byref(cache), ctypes.byref(mom), ctypes.byref(p),
+                                     out, None, None)
+
+
+def test_noalloc_validation_matches_decode(L):
+    """The no-allocation decode rejects what mkv_decode_step rejects, with the
+    same status, before it touches the device (these cases never get there)."""
+    g = mkv.geom(1, 2, 4, 128)
+    cases = [dict(g=mkv.geom(1, 2, 4, 96)), dict(g=mkv.geom(1, 2, 3, 128)), dict(g=mkv.geom(65536, 1, 4, 128)),
+             dict(g=mkv.geom(1, 65536, 4, 128)), dict(q=None), dict(out=FAKE + 8),
+             dict(mom=mkv.mkv_moments(FAKE, FAKE + 4, FAKE, FAKE)),
+             dict(mom=mkv.mkv_moments(FAKE, FAKE, FAKE + 8, FAKE)),
+             dict(cache=mkv.mkv_cache(FAKE + 2, FAKE, FAKE, FAKE, FAKE, 64)),
+             dict(p=mkv.mkv_decode_params(1, 2, 0.0)), dict(p=mkv.mkv_decode_params(1, 1, 0.0, FAKE + 8))]
+    for kw in cases:
+        gg = kw.pop("g", g)
+        want = decode(L, gg, **kw)
+        assert want in (1, 2, 6), kw
+        assert noalloc(L, gg, **kw) == want, kw
+    # more units than the fixed scratch holds even at one split per unit
+    assert noalloc(L, mkv.geom(64, 256, 8, 128)) == 7
 
 
 def test_pack_bf16_validation(L):
