@@ -1,28 +1,35 @@
 """Benchmark of the MomentKV hot path on GB300.
 
-A step is one pass of the whole path over one synthetic layer of the
-Llama-3.1-8B attention geometry (32 query heads, 8 KV heads, d=128, bf16,
-batch 1): compress a T=8192 prompt to a budget of 512 (window 32, one sink,
-moment filter on), then 256 corrected decode steps, each appending its token,
-with a moment-informed eviction back to the budget after every 64 tokens.
-Each part is captured once in a CUDA graph and replayed; CUDA events on the
-launching stream time the segments.  L2 is flushed (a 256 MB write) before
-every timed step, outside the timed region.
+Workload (the headline line): the Qwen3-4B attention geometry, all 36 layers
+(32 query heads, 8 KV heads, d=128, bf16), batch 4 at context 32768, window
+32, one sink, moment filter on, at each of the budgets 128, 256 and 1024.
+A step runs, for each budget in turn, one compress of every layer's prompt,
+then 512 decode steps; a decode step is one corrected decode launch per
+layer, layer after layer, each appending that step's token.  So a step is
+3 x (36 compressions + 18432 decode launches) and generates 3 x 4 x 512
+tokens.  Prompts (19.3 GB over the 36 layers) and per-step queries and new
+tokens are synthetic, drawn on the device (inputs.TorchGenerator), resident
+in HBM before the timed region.  Each part is captured once in a CUDA graph
+and replayed; CUDA events on the launching stream time the parts.  L2 is
+flushed (a 256 MB write) before every timed step, outside the timed region.
 
-value      generated decode tokens per second of whole-step time (device-timed,
-           inputs resident in HBM).
-e2e        the same with the step's inputs copied from pinned host memory and
-           the decode outputs copied back inside the timed region.
+value      generated decode tokens per second of whole-step time (device-timed).
+e2e        the same with every input of the step (the 36 prompts, queries and
+           new tokens) copied from pinned host memory, and the last layer's
+           output of every decode step copied back, inside the timed region.
 roofline   the dominant kernel against the measured HBM copy bandwidth.
-extra keys the decode sweep cells (batch x budget, correction on/off),
-           compress throughput at 32K and 128K context, the continuous
-           eviction mode (one Algorithm 1 step per token at the budget), and
-           32 layers' decode in one launch against one launch per layer.
+extra keys the Llama-3.1-8B 32-layer 128K workload (budget 128, window 64,
+           1024 decode steps, an evict-append on every layer every 64
+           tokens), the one-layer Llama-3.1-8B 8K workload, the decode sweep
+           cells (batch x budget, correction on/off), compress with the
+           budget shared across heads, the continuous eviction mode, and 32
+           layers' decode in one launch against one launch per layer.
 
---impl reference times the fp64 oracle on the host cores instead (a bounded
-sample: one KV-head unit of the same workload per step, scaled to the whole).
+--impl reference times the fp64 oracle on the host cores instead: each step
+is a bounded sample of the same workload (16 (layer, unit, budget) jobs run
+by a process pool), reported as the throughput that sample implies.
 --only LEG runs one of the extra legs alone and prints its result, so that a
-profiler can capture that leg without the step's decode launches.
+profiler can capture that leg without the headline's launches.
 """
 from __future__ import annotations
 
@@ -30,6 +37,7 @@ import argparse
 import hashlib
 import json
 import math
+import multiprocessing as mp
 import os
 import resource
 import subprocess
@@ -42,16 +50,16 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "decode-step attn+correction tokens/s and HBM GB/s frac; compress GB/s at 1 GB300"
-WORKLOAD = "llama8b_layer_t8k"
-EVICT_EVERY = 64
+HEADLINE = "qwen4b_t32k"
+BUDGETS = (128, 256, 1024)
+TAU = 1e-6
+ORACLE_JOBS = 16  # (layer, unit, budget) jobs in one oracle sample
 
-# dram__bytes_read.sum + dram__bytes_write.sum per launch of the dominant
-# kernel from one ncu capture of the bench workload
-# (profiles/decode_kernel_llama8b_layer_t8k.md), valid while the code the
-# kernel compiles from (its .cu file and the library headers, comments
-# aside) is what was captured: code_sha of those sources at capture time.
-NCU_TRAFFIC = {"decode": {"bytes": 2957824,
-                          "code_sha": "91f03de032396f51c39e95e171ace5ef6b207ef5a5e4cec27397692c8a88dba9"}}
+# dram__bytes_read.sum + dram__bytes_write.sum per launch of a kernel on the
+# headline workload from one ncu capture, valid while the code the kernel
+# compiles from (its .cu file and the library headers, comments aside) is
+# what was captured: code_sha of those sources at capture time.
+NCU_TRAFFIC = {}
 
 
 def parse():
@@ -60,11 +68,27 @@ def parse():
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
-    ap.add_argument("--no-extras", action="store_true", help="skip the decode sweep and long-context compress")
+    ap.add_argument("--no-extras", action="store_true", help="skip the extra legs")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--only", choices=["decode_sweep", "compress_long", "continuous_eviction", "layers_one_launch"],
+    ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end measurement")
+    ap.add_argument("--layers", type=int, default=None, help="layers of the headline workload (default: all 36)")
+    ap.add_argument("--only", choices=["t128k", "t8k", "decode_sweep", "compress_adaptive", "continuous_eviction",
+                                       "layers_one_launch"],
                     help="run one extra leg alone and print its result (for profiling that leg)")
     return ap.parse_args()
+
+
+def config_dict(layers=None):
+    """The workload description both arms print."""
+    from paper_2606_01563_gb300 import inputs
+    wl = inputs.WORKLOADS[HEADLINE]
+    L = wl.n_layers if layers is None else layers
+    return {"workload": f"{HEADLINE}: Qwen3-4B attention geometry, {L} layers, batch 4, 32 q heads / 8 kv heads, "
+                        f"d=128, T=32768, budgets 128/256/1024 in turn, window 32, sink 1, mi on; per budget: "
+                        f"compress every layer, then 512 decode steps (one launch per layer, append)",
+            "layers": L, "global_batch": wl.geom.batch, "seq_len": wl.T, "budgets": list(BUDGETS),
+            "decode_steps": wl.decode_steps, "parallelism": "replicas", "accum": "f32",
+            "l2": "flushed (256 MB write) before every timed step; a step reads >19 GB"}
 
 
 def job_throughput(total_ms, steps, tokens_per_rank, dist=None, device=None):
@@ -187,134 +211,247 @@ class Clocks:
 
 
 # --------------------------------------------------------------------------
-# the GPU step
+# a multi-layer workload on the device
 # --------------------------------------------------------------------------
-class Step:
-    """Device state, CUDA graphs and byte counts for one workload replica."""
+class Stack:
+    """Device inputs of a multi-layer workload: each layer's prompt K, V,
+    Q_obs, and each (decode step, layer)'s query and new token, drawn on the
+    device by inputs.TorchGenerator (one generator per layer)."""
 
-    def __init__(self, torch, mkv, inputs, seed, dev):
-        self.t = torch
-        self.mkv = mkv
-        wl = inputs.WORKLOADS[WORKLOAD]
-        self.wl = wl
+    def __init__(self, torch, inputs, wl, seed, dev, layers=None, steps=None):
         G = wl.geom
-        self.G = G
+        self.wl, self.G = wl, G
+        self.L = wl.n_layers if layers is None else layers
+        self.S = wl.decode_steps if steps is None else steps
+        d = G.head_dim
+        bf = torch.bfloat16
+        self.K, self.V, self.Q = [], [], []
+        self.q = torch.empty(self.S, self.L, G.batch, G.n_q_heads, d, dtype=bf, device=dev)
+        self.kn = torch.empty(self.S, self.L, G.batch, G.n_kv_heads, d, dtype=bf, device=dev)
+        self.vn = torch.empty_like(self.kn)
+        for l in range(self.L):
+            gen = inputs.TorchGenerator(wl, seed=seed, layer=l, device=dev)
+            K, V, Q = gen.prefill()
+            self.K.append(K)
+            self.V.append(V)
+            self.Q.append(Q)
+            q, kn, vn = gen.decode(self.S)
+            self.q[:, l] = q
+            self.kn[:, l] = kn
+            self.vn[:, l] = vn
+            del gen
+        torch.cuda.synchronize(dev)
+
+    def tensors(self):
+        return self.K + self.V + self.Q + [self.q, self.kn, self.vn]
+
+    def nbytes(self):
+        return sum(t.numel() * t.element_size() for t in self.tensors())
+
+
+class Run:
+    """One budget of a multi-layer workload on a Stack: compress every layer,
+    then `steps` decode steps, each one mkv_decode_step per layer (layer
+    after layer, appending the step's token), and an mkv_evict_append on
+    every layer back to the budget every `evict_every` steps (0: never)."""
+
+    def __init__(self, torch, mkv, stack, budget, evict_every, dev):
+        self.t, self.mkv, self.st = torch, mkv, stack
+        wl, G = stack.wl, stack.G
+        self.G, self.B, self.ev_every = G, budget, evict_every
         self.g = mkv.geom(G.batch, G.n_kv_heads, G.group, G.head_dim)
-        self.dev = dev
-        gen = inputs.Generator(wl, seed=seed)
-        K, V, Q = gen.prefill()
-        q, kn, vn = gen.decode(wl.decode_steps)
-        tb = inputs.to_bf16_tensor
-        # pinned host copies (e2e) and device copies (value)
-        self.host_in = {k: tb(x).pin_memory() for k, x in (("K", K), ("V", V), ("Q", Q), ("q", q), ("kn", kn),
-                                                          ("vn", vn))}
-        self.dev_in = {k: v.to(dev) for k, v in self.host_in.items()}
-        self.T, self.B, self.S = wl.T, wl.budget, wl.decode_steps
-        self.cap = self.B + EVICT_EVERY
-        self.p = mkv.mkv_compress_params(self.B, wl.window, wl.sink, wl.keep_window, 1, 1, 1, 1e-6)
-        self.dp = mkv.mkv_decode_params(1, 1, 1e-6)
-        self.cache = mkv.alloc_cache(self.g, self.cap, dev)
-        self.mom = mkv.alloc_moments(self.g, dev)
-        self.ws_c = mkv.alloc_workspace(mkv.mkv_compress_workspace_size(self.g, self.T, self.p), dev)
+        self.cap = budget + (evict_every if evict_every else stack.S)
+        self.p = mkv.mkv_compress_params(budget, wl.window, wl.sink, wl.keep_window, wl.pool, 1, 1, TAU)
+        self.dp = mkv.mkv_decode_params(1, 1, TAU)
+        self.caches = [mkv.alloc_cache(self.g, self.cap, dev) for _ in range(stack.L)]
+        self.moms = [mkv.alloc_moments(self.g, dev) for _ in range(stack.L)]
+        # one workspace per kind, shared by the layers (the calls run one after another on one stream)
+        self.ws_c = mkv.alloc_workspace(mkv.mkv_compress_workspace_size(self.g, wl.T, self.p), dev)
         self.ws_d = mkv.alloc_workspace(mkv.mkv_decode_workspace_size(self.g, self.cap), dev)
-        self.ws_e = mkv.alloc_workspace(mkv.mkv_evict_workspace_size(self.g, self.cap), dev)
-        self.out = torch.empty(self.S, G.batch, G.n_q_heads, G.head_dim, device=dev)
-        self.out_host = torch.empty(self.out.shape, dtype=torch.float32).pin_memory()
-        self.stream = torch.cuda.Stream(dev)
-        self.launches_per_step = 8 + self.S + self.S // EVICT_EVERY
+        self.ws_e = mkv.alloc_workspace(mkv.mkv_evict_workspace_size(self.g, self.cap), dev) if evict_every else None
+        self.out = torch.empty(G.batch, G.n_q_heads, G.head_dim, device=dev)        # a layer's output
+        self.final = torch.empty(stack.S, G.batch, G.n_q_heads, G.head_dim, device=dev)  # last layer's, per step
+        self.block = evict_every if evict_every else 64
 
-    # the three parts as plain C-ABI calls on the current stream
     def compress(self):
-        d = self.dev_in
-        self.mkv.mkv_compress(self.g, self.T, d["K"], d["V"], d["Q"], self.p, self.cache, self.mom, self.ws_c)
+        s = self.st
+        for l in range(s.L):
+            self.mkv.mkv_compress(self.g, s.wl.T, s.K[l], s.V[l], s.Q[l], self.p, self.caches[l], self.moms[l],
+                                  self.ws_c)
 
-    def decode(self, s):
-        d = self.dev_in
-        self.mkv.mkv_decode_step(self.g, d["q"][s], d["kn"][s], d["vn"][s], self.cache, self.mom, self.dp,
-                                 self.out[s], None, self.ws_d)
+    def decode(self, i):
+        s = self.st
+        for l in range(s.L):
+            out = self.final[i] if l == s.L - 1 else self.out
+            self.mkv.mkv_decode_step(self.g, s.q[i, l], s.kn[i, l], s.vn[i, l], self.caches[l], self.moms[l],
+                                     self.dp, out, None, self.ws_d)
 
-    def evict(self, s):
-        self.mkv.mkv_evict_append(self.g, self.dev_in["q"][s], None, None, self.B, self.cache, self.mom, 1e-6,
-                                  self.ws_e)
+    def evict(self, i):
+        s = self.st
+        for l in range(s.L):
+            self.mkv.mkv_evict_append(self.g, s.q[i, l], None, None, self.B, self.caches[l], self.moms[l], TAU,
+                                      self.ws_e)
 
-    def eager_step(self):
-        self.compress()
-        for s in range(self.S):
-            self.decode(s)
-            if (s + 1) % EVICT_EVERY == 0:
-                self.evict(s)
+    def parts(self):
+        """(kind, callable) in step order."""
+        out = [("compress", self.compress)]
+        for b0 in range(0, self.st.S, self.block):
+            b1 = min(self.st.S, b0 + self.block)
+            out.append(("decode", lambda b0=b0, b1=b1: [self.decode(i) for i in range(b0, b1)]))
+            if self.ev_every and b1 % self.ev_every == 0:
+                out.append(("evict", lambda i=b1 - 1: self.evict(i)))
+        return out
 
-    def capture(self):
+    def capture(self, stream):
         torch = self.t
-        with torch.cuda.stream(self.stream):
-            self.eager_step()  # warm: function attributes, SM-count cache
-        self.stream.synchronize()
-        self.graphs = []
-        def cap(fn):
-            gr = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(gr, stream=self.stream, capture_error_mode="relaxed"):
+        with torch.cuda.stream(stream):
+            for _, fn in self.parts():  # warm: function attributes, SM-count cache
                 fn()
-            return gr
-        self.g_compress = cap(self.compress)
-        self.g_blocks = []
-        for b0 in range(0, self.S, EVICT_EVERY):
-            gd = cap(lambda b0=b0: [self.decode(s) for s in range(b0, min(self.S, b0 + EVICT_EVERY))])
-            ge = cap(lambda b0=b0: self.evict(min(self.S, b0 + EVICT_EVERY) - 1))
-            self.g_blocks.append((gd, ge))
+        stream.synchronize()
+        self.graphs = []
+        for kind, fn in self.parts():
+            gr = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gr, stream=stream, capture_error_mode="relaxed"):
+                fn()
+            self.graphs.append((kind, gr))
 
-    def replay(self, ev=None):
-        """Replays one step on self.stream; ev: list of 2 + 2*blocks events to record between parts."""
-        torch = self.t
-        with torch.cuda.stream(self.stream):
-            if ev:
-                ev[0].record(self.stream)
-            self.g_compress.replay()
-            k = 1
-            if ev:
-                ev[k].record(self.stream)
-            for gd, ge in self.g_blocks:
-                gd.replay()
-                k += 1
-                if ev:
-                    ev[k].record(self.stream)
-                ge.replay()
-                k += 1
-                if ev:
-                    ev[k].record(self.stream)
+    def launches(self):
+        """Kernels of ours one pass launches (9 per per-unit compress)."""
+        s = self.st
+        n_ev = (s.S // self.ev_every) if self.ev_every else 0
+        return s.L * (9 + s.S + n_ev)
 
-    def n_events(self):
-        return 2 + 2 * len(self.g_blocks)
-
-    def check_errors(self):
+    def check_errors(self, stream):
         for ws in (self.ws_c, self.ws_d, self.ws_e):
-            code, info = self.mkv.mkv_get_device_error(ws, self.stream)
+            if ws is None:
+                continue
+            code, info = self.mkv.mkv_get_device_error(ws, stream)
             if code != 0:
-                raise RuntimeError(f"device error {code} (unit {info})")
+                raise RuntimeError(f"device error {code} (unit {info}) at budget {self.B}")
 
     # algorithmic bytes: every input read once, every output written once
-    def decode_bytes_total(self):
-        G, d = self.G, self.G.head_dim
+    def decode_bytes(self):
+        """Total over the pass's decode launches."""
+        G, d, s = self.G, self.G.head_dim, self.st
         units = G.batch * G.n_kv_heads
-        tot = 0
-        length = self.B
-        for s in range(self.S):
-            tot += units * (length * d * 2 * 2 + d * d * 4 + 2 * d * 4 + 4)   # retained K,V + moments
-            tot += G.batch * G.n_q_heads * d * 2 + units * d * 2 * 2            # q, k_new/v_new
-            tot += units * d * 2 * 2 + G.batch * G.n_q_heads * d * 4            # appended row, out
+        tot, length = 0, self.B
+        for i in range(s.S):
+            per = units * (length * d * 2 * 2 + d * d * 4 + 2 * d * 4 + 4)    # retained K,V + moments
+            per += G.batch * G.n_q_heads * d * 2 + units * d * 2 * 2          # q, k_new/v_new
+            per += units * d * 2 * 2 + G.batch * G.n_q_heads * d * 4          # appended row, out
+            tot += per * s.L
             length += 1
-            if (s + 1) % EVICT_EVERY == 0:
+            if self.ev_every and (i + 1) % self.ev_every == 0:
                 length = self.B
         return tot
 
     def compress_bytes(self):
-        G, d = self.G, self.G.head_dim
+        """Algorithmic bytes of one layer's compress: K and V read once, window queries, outputs written once."""
+        G, d, wl = self.G, self.G.head_dim, self.st.wl
         units = G.batch * G.n_kv_heads
-        return units * (2 * self.T * d * 2 + G.group * self.wl.window * d * 2 + self.B * d * 2 * 2
+        return units * (2 * wl.T * d * 2 + G.group * wl.window * d * 2 + self.B * (d * 2 * 2 + 4)
                         + (d * d + 2 * d + 1) * 4)
 
+    def compress_flops(self):
+        G, d, wl = self.G, self.G.head_dim, self.st.wl
+        units = G.batch * G.n_kv_heads
+        return units * (2 * G.group * wl.window * wl.T * d + 4 * wl.T * d * d)
 
-def l2_flush(torch, buf):
-    buf.zero_()
+
+def replay(runs, stream, ev=None):
+    """One step: every run's parts in order on `stream`; ev[k] recorded before
+    part k and after the last one."""
+    torch = runs[0].t
+    k = 0
+    with torch.cuda.stream(stream):
+        for r in runs:
+            for _, gr in r.graphs:
+                if ev is not None:
+                    ev[k].record(stream)
+                gr.replay()
+                k += 1
+        if ev is not None:
+            ev[k].record(stream)
+
+
+def part_kinds(runs):
+    return [(r.B, kind) for r in runs for kind, _ in r.graphs]
+
+
+def time_steps(torch, runs, stream, flush, steps):
+    """Device time of `steps` steps, L2 flushed before each: per-part times [steps, parts] (ms)."""
+    nparts = sum(len(r.graphs) for r in runs)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(nparts + 1)] for _ in range(steps)]
+    for k in range(steps):
+        with torch.cuda.stream(stream):
+            flush.zero_()
+        replay(runs, stream, evs[k])
+    stream.synchronize()
+    return np.array([[evs[k][i].elapsed_time(evs[k][i + 1]) for i in range(nparts)] for k in range(steps)])
+
+
+def summarise(runs, seg, hbm):
+    """Per budget and kind: ms per step, and the decode / compress roofline figures."""
+    kinds = part_kinds(runs)
+    res = {}
+    for r in runs:
+        cols = {kind: [i for i, (B, k) in enumerate(kinds) if B == r.B and k == kind] for kind in
+                ("compress", "decode", "evict")}
+        ms = {k: float(seg[:, c].sum(axis=1).mean()) if c else 0.0 for k, c in cols.items()}
+        n_dec = r.st.S * r.st.L
+        dec_b = r.decode_bytes()
+        L = r.st.L
+        res[r.B] = {"ms": {k: round(v, 4) for k, v in ms.items()},
+                    "decode": {"launches": n_dec, "avg_launch_us": round(ms["decode"] * 1e3 / n_dec, 3),
+                               "bytes_per_launch": round(dec_b / n_dec), "gbs": round(dec_b / ms["decode"] / 1e6, 1),
+                               "frac": round(dec_b / ms["decode"] / 1e6 / hbm, 4)},
+                    "compress": {"ms_per_layer": round(ms["compress"] / L, 4),
+                                 "gbs": round(r.compress_bytes() * L / ms["compress"] / 1e6, 1),
+                                 "frac": round(r.compress_bytes() * L / ms["compress"] / 1e6 / hbm, 4),
+                                 "tflops": round(r.compress_flops() * L / ms["compress"] / 1e9, 2)},
+                    "decode_bytes": dec_b}
+        if r.ev_every:
+            n_ev = (r.st.S // r.ev_every) * L
+            res[r.B]["evict"] = {"launches": n_ev, "avg_launch_us": round(ms["evict"] * 1e3 / max(1, n_ev), 2)}
+    return res
+
+
+def l2_flush_buffer(torch, dev):
+    return torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=dev)
+
+
+def e2e_measure(torch, stack, runs, stream, flush, steps):
+    """End to end through the C ABI: every input of the step copied from
+    pinned host memory and each budget's last-layer outputs copied back,
+    inside the timed region.  Returns (ms per step list, h2d bytes, d2h bytes)."""
+    dev_in = stack.tensors()
+    host_in = []
+    for t in dev_in:
+        h = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+        h.copy_(t)
+        host_in.append(h)
+    host_out = [torch.empty(r.final.shape, dtype=r.final.dtype, pin_memory=True) for r in runs]
+    times = []
+    for _ in range(steps):
+        with torch.cuda.stream(stream):
+            flush.zero_()
+        stream.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for d, h in zip(dev_in, host_in):
+                d.copy_(h, non_blocking=True)
+        replay(runs, stream)
+        with torch.cuda.stream(stream):
+            for h, r in zip(host_out, runs):
+                h.copy_(r.final, non_blocking=True)
+            e1.record(stream)
+        stream.synchronize()
+        times.append(e0.elapsed_time(e1))
+    h2d = sum(t.numel() * t.element_size() for t in host_in)
+    d2h = sum(t.numel() * t.element_size() for t in host_out)
+    del host_in, host_out
+    return times, h2d, d2h
 
 
 def run_gpu(args):
@@ -328,129 +465,158 @@ def run_gpu(args):
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=dev)
     mkv.lib()
+    hbm, peak_kind = peaks()
+    flush = l2_flush_buffer(torch, dev)
     if args.only:
-        hbm, _ = peaks()
-        flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=dev)
-        legs = {"decode_sweep": lambda: decode_sweep(torch, mkv, dev, flush, hbm),
-                "compress_long": lambda: compress_long(torch, mkv, inputs, dev, flush, hbm),
+        legs = {"t128k": lambda: leg_t128k(torch, mkv, inputs, dev, flush, hbm),
+                "t8k": lambda: leg_t8k(torch, mkv, inputs, dev, flush, hbm),
+                "decode_sweep": lambda: decode_sweep(torch, mkv, dev, flush, hbm),
+                "compress_adaptive": lambda: compress_adaptive(torch, mkv, inputs, dev, flush, hbm),
                 "continuous_eviction": lambda: continuous_eviction(torch, mkv, dev),
                 "layers_one_launch": lambda: layers_one_launch(torch, mkv, dev, flush, hbm)}
         print(json.dumps({"only": args.only, args.only: legs[args.only]()}), flush=True)
         return
-    step = Step(torch, mkv, inputs, seed=1000 * rank, dev=dev)
-    step.capture()
-    flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=dev)
-    st = step.stream
+
+    wl = inputs.WORKLOADS[HEADLINE]
+    t_setup = time.perf_counter()
+    stack = Stack(torch, inputs, wl, seed=1000 * rank, dev=dev, layers=args.layers)
+    runs = [Run(torch, mkv, stack, B, 0, dev) for B in BUDGETS]
+    stream = torch.cuda.Stream(dev)
+    for r in runs:
+        r.capture(stream)
+    setup_s = time.perf_counter() - t_setup
 
     for _ in range(args.warmup):
-        l2_flush(torch, flush)
-        step.replay()
-    st.synchronize()
-    step.check_errors()
+        with torch.cuda.stream(stream):
+            flush.zero_()
+        replay(runs, stream)
+    stream.synchronize()
+    for r in runs:
+        r.check_errors(stream)
 
     # ---- device-timed steps
-    nev = step.n_events()
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(nev)] for _ in range(args.steps)]
     clocks = Clocks(local)
     if dist:
         dist.barrier()
     torch.cuda.synchronize()
     clocks.start()
-    for k in range(args.steps):
-        with torch.cuda.stream(st):
-            l2_flush(torch, flush)
-        step.replay(evs[k])
-    st.synchronize()
+    seg = time_steps(torch, runs, stream, flush, args.steps)
     torch.cuda.synchronize()
     clk = clocks.stop()
     if dist:
         dist.barrier()
-    step.check_errors()
-    seg = np.array([[evs[k][i].elapsed_time(evs[k][i + 1]) for i in range(nev - 1)] for k in range(args.steps)])
+    for r in runs:
+        r.check_errors(stream)
     step_ms = seg.sum(axis=1)
-    compress_ms = seg[:, 0]
-    decode_ms = seg[:, 1::2].sum(axis=1)
-    evict_ms = seg[:, 2::2].sum(axis=1)
-    ms_per_step, value = job_throughput(float(step_ms.sum()), args.steps, step.G.batch * step.S, dist, dev)
+    tokens = sum(stack.G.batch * stack.S for _ in runs)
+    ms_per_step, value = job_throughput(float(step_ms.sum()), args.steps, tokens, dist, dev)
+    per_budget = summarise(runs, seg, hbm)
 
-    # ---- end to end: host inputs in, decode outputs back, inside the timed region
-    e2e_ms = []
-    h2d = sum(v.numel() * v.element_size() for v in step.host_in.values())
-    d2h = step.out.numel() * 4
-    for k in range(max(3, min(args.steps, 10))):
-        l2_flush(torch, flush)
-        torch.cuda.synchronize()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        with torch.cuda.stream(st):
-            e0.record(st)
-            for name, hv in step.host_in.items():
-                step.dev_in[name].copy_(hv, non_blocking=True)
-        step.replay()
-        with torch.cuda.stream(st):
-            step.out_host.copy_(step.out, non_blocking=True)
-            e1.record(st)
-        st.synchronize()
-        e2e_ms.append(e0.elapsed_time(e1))
-    e2e_step, e2e_value = job_throughput(float(np.sum(e2e_ms)), len(e2e_ms), step.G.batch * step.S, dist, dev)
+    # ---- end to end through the C ABI
+    e2e = None
+    if not args.no_e2e:
+        try:
+            times, h2d, d2h = e2e_measure(torch, stack, runs, stream, flush, max(3, min(args.steps, 5)))
+            for r in runs:
+                r.check_errors(stream)
+            e2e_step, e2e_value = job_throughput(float(np.sum(times)), len(times), tokens, dist, dev)
+            e2e = {"value": round(e2e_value, 2), "unit": "tokens/s", "h2d_bytes_per_step": int(h2d),
+                   "d2h_bytes_per_step": int(d2h), "ms_per_step": round(e2e_step, 4)}
+        except RuntimeError as exc:  # pinned host memory for every input could not be had
+            e2e = {"value": None, "unit": "tokens/s", "error": str(exc)[:200]}
 
     # ---- roofline of the dominant kernel
-    hbm, peak_kind = peaks()
-    dec_launch_ms = float(decode_ms.mean()) / step.S
-    dec_bytes = step.decode_bytes_total() / step.S
-    cmp_bytes = step.compress_bytes()
-    shares = {"decode": float(decode_ms.mean() / step_ms.mean()), "compress": float(compress_ms.mean() / step_ms.mean()),
-              "evict": float(evict_ms.mean() / step_ms.mean())}
-    dominant = max(shares, key=shares.get)
-    if dominant == "decode":
-        achieved = dec_bytes / (dec_launch_ms / 1e3) / 1e9
-        src = kernel_sources("decode.cu")
-        kern = "decode_kernel"
-    elif dominant == "compress":
-        achieved = cmp_bytes / (float(compress_ms.mean()) / 1e3) / 1e9
-        src = kernel_sources("compress.cu")
-        kern = "compress (8 launches)"
+    kinds = part_kinds(runs)
+    tot = {k: float(seg[:, [i for i, (_, kk) in enumerate(kinds) if kk == k]].sum(axis=1).mean())
+           for k in ("compress", "decode")}
+    shares = {k: round(v / float(step_ms.mean()), 4) for k, v in tot.items()}
+    dec_bytes = sum(per_budget[r.B]["decode_bytes"] for r in runs)
+    dec_launches = sum(r.st.S * r.st.L for r in runs)
+    cmp_bytes = sum(r.compress_bytes() * r.st.L for r in runs)
+    if shares["decode"] >= shares["compress"]:
+        kern, achieved = "decode_kernel", dec_bytes / (tot["decode"] / 1e3) / 1e9
+        per_launch, src = dec_bytes / dec_launches, kernel_sources("decode.cu")
+        avg_us = tot["decode"] * 1e3 / dec_launches
     else:
-        achieved = None
-        src = kernel_sources("evict.cu")
-        kern = "evict_kernel"
-    tr = NCU_TRAFFIC.get(dominant)
+        kern, achieved = "compress (9 launches per layer)", cmp_bytes / (tot["compress"] / 1e3) / 1e9
+        per_launch, src = cmp_bytes / (stack.L * len(runs)), kernel_sources("compress.cu")
+        avg_us = tot["compress"] * 1e3 / (stack.L * len(runs))
+    tr = NCU_TRAFFIC.get(kern)
     traffic = tr["bytes"] if tr and tr.get("code_sha") == code_sha(src) else None
-    roof = {"kernel": kern, "bound": "hbm", "achieved": None if achieved is None else round(achieved, 1),
-            "peak": hbm, "peak_kind": peak_kind, "unit": "GB/s",
-            "frac": None if achieved is None else round(achieved / hbm, 4), "traffic": traffic,
-            "algorithmic_bytes_per_launch": dec_bytes if dominant == "decode" else cmp_bytes,
-            "shares": {k: round(v, 4) for k, v in shares.items()}}
+    roof = {"kernel": kern, "bound": "hbm", "achieved": round(achieved, 1), "peak": hbm, "peak_kind": peak_kind,
+            "unit": "GB/s", "frac": round(achieved / hbm, 4), "traffic": traffic,
+            "algorithmic_bytes_per_launch": round(per_launch), "avg_launch_us": round(avg_us, 3),
+            "shares": shares}
+    for r in runs:
+        per_budget[r.B].pop("decode_bytes")
 
     line = {"metric": METRIC, "value": round(value, 2), "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": f"{WORKLOAD}: Llama-3.1-8B attention geometry, 1 layer, batch 1, "
-                                   f"32 q heads / 8 kv heads, d=128, T=8192, budget 512, window 32, sink 1, "
-                                   f"mi on, 256 decode steps with append, evict every {EVICT_EVERY}",
-                       "global_batch": step.G.batch * world, "seq_len": step.T, "decode_steps": step.S,
-                       "parallelism": f"replicas x{world}", "accum": "f32", "l2": "flushed (256 MB write) "
-                       "before every timed step", "graphs": "one CUDA graph per part, replayed"},
-            "e2e": {"value": round(e2e_value, 2), "unit": "tokens/s", "h2d_bytes_per_step": int(h2d),
-                    "d2h_bytes_per_step": int(d2h), "ms_per_step": round(e2e_step, 4)},
-            "gpu_launches": step.launches_per_step * args.steps,
-            "parts_ms": {"compress": round(float(compress_ms.mean()), 4), "decode_256": round(float(decode_ms.mean()), 4),
-                         "evict_4": round(float(evict_ms.mean()), 4)},
-            "decode": {"avg_launch_us": round(dec_launch_ms * 1e3, 3), "gbs": round(dec_bytes / dec_launch_ms / 1e6, 1),
-                       "frac": round(dec_bytes / dec_launch_ms / 1e6 / hbm, 4)},
-            "compress": {"gbs": round(cmp_bytes / float(compress_ms.mean()) / 1e6, 1)},
-            "roofline": roof, "clocks": clk}
+            "config": dict(config_dict(stack.L), parallelism=f"replicas x{world}"),
+            "graphs": "one CUDA graph per part (compress of all layers; 64 decode steps x all layers)",
+            "e2e": e2e, "gpu_launches": sum(r.launches() for r in runs) * args.steps,
+            "per_budget": {str(k): v for k, v in per_budget.items()},
+            "roofline": roof, "clocks": clk, "setup_s": round(setup_s, 1),
+            "input_bytes": stack.nbytes()}
+    oracle_in = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        oracle_in = oracle_jobs_from_stack(stack, ORACLE_JOBS)
+    del runs, stack
+    torch.cuda.empty_cache()
     if rank == 0 and not args.no_extras:
+        line["t128k"] = leg_t128k(torch, mkv, inputs, dev, flush, hbm)
+        line["t8k"] = leg_t8k(torch, mkv, inputs, dev, flush, hbm)
         line["decode_sweep"] = decode_sweep(torch, mkv, dev, flush, hbm)
-        line["compress_long"] = compress_long(torch, mkv, inputs, dev, flush, hbm)
+        line["compress_adaptive"] = compress_adaptive(torch, mkv, inputs, dev, flush, hbm)
         line["continuous_eviction"] = continuous_eviction(torch, mkv, dev)
         line["layers_one_launch"] = layers_one_launch(torch, mkv, dev, flush, hbm)
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline()
+    if oracle_in is not None:
+        line["cpu_baseline"] = cpu_baseline(oracle_in, wl, stack_layers=line["config"]["layers"])
     if dist:
         dist.barrier()
         dist.destroy_process_group()
     if rank == 0:
         print(json.dumps(line), flush=True)
+
+
+def run_leg(torch, mkv, inputs, dev, flush, hbm, wl, budget, evict_every, layers=None, steps=None, timed=3):
+    """One multi-layer workload at one budget, timed as the headline is."""
+    stack = Stack(torch, inputs, wl, seed=7, dev=dev, layers=layers, steps=steps)
+    run = Run(torch, mkv, stack, budget, evict_every, dev)
+    stream = torch.cuda.Stream(dev)
+    run.capture(stream)
+    for _ in range(1):
+        replay([run], stream)
+    stream.synchronize()
+    run.check_errors(stream)
+    seg = time_steps(torch, [run], stream, flush, timed)
+    run.check_errors(stream)
+    res = summarise([run], seg, hbm)[budget]
+    step = float(seg.sum(axis=1).mean())
+    res.pop("decode_bytes")
+    out = {"layers": stack.L, "batch": stack.G.batch, "T": wl.T, "budget": budget, "window": wl.window,
+           "decode_steps": stack.S, "evict_every": evict_every, "ms_per_step": round(step, 3),
+           "tokens_per_s": round(stack.G.batch * stack.S / (step / 1e3), 1), "steps_timed": timed, **res,
+           "launches_per_step": run.launches()}
+    del run, stack
+    torch.cuda.empty_cache()
+    return out
+
+
+def leg_t128k(torch, mkv, inputs, dev, flush, hbm):
+    """Llama-3.1-8B geometry, 32 layers, batch 1, T=131072, budget 128,
+    window 64, mixture keys; 1024 decode steps with an evict-append on every
+    layer every 64 tokens (the cache grows from 128 to 192 rows and back)."""
+    wl = inputs.WORKLOADS["llama8b_t128k"]
+    return run_leg(torch, mkv, inputs, dev, flush, hbm, wl, wl.budget, wl.evict_every)
+
+
+def leg_t8k(torch, mkv, inputs, dev, flush, hbm):
+    """Llama-3.1-8B geometry, one layer, batch 1, T=8192, budget 512, window
+    32; 256 decode steps with an evict-append every 64 tokens."""
+    wl = inputs.WORKLOADS["llama8b_layer_t8k"]
+    return run_leg(torch, mkv, inputs, dev, flush, hbm, wl, wl.budget, 64, timed=10)
 
 
 def decode_sweep(torch, mkv, dev, flush, hbm):
@@ -481,7 +647,7 @@ def decode_sweep(torch, mkv, dev, flush, hbm):
             ws = mkv.alloc_workspace(mkv.mkv_decode_workspace_size(g, cap), dev)
             cell = {"batch": b, "budget": B}
             for corr in (1, 0):
-                p = mkv.mkv_decode_params(corr, 1, 1e-6)
+                p = mkv.mkv_decode_params(corr, 1, TAU)
                 with torch.cuda.stream(st):
                     mkv.mkv_decode_step(g, q, None, None, cache, mom, p, out, None, ws, st)
                     gr = torch.cuda.CUDAGraph()
@@ -542,10 +708,10 @@ def decode_layers(torch, mkv, dev, flush, hbm, b, B, gen, st):
         mkv.mkv_moments_pack_bf16(g, moms[l], C16[l])
     res = {}
     for corr in (1, 0, 2):
-        p = mkv.mkv_decode_params(min(corr, 1), 1, 1e-6)
+        p = mkv.mkv_decode_params(min(corr, 1), 1, TAU)
         ps = [p] * layers
         if corr == 2:
-            ps = [mkv.mkv_decode_params(1, 1, 1e-6, C16[l].data_ptr()) for l in range(layers)]
+            ps = [mkv.mkv_decode_params(1, 1, TAU, C16[l].data_ptr()) for l in range(layers)]
         with torch.cuda.stream(st):
             for l in range(layers):
                 mkv.mkv_decode_step(g, q, None, None, caches[l], moms[l], ps[l], out, None, ws, st)
@@ -594,7 +760,7 @@ def layers_one_launch(torch, mkv, dev, flush, hbm, layers=32, B=512):
     lens = torch.full((layers, H), B, dtype=torch.int32, device=dev)
     q = rnd(layers, H * G, D).bfloat16()
     out = torch.empty(layers, H * G, D, device=dev)
-    p = mkv.mkv_decode_params(1, 1, 1e-6)
+    p = mkv.mkv_decode_params(1, 1, TAU)
     st = torch.cuda.Stream(dev)
     gall, g1 = mkv.geom(layers, H, G, D), mkv.geom(1, H, G, D)
     ws_all = mkv.alloc_workspace(mkv.mkv_decode_workspace_size(gall, B), dev)
@@ -650,7 +816,7 @@ def continuous_eviction(torch, mkv, dev, steps=64):
         qs, kn, vn = rnd(steps, b, H * G, D).bfloat16(), rnd(steps, b, H, D).bfloat16(), rnd(steps, b, H, D).bfloat16()
         mom0 = (0.05 * rnd(b, H, D), 0.05 * rnd(b, H, D), 0.01 * rnd(b, H, D, D))
         out = torch.empty(b, H * G, D, device=dev)
-        p = mkv.mkv_decode_params(1, 1, 1e-6)
+        p = mkv.mkv_decode_params(1, 1, TAU)
         st = torch.cuda.Stream(dev)
         cell = {"batch": b, "budget": B}
         for mode in ("one_call", "two_calls"):
@@ -668,7 +834,7 @@ def continuous_eviction(torch, mkv, dev, steps=64):
                     if mode == "one_call":
                         mkv.mkv_decode_evict_step(g, qs[i], kn[i], vn[i], B, cache, mom, p, out, None, wsf, st)
                     else:
-                        mkv.mkv_evict_append(g, qs[i], kn[i], vn[i], B, cache, mom, 1e-6, wse, st)
+                        mkv.mkv_evict_append(g, qs[i], kn[i], vn[i], B, cache, mom, TAU, wse, st)
                         mkv.mkv_decode_step(g, qs[i], None, None, cache, mom, p, out, None, wsd, st)
             with torch.cuda.stream(st):
                 body()
@@ -695,25 +861,22 @@ def continuous_eviction(torch, mkv, dev, steps=64):
     return res
 
 
-def compress_long(torch, mkv, inputs, dev, flush, hbm):
-    """Compress throughput at 32K (Qwen3-4B geometry, batch 4, budget 1024) and 128K
-    (Llama-3.1-8B geometry, batch 1, budget 128, window 64) context, one layer;
-    ms_adaptive is the same compression with the budget shared by the KV heads
-    of each batch item."""
+def compress_adaptive(torch, mkv, inputs, dev, flush, hbm):
+    """One layer's compress at 32K (Qwen3-4B geometry, batch 4, budget 1024) and
+    128K (Llama-3.1-8B geometry, batch 1, budget 128, window 64) context, with
+    the budget per unit and (ms_adaptive) shared by the KV heads of each batch
+    item (Ada-KV allocation)."""
     res = {}
     st = torch.cuda.Stream(dev)
     for name in ("qwen4b_t32k", "llama8b_t128k"):
         wl = inputs.WORKLOADS[name]
         G = wl.geom
         g = mkv.geom(G.batch, G.n_kv_heads, G.group, G.head_dim)
-        gen = inputs.Generator(wl, seed=11)
-        K, V, Q = gen.prefill()
-        tb = inputs.to_bf16_tensor
-        K, V, Q = tb(K).to(dev), tb(V).to(dev), tb(Q).to(dev)
+        K, V, Q = inputs.TorchGenerator(wl, seed=11, device=dev).prefill()
         prot = 1 + wl.window
         for adaptive in (0, 1):
-            p = mkv.mkv_compress_params(wl.budget, wl.window, 1, 1, 1, 1, 1, 1e-6, adaptive)
-            cap = min(wl.T, G.n_kv_heads * (wl.budget - prot) + prot) if adaptive else wl.budget + EVICT_EVERY
+            p = mkv.mkv_compress_params(wl.budget, wl.window, 1, 1, 1, 1, 1, TAU, adaptive)
+            cap = min(wl.T, G.n_kv_heads * (wl.budget - prot) + prot) if adaptive else wl.budget + 64
             cache, mom = mkv.alloc_cache(g, cap, dev), mkv.alloc_moments(g, dev)
             ws = mkv.alloc_workspace(mkv.mkv_compress_workspace_size(g, wl.T, p), dev)
             times = []
@@ -745,80 +908,151 @@ def compress_long(torch, mkv, inputs, dev, flush, hbm):
     return res
 
 
+
 # --------------------------------------------------------------------------
 # the oracle on the host cores
 # --------------------------------------------------------------------------
-def oracle_sample(inputs, O, seed, unit):
-    """One KV-head unit of the bench step through the fp64 oracle; returns seconds (wall, cpu)."""
-    wl = inputs.WORKLOADS[WORKLOAD]
-    G = wl.geom
-    gen = inputs.Generator(wl, seed=seed)
-    K, V, Q = gen.prefill()
-    q, kn, vn = gen.decode(wl.decode_steps)
-    bi, h = divmod(unit, G.n_kv_heads)
-    t0, c0 = time.perf_counter(), resource.getrusage(resource.RUSAGE_SELF)
-    ref = O.compress(K[bi, h], V[bi, h], Q[bi, h], wl.budget, wl.window, wl.sink, True, 1, True, 1e-6)
-    Kr, Vr, m, pos = K[bi, h][ref.idx], V[bi, h][ref.idx], ref.moments, np.array(ref.idx)
-    for s in range(wl.decode_steps):
-        qh = q[s, bi, h * G.group:(h + 1) * G.group]
-        _, _, Kr, Vr = O.decode_step(qh, Kr, Vr, m, kn[s, bi, h], vn[s, bi, h], tau=1e-6)
-        pos = np.append(pos, wl.T + s)
-        if (s + 1) % EVICT_EVERY == 0:
-            ev = O.evict_append(qh, Kr, Vr, pos, m, wl.budget, 1e-6)
-            Kr, Vr, m, pos = ev.K, ev.V, ev.moments, ev.pos
-    t1, c1 = time.perf_counter(), resource.getrusage(resource.RUSAGE_SELF)
-    cpu = (c1.ru_utime - c0.ru_utime) + (c1.ru_stime - c0.ru_stime)
-    return t1 - t0, cpu
-
-
-def cpu_baseline():
+def oracle_job(job):
+    """One (layer, unit) of the headline workload at one budget through the
+    fp64 oracle: compress the prompt, then the decode steps with append.
+    Returns (wall s, CPU s) of this process."""
     import oracle as O
-    from paper_2606_01563_gb300 import inputs
-    wl = inputs.WORKLOADS[WORKLOAD]
+    K, V, Q, q, kn, vn, budget, window, sink, T = job
+    w0, c0 = time.perf_counter(), time.process_time()
+    ref = O.compress(K, V, Q, budget, window, sink, True, 1, True, TAU)
+    Kr, Vr, m = K[ref.idx], V[ref.idx], ref.moments
+    for s in range(q.shape[0]):
+        _, _, Kr, Vr = O.decode_step(q[s], Kr, Vr, m, kn[s], vn[s], tau=TAU)
+    return time.perf_counter() - w0, time.process_time() - c0
+
+
+def _to_np(t):
+    return t.float().cpu().numpy()
+
+
+def oracle_jobs_from_stack(stack, n, step=0):
+    """n oracle jobs on the bytes the GPU consumed: units and budgets rotate
+    with `step`; layers run from 0."""
+    G, wl = stack.G, stack.wl
+    units = G.batch * G.n_kv_heads
+    jobs = []
+    for j in range(n):
+        k = step * n + j
+        u = k % units
+        layer = (k // units) % stack.L
+        B = BUDGETS[k % len(BUDGETS)]
+        bi, h = divmod(u, G.n_kv_heads)
+        g = G.group
+        jobs.append((_to_np(stack.K[layer][bi, h]), _to_np(stack.V[layer][bi, h]), _to_np(stack.Q[layer][bi, h]),
+                     _to_np(stack.q[:, layer, bi, h * g:(h + 1) * g]), _to_np(stack.kn[:, layer, bi, h]),
+                     _to_np(stack.vn[:, layer, bi, h]), B, wl.window, wl.sink, wl.T))
+    return jobs
+
+
+def oracle_pool(n):
+    """A spawn process pool of n single-threaded workers (numpy's BLAS held to
+    one thread each, so that n jobs use n cores)."""
+    keys = ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS")
+    old = {k: os.environ.get(k) for k in keys}
+    for k in keys:
+        os.environ[k] = "1"
+    try:
+        pool = mp.get_context("spawn").Pool(processes=n)
+        pool.map(_noop, range(n))  # workers started and importing done before any timing
+    finally:
+        for k, v in old.items():
+            if v is None:
+                os.environ.pop(k, None)
+            else:
+                os.environ[k] = v
+    return pool
+
+
+def _noop(x):
+    import oracle  # noqa: F401
+    return x
+
+
+def oracle_step(pool, jobs):
+    """Runs the jobs on the pool; (wall s, CPU s summed over the workers)."""
+    t0 = time.perf_counter()
+    res = pool.map(oracle_job, jobs, chunksize=1)
+    return time.perf_counter() - t0, sum(c for _, c in res)
+
+
+def step_tokens_equiv(wl, layers, n_jobs):
+    """Tokens a sample of n_jobs (layer, unit, budget) jobs stands for: the
+    full step has layers x units jobs per budget, each budget producing
+    batch x decode_steps tokens."""
     units = wl.geom.batch * wl.geom.n_kv_heads
-    wall, cpu = 0.0, 0.0
-    n = 0
-    t_start = time.perf_counter()
-    while n < units and (n < 2 or time.perf_counter() - t_start < 20.0):
-        w, c = oracle_sample(inputs, O, 0, n)
-        wall += w
-        cpu += c
-        n += 1
-    est = wall / n * units
-    tokens = wl.geom.batch * wl.decode_steps
-    return {"value": round(tokens / est, 3), "unit": "tokens/s", "cores": max(1, round(cpu / wall)),
-            "kind": "oracle", "sample": f"{n} of {units} KV-head units of the full step (compress T=8192, "
-            f"256 decode steps, 4 evictions), fp64 numpy, scaled by {units}/{n}; "
-            f"{wall:.1f} s wall, host nproc={os.cpu_count()}; cores = CPU time / wall time (numpy's BLAS threads)"}
+    return n_jobs * wl.geom.batch * wl.decode_steps / (layers * units)
+
+
+def cpu_baseline(jobs, wl, stack_layers):
+    n = min(len(jobs), os.cpu_count() or 1)
+    pool = oracle_pool(n)
+    try:
+        wall, cpu = oracle_step(pool, jobs)
+    finally:
+        pool.close()
+        pool.join()
+    tok = step_tokens_equiv(wl, stack_layers, len(jobs))
+    return {"value": round(tok / wall, 3), "unit": "tokens/s", "cores": n, "kind": "oracle",
+            "sample": f"{len(jobs)} (layer, unit, budget) jobs of the headline step on the bytes the GPU consumed "
+                      f"(each: compress T={wl.T}, then {wl.decode_steps} decode steps), fp64 numpy, one job per "
+                      f"worker process, {n} workers; stands for {tok:.1f} of the step's "
+                      f"{len(BUDGETS) * wl.geom.batch * wl.decode_steps} tokens; {wall:.1f} s wall, "
+                      f"{cpu:.1f} s CPU, host nproc={os.cpu_count()}"}
 
 
 def run_reference(args):
     rank, world, _ = dist_env()
     if rank != 0:
         return
-    import oracle as O
+    import torch
     from paper_2606_01563_gb300 import inputs
-    wl = inputs.WORKLOADS[WORKLOAD]
-    units = wl.geom.batch * wl.geom.n_kv_heads
-    for k in range(args.warmup):
-        oracle_sample(inputs, O, 0, k % units)
-    wall, cpu = 0.0, 0.0
-    for k in range(args.steps):
-        w, c = oracle_sample(inputs, O, 0, k % units)
-        wall += w
-        cpu += c
-    est_ms = wall / args.steps * units * 1e3
-    tokens = wl.geom.batch * wl.decode_steps
-    value = tokens / (est_ms / 1e3)
-    cores = max(1, round(cpu / wall))
-    sample = (f"each step: one of {units} KV-head units of the full step (compress T=8192, 256 decode steps, "
-              f"4 evictions) through the fp64 oracle, scaled by {units}; cores = CPU time / wall time")
+    wl = inputs.WORKLOADS[HEADLINE]
+    layers = wl.n_layers if args.layers is None else args.layers
+    n = min(ORACLE_JOBS, os.cpu_count() or 1)
+    pool = oracle_pool(n)
+    # one layer's inputs drawn on the host with the headline's recipe (the
+    # values differ from the GPU arm's device draw, the distribution does not);
+    # the sample's units and budgets rotate from step to step
+    gen = inputs.TorchGenerator(wl, seed=0, layer=0, device="cpu")
+    K, V, Q = gen.prefill()
+    q, kn, vn = gen.decode(wl.decode_steps)
+
+    class One:  # a one-layer stack view for oracle_jobs_from_stack
+        pass
+    st = One()
+    st.G, st.wl, st.L = wl.geom, wl, 1
+    st.K, st.V, st.Q = [K], [V], [Q]
+    st.q, st.kn, st.vn = q[:, None], kn[:, None], vn[:, None]
+    try:
+        for k in range(args.warmup):
+            oracle_step(pool, oracle_jobs_from_stack(st, n, step=k))
+        walls, cpus = [], []
+        for k in range(args.steps):
+            jobs = oracle_jobs_from_stack(st, n, step=args.warmup + k)
+            w, c = oracle_step(pool, jobs)
+            walls.append(w)
+            cpus.append(c)
+    finally:
+        pool.close()
+        pool.join()
+    ms_per_step = float(np.mean(walls)) * 1e3
+    tok = step_tokens_equiv(wl, layers, n)
+    value = tok / (ms_per_step / 1e3)
+    sample = (f"each step: {n} (layer, unit, budget) jobs of the headline step (each: compress T={wl.T}, then "
+              f"{wl.decode_steps} decode steps) through the fp64 oracle, one job per worker process, {n} workers, "
+              f"standing for {tok:.2f} of the step's {len(BUDGETS) * wl.geom.batch * wl.decode_steps} tokens; "
+              f"inputs drawn on the host with the same recipe; {float(np.sum(cpus)) / float(np.sum(walls)):.1f} "
+              f"cores busy on average; host nproc={os.cpu_count()}")
     print(json.dumps({"impl": "reference", "metric": METRIC, "value": round(value, 3), "unit": "tokens/s",
-                      "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(est_ms, 2),
+                      "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 2),
                       "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-                      "data": "synthetic", "config": {"workload": WORKLOAD, "seq_len": wl.T,
-                                                      "decode_steps": wl.decode_steps},
-                      "cpu_baseline": {"value": round(value, 3), "unit": "tokens/s", "cores": cores,
+                      "data": "synthetic", "config": dict(config_dict(layers), parallelism=f"replicas x{world}"),
+                      "cpu_baseline": {"value": round(value, 3), "unit": "tokens/s", "cores": n,
                                        "kind": "oracle", "sample": sample},
                       "e2e": {"value": round(value, 3), "unit": "tokens/s", "h2d_bytes_per_step": 0,
                               "d2h_bytes_per_step": 0}}), flush=True)

@@ -211,6 +211,35 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
     mbar_fence_init();
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
+    // Before the dependency wait: this split's retained rows and moment rows
+    // were written by earlier calls, not by the kernel this launch waits on
+    // (that one produces this step's query and token), so they are pulled
+    // into L2 now, while that kernel still runs.  A prefetch is only a hint
+    // and L2 is the point of coherence: a length read that races with a
+    // writer only moves the prefetched range; the loads after the wait read
+    // the current values.
+    int lp = __ldcg(a.len + u);
+    lp = lp < 0 ? 0 : (lp > a.cap ? a.cap : lp);
+    const int tp = (lp + kTT - 1) / kTT;
+    const int per = (tp + a.S - 1) / a.S;
+    const int pb = min(lp, s * per * kTT), pe = min(lp, pb + per * kTT);
+    if (pe > pb) {
+      const size_t off = ((size_t)u * a.cap + pb) * D * 2;
+      const uint32_t bytes = static_cast<uint32_t>((pe - pb) * D * 2);
+      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(static_cast<const uint8_t*>(a.K) + off),
+                   "r"(bytes) : "memory");
+      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(static_cast<const uint8_t*>(a.V) + off),
+                   "r"(bytes) : "memory");
+    }
+    if (a.correction && a.n != nullptr && a.order == 1) {
+      const int rp = (D + a.S - 1) / a.S, c0 = s * rp, c1 = min(D, c0 + rp);
+      if (c1 > c0) {
+        const void* base = C16 ? static_cast<const void*>(a.C16 + ((size_t)u * D + c0) * D)
+                               : static_cast<const void*>(a.C + ((size_t)u * D + c0) * D);
+        asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base),
+                     "r"((uint32_t)((c1 - c0) * D * (C16 ? 2 : 4))) : "memory");
+      }
+    }
   }
   grid_dependency_wait();
   grid_launch_dependents();
@@ -299,9 +328,9 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
     mkp[kk][0] = v ? __ldg(reinterpret_cast<const float2*>(a.mu_k + (size_t)u * D + kk * 16 + 2 * t)) : make_float2(0.f, 0.f);
     mkp[kk][1] = v ? __ldg(reinterpret_cast<const float2*>(a.mu_k + (size_t)u * D + kk * 16 + 8 + 2 * t)) : make_float2(0.f, 0.f);
   }
-  const int n_e = corr ? a.n[u] : 0;
-  const int seen0 = (CL && s == 0 && tid == 0 && a.k_new != nullptr) ? a.seen[u] : 0;  // for the bookkeeping
-  int len0 = a.len[u];
+  const int n_e = corr ? __ldcg(a.n + u) : 0;
+  const int seen0 = (CL && s == 0 && tid == 0 && a.k_new != nullptr) ? __ldcg(a.seen + u) : 0;  // bookkeeping
+  int len0 = __ldcg(a.len + u);
   if (len0 < 0 || len0 > a.cap) {  // corrupt cache state: never read past the slab
     if (tid == 0 && s == 0) record_error(a.ws, MKV_ERR_CAPACITY, u);
     len0 = len0 < 0 ? 0 : a.cap;
@@ -368,22 +397,31 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
       const float y = (fabsf(f[i].y * nf) < tau) ? 0.f : f[i].y;
       split_bf16x2(x, y, hi[i], lo[i]);
     }
-    mma_bf16_full(d, hi[0], hi[1], hi[2], hi[3], qa[kk][0], qa[kk][1]);
-    mma_bf16_full(d, lo[0], lo[1], lo[2], lo[3], qa[kk][0], qa[kk][1]);  // zero for a bf16 copy of C
+    // the q fragment of k-step kk, selected without indexing the register
+    // array by a runtime value (which would move qa to local memory)
+    uint32_t b0 = 0u, b1 = 0u;
+#pragma unroll
+    for (int k = 0; k < D / 16; ++k) {
+      b0 = (k == kk) ? qa[k][0] : b0;
+      b1 = (k == kk) ? qa[k][1] : b1;
+    }
+    mma_bf16_full(d, hi[0], hi[1], hi[2], hi[3], b0, b1);
+    mma_bf16_full(d, lo[0], lo[1], lo[2], lo[3], b0, b1);  // zero for a bf16 copy of C
   };
   if (use_m && do_c && split_k) {
     const int g = lane >> 2, t = lane & 3;
 #pragma unroll
     for (int j = 0; j < 2; ++j) {
-      if (j >= n_mt) break;  // warp-uniform
-      float d[4] = {0.f, 0.f, 0.f, 0.f};
+      if (j < n_mt) {  // warp-uniform; no early exit, so cfr stays in registers
+        float d[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-      for (int kp = 0; kp < KPW; ++kp) mma_c(d, cfr[j][kp], warp * KPW + kp);
-      float(*fp)[8] = sFp[j][warp];
-      fp[g][2 * t] = d[0];
-      fp[g][2 * t + 1] = d[1];
-      fp[g + 8][2 * t] = d[2];
-      fp[g + 8][2 * t + 1] = d[3];
+        for (int kp = 0; kp < KPW; ++kp) mma_c(d, cfr[j][kp], warp * KPW + kp);
+        float(*fp)[8] = sFp[j][warp];
+        fp[g][2 * t] = d[0];
+        fp[g][2 * t + 1] = d[1];
+        fp[g + 8][2 * t] = d[2];
+        fp[g + 8][2 * t + 1] = d[3];
+      }
     }
   }
   __syncthreads();
@@ -811,12 +849,69 @@ cudaError_t launch_dg(const DecodeArgs& a, cudaStream_t stream) {
 
 }  // namespace
 
-// Split count per unit.  All CTAs of a launch should be resident at once (two
-// per SM at d = 128, three at d = 64, limited by shared memory): a second wave
-// costs a whole CTA latency.  Within that, one tile per CTA up to ten tiles,
-// at least two tiles per CTA beyond, and past 12 splits the merge costs more
-// than the extra parallelism saves (measured on the Llama-3.1-8B decode
-// geometry over batch 1..64 and caches of 256..4096 rows).
+// Split count per unit.  One CTA per SM at most, so that the next launch's
+// CTAs (programmatic dependents) can be resident beside this launch's and
+// prefetch their rows while it runs; and units * S clusters of S CTAs must
+// fit the GPU twice over (clusters are placed within one GPC, so the query
+// asks the driver rather than dividing SM counts).  Within that, one tile per
+// CTA up to ten tiles, at least two tiles per CTA beyond, and at most 12
+// splits, past which the merge costs more than the extra parallelism saves.
+namespace {
+template <int D, int G>
+int active_clusters(int S) {
+  constexpr int kMaxDev = 64;
+  static std::mutex mu;
+  static int known[kMaxDev][kMaxClusterSplits + 1] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) return 0;
+  std::lock_guard<std::mutex> lock(mu);
+  if (known[dev][S] == 0) {
+    const size_t ring = (size_t)2 * kStages * kTT * D * 2 + 1024;
+    const size_t smem = ring + ((size_t)S * G * (D + 4) + (size_t)G * D + 2 * (size_t)S * G) * sizeof(float);
+    int n = 0;
+    cudaError_t e = cudaFuncSetAttribute(decode_kernel<D, G, true, false>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    if (e == cudaSuccess && S > 8)
+      e = cudaFuncSetAttribute(decode_kernel<D, G, true, false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e == cudaSuccess) {
+      cudaLaunchConfig_t cfg{};
+      cfg.gridDim = dim3(S, 1, 1);
+      cfg.blockDim = dim3(kThreads, 1, 1);
+      cfg.dynamicSmemBytes = smem;
+      cudaLaunchAttribute at[1];
+      at[0].id = cudaLaunchAttributeClusterDimension;
+      at[0].val.clusterDim.x = S;
+      at[0].val.clusterDim.y = 1;
+      at[0].val.clusterDim.z = 1;
+      cfg.attrs = at;
+      cfg.numAttrs = 1;
+      e = cudaOccupancyMaxActiveClusters(&n, decode_kernel<D, G, true, false>, &cfg);
+    }
+    if (e != cudaSuccess) {
+      (void)cudaGetLastError();
+      n = 0;
+    }
+    known[dev][S] = n > 0 ? n : -1;
+  }
+  return known[dev][S];
+}
+
+int active_clusters_dg(int head_dim, int group, int S) {
+#define MKV_AC_CASE(D, G) \
+  if (head_dim == D && group == G) return active_clusters<D, G>(S);
+  MKV_AC_CASE(128, 1)
+  MKV_AC_CASE(128, 2)
+  MKV_AC_CASE(128, 4)
+  MKV_AC_CASE(128, 8)
+  MKV_AC_CASE(64, 1)
+  MKV_AC_CASE(64, 2)
+  MKV_AC_CASE(64, 4)
+  MKV_AC_CASE(64, 8)
+#undef MKV_AC_CASE
+  return 0;
+}
+}  // namespace
+
 namespace {
 __global__ void __launch_bounds__(256) pack_bf16_kernel(const float* __restrict__ C, __nv_bfloat16* __restrict__ C16,
                                                         size_t n4) {
@@ -841,11 +936,9 @@ cudaError_t launch_pack_bf16(const float* C, __nv_bfloat16* C16, size_t n, cudaS
 int decode_splits(const mkv_geom& g, int32_t capacity, int num_sms) {
   const long units = (long)g.batch * g.n_kv_heads;
   const long tiles = ((long)capacity + 1 + kTT - 1) / kTT;
-  const long slots = (g.head_dim == 64 ? 3L : 2L) * num_sms;
-  long S = slots / units;
   const long by_tiles = tiles <= 10 ? tiles : std::max(10L, (tiles + 1) / 2);
-  S = std::min(S, by_tiles);
-  S = std::min(S, 12L);
+  long S = std::min<long>(std::min(by_tiles, 12L), num_sms / units);
+  while (S > 1 && 2 * units > active_clusters_dg(g.head_dim, g.group, static_cast<int>(S))) --S;
   if (S < 1) S = 1;
   return static_cast<int>(S);
 }

@@ -19,6 +19,8 @@ Recipes (one numpy PCG64 stream per seed):
                    rows ("outlier"), a fixed random 5% of rows ("logscale"),
                    or the rows of 2 fixed components ("mixture").
 Everything is rounded to bf16 (round to nearest even) before use.
+Generator draws with numpy on the host; TorchGenerator draws the same
+recipes with torch on a device, for the multi-layer workloads.
 """
 from __future__ import annotations
 
@@ -186,6 +188,111 @@ class Generator:
         b, H = g.batch, g.n_kv_heads
         return (bf16_round(q).reshape(steps, b, H * g.group, d),
                 bf16_round(kn).reshape(steps, b, H, d), bf16_round(vn).reshape(steps, b, H, d))
+
+
+class TorchGenerator:
+    """The same recipes as Generator, drawn with torch's generator on any
+    device.  A multi-layer workload's prompts (about 19 GB at 36 layers of
+    batch 4 x 32K) take minutes to draw with numpy on the host; on the GPU
+    they take seconds.  The random streams differ from Generator's (and
+    between devices), the distributions are the same.  Tensors come back as
+    bf16 on `device`.  One generator per (seed, layer)."""
+
+    def __init__(self, wl: Workload, seed: int = 0, layer: int = 0, device="cpu"):
+        self.wl = wl
+        self.dev = torch.device(device)
+        self.gen = torch.Generator(device=self.dev)
+        self.gen.manual_seed(int(seed) * 1000003 + int(layer) * 7919 + 17)
+        g = wl.geom
+        self.units = g.batch * g.n_kv_heads
+        d = g.head_dim
+        if wl.key_dist == "outlier":
+            scale = torch.ones(self.units, d, device=self.dev)
+            idx = torch.argsort(self._rand(self.units, d), dim=1)[:, :4]
+            self.scale = scale.scatter_(1, idx, 6.0)
+        elif wl.key_dist == "logscale":
+            lo, hi = np.log(0.5), np.log(4.0)
+            self.scale = torch.exp(lo + (hi - lo) * self._rand(self.units, d))
+        elif wl.key_dist == "mixture":
+            A = self._randn(self.units, d, 16).double()
+            Qm, _ = torch.linalg.qr(A.cpu())                   # orthonormal columns, [units, d, 16]
+            self.means = (Qm.transpose(1, 2) * np.sqrt(d)).float().to(self.dev)   # [units, 16, d]
+            self.hot_comps = torch.argsort(self._rand(self.units, 16), dim=1)[:, :2]
+        else:
+            raise ValueError(wl.key_dist)
+        self.scale = getattr(self, "scale", None)
+        self._K = None
+        self._pool = None
+
+    def _rand(self, *shape):
+        return torch.rand(*shape, generator=self.gen, device=self.dev)
+
+    def _randn(self, *shape):
+        return torch.randn(*shape, generator=self.gen, device=self.dev)
+
+    def _randint(self, hi, shape):
+        return torch.randint(0, hi, shape, generator=self.gen, device=self.dev)
+
+    def _keys(self, n):
+        d = self.wl.geom.head_dim
+        if self.scale is not None:
+            return self._randn(self.units, n, d) * self.scale[:, None, :], None
+        comp = self._randint(16, (self.units, n))
+        u = torch.arange(self.units, device=self.dev)[:, None]
+        return self.means[u, comp] + 0.5 * self._randn(self.units, n, d), comp
+
+    def _pools(self, comp, T):
+        """Per unit, the candidate rows of the query recipe (None: all rows)."""
+        if self.wl.key_dist == "outlier":
+            return None
+        if self.wl.key_dist == "logscale":
+            n = max(3, T // 20)
+            return [torch.sort(torch.argsort(self._rand(T), dim=0)[:n]).values for _ in range(self.units)]
+        return [torch.nonzero(torch.isin(comp[u], self.hot_comps[u]))[:, 0] for u in range(self.units)]
+
+    def _queries(self, n):
+        """n queries per unit from its pool over the prefill keys: [units, n, d] float32."""
+        K, pool = self._K, self._pool
+        d = K.shape[-1]
+        out = torch.empty(self.units, n, d, device=self.dev)
+        for u in range(self.units):
+            if pool is None:
+                rows = self._randint(K.shape[1], (n, 3))
+            else:
+                rows = pool[u][self._randint(len(pool[u]), (n, 3))]
+            v = K[u][rows].float().sum(dim=1)
+            v = np.sqrt(d) * v / torch.linalg.norm(v, dim=1, keepdim=True)
+            out[u] = v + 0.3 * self._randn(n, d)
+        return out
+
+    def prefill(self, T=None):
+        """K, V [b, Hkv, T, d] and Q_obs [b, Hkv, g, w, d], bf16 on the device."""
+        wl, g = self.wl, self.wl.geom
+        T = wl.T if T is None else T
+        d, w = g.head_dim, wl.window
+        K, comp = self._keys(T)
+        K = K.to(torch.bfloat16)
+        V = self._randn(self.units, T, d).to(torch.bfloat16)
+        self._K = K
+        self._pool = self._pools(comp, T)
+        Q = self._queries(g.group * w).to(torch.bfloat16)
+        shp = (g.batch, g.n_kv_heads)
+        return K.view(*shp, T, d), V.view(*shp, T, d), Q.view(*shp, g.group, w, d)
+
+    def decode(self, steps=None):
+        """q [steps, b, Hq, d], k_new, v_new [steps, b, Hkv, d], bf16 on the device;
+        queries follow the window-query recipe over the prefill keys."""
+        wl, g = self.wl, self.wl.geom
+        steps = wl.decode_steps if steps is None else steps
+        d = g.head_dim
+        q = self._queries(steps * g.group).view(self.units, steps, g.group, d)
+        kn, _ = self._keys(steps)
+        vn = self._randn(self.units, steps, d)
+        b, H = g.batch, g.n_kv_heads
+        q = q.permute(1, 0, 2, 3).reshape(steps, b, H * g.group, d)
+        kn = kn.permute(1, 0, 2).reshape(steps, b, H, d)
+        vn = vn.permute(1, 0, 2).reshape(steps, b, H, d)
+        return q.to(torch.bfloat16), kn.to(torch.bfloat16), vn.to(torch.bfloat16)
 
 
 def random_moments(rng, batch, n_kv_heads, d, n=4096, scale=0.05):

@@ -49,14 +49,15 @@ def test_kernel_sources_exist():
         assert len(bench.code_sha(paths)) == 64
 
 
-def _fake_step(B, S, T=8192):
-    """A bench.Step holding only what the byte accounting reads (no GPU state)."""
+def _fake_run(name, B, S, L=1, evict_every=0):
+    """A bench.Run holding only what the byte accounting reads (no GPU state)."""
     from paper_2606_01563_gb300.inputs import WORKLOADS
-    st = bench.Step.__new__(bench.Step)
-    st.wl = WORKLOADS[bench.WORKLOAD]
-    st.G = st.wl.geom
-    st.B, st.S, st.T = B, S, T
-    return st
+    st = type("FakeStack", (), {})()
+    st.wl = WORKLOADS[name]
+    st.G, st.S, st.L = st.wl.geom, S, L
+    r = bench.Run.__new__(bench.Run)
+    r.st, r.G, r.B, r.ev_every = st, st.G, B, evict_every
+    return r
 
 
 def test_decode_bytes_per_launch():
@@ -67,15 +68,55 @@ def test_decode_bytes_per_launch():
     q, out = hq * d * 2, hq * d * 4
     assert retained + moments + q + out == 1605664  # 1.61 MB at budget 256
     new_row = units * d * 2 * 2                  # k_new, v_new read, and the row written
-    assert _fake_step(256, 1).decode_bytes_total() == 1605664 + 2 * new_row
-    # the bench step: 256 launches over 512..575 rows (an eviction back to 512 every 64)
-    assert _fake_step(512, 256).decode_bytes_total() / 256 == 2791456
+    assert _fake_run("llama8b_layer_t8k", 256, 1).decode_bytes() == 1605664 + 2 * new_row
+    # 256 launches over 512..575 rows (an eviction back to 512 every 64)
+    assert _fake_run("llama8b_layer_t8k", 512, 256, evict_every=64).decode_bytes() / 256 == 2791456
+    # the headline at budget 1024: 36 layers, 512 steps over 1024..1535 rows, batch 4 (32 units, 128 q heads)
+    r = _fake_run("qwen4b_t32k", 1024, 512, L=36)
+    units, hq = 32, 128
+    per_row = units * d * 4
+    fixed = units * (d * d * 4 + 2 * d * 4 + 4) + hq * d * (2 + 4) + 2 * units * d * 4
+    want = 36 * sum(fixed + (1024 + i) * per_row for i in range(512))
+    assert r.decode_bytes() == want
+    assert abs(want / (36 * 512) - 23.22e6) < 0.01e6
 
 
 def test_compress_bytes():
     units, d, T, B, g, w = 8, 128, 8192, 512, 4, 32
-    want = units * (2 * T * d * 2 + g * w * d * 2 + B * d * 2 * 2 + (d * d + 2 * d + 1) * 4)
-    assert _fake_step(B, 256, T).compress_bytes() == want == 36446240
+    want = units * (2 * T * d * 2 + g * w * d * 2 + B * (d * 2 * 2 + 4) + (d * d + 2 * d + 1) * 4)
+    assert _fake_run("llama8b_layer_t8k", B, 256).compress_bytes() == want == 36462624
+    # the headline layer at 32K, batch 4: 537 MB of K and V dominate
+    assert abs(_fake_run("qwen4b_t32k", 1024, 512).compress_bytes() - 557.0e6) < 0.1e6
+
+
+def test_oracle_sample_stands_for_its_share_of_the_step():
+    from paper_2606_01563_gb300.inputs import WORKLOADS
+    wl = WORKLOADS["qwen4b_t32k"]
+    # 16 of the step's 36 x 32 (layer, unit) jobs per budget; each budget makes 4 x 512 tokens
+    assert bench.step_tokens_equiv(wl, 36, 16) == 16 * 4 * 512 / (36 * 32)
+    cfg = bench.config_dict(36)
+    assert cfg["layers"] == 36 and cfg["budgets"] == [128, 256, 1024] and cfg["seq_len"] == 32768
+    assert cfg["decode_steps"] == 512 and cfg["global_batch"] == 4
+
+
+def test_oracle_jobs_rotate_units_and_budgets():
+    import torch
+    from paper_2606_01563_gb300.inputs import WORKLOADS, TorchGenerator
+    wl = WORKLOADS["tiny_d64_t1k"]
+    gen = TorchGenerator(wl, seed=0)
+    K, V, Q = gen.prefill()
+    q, kn, vn = gen.decode(3)
+    st = type("S", (), {})()
+    st.G, st.wl, st.L = wl.geom, wl, 1
+    st.K, st.V, st.Q, st.q, st.kn, st.vn = [K], [V], [Q], q[:, None], kn[:, None], vn[:, None]
+    jobs = bench.oracle_jobs_from_stack(st, 4)
+    assert [j[6] for j in jobs] == [128, 256, 1024, 128]
+    # unit 1 = (batch 0, KV head 1): its rows and its group's query heads 2..3
+    assert torch.equal(torch.from_numpy(jobs[1][0]), K[0, 1].float())
+    assert torch.equal(torch.from_numpy(jobs[1][3]), q[:, 0, 2:4].float())
+    assert jobs[0][3].shape == (3, 2, 64) and jobs[0][4].shape == (3, 64)
+    nxt = bench.oracle_jobs_from_stack(st, 4, step=1)
+    assert [j[6] for j in nxt] == [256, 1024, 128, 256]
 
 
 class _FakeProc:

@@ -116,3 +116,67 @@ def test_bench_workloads_match_their_configurations():
     g = wl.geom
     assert (g.batch, g.n_kv_heads, g.group, g.head_dim) == (1, 2, 2, 64)
     assert (wl.T, wl.budget, wl.window, wl.decode_steps, wl.key_dist) == (1024, 128, 16, 16, "outlier")
+
+
+# ---------------------------------------------------------------------------
+# TorchGenerator: the same recipes drawn with torch (here on the CPU; the
+# bench draws the multi-layer prompts on the GPU with the same code)
+# ---------------------------------------------------------------------------
+def _torch_unit(wl, seed=0, layer=0, T=None, steps=4):
+    import torch  # noqa: F401
+    from paper_2606_01563_gb300.inputs import TorchGenerator
+    gen = TorchGenerator(wl, seed=seed, layer=layer)
+    K, V, Q = gen.prefill(T)
+    q, kn, vn = gen.decode(steps)
+    return gen, [x.float().numpy() for x in (K, V, Q, q, kn, vn)]
+
+
+def test_torch_generator_shapes_bf16_determinism():
+    wl = WORKLOADS["tiny_d64_t1k"]
+    _, A = _torch_unit(wl, seed=0, layer=1)
+    _, B = _torch_unit(wl, seed=0, layer=1)
+    _, C = _torch_unit(wl, seed=0, layer=2)
+    G = wl.geom
+    shapes = [(1, 2, 1024, 64), (1, 2, 1024, 64), (1, 2, 2, 16, 64), (4, 1, 4, 64), (4, 1, 2, 64), (4, 1, 2, 64)]
+    for x, y, z, shp in zip(A, B, C, shapes):
+        assert x.shape == shp and _is_bf16(x)
+        assert np.array_equal(x, y)
+        assert not np.array_equal(x, z)
+    assert G.n_q_heads == 4
+
+
+def test_torch_generator_logscale_recipe():
+    wl = Workload("l", Geometry(1, 2, 4, 128), 8192, 512, 32, "logscale")
+    gen, (K, V, Q, q, kn, vn) = _torch_unit(wl, seed=5, steps=64)
+    d = 128
+    for u in range(2):
+        scale = gen.scale[u].numpy()
+        assert scale.min() >= 0.5 and scale.max() <= 4.0
+        assert abs(np.log(scale).mean() - 0.5 * (np.log(0.5) + np.log(4.0))) < 0.2
+        np.testing.assert_allclose(K[0, u].std(axis=0), scale, rtol=0.06)
+        assert abs(V[0, u].std() - 1.0) < 0.02
+        hot = gen._pool[u].numpy()
+        assert len(hot) == wl.T // 20 and len(np.unique(hot)) == len(hot)
+        for qq in (Q[0, u].reshape(-1, d), q[:, 0, 4 * u:4 * u + 4].reshape(-1, d)):
+            norms = np.linalg.norm(qq, axis=1)
+            assert abs(np.median(norms) / np.sqrt(d * (1 + 0.3 ** 2)) - 1) < 0.1
+            assert np.isin(_aim(qq, K[0, u]), hot).mean() > 0.9
+        np.testing.assert_allclose(kn[:, 0, u].std(axis=0).mean(), np.sqrt((scale ** 2).mean()), rtol=0.25)
+
+
+def test_torch_generator_mixture_recipe():
+    wl = Workload("m", Geometry(1, 2, 4, 128), 8192, 128, 64, "mixture")
+    gen, (K, V, Q, q, kn, vn) = _torch_unit(wl, seed=7)
+    d = 128
+    for u in range(2):
+        means = gen.means[u].double().numpy()
+        np.testing.assert_allclose(means @ means.T, d * np.eye(16), atol=1e-4)
+        hot_comps = gen.hot_comps[u].numpy()
+        assert len(set(hot_comps)) == 2
+        # every key is a component mean plus N(0, 0.5^2) noise: the nearest mean explains it
+        dist = ((K[0, u][:, None, :] - means[None].astype(np.float32)) ** 2).sum(-1)
+        comp = dist.argmin(1)
+        assert abs((K[0, u] - means[comp]).std() - 0.5) < 0.01
+        hot_rows = np.nonzero(np.isin(comp, hot_comps))[0]
+        assert np.array_equal(hot_rows, gen._pool[u].numpy())
+        assert np.isin(_aim(Q[0, u].reshape(-1, d), K[0, u]), hot_rows).mean() > 0.9
