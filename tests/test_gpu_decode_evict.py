@@ -1,6 +1,8 @@
 """One decoding step of Algorithm 1 (append, Phase 1 down to the budget,
-Phase 2) on the GPU against the fp64 oracle's evict_append followed by its
-decode_step, through the C ABI: the corrected output and its log-normaliser
+Phase 2) on the GPU against the fp64 oracle, through the C ABI: the oracle
+follows the kernel's evictions (each the argmin of Algorithm 1's scores under
+the state reached, or at a near tie one of the near-minimal rows), then
+decodes over the state reached; the corrected output and its log-normaliser
 (2e-3 of the output's max-abs), the surviving rows (exact), and the updated
 moments (1e-4 relative).  Covers the register eviction kernel and the
 larger-cache eviction kernels ahead of the decode kernel, steps with nothing
@@ -12,17 +14,11 @@ import torch
 import oracle as O
 from paper_2606_01563_gb300 import mkv
 from paper_2606_01563_gb300.inputs import bf16_round
-from gpu_util import GAP_EXACT, assert_moment_close, assert_output_close, bf16, f32, host, i32
+from gpu_util import assert_output_close, bf16, f32, host, i32
+from parity import check_evicted_unit
 from test_gpu_evict import setup
 
 pytestmark = pytest.mark.gpu
-
-
-def oracle_step(st, bi, h, G, budget, tau, correction, order, K, V, pos, m, kn, vn, pos_new):
-    q = st["q"][bi, h * G:(h + 1) * G]
-    r = O.evict_append(q, K, V, pos, m, budget, tau, kn, vn, pos_new)
-    o, lse, _, _ = O.decode_step(q, r.K, r.V, r.moments, None, None, bool(correction), order, tau)
-    return r, o, lse
 
 
 def run_steps(st, b, H, G, D, budget, steps=1, correction=1, order=1, tau=1e-6, seed=0):
@@ -58,24 +54,19 @@ def run_steps(st, b, H, G, D, budget, steps=1, correction=1, order=1, tau=1e-6, 
                    len=host(cache.len), seen=host(cache.seen), n=host(mom.n), mu_k=host(mom.mu_k),
                    mu_v=host(mom.mu_v), C=host(mom.C))
         for (bi, h), s in ref.items():
-            r, o, l = oracle_step(st, bi, h, G, budget, tau, correction, order, s["K"], s["V"], s["pos"], s["m"],
-                                  st["kn"][bi, h], st["vn"][bi, h], seen0 + step)
-            if r.gaps:
-                assert min(r.gaps) > GAP_EXACT, "fixture has a near-tie; pick another seed"
-            n_r = len(r.pos)
-            assert got["len"][bi, h] == n_r and got["seen"][bi, h] == seen0 + step + 1
-            np.testing.assert_array_equal(got["pos"][bi, h, :n_r], r.pos)
-            if n_r:
-                np.testing.assert_array_equal(got["K"][bi, h, :n_r], r.K)
-                np.testing.assert_array_equal(got["V"][bi, h, :n_r], r.V)
-            assert got["n"][bi, h] == r.moments.n
-            if r.moments.n:
-                assert_moment_close(got["mu_k"][bi, h], r.moments.mu_k, "mu_k")
-                assert_moment_close(got["mu_v"][bi, h], r.moments.mu_v, "mu_v")
-                assert_moment_close(got["C"][bi, h], r.moments.C, "C")
+            q = st["q"][bi, h * G:(h + 1) * G]
+            K = np.vstack([s["K"], st["kn"][bi, h][None]])
+            V = np.vstack([s["V"], st["vn"][bi, h][None]])
+            pos = np.append(s["pos"], seen0 + step)
+            # Phase 1: the oracle follows the kernel's evictions (exact argmin,
+            # or one of the near-minimal rows at a near tie)
+            f = check_evicted_unit(got, bi, h, q, K, V, pos, s["m"], budget, tau)
+            assert got["seen"][bi, h] == seen0 + step + 1
+            # Phase 2 over the state reached
+            o, l, _, _ = O.decode_step(q, f.K, f.V, f.moments, None, None, bool(correction), order, tau)
             assert_output_close(got["out"][bi, h * G:(h + 1) * G], o, f"out step {step} unit {(bi, h)}")
             np.testing.assert_allclose(got["lse"][bi, h * G:(h + 1) * G], l, rtol=1e-4, atol=1e-4)
-            s.update(K=r.K, V=r.V, pos=r.pos, m=r.moments)
+            s.update(K=f.K, V=f.V, pos=f.pos, m=f.moments)
     return got
 
 

@@ -24,10 +24,10 @@ import numpy as np
 import pytest
 import torch
 
-import oracle as O
 from paper_2606_01563_gb300 import mkv
 from paper_2606_01563_gb300.inputs import WORKLOADS, Generator
-from gpu_util import GAP_EXACT, assert_moment_close, bf16, host
+from gpu_util import bf16, host
+from parity import check_compress_item_adaptive, check_compress_unit
 
 pytestmark = pytest.mark.gpu
 
@@ -66,101 +66,14 @@ def _compress_gpu(wl, K, V, Q, adaptive):
     return out
 
 
-def _score2_under(K, V, s, R0):
-    """Oracle score2 (Eq. residual under the moments of all \\ R0, times s)
-    for a given stage-1 set R0."""
-    keep0 = np.zeros(K.shape[0], bool)
-    keep0[R0] = True
-    r = O.residual(K, V, O.moments_of(K[~keep0], V[~keep0]), TAU)
-    return s * np.sqrt((r * r).sum(axis=1))
-
-
-def _check_rows_and_moments(out, bi, h, K, V, R, m):
-    n_r = len(R)
-    np.testing.assert_array_equal(out["K"][bi, h, :n_r], K[R])
-    np.testing.assert_array_equal(out["V"][bi, h, :n_r], V[R])
-    assert out["n"][bi, h] == m.n
-    if m.n:
-        assert_moment_close(out["mu_k"][bi, h], m.mu_k, "mu_k")
-        assert_moment_close(out["mu_v"][bi, h], m.mu_v, "mu_v")
-        assert_moment_close(out["C"][bi, h], m.C, "C")
-    else:
-        assert not out["C"][bi, h].any()
-
-
-def _evicted_moments(K, V, R):
-    keep = np.zeros(K.shape[0], bool)
-    keep[R] = True
-    return O.moments_of(K[~keep], V[~keep])
-
-
 def check_unit(out, wl, bi, h, K, V, Q):
-    """One (batch, KV head) unit of a per-unit-budget compress."""
-    T, B = wl.T, wl.budget
-    ref = O.compress(K, V, Q, B, wl.window, wl.sink, bool(wl.keep_window), 1, True, TAU)
-    prot = O.protected_mask(T, wl.window, wl.sink, bool(wl.keep_window))
-    free = ~prot
-    k = B - int(prot.sum())
-    s_g, s2_g = out["s"][bi, h], out["s2"][bi, h]
-    np.testing.assert_allclose(s_g, ref.scores, rtol=2e-5, atol=2e-6 * ref.scores.max())
-    # stage 1: the kernel's choice is the exact top k of its own scores
-    R0 = out["i1"][bi, h]
-    np.testing.assert_array_equal(R0, O.select_topk(s_g, k, prot)[0])
-    if ref.gap1 > GAP_EXACT:
-        np.testing.assert_array_equal(R0, ref.idx_stage1)
-        score2 = ref.score2
-    else:
-        score2 = _score2_under(K, V, ref.scores, R0)
-    np.testing.assert_allclose(s2_g[free], score2[free], rtol=1e-4, atol=1e-5 * score2[free].max())
-    # stage 2 into the cache
-    assert out["len"][bi, h] == B and out["seen"][bi, h] == T
-    R = out["pos"][bi, h, :B]
-    np.testing.assert_array_equal(R, O.select_topk(s2_g, k, prot)[0])
-    if ref.gap1 > GAP_EXACT and ref.gap2 > GAP_EXACT:
-        np.testing.assert_array_equal(R, ref.idx)
-        m = ref.moments
-    else:
-        m = _evicted_moments(K, V, R)
-    _check_rows_and_moments(out, bi, h, K, V, R, m)
-    return ref.gap1 > GAP_EXACT and ref.gap2 > GAP_EXACT
+    return check_compress_unit(out, bi, h, K, V, Q, wl.T, wl.budget, wl.window, wl.sink, bool(wl.keep_window), 1, 1,
+                               TAU)
 
 
 def check_item_adaptive(out, wl, bi, K, V, Q):
-    """The KV heads of batch item bi, budget shared across them (K, V: [H, T, d])."""
-    T, B = wl.T, wl.budget
-    H = K.shape[0]
-    ref = O.compress_adaptive(K, V, Q, B, wl.window, wl.sink, bool(wl.keep_window), 1, True, TAU)
-    prot = np.stack([O.protected_mask(T, wl.window, wl.sink, bool(wl.keep_window))] * H)
-    k = H * B - int(prot.sum())
-    s_g, s2_g = out["s"][bi], out["s2"][bi]
-    for h in range(H):
-        np.testing.assert_allclose(s_g[h], ref.scores[h], rtol=2e-5, atol=2e-6 * ref.scores[h].max())
-
-    def flat(lists):
-        return np.concatenate([h * T + r for h, r in enumerate(lists)])
-
-    R0 = O.select_topk_joint(s_g, k, prot)[0]
-    np.testing.assert_array_equal(out["i1"][bi], flat(R0))
-    if ref.gap1 > GAP_EXACT:
-        np.testing.assert_array_equal(flat(R0), flat(ref.idx_stage1))
-        score2 = ref.score2
-    else:
-        score2 = np.stack([_score2_under(K[h], V[h], ref.scores[h], R0[h]) for h in range(H)])
-    for h in range(H):
-        free = ~prot[h]
-        np.testing.assert_allclose(s2_g[h][free], score2[h][free], rtol=1e-4,
-                                   atol=1e-5 * score2[h][free].max())
-    assert (out["seen"][bi] == T).all() and out["len"][bi].sum() == H * B
-    R = [out["pos"][bi, h, :out["len"][bi, h]] for h in range(H)]
-    want = O.select_topk_joint(s2_g, k, prot)[0]
-    np.testing.assert_array_equal(flat(R), flat(want))
-    exact = ref.gap1 > GAP_EXACT and ref.gap2 > GAP_EXACT
-    if exact:
-        np.testing.assert_array_equal(flat(R), flat(ref.idx))
-    for h in range(H):
-        m = ref.moments[h] if exact else _evicted_moments(K[h], V[h], R[h])
-        _check_rows_and_moments(out, bi, h, K[h], V[h], R[h], m)
-    return exact
+    return check_compress_item_adaptive(out, bi, K, V, Q, wl.T, wl.budget, wl.window, wl.sink,
+                                        bool(wl.keep_window), 1, 1, TAU)
 
 
 @pytest.fixture(scope="module")

@@ -60,3 +60,75 @@ def test_noalloc_rejects_oversized_geometry():
     with pytest.raises(mkv.MKVError) as e:
         mkv.mkv_decode_step_noalloc(g, out, None, None, cache, None, p, out, None)
     assert e.value.code == 7
+
+
+def _oracle_decode(q, K, V, lens, n, mu_k, mu_v, C, kn, vn, G, tau=1e-6):
+    import oracle as O
+    b, H = lens.shape
+    D = K.shape[-1]
+    out = np.zeros((b, H * G, D))
+    lse = np.zeros((b, H * G))
+    for bi in range(b):
+        for h in range(H):
+            L = lens[bi, h]
+            m = O.Moments(int(n[bi, h]), mu_k[bi, h], mu_v[bi, h], C[bi, h])
+            o, l, _, _ = O.decode_step(q[bi, h * G:(h + 1) * G], K[bi, h, :L], V[bi, h, :L], m, kn[bi, h], vn[bi, h],
+                                       True, 1, tau)
+            out[bi, h * G:(h + 1) * G] = o
+            lse[bi, h * G:(h + 1) * G] = l
+    return out, lse
+
+
+def _case(rng, b, H, G, D, cap):
+    """Host arrays of one decode call (cache, moments, query, new token)."""
+    K = bf16_round(rng.standard_normal((b, H, cap, D)))
+    V = bf16_round(rng.standard_normal((b, H, cap, D)))
+    lens = rng.integers(1, cap - 1, (b, H)).astype(np.int32)
+    n = rng.integers(0, 5000, (b, H)).astype(np.int32)
+    mu_k = (0.3 * rng.standard_normal((b, H, D))).astype(np.float32)
+    mu_v = (0.3 * rng.standard_normal((b, H, D))).astype(np.float32)
+    C = (0.05 * rng.standard_normal((b, H, D, D))).astype(np.float32)
+    q = bf16_round(2.0 * rng.standard_normal((b, H * G, D)))
+    kn = bf16_round(rng.standard_normal((b, H, D)))
+    vn = bf16_round(rng.standard_normal((b, H, D)))
+    return dict(K=K, V=V, lens=lens, n=n, mu_k=mu_k, mu_v=mu_v, C=C, q=q, kn=kn, vn=vn, cap=cap)
+
+
+def _noalloc_vs_oracle(c, b, H, G, D, what):
+    g = mkv.geom(b, H, G, D)
+    cache = mkv.Cache(bf16(c["K"]), bf16(c["V"]), i32(np.zeros((b, H, c["cap"]))), i32(c["lens"]), i32(c["lens"]))
+    mom = mkv.Moments(i32(c["n"]), f32(c["mu_k"]), f32(c["mu_v"]), f32(c["C"]))
+    out = torch.full((b, H * G, D), float("nan"), device="cuda")
+    lse = torch.full((b, H * G), float("nan"), device="cuda")
+    mkv.mkv_decode_step_noalloc(g, bf16(c["q"]), bf16(c["kn"]), bf16(c["vn"]), cache, mom,
+                                mkv.mkv_decode_params(1, 1, 1e-6), out, lse)
+    torch.cuda.synchronize()
+    want, want_lse = _oracle_decode(c["q"], c["K"], c["V"], c["lens"], c["n"], c["mu_k"], c["mu_v"], c["C"], c["kn"],
+                                    c["vn"], G)
+    assert_output_close(host(out), want, what)
+    np.testing.assert_allclose(host(lse), want_lse, rtol=1e-4, atol=1e-4)
+    np.testing.assert_array_equal(host(cache.len), c["lens"] + 1)
+
+
+def test_noalloc_against_oracle_alternating_geometries():
+    """A geometry with few units and one with many, alternating, each call
+    against the fp64 oracle: one call's partial records must not disturb the
+    next call's ticket counters or results (the counters sit in a region of
+    their own in the shared array)."""
+    rng = np.random.default_rng(78)
+    small = (1, 2, 2, 64, 200)
+    large = (8, 8, 4, 128, 700)   # 64 units, two splits each
+    for k, geom in enumerate([small, large, small, large]):
+        b, H, G, D, cap = geom
+        _noalloc_vs_oracle(_case(rng, b, H, G, D, cap), b, H, G, D, f"call {k} geometry {geom}")
+
+
+def test_noalloc_near_largest_accepted_geometry():
+    """1024 units (one split each: more units than SMs), about half of the
+    fixed scratch.  With at most one CTA per SM per launch the split count
+    times the units never exceeds the SM count, so the partial records stay
+    far below the array's size and every accepted geometry runs with its
+    full split count; the size check rejects by units (the f_hat rows)."""
+    rng = np.random.default_rng(79)
+    b, H, G, D, cap = 16, 64, 4, 64, 40
+    _noalloc_vs_oracle(_case(rng, b, H, G, D, cap), b, H, G, D, "1024 units")
