@@ -6,6 +6,7 @@
 #include "common.cuh"
 #include "kernels.h"
 #include "validate.h"
+#include "../../include/mkv_debug.h"
 
 using namespace mkv;
 
@@ -60,6 +61,7 @@ size_t mkv_decode_workspace_size(mkv_geom geom, int32_t capacity) {
 mkv_status mkv_decode_step(mkv_geom geom, const void* q, const void* k_new, const void* v_new,
                            const mkv_cache* cache, const mkv_moments* mom, const mkv_decode_params* p,
                            float* out, float* lse, void* workspace, size_t workspace_bytes, void* stream) {
+  NvtxRange nvtx("mkv_decode_step");
   const mkv_status chk = decode_args_status(geom, q, k_new, v_new, cache, mom, p, out);
   if (chk != MKV_OK) return chk;
   const int sms = num_sms_current();
@@ -92,6 +94,7 @@ mkv_status mkv_decode_step(mkv_geom geom, const void* q, const void* k_new, cons
 }
 
 mkv_status mkv_moments_pack_bf16(mkv_geom geom, const mkv_moments* mom, void* C16, void* stream) {
+  NvtxRange nvtx("mkv_moments_pack_bf16");
   if (!geom_ok(geom)) return geom_status(geom);
   if (!moments_ok(mom) || !C16 || !aligned(C16, 16)) return MKV_ERR_INVALID_ARG;
   const size_t n = (size_t)geom.batch * geom.n_kv_heads * geom.head_dim * geom.head_dim;
@@ -107,6 +110,7 @@ size_t mkv_evict_workspace_size(mkv_geom geom, int32_t capacity) {
 mkv_status mkv_evict_append(mkv_geom geom, const void* q, const void* k_new, const void* v_new, int32_t budget,
                             const mkv_cache* cache, const mkv_moments* mom, float tau, void* workspace,
                             size_t workspace_bytes, void* stream) {
+  NvtxRange nvtx("mkv_evict_append");
   if (!geom_ok(geom)) return geom_status(geom);
   if (!q || !cache_ok(cache) || !moments_ok(mom) || budget < 0 || !(tau >= 0.f)) return MKV_ERR_INVALID_ARG;
   if ((k_new == nullptr) != (v_new == nullptr)) return MKV_ERR_INVALID_ARG;
@@ -151,6 +155,7 @@ size_t mkv_decode_evict_workspace_size(mkv_geom geom, int32_t capacity) {
 mkv_status mkv_decode_evict_step(mkv_geom geom, const void* q, const void* k_new, const void* v_new, int32_t budget,
                                  const mkv_cache* cache, const mkv_moments* mom, const mkv_decode_params* p,
                                  float* out, float* lse, void* workspace, size_t workspace_bytes, void* stream) {
+  NvtxRange nvtx("mkv_decode_evict_step");
   if (!geom_ok(geom)) return geom_status(geom);
   if (!q || !k_new || !v_new || !out || !p || !cache_ok(cache) || !moments_ok(mom) || budget < 0)
     return MKV_ERR_INVALID_ARG;
@@ -250,6 +255,7 @@ size_t mkv_compress_workspace_size(mkv_geom geom, int32_t T, const mkv_compress_
 mkv_status mkv_compress(mkv_geom geom, int32_t T, const void* K, const void* V, const void* Q_obs,
                         const mkv_compress_params* p, const mkv_cache* out_cache, const mkv_moments* out_mom,
                         const mkv_compress_diag* diag, void* workspace, size_t workspace_bytes, void* stream) {
+  NvtxRange nvtx("mkv_compress");
   mkv_status st = compress_params_ok(geom, T, p);
   if (st != MKV_OK) return st;
   if (!K || !V || !Q_obs || !cache_ok(out_cache) || !moments_ok(out_mom)) return MKV_ERR_INVALID_ARG;
@@ -282,6 +288,14 @@ mkv_status mkv_compress(mkv_geom geom, int32_t T, const void* K, const void* V, 
   a.n_kv = geom.n_kv_heads;
   return cuda_status(launch_compress(a, geom, workspace_bytes, sms, static_cast<cudaStream_t>(stream)));
 }
+
+// ------------------------------------------------------------- test hooks
+int64_t mkv_debug_set_poll_limit(int64_t polls) {
+  const uint32_t v = polls < 0 ? kMaxPolls : (polls > (int64_t)kMaxPolls ? kMaxPolls : static_cast<uint32_t>(polls));
+  return static_cast<int64_t>(g_poll_limit.exchange(v));
+}
+
+int32_t mkv_debug_force_ticket_merge(int32_t on) { return g_force_ticket_merge.exchange(on != 0 ? 1 : 0); }
 
 // ------------------------------------------------------------------ errors
 mkv_status mkv_get_device_error(void* workspace, void* stream, int32_t* info) {

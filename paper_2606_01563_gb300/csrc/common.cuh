@@ -11,6 +11,7 @@
 #include <cudaTypedefs.h>
 #include <stdint.h>
 
+#include <atomic>
 #include <mutex>
 
 #include "../../include/mkv.h"
@@ -24,6 +25,16 @@ constexpr float kLn2 = 0.6931471805599453f;
 // poll is a try_wait that may itself suspend for a while, so this is well
 // over a second -- far beyond any legitimate copy latency.
 constexpr uint32_t kMaxPolls = 1u << 22;
+
+// Poll limit of the pipeline waits (tile copies, MMA commits), passed to the
+// kernels in their arguments.  Normally kMaxPolls; mkv_debug_set_poll_limit
+// lowers it so that a test can make those waits run out.  The waits that
+// drain a CTA's copies in flight before it exits always use kMaxPolls.
+inline std::atomic<uint32_t> g_poll_limit{kMaxPolls};
+inline uint32_t pipeline_poll_limit() { return g_poll_limit.load(std::memory_order_relaxed); }
+// Test switch: the decode merges through global partial records (the variant
+// that runs when a cluster of the split count cannot be co-scheduled).
+inline std::atomic<int> g_force_ticket_merge{0};
 
 struct ErrorWord {
   uint32_t code;
@@ -73,9 +84,9 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
-// Bounded wait on one phase; returns false if it gave up.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
-  for (uint32_t i = 0; i < kMaxPolls; ++i) {
+// Bounded wait on one phase (at most `polls` polls); returns false if it gave up.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint32_t polls = kMaxPolls) {
+  for (uint32_t i = 0; i < polls; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
   }
   return false;

@@ -163,15 +163,43 @@ __device__ __forceinline__ bool is_protected(int t, int T, int W, int sink, int 
 }
 
 __device__ __forceinline__ void epi_sync() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+// whether v holds in all 128 threads of the first epilogue group (barrier 1)
+__device__ __forceinline__ bool epi_all(bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\tsetp.ne.u32 p, %1, 0;\n\tbar.red.and.pred q, 1, 128, p;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"((uint32_t)v)
+      : "memory");
+  return r != 0;
+}
 
-// Pipeline wait that gives up after the bounded poll count: records the
-// timeout once and raises the CTA's abort flag so that no other role waits on.
-__device__ __forceinline__ bool pwait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, void* ws, int u) {
+// Pipeline wait that gives up after `polls` polls: records the timeout once
+// and raises the CTA's abort flag so that no other role waits on.
+__device__ __forceinline__ bool pwait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, void* ws, int u,
+                                      uint32_t polls) {
   if (*abort_flag) return false;
-  if (mbar_wait(bar, parity)) return true;
+  if (mbar_wait(bar, parity, polls)) return true;
   *abort_flag = 1;
   record_error(ws, MKV_ERR_TIMEOUT, u);
   return false;
+}
+
+// After an abort, before a CTA frees its tensor memory and exits: wait (with
+// the full poll limit) for the last tile copy issued into each of the kS
+// stages, for the window-query copy if one was issued, and for the MMA
+// thread's final commit (every MMA it issued has completed, so none still
+// reads shared memory or writes TMEM).  `issued` tiles went out in order,
+// tile i into stage i % kS.
+__device__ __forceinline__ void drain_after_abort(uint64_t* full, int kS, int issued, uint64_t* qfull,
+                                                  uint64_t* mma_done) {
+  for (int st = 0; st < kS; ++st) {
+    const int last = issued - 1 - ((issued - 1 - st) % kS + kS) % kS;  // largest i < issued with i % kS == st
+    if (last >= 0 && last % kS == st) (void)mbar_wait(&full[st], (last / kS) & 1);
+  }
+  if (qfull != nullptr) (void)mbar_wait(qfull, 0);
+  (void)mbar_wait(mma_done, 0);
 }
 
 struct TcArgs {
@@ -191,6 +219,7 @@ struct TcArgs {
   float* diag;
   const float* m0;
   void* ws;
+  uint32_t polls;  // poll limit of the pipeline waits
 };
 
 // --------------------------------------------------------------- stats_tc
@@ -213,7 +242,7 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
   uint8_t* sOnes = sQ + (LOGITS ? 2 * 2 * kBoxBytes : 0);  // [2 boxes][16 rows][128 B] of bf16 1.0
   __shared__ __align__(8) uint64_t full[kS], empty[kS], lfull, lempty, qfull, sdone;
   __shared__ uint32_t tmem_base;
-  __shared__ int abort_flag;
+  __shared__ int abort_flag, s_issued;
   __shared__ float sum_k[kDP], sum_v[kDP];
   __shared__ float s_m1[2][128], s_l1[2][128];  // the second epilogue group's row stats
 
@@ -249,6 +278,7 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
     mbar_init(&qfull, 1);
     mbar_init(&sdone, 1);
     abort_flag = 0;
+    s_issued = 0;
     mbar_fence_init();
   }
   if (warp == 1) tmem_alloc(&tmem_base, kTmemCols);
@@ -280,12 +310,13 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
             tma_prefetch_3d(&tmK, bx * 64, t_begin + (i + kPF) * kTok, u);
             tma_prefetch_3d(&tmV, bx * 64, t_begin + (i + kPF) * kTok, u);
           }
-        if (j >= 1 && !pwait(&empty[s], (j - 1) & 1, abrt, p.ws, u)) break;
+        if (j >= 1 && !pwait(&empty[s], (j - 1) & 1, abrt, p.ws, u, p.polls)) break;
         mbar_arrive_expect_tx(&full[s], 2u * kTileBytes);
         for (int bx = 0; bx < 2; ++bx) {
           tma_load_3d(sK + s * kTileBytes + bx * kBoxBytes, &tmK, bx * 64, t_begin + i * kTok, u, &full[s]);
           tma_load_3d(sV + s * kTileBytes + bx * kBoxBytes, &tmV, bx * 64, t_begin + i * kTok, u, &full[s]);
         }
+        s_issued = i + 1;
       }
     }
   } else if (warp == 1) {
@@ -294,14 +325,14 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
       const uint32_t idS = idesc_bf16(128, 128, 1, 1);  // V^T K: both MN-major (reduction over tokens)
       const uint32_t id1 = idesc_bf16(128, 16, 1, 0);   // X^T 1: X MN-major, ones K-major
       const uint32_t aQ = smem_addr(sQ), a1 = smem_addr(sOnes);
-      const bool ok = !LOGITS || pwait(&qfull, 0, abrt, p.ws, u);
+      const bool ok = !LOGITS || pwait(&qfull, 0, abrt, p.ws, u, p.polls);
       for (int i = 0; ok && i < n_tiles; ++i) {
         const int s = i % kS, j = i / kS;
-        if (!pwait(&full[s], j & 1, abrt, p.ws, u)) break;
+        if (!pwait(&full[s], j & 1, abrt, p.ws, u, p.polls)) break;
         tc_fence_after();
         const uint32_t aK = smem_addr(sK + s * kTileBytes), aV = smem_addr(sV + s * kTileBytes);
         if (LOGITS) {
-          if (i >= 1 && !pwait(&lempty, (i - 1) & 1, abrt, p.ws, u)) break;
+          if (i >= 1 && !pwait(&lempty, (i - 1) & 1, abrt, p.ws, u, p.polls)) break;
           tc_fence_after();
           for (int rb = 0; rb < RWb; ++rb)
             for (int kk = 0; kk < 8; ++kk) {
@@ -339,11 +370,15 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
     }
     const int t_safe = p.causal ? p.T - p.W : 0x7fffffff;  // tokens every window row sees
     for (int i = 0; LOGITS && i < n_tiles; ++i) {
-      if (!pwait(&lfull, i & 1, abrt, p.ws, u)) break;
+      if (!pwait(&lfull, i & 1, abrt, p.ws, u, p.polls)) break;
       tc_fence_after();
       const int tt0 = t_begin + i * kTok;
       const bool fast = tt0 + kTok <= t_end && tt0 + kTok - 1 <= t_safe;  // no masking in this tile
-      for (int rb = 0; rb < RWb; ++rb) {
+      // rb runs over a constant range (guarded by RWb), so that m, l and
+      // tmax_vis stay in registers
+#pragma unroll
+      for (int rb = 0; rb < 2; ++rb) {
+        if (rb >= RWb) break;
         for (int c0 = grp * 64; c0 < grp * 64 + 64; c0 += 32) {
           float x[32];
           tmem_ld32(tm + lane_base + rb * 128 + c0, x);
@@ -381,13 +416,18 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
     }
     if (LOGITS) {  // merge the two groups' (max, sum) of each row
       if (grp == 1)
-        for (int rb = 0; rb < RWb; ++rb) {
-          s_m1[rb][qd * 32 + lane] = m[rb];
-          s_l1[rb][qd * 32 + lane] = l[rb];
+#pragma unroll
+        for (int rb = 0; rb < 2; ++rb) {
+          if (rb < RWb) {
+            s_m1[rb][qd * 32 + lane] = m[rb];
+            s_l1[rb][qd * 32 + lane] = l[rb];
+          }
         }
       asm volatile("bar.sync 2, 256;" ::: "memory");
       if (grp == 0)
-        for (int rb = 0; rb < RWb; ++rb) {
+#pragma unroll
+        for (int rb = 0; rb < 2; ++rb) {
+          if (rb >= RWb) break;
           const int r = rb * 128 + qd * 32 + lane;
           const float m1 = s_m1[rb][qd * 32 + lane], l1 = s_l1[rb][qd * 32 + lane];
           const float M = fmaxf(m[rb], m1);
@@ -404,7 +444,12 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
         }
     }
     if (grp == 0) {
-    const bool got = pwait(&sdone, 0, abrt, p.ws, u);
+    // uniform over the group: after an abort the MMAs may still write TMEM,
+    // so it is not read and the chunk's record is left empty
+    const bool got = epi_all(pwait(&sdone, 0, abrt, p.ws, u, p.polls));
+    float* rec = p.mrec + ((size_t)u * p.n_chunks + chunk) * rec_floats(p.D);
+    const float nc = got ? static_cast<float>(max(0, t_end - t_begin)) : 0.f;
+    if (got) {
     tc_fence_after();
     {
       float x[32];
@@ -413,9 +458,7 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
       sum_v[qd * 32 + lane] = x[16];
     }
     epi_sync();
-    const float nc = static_cast<float>(max(0, t_end - t_begin));
     const float inv_nc = nc > 0.f ? 1.f / nc : 0.f;
-    float* rec = p.mrec + ((size_t)u * p.n_chunks + chunk) * rec_floats(p.D);
     const int a = qd * 32 + lane;  // value dim = TMEM lane
     // centred co-moment rows staged 32 columns at a time through the (now
     // free) K stage, so that the record is written in coalesced rows
@@ -437,11 +480,18 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
       rec[4 + a] = nc > 0.f ? sum_k[a] / nc : 0.f;
       rec[4 + p.D + a] = nc > 0.f ? sum_v[a] / nc : 0.f;
     }
-    if (et == 0) rec[0] = got ? nc : 0.f;
+    } else if (et < 4 + 2 * p.D) {
+      rec[et] = 0.f;  // an empty record: n = 0, zero means
+    }
+    if (et == 0) rec[0] = nc;
     }
   }
   tc_fence_before();
   __syncthreads();
+  if (abort_flag) {  // uniform: every role has left its loop
+    if (tid == 0) drain_after_abort(full, kS, s_issued, LOGITS ? &qfull : nullptr, &sdone);
+    __syncthreads();
+  }
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tm, kTmemCols);
@@ -456,9 +506,9 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
   uint8_t* sK = sm;                    // [kS][128 x 128]
   uint8_t* sQ = sm + kS * kTileBytes;  // [2 boxes][RWb*128][128 B]
-  __shared__ __align__(8) uint64_t full[kS], empty[kS], lfull[2], lempty[2], qfull;
+  __shared__ __align__(8) uint64_t full[kS], empty[kS], lfull[2], lempty[2], qfull, mma_done;
   __shared__ uint32_t tmem_base;
-  __shared__ int abort_flag;
+  __shared__ int abort_flag, s_issued;
   __shared__ __align__(16) float s_b[256];  // log2(1 / l_r) - m_r (-inf for padding rows)
   __shared__ int s_wi[256];                   // window index of row r (r mod W)
 
@@ -480,7 +530,9 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
       mbar_init(&lempty[i], 4);
     }
     mbar_init(&qfull, 1);
+    mbar_init(&mma_done, 1);
     abort_flag = 0;
+    s_issued = 0;
     mbar_fence_init();
   }
   if (warp == 1) tmem_alloc(&tmem_base, 512);
@@ -499,21 +551,22 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
         const int s = i % kS, j = i / kS;
         if (kPF > 0 && i + kS + kPF < n_tiles)
           for (int bx = 0; bx < 2; ++bx) tma_prefetch_3d(&tmK, bx * 64, t_begin + (i + kS + kPF) * kTok, u);
-        if (j >= 1 && !pwait(&empty[s], (j - 1) & 1, abrt, p.ws, u)) break;
+        if (j >= 1 && !pwait(&empty[s], (j - 1) & 1, abrt, p.ws, u, p.polls)) break;
         mbar_arrive_expect_tx(&full[s], kTileBytes);
         for (int bx = 0; bx < 2; ++bx)
           tma_load_3d(sK + s * kTileBytes + bx * kBoxBytes, &tmK, bx * 64, t_begin + i * kTok, u, &full[s]);
+        s_issued = i + 1;
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {
       const uint32_t id = idesc_bf16(128, RWp, 0, 0);  // tokens x window rows, both K-major
       const uint32_t aQ = smem_addr(sQ);
-      const bool ok = pwait(&qfull, 0, abrt, p.ws, u);
+      const bool ok = pwait(&qfull, 0, abrt, p.ws, u, p.polls);
       for (int i = 0; ok && i < n_tiles; ++i) {
         const int s = i % kS, j = i / kS, b = i & 1;
-        if (!pwait(&full[s], j & 1, abrt, p.ws, u)) break;
-        if (i >= 2 && !pwait(&lempty[b], ((i >> 1) - 1) & 1, abrt, p.ws, u)) break;
+        if (!pwait(&full[s], j & 1, abrt, p.ws, u, p.polls)) break;
+        if (i >= 2 && !pwait(&lempty[b], ((i >> 1) - 1) & 1, abrt, p.ws, u, p.polls)) break;
         tc_fence_after();
         const uint32_t aK = smem_addr(sK + s * kTileBytes);
         for (int kk = 0; kk < 8; ++kk) {
@@ -524,6 +577,7 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
         umma_commit(&lfull[b]);
         umma_commit(&empty[s]);
       }
+      umma_commit(&mma_done);  // every MMA issued has completed
     }
   } else {
     // two epilogue groups (warps 2..5 and 6..9) take alternate tiles; group g
@@ -549,7 +603,7 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
     const int t_safe = p.causal ? p.T - p.W : 0x7fffffff;  // tokens every window row sees
     for (int i = grp; i < n_tiles; i += 2) {
       const int b = i & 1;
-      if (!pwait(&lfull[b], (i >> 1) & 1, abrt, p.ws, u)) break;
+      if (!pwait(&lfull[b], (i >> 1) & 1, abrt, p.ws, u, p.polls)) break;
       tc_fence_after();
       const int t = t_begin + i * kTok + qd * 32 + lane;  // token of this thread (TMEM lane)
       const bool fast = t <= t_safe;  // every window row sees this token
@@ -584,6 +638,9 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
   }
   tc_fence_before();
   __syncthreads();
+  // the MMA thread's final commit, and after an abort the copies in flight
+  if (tid == 0) drain_after_abort(full, kS, abort_flag ? s_issued : 0, abort_flag ? &qfull : nullptr, &mma_done);
+  __syncthreads();
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tm, 512);
@@ -599,9 +656,9 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
   uint8_t* sK = sm;                        // [kS][128 x 128]
   uint8_t* sV = sm + kS * kTileBytes;      // [kS][128 x 128]
   uint8_t* sC = sm + 2 * kS * kTileBytes;  // [3 parts][128 x 128]: C0' = hi + mid + lo
-  __shared__ __align__(8) uint64_t full[kS], empty[kS], yfull[2], yempty[2];
+  __shared__ __align__(8) uint64_t full[kS], empty[kS], yfull[2], yempty[2], mma_done;
   __shared__ uint32_t tmem_base;
-  __shared__ int abort_flag;
+  __shared__ int abort_flag, s_issued;
   __shared__ float s_mv[kDP];
 
   const int chunk = blockIdx.x, u = blockIdx.y;
@@ -622,6 +679,7 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
       mbar_init(&yfull[i], 1);
       mbar_init(&yempty[i], 4);
     }
+    mbar_init(&mma_done, 1);
     abort_flag = 0;
     mbar_fence_init();
     // the first stages' copies go out while C0' is being prepared
@@ -637,6 +695,7 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
         tma_load_3d(sV + i * kTileBytes + bx * kBoxBytes, &tmV, bx * 64, t_begin + i * kTok, u, &full[i]);
       }
     }
+    s_issued = min(kS, n_tiles);
   }
   if (warp == 1) tmem_alloc(&tmem_base, 256);
   if (warp >= 2 && warp < 6) {
@@ -683,12 +742,13 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
             tma_prefetch_3d(&tmK, bx * 64, t_begin + (i + kPF) * kTok, u);
             tma_prefetch_3d(&tmV, bx * 64, t_begin + (i + kPF) * kTok, u);
           }
-        if (!pwait(&empty[s], (j - 1) & 1, abrt, p.ws, u)) break;
+        if (!pwait(&empty[s], (j - 1) & 1, abrt, p.ws, u, p.polls)) break;
         mbar_arrive_expect_tx(&full[s], 2u * kTileBytes);
         for (int bx = 0; bx < 2; ++bx) {
           tma_load_3d(sK + s * kTileBytes + bx * kBoxBytes, &tmK, bx * 64, t_begin + i * kTok, u, &full[s]);
           tma_load_3d(sV + s * kTileBytes + bx * kBoxBytes, &tmV, bx * 64, t_begin + i * kTok, u, &full[s]);
         }
+        s_issued = i + 1;
       }
     }
   } else if (warp == 1) {
@@ -697,8 +757,8 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
       const uint32_t aC = smem_addr(sC);
       for (int i = 0; i < n_tiles; ++i) {
         const int s = i % kS, j = i / kS, b = i & 1;
-        if (!pwait(&full[s], j & 1, abrt, p.ws, u)) break;
-        if (i >= 2 && !pwait(&yempty[b], ((i >> 1) - 1) & 1, abrt, p.ws, u)) break;
+        if (!pwait(&full[s], j & 1, abrt, p.ws, u, p.polls)) break;
+        if (i >= 2 && !pwait(&yempty[b], ((i >> 1) - 1) & 1, abrt, p.ws, u, p.polls)) break;
         tc_fence_after();
         const uint32_t aK = smem_addr(sK + s * kTileBytes);
         for (int part = 0; part < 3; ++part)
@@ -711,6 +771,7 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
         umma_commit(&yfull[b]);
         umma_commit(&empty[s]);
       }
+      umma_commit(&mma_done);  // every MMA issued has completed
     }
   } else {
     // two epilogue groups (warps 2..5 and 6..9) take alternate tiles; group g
@@ -720,8 +781,8 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
     const int row = qd * 32 + lane;  // token within the tile = TMEM lane
     for (int i = grp; i < n_tiles; i += 2) {
       const int s = i % kS, j = i / kS, b = i & 1;
-      if (!pwait(&yfull[b], (i >> 1) & 1, abrt, p.ws, u)) break;
-      if (!pwait(&full[s], j & 1, abrt, p.ws, u)) break;
+      if (!pwait(&yfull[b], (i >> 1) & 1, abrt, p.ws, u, p.polls)) break;
+      if (!pwait(&full[s], j & 1, abrt, p.ws, u, p.polls)) break;
       tc_fence_after();
       const uint8_t* tv = sV + s * kTileBytes;
       float ss = 0.f;
@@ -760,6 +821,9 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
     }
   }
   tc_fence_before();
+  __syncthreads();
+  // the MMA thread's final commit, and after an abort the copies in flight
+  if (tid == 0) drain_after_abort(full, kS, abort_flag ? s_issued : 0, nullptr, &mma_done);
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
@@ -864,7 +928,8 @@ __global__ void __cluster_dims__(kSelCL, 1, 1) __launch_bounds__(kSelThreads, 2)
   const int k = hs * (a.B - protected_count(T, W, a.sink, a.keep_window));
 
   // The CTA's keys are cached in shared memory when they fit (protected
-  // positions hold key 0, which no score maps to: scores are >= 0); larger
+  // positions hold key 0; every other position's key is at least 1, whatever
+  // the bits of its score, so at most k of them are ever selected); larger
   // ranges are read from global memory on every pass.
   extern __shared__ uint32_t ks[];
   const int nk = r1 - r0;
@@ -872,7 +937,7 @@ __global__ void __cluster_dims__(kSelCL, 1, 1) __launch_bounds__(kSelThreads, 2)
   auto key_of = [&](int f) -> uint32_t {
     int h;
     const int t = pos_of(f, h);
-    return is_protected(t, T, W, a.sink, a.keep_window) ? 0u : float_key(sc[(size_t)h * T + t]);
+    return is_protected(t, T, W, a.sink, a.keep_window) ? 0u : max(1u, float_key(sc[(size_t)h * T + t]));
   };
   auto key_at = [&](int f) -> uint32_t {  // 0 for protected positions
     return cached ? ks[f - r0] : key_of(f);
@@ -1315,6 +1380,7 @@ cudaError_t run(const CompressArgs& a, const mkv_geom& g, int num_sms, cudaStrea
   tp.qscale = rsqrtf(static_cast<float>(D)) * kLog2e;
   tp.tau = a.tau;
   tp.ws = a.ws;
+  tp.polls = pipeline_poll_limit();
   const dim3 cg(L.n_chunks, U);
 
   if (!keep_all || a.diag_scores != nullptr) {

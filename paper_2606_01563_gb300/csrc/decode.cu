@@ -485,7 +485,7 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
   for (; it < n_tiles; ++it) {
     const int stg = it % kStages;
     const int rows = min(kTT, n_cached - it * kTT);
-    const bool got = mbar_wait(&bars[stg], (it / kStages) & 1);
+    const bool got = mbar_wait(&bars[stg], (it / kStages) & 1, a.polls);
     if (!__syncthreads_and(got)) {
       ok = false;
       break;
@@ -795,7 +795,9 @@ bool cluster_fits(int S, size_t smem) {
 }
 
 template <int D, int G, bool C16>
-cudaError_t launch_dgc(const DecodeArgs& a, cudaStream_t stream) {
+cudaError_t launch_dgc(const DecodeArgs& args, cudaStream_t stream) {
+  DecodeArgs a = args;
+  a.polls = pipeline_poll_limit();
   const size_t ring = (size_t)2 * kStages * kTT * D * 2 + 1024;  // + alignment slack
   const size_t rcv = ((size_t)a.S * G * (D + 4) + (size_t)G * D + 2 * (size_t)a.S * G) * sizeof(float);
   const bool cl = a.S <= kMaxClusterSplits;
@@ -812,7 +814,7 @@ cudaError_t launch_dgc(const DecodeArgs& a, cudaStream_t stream) {
                              static_cast<int>(smem));
   }
   if (e != cudaSuccess) return e;
-  const bool use_cl = cl && cluster_fits<D, G, C16>(a.S, smem);
+  const bool use_cl = cl && cluster_fits<D, G, C16>(a.S, smem) && g_force_ticket_merge.load() == 0;
   // the cache slabs of all units as one [units * cap][D] matrix
   const uint64_t rows = (uint64_t)a.batch * a.n_kv * a.cap;
   CUtensorMap tmK, tmV;

@@ -38,6 +38,7 @@ struct DecodeArgs {
   int32_t batch;
   int32_t n_kv;
   int32_t S;
+  uint32_t polls;  // poll limit of the tile waits (the drain after a timeout uses kMaxPolls)
 };
 
 constexpr int kDecodeTile = 64;  // tokens per pipeline stage

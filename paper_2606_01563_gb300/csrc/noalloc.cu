@@ -89,6 +89,7 @@ extern "C" MKV_API mkv_status mkv_decode_step_noalloc(mkv_geom geom, const void*
                                                       const void* v_new, const mkv_cache* cache,
                                                       const mkv_moments* mom, const mkv_decode_params* p,
                                                       float* out, float* lse, void* stream) {
+  NvtxRange nvtx("mkv_decode_step_noalloc");
   const mkv_status chk = decode_args_status(geom, q, k_new, v_new, cache, mom, p, out);
   if (chk != MKV_OK) return chk;
   // The smallest split count needs one partial record per query head: reject

@@ -53,6 +53,8 @@ EXPORTS = ("mkv_status_str", "mkv_version", "mkv_compress_workspace_size", "mkv_
            "mkv_decode_workspace_size", "mkv_decode_step", "mkv_evict_workspace_size",
            "mkv_evict_append", "mkv_get_device_error", "mkv_decode_step_noalloc", "mkv_moments_pack_bf16",
            "mkv_decode_evict_workspace_size", "mkv_decode_evict_step")
+# test hooks declared in include/mkv_debug.h
+DEBUG_EXPORTS = ("mkv_debug_set_poll_limit", "mkv_debug_force_ticket_merge")
 
 
 class MKVError(RuntimeError):
@@ -104,6 +106,10 @@ def lib():
                                             c_vp, c_vp, c_vp, ctypes.c_size_t, c_vp]
         L.mkv_moments_pack_bf16.restype = c_i32
         L.mkv_moments_pack_bf16.argtypes = [mkv_geom, ctypes.POINTER(mkv_moments), c_vp, c_vp]
+        L.mkv_debug_set_poll_limit.restype = ctypes.c_int64
+        L.mkv_debug_set_poll_limit.argtypes = [ctypes.c_int64]
+        L.mkv_debug_force_ticket_merge.restype = c_i32
+        L.mkv_debug_force_ticket_merge.argtypes = [c_i32]
         L.mkv_get_device_error.restype = c_i32
         L.mkv_get_device_error.argtypes = [c_vp, c_vp, ctypes.POINTER(c_i32)]
         _lib = L
@@ -260,6 +266,17 @@ def mkv_moments_pack_bf16(g, mom: Moments, C16, stream=None):
     """C16 (bf16 [b, h_kv, d, d]) = bf16(mom.C): the 16-bit copy mkv_decode_params.C16 points at."""
     m = mom.c()
     _check(lib().mkv_moments_pack_bf16(g, ctypes.byref(m), _ptr(C16), _stream(stream)), "mkv_moments_pack_bf16")
+
+
+def mkv_debug_set_poll_limit(polls):
+    """Test hook (include/mkv_debug.h): poll limit of the kernels' pipeline
+    waits; negative restores the default.  Returns the previous limit."""
+    return lib().mkv_debug_set_poll_limit(int(polls))
+
+
+def mkv_debug_force_ticket_merge(on):
+    """Test hook (include/mkv_debug.h): decode merges through global partials."""
+    return lib().mkv_debug_force_ticket_merge(1 if on else 0)
 
 
 def mkv_get_device_error(ws, stream=None):

@@ -20,8 +20,8 @@ def L():
     return mkv.lib()
 
 
-def declared_functions():
-    src = open(os.path.join(ROOT, "include", "mkv.h")).read()
+def declared_functions(header="mkv.h"):
+    src = open(os.path.join(ROOT, "include", header)).read()
     return sorted(set(re.findall(r"MKV_API\s+[\w\s\*]+?\b(mkv_\w+)\s*\(", src)))
 
 
@@ -31,6 +31,20 @@ def test_every_declared_symbol_is_exported(L):
     assert set(names) == set(mkv.EXPORTS)
     for n in names:
         assert hasattr(L, n), n
+    debug = declared_functions("mkv_debug.h")
+    assert set(debug) == set(mkv.DEBUG_EXPORTS) and len(debug) == 2
+    for n in debug:
+        assert hasattr(L, n), n
+
+
+def test_debug_hooks_round_trip(L):
+    """The test hooks only set process-wide values read at the next launch."""
+    default = mkv.mkv_debug_set_poll_limit(5)
+    assert default == 1 << 22
+    assert mkv.mkv_debug_set_poll_limit(-1) == 5
+    assert mkv.mkv_debug_set_poll_limit(-1) == default
+    assert mkv.mkv_debug_force_ticket_merge(1) == 0
+    assert mkv.mkv_debug_force_ticket_merge(0) == 1
 
 
 def test_version_and_status_strings(L):

@@ -132,3 +132,21 @@ def test_noalloc_near_largest_accepted_geometry():
     rng = np.random.default_rng(79)
     b, H, G, D, cap = 16, 64, 4, 64, 40
     _noalloc_vs_oracle(_case(rng, b, H, G, D, cap), b, H, G, D, "1024 units")
+
+
+def test_noalloc_ticket_merge_alternating_geometries():
+    """The merge through the array's partial records and ticket counters (the
+    variant for clusters that cannot be co-scheduled, forced by a test hook),
+    alternating a geometry with few units and one with many: the counters a
+    call leaves at zero must still be zero for the next call, whatever the
+    previous call's partial records overwrote."""
+    rng = np.random.default_rng(80)
+    small = (1, 2, 2, 64, 200)
+    large = (8, 8, 4, 128, 700)
+    prev = mkv.mkv_debug_force_ticket_merge(1)
+    try:
+        for k, geom in enumerate([large, small, large, small, large]):
+            b, H, G, D, cap = geom
+            _noalloc_vs_oracle(_case(rng, b, H, G, D, cap), b, H, G, D, f"ticket call {k} geometry {geom}")
+    finally:
+        mkv.mkv_debug_force_ticket_merge(prev)
