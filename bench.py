@@ -263,7 +263,10 @@ class Run:
         self.g = mkv.geom(G.batch, G.n_kv_heads, G.group, G.head_dim)
         self.cap = budget + (evict_every if evict_every else stack.S)
         self.p = mkv.mkv_compress_params(budget, wl.window, wl.sink, wl.keep_window, wl.pool, 1, 1, TAU)
-        self.dp = mkv.mkv_decode_params(1, 1, TAU)
+        # a layer chain: the kernel before each decode launch belongs to another
+        # layer (or is a compress or eviction of another layer), so the launch
+        # may read its cache and moments before its dependency wait
+        self.dp = mkv.mkv_decode_params(1, 1, TAU, None, 1 if stack.L > 1 else 0)
         self.caches = [mkv.alloc_cache(self.g, self.cap, dev) for _ in range(stack.L)]
         self.moms = [mkv.alloc_moments(self.g, dev) for _ in range(stack.L)]
         # one workspace per kind, shared by the layers (the calls run one after another on one stream)

@@ -146,6 +146,20 @@ typedef struct {
                       /* (16-bit moment storage, Sec. C.2; mkv_moments_pack_bf16): */
                       /* when set, the order-1 term reads C from it (half the  */
                       /* bytes) instead of mkv_moments.C; 16-byte aligned.     */
+  int32_t early_load; /* 1: the caller guarantees that no kernel which may still */
+                      /* run when this call's kernel starts writes this cache   */
+                      /* or these moments: in a model's layer chain, the        */
+                      /* previous layer's kernels (and, if the preceding kernel */
+                      /* releases its dependents before waiting on its own      */
+                      /* predecessor, that predecessor too).  The kernel then   */
+                      /* reads the cache length and moment rows and starts the  */
+                      /* first tile copies before its programmatic dependency   */
+                      /* wait, overlapping the preceding kernel; only q, k_new  */
+                      /* and v_new are read after it.  A length that changed in */
+                      /* between is recorded as MKV_ERR_INVALID_ARG (outputs    */
+                      /* undefined); other violations go undetected.  0: every */
+                      /* read waits (always safe).  mkv_decode_evict_step        */
+                      /* ignores it (its own eviction kernel writes the cache). */
 } mkv_decode_params;
 
 /*

@@ -50,7 +50,7 @@ const char* mkv_status_str(mkv_status s) {
   return "unknown status";
 }
 
-int32_t mkv_version(void) { return 200; }
+int32_t mkv_version(void) { return 201; }
 
 // ------------------------------------------------------------------ decode
 size_t mkv_decode_workspace_size(mkv_geom geom, int32_t capacity) {
@@ -89,6 +89,7 @@ mkv_status mkv_decode_step(mkv_geom geom, const void* q, const void* k_new, cons
   a.lse = lse;
   a.batch = geom.batch;
   a.n_kv = geom.n_kv_heads;
+  a.early = p->early_load;
   decode_carve(a, geom, cache->capacity, sms, workspace);
   return cuda_status(launch_decode(a, geom.head_dim, geom.group, static_cast<cudaStream_t>(stream)));
 }
@@ -161,7 +162,7 @@ mkv_status mkv_decode_evict_step(mkv_geom geom, const void* q, const void* k_new
     return MKV_ERR_INVALID_ARG;
   if (!aligned(q, 16) || !aligned(out, 16) || !aligned(k_new, 16) || !aligned(v_new, 16)) return MKV_ERR_INVALID_ARG;
   if ((p->correction != 0 && p->correction != 1) || (p->order != 0 && p->order != 1) || !(p->tau >= 0.f) ||
-      p->C16 != nullptr)
+      p->C16 != nullptr || (p->early_load != 0 && p->early_load != 1))
     return MKV_ERR_INVALID_ARG;
   if (cache->capacity > 65536) return MKV_ERR_SHAPE;
   const int sms = num_sms_current();

@@ -173,7 +173,7 @@ __device__ __forceinline__ void process16(WarpState<D>& st, const uint32_t (&qa)
   }
 }
 
-template <int D, int G, bool CL, bool C16>
+template <int D, int G, bool CL, bool C16, bool EARLY>
 __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, const __grid_constant__ CUtensorMap tmK,
                                                           const __grid_constant__ CUtensorMap tmV) {
   constexpr int DPL = D / 32;
@@ -211,6 +211,8 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
     mbar_fence_init();
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
+  }
+  if (tid == 0 && !EARLY) {
     // Before the dependency wait: this split's retained rows and moment rows
     // were written by earlier calls, not by the kernel this launch waits on
     // (that one produces this step's query and token), so they are pulled
@@ -241,20 +243,13 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
       }
     }
   }
-  grid_dependency_wait();
-  grid_launch_dependents();
-
-  // ---- loads that do not depend on the cache length go out first
-  const __nv_bfloat16* qg = reinterpret_cast<const __nv_bfloat16*>(a.q) + ((size_t)u * G) * D;
-  uint32_t qa[D / 16][2];  // Q as the A operand: rows = heads (g = lane/4 < G), 16 dims per k-step
-  {
-    const int g = lane >> 2, t = lane & 3;
-#pragma unroll
-    for (int kk = 0; kk < D / 16; ++kk) {
-      qa[kk][0] = (g < G) ? *reinterpret_cast<const uint32_t*>(qg + g * D + kk * 16 + 2 * t) : 0u;
-      qa[kk][1] = (g < G) ? *reinterpret_cast<const uint32_t*>(qg + g * D + kk * 16 + 8 + 2 * t) : 0u;
-    }
-  }
+  // ---- the unit's cache length, its first tiles and its moment rows.  With
+  // EARLY the caller guarantees that the kernels that may still run when
+  // this launch starts (in a layer chain: the previous layer's) write
+  // neither this cache nor these moments, so they are read, and the first
+  // tile copies go out, before the dependency wait, overlapping that
+  // kernel's tail; only the query and the new token, which it may produce,
+  // wait.  Otherwise everything is read after the wait.
   const bool corr = a.correction != 0 && a.n != nullptr;
   // Moment rows [r0, r1) of this split: C'q on the tensor cores.  The rows
   // form m16 tiles (A = C' rows, split into bf16 hi + lo parts: about 16
@@ -277,87 +272,54 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
     else return __ldg(reinterpret_cast<const float2*>(a.C + off));
   };
   float2 cfr[2][KPW][4];
-  {
-    const int g = lane >> 2, t = lane & 3;
-    auto load_frags = [&](auto ld) {
-#pragma unroll
-      for (int j = 0; j < 2; ++j) {
-        const int ra = r0 + j * 16 + g, rb = ra + 8;
-#pragma unroll
-        for (int kp = 0; kp < KPW; ++kp) {
-          const int c0 = (warp * KPW + kp) * 16 + 2 * t;
-          const bool va = do_c && split_k && ra < r1, vb = do_c && split_k && rb < r1;
-          cfr[j][kp][0] = va ? ld(ra, c0) : make_float2(0.f, 0.f);
-          cfr[j][kp][1] = vb ? ld(rb, c0) : make_float2(0.f, 0.f);
-          cfr[j][kp][2] = va ? ld(ra, c0 + 8) : make_float2(0.f, 0.f);
-          cfr[j][kp][3] = vb ? ld(rb, c0 + 8) : make_float2(0.f, 0.f);
-        }
-      }
-    };
-    if constexpr (c16)
-      load_frags([&](int row, int c0) {
-        return __bfloat1622float2(
-            __ldg(reinterpret_cast<const __nv_bfloat162*>(a.C16 + ((size_t)u * D + row) * D + c0)));
-      });
-    else
-      load_frags([&](int row, int c0) {
-        return __ldg(reinterpret_cast<const float2*>(a.C + ((size_t)u * D + row) * D + c0));
-      });
-  }
-  if (do_c && !split_k && tid == 0 && r1 > r0) {  // whole-tile case: the rows are read after the tiles
-    const void* base = c16 ? static_cast<const void*>(a.C16 + ((size_t)u * D + r0) * D)
-                           : static_cast<const void*>(a.C + ((size_t)u * D + r0) * D);
-    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base),
-                 "r"((uint32_t)((r1 - r0) * D * (c16 ? 2 : 4)))
-                 : "memory");
-  }
   // mu_v of the (row, head) pairs this thread finishes in the two-tile case
   constexpr int kPairs = 2 * 16 * 8 / kThreads;  // at most 32 rows x 8 heads
   float muv_pre[kPairs];
-#pragma unroll
-  for (int j = 0; j < kPairs; ++j) {
-    const int idx = tid + j * kThreads, row = r0 + idx / G;
-    muv_pre[j] = (do_c && split_k && row < r1) ? __ldg(a.mu_v + (size_t)u * D + row) : 0.f;
-  }
   // mu_k at this lane's q dims (warp 1 computes scale q . mu_k for its head)
   float2 mkp[D / 16][2];
+  int n_e = 0;
+  auto load_moments = [&]() {
+    const int g = lane >> 2, t = lane & 3;
 #pragma unroll
-  for (int kk = 0; kk < D / 16; ++kk) {
-    const int t = lane & 3;
-    const bool v = corr && warp == 1 && (lane >> 2) < G;
-    mkp[kk][0] = v ? __ldg(reinterpret_cast<const float2*>(a.mu_k + (size_t)u * D + kk * 16 + 2 * t)) : make_float2(0.f, 0.f);
-    mkp[kk][1] = v ? __ldg(reinterpret_cast<const float2*>(a.mu_k + (size_t)u * D + kk * 16 + 8 + 2 * t)) : make_float2(0.f, 0.f);
-  }
-  const int n_e = corr ? __ldcg(a.n + u) : 0;
-  const int seen0 = (CL && s == 0 && tid == 0 && a.k_new != nullptr) ? __ldcg(a.seen + u) : 0;  // bookkeeping
-  int len0 = __ldcg(a.len + u);
-  if (len0 < 0 || len0 > a.cap) {  // corrupt cache state: never read past the slab
-    if (tid == 0 && s == 0) record_error(a.ws, MKV_ERR_CAPACITY, u);
-    len0 = len0 < 0 ? 0 : a.cap;
-  }
-  const bool has_new = a.k_new != nullptr;
-  const bool use_m = n_e > 0;
-  // the cached rows are split into whole tiles over the S CTAs; the appended
-  // token is attended to by the last CTA (which holds the fewest rows), whose
-  // threads fetch it now: threads 0..D/8-1 hold 16 bytes of k each, the next
-  // D/8 threads 16 bytes of v
-  const bool own_new = has_new && s == a.S - 1;
-  uint4 new_part = make_uint4(0u, 0u, 0u, 0u);
-  if (own_new && tid < D / 4) {
-    const __nv_bfloat16* src = reinterpret_cast<const __nv_bfloat16*>(tid < D / 8 ? a.k_new : a.v_new) + (size_t)u * D;
-    new_part = reinterpret_cast<const uint4*>(src)[tid % (D / 8)];
-  }
-  const int tiles_total = (len0 + kTT - 1) / kTT;
-  const int tiles_per = (tiles_total + a.S - 1) / a.S;
-  const int t_begin = min(len0, s * tiles_per * kTT);
-  const int t_end = min(len0, t_begin + tiles_per * kTT);
-  const int n_cached = t_end - t_begin;
-  const int n_tiles = (n_cached + kTT - 1) / kTT;
-
-  // one thread fills a stage: a 64-row box per 64 columns, for K and for V
-  // (rows past the unit's slab belong to the next unit or are zero-filled by
-  // the TMA unit; they are masked below)
-  const int row_base = u * a.cap + t_begin;
+    for (int j = 0; j < 2; ++j) {
+      const int ra = r0 + j * 16 + g, rb = ra + 8;
+#pragma unroll
+      for (int kp = 0; kp < KPW; ++kp) {
+        const int c0 = (warp * KPW + kp) * 16 + 2 * t;
+        const bool va = do_c && split_k && ra < r1, vb = do_c && split_k && rb < r1;
+        cfr[j][kp][0] = va ? ld_c2(ra, c0) : make_float2(0.f, 0.f);
+        cfr[j][kp][1] = vb ? ld_c2(rb, c0) : make_float2(0.f, 0.f);
+        cfr[j][kp][2] = va ? ld_c2(ra, c0 + 8) : make_float2(0.f, 0.f);
+        cfr[j][kp][3] = vb ? ld_c2(rb, c0 + 8) : make_float2(0.f, 0.f);
+      }
+    }
+    if (do_c && !split_k && tid == 0 && r1 > r0) {  // whole-tile case: the rows are read after the tiles
+      const void* base = c16 ? static_cast<const void*>(a.C16 + ((size_t)u * D + r0) * D)
+                             : static_cast<const void*>(a.C + ((size_t)u * D + r0) * D);
+      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base),
+                   "r"((uint32_t)((r1 - r0) * D * (c16 ? 2 : 4)))
+                   : "memory");
+    }
+#pragma unroll
+    for (int j = 0; j < kPairs; ++j) {
+      const int idx = tid + j * kThreads, row = r0 + idx / G;
+      muv_pre[j] = (do_c && split_k && row < r1) ? __ldg(a.mu_v + (size_t)u * D + row) : 0.f;
+    }
+#pragma unroll
+    for (int kk = 0; kk < D / 16; ++kk) {
+      const bool v = corr && warp == 1 && g < G;
+      mkp[kk][0] = v ? __ldg(reinterpret_cast<const float2*>(a.mu_k + (size_t)u * D + kk * 16 + 2 * t))
+                     : make_float2(0.f, 0.f);
+      mkp[kk][1] = v ? __ldg(reinterpret_cast<const float2*>(a.mu_k + (size_t)u * D + kk * 16 + 8 + 2 * t))
+                     : make_float2(0.f, 0.f);
+    }
+    n_e = corr ? __ldcg(a.n + u) : 0;
+  };
+  // the cached rows are split into whole tiles over the S CTAs; one thread
+  // fills a stage: a 64-row box per 64 columns, for K and for V (rows past
+  // the unit's slab belong to the next unit or are zero-filled by the TMA
+  // unit; they are masked below)
+  int len_read = 0, len0 = 0, t_begin = 0, n_cached = 0, n_tiles = 0, row_base = 0;
   auto issue = [&](int it) {
     const int st = it % kStages;
     mbar_arrive_expect_tx(&bars[st], 2u * kTileBytes);
@@ -367,9 +329,68 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
       tma_load_2d(sV + st * kTileBytes + bx * kTT * 128, &tmV, bx * 64, row_base + it * kTT, &bars[st]);
     }
   };
+  auto load_len_and_issue = [&]() {
+    len_read = __ldcg(a.len + u);
+    len0 = len_read;
+    if (len0 < 0 || len0 > a.cap) {  // corrupt cache state: never read past the slab
+      if (tid == 0 && s == 0) record_error(a.ws, MKV_ERR_CAPACITY, u);
+      len0 = len0 < 0 ? 0 : a.cap;
+    }
+    const int tiles_total = (len0 + kTT - 1) / kTT;
+    const int tiles_per = (tiles_total + a.S - 1) / a.S;
+    t_begin = min(len0, s * tiles_per * kTT);
+    n_cached = min(len0, t_begin + tiles_per * kTT) - t_begin;
+    n_tiles = (n_cached + kTT - 1) / kTT;
+    row_base = u * a.cap + t_begin;
+    if (tid == 0)
+      for (int i = 0; i < min(kStages, n_tiles); ++i) issue(i);
+  };
+  if constexpr (EARLY) {
+    load_len_and_issue();
+    if (tid == 0) {  // the split's tiles past the first stages: into L2 now
+      const int first = min(kStages, n_tiles);
+      if (n_tiles > first) {
+        const size_t off = ((size_t)row_base + first * kTT) * D * 2;
+        const uint32_t bytes = static_cast<uint32_t>((n_cached - first * kTT) * D * 2);
+        asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(static_cast<const uint8_t*>(a.K) + off),
+                     "r"(bytes) : "memory");
+        asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(static_cast<const uint8_t*>(a.V) + off),
+                     "r"(bytes) : "memory");
+      }
+    }
+    load_moments();
+  }
+  grid_dependency_wait();
+  grid_launch_dependents();
 
-  if (tid == 0) {
-    for (int i = 0; i < min(kStages, n_tiles); ++i) issue(i);
+  // ---- the query: the A operand, rows = heads (g = lane/4 < G), 16 dims per k-step
+  const __nv_bfloat16* qg = reinterpret_cast<const __nv_bfloat16*>(a.q) + ((size_t)u * G) * D;
+  uint32_t qa[D / 16][2];
+  {
+    const int g = lane >> 2, t = lane & 3;
+#pragma unroll
+    for (int kk = 0; kk < D / 16; ++kk) {
+      qa[kk][0] = (g < G) ? *reinterpret_cast<const uint32_t*>(qg + g * D + kk * 16 + 2 * t) : 0u;
+      qa[kk][1] = (g < G) ? *reinterpret_cast<const uint32_t*>(qg + g * D + kk * 16 + 8 + 2 * t) : 0u;
+    }
+  }
+  if constexpr (!EARLY) {
+    load_moments();
+    load_len_and_issue();
+  } else if (tid == 0 && s == 0 && __ldcg(a.len + u) != len_read) {
+    record_error(a.ws, MKV_ERR_INVALID_ARG, u);  // the cache changed under an early load
+  }
+  const int seen0 = (CL && s == 0 && tid == 0 && a.k_new != nullptr) ? __ldcg(a.seen + u) : 0;  // bookkeeping
+  const bool has_new = a.k_new != nullptr;
+  const bool use_m = n_e > 0;
+  // the appended token is attended to by the last CTA (which holds the
+  // fewest rows), whose threads fetch it now: threads 0..D/8-1 hold 16 bytes
+  // of k each, the next D/8 threads 16 bytes of v
+  const bool own_new = has_new && s == a.S - 1;
+  uint4 new_part = make_uint4(0u, 0u, 0u, 0u);
+  if (own_new && tid < D / 4) {
+    const __nv_bfloat16* src = reinterpret_cast<const __nv_bfloat16*>(tid < D / 8 ? a.k_new : a.v_new) + (size_t)u * D;
+    new_part = reinterpret_cast<const uint4*>(src)[tid % (D / 8)];
   }
   if (use_m && warp == 1) {  // scale * q . mu_k per head from the qa fragments (lanes 4h..4h+3)
     const int g = lane >> 2;
@@ -768,7 +789,7 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
 
 // Whether clusters of S CTAs with `smem` bytes each can be resident (checked
 // once per split count; portable sizes always can).
-template <int D, int G, bool C16>
+template <int D, int G, bool C16, bool EARLY>
 bool cluster_fits(int S, size_t smem) {
   if (S <= 8) return true;
   static std::mutex mu;
@@ -787,14 +808,14 @@ bool cluster_fits(int S, size_t smem) {
     cfg.attrs = at;
     cfg.numAttrs = 1;
     int n = 0;
-    const cudaError_t e = cudaOccupancyMaxActiveClusters(&n, decode_kernel<D, G, true, C16>, &cfg);
+    const cudaError_t e = cudaOccupancyMaxActiveClusters(&n, decode_kernel<D, G, true, C16, EARLY>, &cfg);
     if (e != cudaSuccess) (void)cudaGetLastError();
     known[S] = (e == cudaSuccess && n > 0) ? 1 : -1;
   }
   return known[S] > 0;
 }
 
-template <int D, int G, bool C16>
+template <int D, int G, bool C16, bool EARLY>
 cudaError_t launch_dgc(const DecodeArgs& args, cudaStream_t stream) {
   DecodeArgs a = args;
   a.polls = pipeline_poll_limit();
@@ -805,16 +826,16 @@ cudaError_t launch_dgc(const DecodeArgs& args, cudaStream_t stream) {
   // per-device function attributes; setting them again is harmless
   cudaError_t e;
   if (cl) {
-    e = cudaFuncSetAttribute(decode_kernel<D, G, true, C16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    e = cudaFuncSetAttribute(decode_kernel<D, G, true, C16, EARLY>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(smem));
     if (e == cudaSuccess && a.S > 8)
-      e = cudaFuncSetAttribute(decode_kernel<D, G, true, C16>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+      e = cudaFuncSetAttribute(decode_kernel<D, G, true, C16, EARLY>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   } else {
-    e = cudaFuncSetAttribute(decode_kernel<D, G, false, C16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    e = cudaFuncSetAttribute(decode_kernel<D, G, false, C16, EARLY>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(smem));
   }
   if (e != cudaSuccess) return e;
-  const bool use_cl = cl && cluster_fits<D, G, C16>(a.S, smem) && g_force_ticket_merge.load() == 0;
+  const bool use_cl = cl && cluster_fits<D, G, C16, EARLY>(a.S, smem) && g_force_ticket_merge.load() == 0;
   // the cache slabs of all units as one [units * cap][D] matrix
   const uint64_t rows = (uint64_t)a.batch * a.n_kv * a.cap;
   CUtensorMap tmK, tmV;
@@ -835,18 +856,20 @@ cudaError_t launch_dgc(const DecodeArgs& args, cudaStream_t stream) {
   at[1].val.clusterDim.z = 1;
   cfg.attrs = at;
   cfg.numAttrs = use_cl ? 2 : 1;
-  if (use_cl) return cudaLaunchKernelEx(&cfg, decode_kernel<D, G, true, C16>, a, tmK, tmV);
+  if (use_cl) return cudaLaunchKernelEx(&cfg, decode_kernel<D, G, true, C16, EARLY>, a, tmK, tmV);
   if (cl) {  // the cluster did not fit: the ticket variant with the ring only
-    e = cudaFuncSetAttribute(decode_kernel<D, G, false, C16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    e = cudaFuncSetAttribute(decode_kernel<D, G, false, C16, EARLY>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(ring));
     if (e != cudaSuccess) return e;
   }
-  return cudaLaunchKernelEx(&cfg, decode_kernel<D, G, false, C16>, a, tmK, tmV);
+  return cudaLaunchKernelEx(&cfg, decode_kernel<D, G, false, C16, EARLY>, a, tmK, tmV);
 }
 
 template <int D, int G>
 cudaError_t launch_dg(const DecodeArgs& a, cudaStream_t stream) {
-  return a.C16 != nullptr ? launch_dgc<D, G, true>(a, stream) : launch_dgc<D, G, false>(a, stream);
+  if (a.early)
+    return a.C16 != nullptr ? launch_dgc<D, G, true, true>(a, stream) : launch_dgc<D, G, false, true>(a, stream);
+  return a.C16 != nullptr ? launch_dgc<D, G, true, false>(a, stream) : launch_dgc<D, G, false, false>(a, stream);
 }
 
 }  // namespace
@@ -871,10 +894,10 @@ int active_clusters(int S) {
     const size_t ring = (size_t)2 * kStages * kTT * D * 2 + 1024;
     const size_t smem = ring + ((size_t)S * G * (D + 4) + (size_t)G * D + 2 * (size_t)S * G) * sizeof(float);
     int n = 0;
-    cudaError_t e = cudaFuncSetAttribute(decode_kernel<D, G, true, false>,
+    cudaError_t e = cudaFuncSetAttribute(decode_kernel<D, G, true, false, false>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
     if (e == cudaSuccess && S > 8)
-      e = cudaFuncSetAttribute(decode_kernel<D, G, true, false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+      e = cudaFuncSetAttribute(decode_kernel<D, G, true, false, false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (e == cudaSuccess) {
       cudaLaunchConfig_t cfg{};
       cfg.gridDim = dim3(S, 1, 1);
@@ -887,7 +910,7 @@ int active_clusters(int S) {
       at[0].val.clusterDim.z = 1;
       cfg.attrs = at;
       cfg.numAttrs = 1;
-      e = cudaOccupancyMaxActiveClusters(&n, decode_kernel<D, G, true, false>, &cfg);
+      e = cudaOccupancyMaxActiveClusters(&n, decode_kernel<D, G, true, false, false>, &cfg);
     }
     if (e != cudaSuccess) {
       (void)cudaGetLastError();

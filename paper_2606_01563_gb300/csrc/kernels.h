@@ -39,6 +39,7 @@ struct DecodeArgs {
   int32_t n_kv;
   int32_t S;
   uint32_t polls;  // poll limit of the tile waits (the drain after a timeout uses kMaxPolls)
+  int32_t early;   // cache and moments read before the dependency wait (mkv_decode_params.early_load)
 };
 
 constexpr int kDecodeTile = 64;  // tokens per pipeline stage

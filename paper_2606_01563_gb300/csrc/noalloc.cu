@@ -126,6 +126,7 @@ extern "C" MKV_API mkv_status mkv_decode_step_noalloc(mkv_geom geom, const void*
   a.lse = lse;
   a.batch = geom.batch;
   a.n_kv = geom.n_kv_heads;
+  a.early = p->early_load;
   carve(a, geom, S, scratch);
   return launch_decode(a, geom.head_dim, geom.group, static_cast<cudaStream_t>(stream)) == cudaSuccess
              ? MKV_OK

@@ -43,7 +43,8 @@ class mkv_compress_diag(ctypes.Structure):
 
 
 class mkv_decode_params(ctypes.Structure):
-    _fields_ = [("correction", c_i32), ("order", c_i32), ("tau", ctypes.c_float), ("C16", c_vp)]
+    _fields_ = [("correction", c_i32), ("order", c_i32), ("tau", ctypes.c_float), ("C16", c_vp),
+                ("early_load", c_i32)]
 
 
 STATUS = {0: "MKV_OK", 1: "MKV_ERR_INVALID_ARG", 2: "MKV_ERR_SHAPE", 3: "MKV_ERR_CAPACITY",

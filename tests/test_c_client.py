@@ -41,7 +41,7 @@ int main(void) {
   const mkv_geom bad_group = {1, 2, 3, 128};
   mkv_cache c = {FAKE, FAKE, (int32_t*)FAKE, (int32_t*)FAKE, (int32_t*)FAKE, 64};
   mkv_moments m = {(int32_t*)FAKE, (float*)FAKE, (float*)FAKE, (float*)FAKE};
-  mkv_decode_params dp = {1, 1, 1e-6f, NULL};
+  mkv_decode_params dp = {1, 1, 1e-6f, NULL, 0};
   mkv_compress_params cp = {128, 16, 1, 1, 1, 1, 1, 1e-6f, 0};
   mkv_compress_params small = cp;
   const size_t big = (size_t)1 << 30;
@@ -52,11 +52,12 @@ int main(void) {
   CHECK(sizeof(mkv_cache) == 48 && offsetof(mkv_cache, capacity) == 40);
   CHECK(sizeof(mkv_compress_params) == 36);
   CHECK(offsetof(mkv_compress_params, tau) == 28 && offsetof(mkv_compress_params, adaptive) == 32);
-  CHECK(sizeof(mkv_decode_params) == 24 && offsetof(mkv_decode_params, C16) == 16);
+  CHECK(sizeof(mkv_decode_params) == 32 && offsetof(mkv_decode_params, C16) == 16 &&
+        offsetof(mkv_decode_params, early_load) == 24);
   CHECK(sizeof(mkv_compress_diag) == 24);
   CHECK(sizeof(mkv_status) == 4 && MKV_ERR_WORKSPACE == 7);
 
-  CHECK(mkv_version() == 200);
+  CHECK(mkv_version() == 201);
   CHECK(strcmp(mkv_status_str(MKV_OK), "ok") == 0);
   CHECK(strcmp(mkv_status_str((mkv_status)99), "unknown status") == 0);
 
@@ -129,7 +130,7 @@ def test_header_compiles_as_cpp(tmp_path):
     if cxx is None:
         pytest.skip("no C++ compiler")
     src = tmp_path / "h.cpp"
-    src.write_text('#include "mkv.h"\nint main() { return mkv_version() == 200 ? 0 : 1; }\n')
+    src.write_text('#include "mkv.h"\nint main() { return mkv_version() == 201 ? 0 : 1; }\n')
     r = subprocess.run([cxx, "-std=c++17", "-Wall", "-Wextra", "-Werror", "-fsyntax-only", "-I", INCLUDE, str(src)],
                        capture_output=True, text=True)
     assert r.returncode == 0, r.stderr
@@ -142,5 +143,6 @@ def test_binding_structs_match_the_c_layout():
     assert ctypes.sizeof(mkv.mkv_cache) == 48 and mkv.mkv_cache.capacity.offset == 40
     assert ctypes.sizeof(mkv.mkv_compress_params) == 36
     assert mkv.mkv_compress_params.tau.offset == 28 and mkv.mkv_compress_params.adaptive.offset == 32
-    assert ctypes.sizeof(mkv.mkv_decode_params) == 24 and mkv.mkv_decode_params.C16.offset == 16
+    assert ctypes.sizeof(mkv.mkv_decode_params) == 32 and mkv.mkv_decode_params.C16.offset == 16
+    assert mkv.mkv_decode_params.early_load.offset == 24
     assert ctypes.sizeof(mkv.mkv_compress_diag) == 24

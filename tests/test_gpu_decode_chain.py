@@ -1,0 +1,80 @@
+"""Decode in a model's layer chain with early loads (mkv_decode_params.early_load
+= 1): several layers' caches, each decode step one launch per layer, layer
+after layer, each appending its token, back to back on one stream, so that
+every launch starts while the previous layer's is still running and reads its
+own cache and moments before its dependency wait.  Every output of every
+launch against the fp64 oracle; also with the bf16 copy of C, batch 1 (many
+splits) and the large-batch one-split case."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2606_01563_gb300 import mkv
+from paper_2606_01563_gb300.inputs import bf16_round
+from gpu_util import assert_output_close, bf16, f32, host, i32
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.mark.parametrize("b,H,G,D,L,lens,cap,c16", [
+    (2, 8, 4, 128, 3, (300, 420), 440, False),
+    (1, 8, 4, 128, 4, (130, 510), 520, False),
+    (1, 8, 4, 128, 3, (200, 260), 270, True),
+    (24, 8, 2, 64, 2, (60, 90), 100, False),
+])
+def test_layer_chain_early_load(b, H, G, D, L, lens, cap, c16):
+    rng = np.random.default_rng(b * 1000 + L * 10 + D)
+    steps = 3
+    layers = []
+    for l in range(L):
+        K = bf16_round(rng.standard_normal((b, H, cap, D)))
+        V = bf16_round(rng.standard_normal((b, H, cap, D)))
+        ln = rng.integers(lens[0], lens[1], (b, H)).astype(np.int32)
+        n = rng.integers(0, 6000, (b, H)).astype(np.int32)
+        mk = (0.3 * rng.standard_normal((b, H, D))).astype(np.float32)
+        mv = (0.3 * rng.standard_normal((b, H, D))).astype(np.float32)
+        C = (0.05 * rng.standard_normal((b, H, D, D))).astype(np.float32)
+        if c16:
+            C = bf16_round(C)  # the oracle sees what the bf16 copy holds
+        layers.append(dict(K=K, V=V, len=ln, n=n, mu_k=mk, mu_v=mv, C=C))
+    q = bf16_round(2.0 * rng.standard_normal((steps, L, b, H * G, D)))
+    kn = bf16_round(rng.standard_normal((steps, L, b, H, D)))
+    vn = bf16_round(rng.standard_normal((steps, L, b, H, D)))
+    g = mkv.geom(b, H, G, D)
+    dev = []
+    for st in layers:
+        cache = mkv.Cache(bf16(st["K"]), bf16(st["V"]), i32(np.zeros((b, H, cap))), i32(st["len"]),
+                          i32(st["len"]))
+        mom = mkv.Moments(i32(st["n"]), f32(st["mu_k"]), f32(st["mu_v"]), f32(st["C"]))
+        C16 = None
+        if c16:
+            C16 = torch.empty(b, H, D, D, dtype=torch.bfloat16, device="cuda")
+            mkv.mkv_moments_pack_bf16(g, mom, C16)
+        dev.append((cache, mom, C16))
+    qd, knd, vnd = bf16(q), bf16(kn), bf16(vn)
+    outs = torch.full((steps, L, b, H * G, D), float("nan"), device="cuda")
+    ws = mkv.alloc_workspace(mkv.mkv_decode_workspace_size(g, cap))
+    torch.cuda.synchronize()
+    stream = torch.cuda.Stream()
+    with torch.cuda.stream(stream):
+        for i in range(steps):
+            for l in range(L):
+                cache, mom, C16 = dev[l]
+                p = mkv.mkv_decode_params(1, 1, 1e-6, None if C16 is None else C16.data_ptr(), 1)
+                mkv.mkv_decode_step(g, qd[i, l], knd[i, l], vnd[i, l], cache, mom, p, outs[i, l], None, ws, stream)
+    stream.synchronize()
+    code, info = mkv.mkv_get_device_error(ws)
+    assert code == 0, (code, info)
+    got = host(outs)
+    for l, st in enumerate(layers):
+        for bi in range(b):
+            for h in range(H):
+                n0 = st["len"][bi, h]
+                Kr, Vr = st["K"][bi, h, :n0], st["V"][bi, h, :n0]
+                m = O.Moments(int(st["n"][bi, h]), st["mu_k"][bi, h], st["mu_v"][bi, h], st["C"][bi, h])
+                for i in range(steps):
+                    o, _, Kr, Vr = O.decode_step(q[i, l, bi, h * G:(h + 1) * G], Kr, Vr, m, kn[i, l, bi, h],
+                                                 vn[i, l, bi, h], True, 1, 1e-6)
+                    assert_output_close(got[i, l, bi, h * G:(h + 1) * G], o, f"step {i} layer {l} unit {(bi, h)}")
+        np.testing.assert_array_equal(host(dev[l][0].len), st["len"] + steps)

@@ -48,7 +48,7 @@ def test_debug_hooks_round_trip(L):
 
 
 def test_version_and_status_strings(L):
-    assert mkv.mkv_version() == 200
+    assert mkv.mkv_version() == 201
     for code in range(8):
         assert mkv.mkv_status_str(code)
     assert mkv.mkv_status_str(99) == "unknown status"
@@ -92,6 +92,7 @@ def test_decode_validation(L):
     assert decode(L, g, ws=FAKE + 8) == 7                    # misaligned workspace
     assert decode(L, g, p=mkv.mkv_decode_params(1, 1, 0.0, FAKE + 8)) == 1  # misaligned bf16 C copy
     assert decode(L, g, q=FAKE + 4) == 1                     # misaligned q
+    assert decode(L, g, p=mkv.mkv_decode_params(1, 1, 0.0, None, 2)) == 1   # early_load not 0/1
     # mu_k is read as float2 and mu_v as float4: 4-byte alignment is not enough
     assert decode(L, g, mom=mkv.mkv_moments(FAKE, FAKE + 4, FAKE, FAKE)) == 1
     assert decode(L, g, mom=mkv.mkv_moments(FAKE, FAKE, FAKE + 8, FAKE)) == 1
