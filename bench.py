@@ -267,7 +267,8 @@ class Run:
         # layer (or is a compress or eviction of another layer), so the launch
         # may read its cache and moments before its dependency wait
         self.dp = mkv.mkv_decode_params(1, 1, TAU, None, 1 if stack.L > 1 else 0)
-        self.caches = [mkv.alloc_cache(self.g, self.cap, dev) for _ in range(stack.L)]
+        # with periodic eviction the caches keep y_j = S_tilde k_j across calls
+        self.caches = [mkv.alloc_cache(self.g, self.cap, dev, evict_state=bool(evict_every)) for _ in range(stack.L)]
         self.moms = [mkv.alloc_moments(self.g, dev) for _ in range(stack.L)]
         # one workspace per kind, shared by the layers (the calls run one after another on one stream)
         self.ws_c = mkv.alloc_workspace(mkv.mkv_compress_workspace_size(self.g, wl.T, self.p), dev)
@@ -808,8 +809,10 @@ def layers_one_launch(torch, mkv, dev, flush, hbm, layers=32, B=512):
 def continuous_eviction(torch, mkv, dev, steps=64):
     """Algorithm 1 once per generated token with the cache at its budget (one
     append and one eviction per step, Llama-3.1-8B geometry, budget 512):
-    mkv_decode_evict_step, and the two calls it stands for (mkv_evict_append,
-    then mkv_decode_step), each as a graph of `steps` steps."""
+    mkv_decode_evict_step with the cache keeping y_j = S_tilde k_j across
+    calls, the same without that state, and the two calls it stands for
+    (mkv_evict_append, then mkv_decode_step), each as a graph of `steps`
+    steps."""
     res = []
     for b in (1, 8):
         H, G, D, B, cap = 8, 4, 128, 512, 576
@@ -823,11 +826,14 @@ def continuous_eviction(torch, mkv, dev, steps=64):
         p = mkv.mkv_decode_params(1, 1, TAU)
         st = torch.cuda.Stream(dev)
         cell = {"batch": b, "budget": B}
-        for mode in ("one_call", "two_calls"):
+        for mode in ("one_call_state", "one_call", "two_calls"):
             cache = mkv.Cache(K0.clone(), V0.clone(),
                               torch.arange(cap, dtype=torch.int32, device=dev).expand(b, H, cap).contiguous(),
                               torch.full((b, H), B, dtype=torch.int32, device=dev),
                               torch.full((b, H), 10 ** 4, dtype=torch.int32, device=dev))
+            if mode == "one_call_state":
+                cache.y = torch.zeros(b, H, cap, D, device=dev)
+                cache.y_len = torch.zeros(b, H, dtype=torch.int32, device=dev)
             mom = mkv.Moments(torch.full((b, H), 7000, dtype=torch.int32, device=dev), *(x.clone() for x in mom0))
             wsf = mkv.alloc_workspace(mkv.mkv_decode_evict_workspace_size(g, cap), dev)
             wse = mkv.alloc_workspace(mkv.mkv_evict_workspace_size(g, cap), dev)
@@ -835,7 +841,7 @@ def continuous_eviction(torch, mkv, dev, steps=64):
 
             def body():
                 for i in range(steps):
-                    if mode == "one_call":
+                    if mode in ("one_call", "one_call_state"):
                         mkv.mkv_decode_evict_step(g, qs[i], kn[i], vn[i], B, cache, mom, p, out, None, wsf, st)
                     else:
                         mkv.mkv_evict_append(g, qs[i], kn[i], vn[i], B, cache, mom, TAU, wse, st)

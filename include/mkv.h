@@ -102,6 +102,20 @@ typedef struct {
  *   len   int32 [b, h_kv]                rows in use
  *   seen  int32 [b, h_kv]                tokens seen so far; an appended token
  *                                        takes position `seen`, then seen += 1
+ * Optional eviction state (both NULL, or both set):
+ *   y     fp32  [b, h_kv, capacity, d]   y_j = S_tilde k_j of each row under
+ *                                        the current moments (the products
+ *                                        Algorithm 1's residual needs), 16-byte
+ *                                        aligned
+ *   y_len int32 [b, h_kv]                rows 0..y_len-1 of y are current
+ * With them, mkv_evict_append and mkv_decode_evict_step compute S_tilde k_j
+ * only for rows at or above y_len (the rows appended since the last
+ * eviction), O(d^2) each, instead of for every row, and leave y current for
+ * the surviving rows; mkv_compress sets y_len to 0.  Appends by
+ * mkv_decode_step need no update (they add rows above y_len).  A caller that
+ * changes the cache or the moments in any other way sets y_len to 0.
+ * Capacities above 1152 rows run an eviction kernel that does not keep y: it
+ * sets y_len to 0.
  */
 typedef struct {
   void* K;
@@ -110,6 +124,8 @@ typedef struct {
   int32_t* len;
   int32_t* seen;
   int32_t capacity;
+  float* y;
+  int32_t* y_len;
 } mkv_cache;
 
 /* Prefill compression parameters (SnapKV protocol of Sec. 5.1 plus the

@@ -132,6 +132,8 @@ mkv_status mkv_evict_append(mkv_geom geom, const void* q, const void* k_new, con
   a.mu_k = mom->mu_k;
   a.mu_v = mom->mu_v;
   a.C = mom->C;
+  a.Y = cache->y;
+  a.y_len = cache->y_len;
   a.budget = budget;
   a.tau = tau;
   a.batch = geom.batch;
@@ -182,6 +184,8 @@ mkv_status mkv_decode_evict_step(mkv_geom geom, const void* q, const void* k_new
   e.mu_k = mom->mu_k;
   e.mu_v = mom->mu_v;
   e.C = mom->C;
+  e.Y = cache->y;
+  e.y_len = cache->y_len;
   e.budget = budget;
   e.tau = p->tau;
   e.batch = geom.batch;
@@ -287,6 +291,11 @@ mkv_status mkv_compress(mkv_geom geom, int32_t T, const void* K, const void* V, 
   a.ws = workspace;
   a.batch = geom.batch;
   a.n_kv = geom.n_kv_heads;
+  // the cache's rows and the moments are replaced: no y row stays current
+  if (out_cache->y_len != nullptr &&
+      cudaMemsetAsync(out_cache->y_len, 0, (size_t)geom.batch * geom.n_kv_heads * sizeof(int32_t),
+                      static_cast<cudaStream_t>(stream)) != cudaSuccess)
+    return MKV_ERR_CUDA;
   return cuda_status(launch_compress(a, geom, workspace_bytes, sms, static_cast<cudaStream_t>(stream)));
 }
 

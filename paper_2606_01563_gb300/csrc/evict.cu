@@ -303,6 +303,7 @@ __global__ void __launch_bounds__(kThreads) evict_kernel(const EvictArgs a) {
   if (tid == 0) {
     a.n[u] = n;
     a.len[u] = a.budget;
+    if (a.y_len != nullptr) a.y_len[u] = 0;  // rows moved and the moments changed: no y row is current
   }
 
   // ---- ordered in-place compaction, 32 rows per step (destination <= source)
@@ -939,6 +940,7 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kCT, 1)
       a.n[u] = n;
       a.len[u] = a.budget;
       a.seen[u] = seen_in + (has_new ? 1 : 0);
+      if (a.y_len != nullptr) a.y_len[u] = 0;  // rows moved and the moments changed: no y row is current
     }
   }
 }
@@ -1068,6 +1070,8 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
     return;  // uniform over the cluster
   }
   const int len = len_in + (has_new ? 1 : 0);
+  // rows 0..y_cur-1 of the cache's y rows are current (none without them)
+  const int y_cur = (a.Y != nullptr && a.y_len != nullptr) ? max(0, min(a.y_len[u], len_in)) : 0;
   const int rows_per = (len + kCL - 1) / kCL;
   const int j0 = min(len, rank * rows_per), j1 = min(len, j0 + rows_per);
   const int nr = j1 - j0;
@@ -1258,23 +1262,49 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
     if (warp + kRW * i < nr) alive |= 1u << i;
   }
   if (n > 0) {
-    for (int c = 0; c < D; ++c) {
-      float cv[DPL];
-      ld_vec<DPL>(Ct + (size_t)c * D + lane * DPL, cv);
+    // rows below the cache's y_len carry y_j = S_tilde k_j from the call that
+    // last changed the moments (kept in the cache across calls); the others
+    // (the rows appended since) are computed here, O(d^2) each
+    unsigned fresh = 0u;
 #pragma unroll
-      for (int i = 0; i < RPW; ++i) {
-        const int r = warp + kRW * i;
-        if (r < nr) {
-          const float kv = __bfloat162float(Kr[(size_t)r * D + c]);
-#pragma unroll
-          for (int d = 0; d < DPL; ++d) y[i][d] = fmaf(cv[d], kv, y[i][d]);
+    for (int i = 0; i < RPW; ++i) {
+      const int r = warp + kRW * i;
+      if (r < nr && j0 + r < y_cur) {
+        const float* src = a.Y + (row0 + j0 + r) * D + lane * DPL;
+        if constexpr (DPL == 4) {
+          const float4 t = *reinterpret_cast<const float4*>(src);
+          y[i][0] = t.x;
+          y[i][1] = t.y;
+          y[i][2] = t.z;
+          y[i][3] = t.w;
+        } else {
+          const float2 t = *reinterpret_cast<const float2*>(src);
+          y[i][0] = t.x;
+          y[i][1] = t.y;
         }
+      } else if (r < nr) {
+        fresh |= 1u << i;
       }
     }
+    if (fresh != 0u) {  // warp-uniform
+      for (int c = 0; c < D; ++c) {
+        float cv[DPL];
+        ld_vec<DPL>(Ct + (size_t)c * D + lane * DPL, cv);
 #pragma unroll
-    for (int i = 0; i < RPW; ++i)
+        for (int i = 0; i < RPW; ++i) {
+          if ((fresh >> i) & 1u) {
+            const float kv = __bfloat162float(Kr[(size_t)(warp + kRW * i) * D + c]);
 #pragma unroll
-      for (int d = 0; d < DPL; ++d) y[i][d] *= nf0;
+            for (int d = 0; d < DPL; ++d) y[i][d] = fmaf(cv[d], kv, y[i][d]);
+          }
+        }
+      }
+#pragma unroll
+      for (int i = 0; i < RPW; ++i)
+        if ((fresh >> i) & 1u)
+#pragma unroll
+          for (int d = 0; d < DPL; ++d) y[i][d] *= nf0;
+    }
   }
   float creg[CJ][DPL];
 #pragma unroll
@@ -1555,6 +1585,49 @@ __global__ void __cluster_dims__(kCL, 1, 1) __launch_bounds__(kRT, 1)
   int base = 0;
   for (int r = 0; r < rank; ++r) base += *cluster.map_shared_rank(&ex_cnt, r);
   const int mine = ex_cnt;
+  if (a.Y != nullptr && a.y_len != nullptr) {
+    // the loop left the last eviction folded into S_tilde but not yet into
+    // y: y_j += (dk . k_j) dv for the surviving rows, as in the loop
+    {
+      float part[RPW];
+#pragma unroll
+      for (int i = 0; i < RPW; ++i) {
+        part[i] = 0.f;
+        if ((alive >> i) & 1u) {
+          float kf[DPL];
+          load_bf16<DPL>(Kr + (size_t)(warp + kRW * i) * D + lane * DPL, kf);
+#pragma unroll
+          for (int d = 0; d < DPL; ++d) part[i] = fmaf(sdk[d], kf[d], part[i]);
+        }
+      }
+      float pv[P];
+#pragma unroll
+      for (int i = 0; i < P; ++i) pv[i] = i < RPW ? part[i] : 0.f;
+      const float dsum = transpose_sum<P>(pv, lane);
+#pragma unroll
+      for (int i = 0; i < RPW; ++i) {
+        const float dot = __shfl_sync(kFull, dsum, i << SH);
+#pragma unroll
+        for (int d = 0; d < DPL; ++d) y[i][d] = fmaf(dot, sdv[d], y[i][d]);
+      }
+    }
+    // y_j of the surviving rows to their compacted rows: each warp writes its
+    // own rows' registers (every read of the y rows was in the set-up, before
+    // the cluster barriers of the loop)
+#pragma unroll
+    for (int i = 0; i < RPW; ++i) {
+      const int r = warp + kRW * i;
+      if (r < nr && ((alive >> i) & 1u)) {  // warp-uniform
+        int before = 0;  // survivors of this CTA ahead of row r
+        for (int c0 = 0; c0 < r; c0 += 32)
+          before += __popc(__ballot_sync(kFull, c0 + lane < r && alv[c0 + lane]));
+        float* dst = a.Y + (row0 + base + before) * D + lane * DPL;
+        if constexpr (DPL == 4) *reinterpret_cast<float4*>(dst) = make_float4(y[i][0], y[i][1], y[i][2], y[i][3]);
+        else *reinterpret_cast<float2*>(dst) = make_float2(y[i][0], y[i][1]);
+      }
+    }
+    if (rank == 0 && tid == 0) a.y_len[u] = a.budget;  // ordered after the other CTAs' writes by the kernel end
+  }
   uint8_t* st = static_cast<uint8_t*>(a.stage) + (size_t)u * stage_stride(a.cap, D);
   __nv_bfloat16* SK = reinterpret_cast<__nv_bfloat16*>(st);
   __nv_bfloat16* SV = SK + (size_t)a.cap * D;

@@ -71,6 +71,8 @@ struct EvictArgs {
   void* ws;
   float* scratch;  // [units][G][cap] logits (single-CTA kernel)
   void* stage;     // [units][cap] rows staged by the cluster kernel's compaction
+  float* Y;          // optional fp32 [units][cap][D]: y_j = S_tilde k_j of each row (mkv_cache.y)
+  int32_t* y_len;    // optional [units]: rows 0..y_len-1 of Y are current (mkv_cache.y_len)
   int32_t rows_max;  // cluster kernel: rows per CTA slice = ceil(cap / CTAs per unit)
   int32_t kv_smem;   // cluster kernel: the slice's K/V rows are cached in shared memory
   int32_t batch;

@@ -34,10 +34,11 @@ inline mkv_status geom_status(const mkv_geom& g) {
   return (g.head_dim == 64 || g.head_dim == 128) ? MKV_ERR_SHAPE : MKV_ERR_UNSUPPORTED;
 }
 
-// K and V rows are read by 16-byte tensor copies
+// K and V rows are read by 16-byte tensor copies; the optional y rows by
+// vector loads, and y comes with y_len or not at all
 inline bool cache_ok(const mkv_cache* c) {
   return c && c->K && c->V && c->pos && c->len && c->seen && c->capacity >= 1 && aligned(c->K, 16) &&
-         aligned(c->V, 16);
+         aligned(c->V, 16) && ((c->y == nullptr) == (c->y_len == nullptr)) && aligned(c->y, 16);
 }
 
 // The decode kernel reads mu_k as float2 and mu_v (and C) as float4, so mu_k

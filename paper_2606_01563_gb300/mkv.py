@@ -30,7 +30,8 @@ class mkv_moments(ctypes.Structure):
 
 
 class mkv_cache(ctypes.Structure):
-    _fields_ = [("K", c_vp), ("V", c_vp), ("pos", c_vp), ("len", c_vp), ("seen", c_vp), ("capacity", c_i32)]
+    _fields_ = [("K", c_vp), ("V", c_vp), ("pos", c_vp), ("len", c_vp), ("seen", c_vp), ("capacity", c_i32),
+                ("y", c_vp), ("y_len", c_vp)]
 
 
 class mkv_compress_params(ctypes.Structure):
@@ -142,6 +143,8 @@ class Cache:
     pos: torch.Tensor
     len: torch.Tensor
     seen: torch.Tensor
+    y: torch.Tensor | None = None      # optional eviction state: fp32 [b, h_kv, cap, d]
+    y_len: torch.Tensor | None = None  # int32 [b, h_kv]
 
     @property
     def capacity(self):
@@ -149,7 +152,8 @@ class Cache:
 
     def c(self):
         return mkv_cache(self.K.data_ptr(), self.V.data_ptr(), self.pos.data_ptr(), self.len.data_ptr(),
-                         self.seen.data_ptr(), self.capacity)
+                         self.seen.data_ptr(), self.capacity, None if self.y is None else self.y.data_ptr(),
+                         None if self.y_len is None else self.y_len.data_ptr())
 
 
 @dataclass
@@ -168,13 +172,16 @@ def geom(batch, n_kv_heads, group, head_dim):
     return mkv_geom(batch, n_kv_heads, group, head_dim)
 
 
-def alloc_cache(g: mkv_geom, capacity, device="cuda"):
+def alloc_cache(g: mkv_geom, capacity, device="cuda", evict_state=False):
+    """A zero cache; evict_state adds the y rows and y_len of the eviction state."""
     shp = (g.batch, g.n_kv_heads)
+    y = torch.zeros(*shp, capacity, g.head_dim, dtype=torch.float32, device=device) if evict_state else None
+    y_len = torch.zeros(*shp, dtype=torch.int32, device=device) if evict_state else None
     return Cache(torch.zeros(*shp, capacity, g.head_dim, dtype=torch.bfloat16, device=device),
                  torch.zeros(*shp, capacity, g.head_dim, dtype=torch.bfloat16, device=device),
                  torch.zeros(*shp, capacity, dtype=torch.int32, device=device),
                  torch.zeros(*shp, dtype=torch.int32, device=device),
-                 torch.zeros(*shp, dtype=torch.int32, device=device))
+                 torch.zeros(*shp, dtype=torch.int32, device=device), y, y_len)
 
 
 def alloc_moments(g: mkv_geom, device="cuda"):

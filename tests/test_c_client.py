@@ -39,7 +39,7 @@ int main(void) {
   const mkv_geom g = {1, 2, 4, 128};
   const mkv_geom bad_dim = {1, 2, 4, 96};
   const mkv_geom bad_group = {1, 2, 3, 128};
-  mkv_cache c = {FAKE, FAKE, (int32_t*)FAKE, (int32_t*)FAKE, (int32_t*)FAKE, 64};
+  mkv_cache c = {FAKE, FAKE, (int32_t*)FAKE, (int32_t*)FAKE, (int32_t*)FAKE, 64, NULL, NULL};
   mkv_moments m = {(int32_t*)FAKE, (float*)FAKE, (float*)FAKE, (float*)FAKE};
   mkv_decode_params dp = {1, 1, 1e-6f, NULL, 0};
   mkv_compress_params cp = {128, 16, 1, 1, 1, 1, 1, 1e-6f, 0};
@@ -49,7 +49,7 @@ int main(void) {
   /* layouts (LP64) as the Python binding declares them */
   CHECK(sizeof(mkv_geom) == 16);
   CHECK(sizeof(mkv_moments) == 32);
-  CHECK(sizeof(mkv_cache) == 48 && offsetof(mkv_cache, capacity) == 40);
+  CHECK(sizeof(mkv_cache) == 64 && offsetof(mkv_cache, capacity) == 40 && offsetof(mkv_cache, y_len) == 56);
   CHECK(sizeof(mkv_compress_params) == 36);
   CHECK(offsetof(mkv_compress_params, tau) == 28 && offsetof(mkv_compress_params, adaptive) == 32);
   CHECK(sizeof(mkv_decode_params) == 32 && offsetof(mkv_decode_params, C16) == 16 &&
@@ -140,7 +140,8 @@ def test_binding_structs_match_the_c_layout():
     import ctypes
     assert ctypes.sizeof(mkv.mkv_geom) == 16
     assert ctypes.sizeof(mkv.mkv_moments) == 32
-    assert ctypes.sizeof(mkv.mkv_cache) == 48 and mkv.mkv_cache.capacity.offset == 40
+    assert ctypes.sizeof(mkv.mkv_cache) == 64 and mkv.mkv_cache.capacity.offset == 40
+    assert mkv.mkv_cache.y.offset == 48 and mkv.mkv_cache.y_len.offset == 56
     assert ctypes.sizeof(mkv.mkv_compress_params) == 36
     assert mkv.mkv_compress_params.tau.offset == 28 and mkv.mkv_compress_params.adaptive.offset == 32
     assert ctypes.sizeof(mkv.mkv_decode_params) == 32 and mkv.mkv_decode_params.C16.offset == 16

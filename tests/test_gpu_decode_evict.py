@@ -21,15 +21,19 @@ from test_gpu_evict import setup
 pytestmark = pytest.mark.gpu
 
 
-def run_steps(st, b, H, G, D, budget, steps=1, correction=1, order=1, tau=1e-6, seed=0):
+def run_steps(st, b, H, G, D, budget, steps=1, correction=1, order=1, tau=1e-6, seed=0, evict_state=False):
     """`steps` calls of mkv_decode_evict_step, each with fresh queries and a
-    new token, against the oracle carrying its own state."""
+    new token, against the oracle carrying its own state.  evict_state: the
+    cache keeps y_j = S_tilde k_j across calls (mkv_cache.y, y_len)."""
     rng = np.random.default_rng(seed)
     g = mkv.geom(b, H, G, D)
     cap = st["cap"]
     pos0 = np.broadcast_to(np.arange(cap, dtype=np.int32) * 3, (b, H, cap)).copy()
     seen0 = 10 ** 6
     cache = mkv.Cache(bf16(st["K"]), bf16(st["V"]), i32(pos0), i32(st["lens"]), i32(np.full((b, H), seen0)))
+    if evict_state:
+        cache.y = torch.zeros(b, H, cap, D, device="cuda")
+        cache.y_len = torch.zeros(b, H, dtype=torch.int32, device="cuda")
     mom = mkv.Moments(i32(st["n"]), f32(st["mu_k"]), f32(st["mu_v"]), f32(st["C"]))
     ws = mkv.alloc_workspace(mkv.mkv_decode_evict_workspace_size(g, cap))
     p = mkv.mkv_decode_params(correction, order, tau)
@@ -67,7 +71,25 @@ def run_steps(st, b, H, G, D, budget, steps=1, correction=1, order=1, tau=1e-6, 
             assert_output_close(got["out"][bi, h * G:(h + 1) * G], o, f"out step {step} unit {(bi, h)}")
             np.testing.assert_allclose(got["lse"][bi, h * G:(h + 1) * G], l, rtol=1e-4, atol=1e-4)
             s.update(K=f.K, V=f.V, pos=f.pos, m=f.moments)
+        if evict_state:
+            check_y_rows(cache, mom)
     return got
+
+
+def check_y_rows(cache, mom):
+    """The cache's current y rows equal S_tilde k_j = n C k_j of the kernel's
+    own moments and rows (1e-4 of the largest, per unit)."""
+    y, y_len, K = host(cache.y), host(cache.y_len), host(cache.K).astype(np.float64)
+    n, C = host(mom.n), host(mom.C).astype(np.float64)
+    for bi in range(y.shape[0]):
+        for h in range(y.shape[1]):
+            L = int(y_len[bi, h])
+            assert 0 <= L <= int(host(cache.len)[bi, h])
+            if L == 0 or n[bi, h] == 0:
+                continue
+            want = K[bi, h, :L] @ (n[bi, h] * C[bi, h]).T
+            err = np.abs(y[bi, h, :L] - want).max()
+            assert err <= 1e-4 * np.abs(want).max(), (bi, h, err, np.abs(want).max())
 
 
 def test_tiny_several_evictions_in_one_step():
@@ -107,3 +129,20 @@ def test_group_8_d64_batch():
     rng = np.random.default_rng(36)
     st = setup(rng, 2, 2, 8, 64, [100, 64, 65, 99], 128, [10, 0, 200, 3])
     run_steps(st, 2, 2, 8, 64, 64, steps=2, seed=7)
+
+
+@pytest.mark.parametrize("G", [4, 1])
+def test_continuous_with_eviction_state(G):
+    """Continuous eviction with y_j = S_tilde k_j kept in the cache across
+    calls: the first call fills it, the next ones compute it only for the
+    appended token; every step against the oracle, and the kept y rows
+    against n C k_j of the kernel's own moments."""
+    rng = np.random.default_rng(40 + G)
+    st = setup(rng, 1, 8, G, 128, [512] * 8, 576, [3000] * 6 + [0] * 2)
+    run_steps(st, 1, 8, G, 128, 512, steps=4, seed=8, evict_state=True)
+
+
+def test_eviction_state_several_evictions_per_step_d64():
+    rng = np.random.default_rng(42)
+    st = setup(rng, 2, 2, 2, 64, [40, 33, 45, 20], 48, [0, 25, 3, 7])
+    run_steps(st, 2, 2, 2, 64, 24, steps=3, seed=9, evict_state=True)

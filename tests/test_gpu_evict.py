@@ -162,3 +162,77 @@ def test_evict_many_units():
     st = setup(rng, 3, 8, 2, 128, [190] * 24, 200, [400, 0] * 12)
     gpu = run_case(st, 3, 8, 2, 128, 140, True)
     check(gpu, st)
+
+
+def test_periodic_rounds_with_eviction_state():
+    """Rounds of 64 appended tokens (mkv_decode_step appends, which leave the
+    kept y rows alone) and one mkv_evict_append back to the budget, the cache
+    keeping y_j = S_tilde k_j across calls: each round against the oracle
+    following the kernel's evictions, and the kept y rows against n C k_j."""
+    from test_gpu_decode_evict import check_y_rows
+    rng = np.random.default_rng(51)
+    b, H, G, D, B, cap, every = 1, 8, 4, 128, 128, 192, 64
+    st = setup(rng, b, H, G, D, [B] * H, cap, [4000] * 5 + [0] * 3)
+    g = mkv.geom(b, H, G, D)
+    pos0 = np.broadcast_to(np.arange(cap, dtype=np.int32) * 3, (b, H, cap)).copy()
+    cache = mkv.Cache(bf16(st["K"]), bf16(st["V"]), i32(pos0), i32(st["lens"]), i32(np.full((b, H), 10 ** 6)),
+                      torch.zeros(b, H, cap, D, device="cuda"), torch.zeros(b, H, dtype=torch.int32, device="cuda"))
+    mom = mkv.Moments(i32(st["n"]), f32(st["mu_k"]), f32(st["mu_v"]), f32(st["C"]))
+    ws_d = mkv.alloc_workspace(mkv.mkv_decode_workspace_size(g, cap))
+    ws_e = mkv.alloc_workspace(mkv.mkv_evict_workspace_size(g, cap))
+    out = torch.empty(b, H * G, D, device="cuda")
+    state = {}
+    for h in range(H):
+        state[h] = dict(K=st["K"][0, h, :B], V=st["V"][0, h, :B], pos=pos0[0, h, :B].astype(np.int64),
+                        m=O.Moments(int(st["n"][0, h]), st["mu_k"][0, h], st["mu_v"][0, h], st["C"][0, h]))
+    seen = 10 ** 6
+    for rnd in range(3):
+        kn = bf16_round(1.5 * rng.standard_normal((every, b, H, D)))
+        vn = bf16_round(rng.standard_normal((every, b, H, D)))
+        q = bf16_round(2.0 * rng.standard_normal((b, H * G, D)))
+        for i in range(every):
+            mkv.mkv_decode_step(g, bf16(q), bf16(kn[i]), bf16(vn[i]), cache, mom, mkv.mkv_decode_params(1, 1, 1e-6),
+                                out, None, ws_d)
+        mkv.mkv_evict_append(g, bf16(q), None, None, B, cache, mom, 1e-6, ws_e)
+        assert mkv.mkv_get_device_error(ws_d)[0] == 0 and mkv.mkv_get_device_error(ws_e)[0] == 0
+        gpu = dict(K=host(cache.K), V=host(cache.V), pos=host(cache.pos), len=host(cache.len), n=host(mom.n),
+                   mu_k=host(mom.mu_k), mu_v=host(mom.mu_v), C=host(mom.C))
+        assert (host(cache.y_len) == B).all()
+        for h in range(H):
+            s0 = state[h]
+            K = np.vstack([s0["K"], kn[:, 0, h]])
+            V = np.vstack([s0["V"], vn[:, 0, h]])
+            pos = np.append(s0["pos"], seen + np.arange(every))
+            f = check_evicted_unit(gpu, 0, h, q[0, h * G:(h + 1) * G], K, V, pos, s0["m"], B, 1e-6)
+            state[h] = dict(K=f.K, V=f.V, pos=f.pos, m=f.moments)
+        seen += every
+        check_y_rows(cache, mom)
+
+
+def test_eviction_state_reset_by_compress_and_large_capacity():
+    """mkv_compress leaves no y row current; the eviction kernel for
+    capacities past the register kernel's does not keep y either."""
+    from paper_2606_01563_gb300.inputs import WORKLOADS, Generator
+    wl = WORKLOADS["tiny_d64_t1k"]
+    K, V, Q = Generator(wl, seed=2).prefill()
+    G_ = wl.geom
+    g = mkv.geom(G_.batch, G_.n_kv_heads, G_.group, G_.head_dim)
+    cache = mkv.alloc_cache(g, wl.budget + 4, evict_state=True)
+    cache.y_len.fill_(7)
+    p = mkv.mkv_compress_params(wl.budget, wl.window, 1, 1, 1, 1, 1, 1e-6)
+    ws = mkv.alloc_workspace(mkv.mkv_compress_workspace_size(g, wl.T, p))
+    mkv.mkv_compress(g, wl.T, bf16(K), bf16(V), bf16(Q), p, cache, mkv.alloc_moments(g), ws)
+    assert mkv.mkv_get_device_error(ws)[0] == 0
+    assert (host(cache.y_len) == 0).all()
+    # capacity 2400 runs the single-CTA kernel: y_len goes to 0 after its evictions
+    rng = np.random.default_rng(32)
+    st = setup(rng, 1, 1, 4, 128, [2300], 2400, [500])
+    g = mkv.geom(1, 1, 4, 128)
+    pos0 = np.arange(2400, dtype=np.int32)[None, None] * 3
+    c = mkv.Cache(bf16(st["K"]), bf16(st["V"]), i32(pos0), i32(st["lens"]), i32(np.full((1, 1), 10 ** 6)),
+                  torch.zeros(1, 1, 2400, 128, device="cuda"), torch.full((1, 1), 2300, dtype=torch.int32, device="cuda"))
+    mom = mkv.Moments(i32(st["n"]), f32(st["mu_k"]), f32(st["mu_v"]), f32(st["C"]))
+    ws = mkv.alloc_workspace(mkv.mkv_evict_workspace_size(g, 2400))
+    mkv.mkv_evict_append(g, bf16(st["q"]), None, None, 2290, c, mom, 1e-6, ws)
+    assert mkv.mkv_get_device_error(ws)[0] == 0
+    assert int(host(c.y_len)[0, 0]) == 0 and int(host(c.len)[0, 0]) == 2290

@@ -87,6 +87,9 @@ def test_decode_validation(L):
     assert decode(L, g, p=mkv.mkv_decode_params(1, 1, -1.0)) == 1  # tau
     assert decode(L, g, cache=mkv.mkv_cache(FAKE, FAKE, FAKE, FAKE, FAKE, 0)) == 1
     assert decode(L, g, cache=mkv.mkv_cache(FAKE + 2, FAKE, FAKE, FAKE, FAKE, 64)) == 1  # misaligned K
+    assert decode(L, g, cache=mkv.mkv_cache(FAKE, FAKE, FAKE, FAKE, FAKE, 64, FAKE, None)) == 1  # y without y_len
+    assert decode(L, g, cache=mkv.mkv_cache(FAKE, FAKE, FAKE, FAKE, FAKE, 64, None, FAKE)) == 1  # y_len without y
+    assert decode(L, g, cache=mkv.mkv_cache(FAKE, FAKE, FAKE, FAKE, FAKE, 64, FAKE + 8, FAKE)) == 1  # misaligned y
     assert decode(L, g, ws=None) == 7
     assert decode(L, g, wsb=16) == 7
     assert decode(L, g, ws=FAKE + 8) == 7                    # misaligned workspace
