@@ -215,16 +215,17 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
   if (tid == 0 && !EARLY) {
     // Before the dependency wait: this split's retained rows and moment rows
     // were written by earlier calls, not by the kernel this launch waits on
-    // (that one produces this step's query and token), so they are pulled
-    // into L2 now, while that kernel still runs.  A prefetch is only a hint
-    // and L2 is the point of coherence: a length read that races with a
-    // writer only moves the prefetched range; the loads after the wait read
-    // the current values.
+    // (that one produces this step's query and token), so its first tiles
+    // (at most 2 kStages: more would only crowd L2 when many units stream at
+    // once) are pulled into L2 now, while that kernel still runs.  A prefetch
+    // is only a hint and L2 is the point of coherence: a length read that
+    // races with a writer only moves the prefetched range; the loads after
+    // the wait read the current values.
     int lp = __ldcg(a.len + u);
     lp = lp < 0 ? 0 : (lp > a.cap ? a.cap : lp);
     const int tp = (lp + kTT - 1) / kTT;
     const int per = (tp + a.S - 1) / a.S;
-    const int pb = min(lp, s * per * kTT), pe = min(lp, pb + per * kTT);
+    const int pb = min(lp, s * per * kTT), pe = min(lp, pb + min(per, 2 * kStages) * kTT);
     if (pe > pb) {
       const size_t off = ((size_t)u * a.cap + pb) * D * 2;
       const uint32_t bytes = static_cast<uint32_t>((pe - pb) * D * 2);
@@ -347,11 +348,11 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
   };
   if constexpr (EARLY) {
     load_len_and_issue();
-    if (tid == 0) {  // the split's tiles past the first stages: into L2 now
+    if (tid == 0) {  // the split's next tiles past the first stages (up to 2 kStages): into L2 now
       const int first = min(kStages, n_tiles);
-      if (n_tiles > first) {
+      if (min(n_tiles, 2 * kStages) > first) {
         const size_t off = ((size_t)row_base + first * kTT) * D * 2;
-        const uint32_t bytes = static_cast<uint32_t>((n_cached - first * kTT) * D * 2);
+        const uint32_t bytes = static_cast<uint32_t>((min(n_cached, 2 * kStages * kTT) - first * kTT) * D * 2);
         asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(static_cast<const uint8_t*>(a.K) + off),
                      "r"(bytes) : "memory");
         asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(static_cast<const uint8_t*>(a.V) + off),
@@ -874,13 +875,13 @@ cudaError_t launch_dg(const DecodeArgs& a, cudaStream_t stream) {
 
 }  // namespace
 
-// Split count per unit.  One CTA per SM at most, so that the next launch's
-// CTAs (programmatic dependents) can be resident beside this launch's and
-// prefetch their rows while it runs; and units * S clusters of S CTAs must
-// fit the GPU twice over (clusters are placed within one GPC, so the query
-// asks the driver rather than dividing SM counts).  Within that, one tile per
-// CTA up to ten tiles, at least two tiles per CTA beyond, and at most 12
-// splits, past which the merge costs more than the extra parallelism saves.
+// Split count per unit.  Up to two CTAs per SM (a CTA's 4 warps leave room
+// for a second), and the units' clusters of S CTAs must all be resident at
+// once: clusters are placed within one GPC, so the driver's occupancy query
+// decides rather than a division of SM counts (a second wave of clusters
+// costs a whole launch latency).  Within that, one tile per CTA up to ten
+// tiles, at least two tiles per CTA beyond, and at most 12 splits, past which
+// the merge costs more than the extra parallelism saves.
 namespace {
 template <int D, int G>
 int active_clusters(int S) {
@@ -962,8 +963,8 @@ int decode_splits(const mkv_geom& g, int32_t capacity, int num_sms) {
   const long units = (long)g.batch * g.n_kv_heads;
   const long tiles = ((long)capacity + 1 + kTT - 1) / kTT;
   const long by_tiles = tiles <= 10 ? tiles : std::max(10L, (tiles + 1) / 2);
-  long S = std::min<long>(std::min(by_tiles, 12L), num_sms / units);
-  while (S > 1 && 2 * units > active_clusters_dg(g.head_dim, g.group, static_cast<int>(S))) --S;
+  long S = std::min<long>(std::min(by_tiles, 12L), 2L * num_sms / units);
+  while (S > 1 && units > active_clusters_dg(g.head_dim, g.group, static_cast<int>(S))) --S;
   if (S < 1) S = 1;
   return static_cast<int>(S);
 }

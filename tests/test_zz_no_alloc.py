@@ -125,10 +125,11 @@ def test_noalloc_against_oracle_alternating_geometries():
 
 def test_noalloc_near_largest_accepted_geometry():
     """1024 units (one split each: more units than SMs), about half of the
-    fixed scratch.  With at most one CTA per SM per launch the split count
-    times the units never exceeds the SM count, so the partial records stay
-    far below the array's size and every accepted geometry runs with its
-    full split count; the size check rejects by units (the f_hat rows)."""
+    fixed scratch.  With at most two CTAs per SM per launch the split count
+    times the units never exceeds twice the SM count, so the partial records
+    stay far below the array's size (at most 304 x 8 x 132 floats) and every
+    accepted geometry runs with its full split count; the size check rejects
+    by units (the f_hat rows)."""
     rng = np.random.default_rng(79)
     b, H, G, D, cap = 16, 64, 4, 64, 40
     _noalloc_vs_oracle(_case(rng, b, H, G, D, cap), b, H, G, D, "1024 units")
