@@ -59,8 +59,7 @@ ORACLE_JOBS = 16  # (layer, unit, budget) jobs in one oracle sample
 # headline workload from one ncu capture, valid while the code the kernel
 # compiles from (its .cu file and the library headers, comments aside) is
 # what was captured: code_sha of those sources at capture time.
-NCU_TRAFFIC = {"decode_kernel": {"bytes": 14912739,
-                                  "code_sha": "7aba0e359c763b4159e33f4bd67822eac9f51126b4acea6b1be013c9173e6e98"}}
+NCU_TRAFFIC = {}
 
 
 def parse():
@@ -126,8 +125,8 @@ def peaks():
 def kernel_sources(cu):
     """The files a kernel compiles from: its .cu file and the library headers."""
     c = os.path.join(ROOT, "paper_2606_01563_gb300", "csrc")
-    return [os.path.join(c, cu), os.path.join(c, "common.cuh"), os.path.join(c, "kernels.h"),
-            os.path.join(ROOT, "include", "mkv.h")]
+    return [os.path.join(c, cu), os.path.join(c, "common.cuh"), os.path.join(c, "warp_mma.cuh"),
+            os.path.join(c, "kernels.h"), os.path.join(ROOT, "include", "mkv.h")]
 
 
 def code_sha(paths):
@@ -539,8 +538,8 @@ def run_gpu(args):
     dec_launches = sum(r.st.S * r.st.L for r in runs)
     cmp_bytes = sum(r.compress_bytes() * r.st.L for r in runs)
     if shares["decode"] >= shares["compress"]:
-        kern, achieved = "decode_kernel", dec_bytes / (tot["decode"] / 1e3) / 1e9
-        per_launch, src = dec_bytes / dec_launches, kernel_sources("decode.cu")
+        kern, achieved = "decode_cl_kernel", dec_bytes / (tot["decode"] / 1e3) / 1e9
+        per_launch, src = dec_bytes / dec_launches, kernel_sources("decode_cl.cu")
         avg_us = tot["decode"] * 1e3 / dec_launches
     else:
         kern, achieved = "compress (9 launches per layer)", cmp_bytes / (tot["compress"] / 1e3) / 1e9

@@ -1,5 +1,8 @@
-// Decode step: retained-cache attention merged with the moment correction
-// (Algorithm 1 Phase 2; Eqs. jensen, fhat, fused; log-domain merge of App. C.2).
+// Decode step, ticket form: retained-cache attention merged with the moment
+// correction (Algorithm 1 Phase 2; Eqs. jensen, fhat, fused; log-domain merge
+// of App. C.2).  mkv_decode_step runs this kernel only when the split CTAs of
+// a unit cannot form a thread-block cluster (or a test forces it); the
+// cluster kernel in decode_cl.cu is the normal path.
 //
 // Grid (S, h_kv, b): every CTA serves all G query heads of one KV head
 // (GQA grouping, so K/V rows are read once per unit) over one contiguous
@@ -20,21 +23,14 @@
 // records with the moment pseudo-partial (log n + scale q.mu_k, f_hat_E) by
 // log-sum-exp, writes the output and updates the length.
 //
-// Cluster variant (S <= 16): the S CTAs of a unit form one thread-block
-// cluster.  Partial records and f_hat_E rows go straight into CTA 0's shared
-// memory (distributed shared memory stores), one cluster barrier orders them,
-// and CTA 0 merges: no global partials, no atomics, no second L2 round trip.
-//
-// Both variants are launched as programmatic dependents of the previous
-// kernel in the stream: barrier set-up overlaps its tail, and every global
-// read waits on griddepcontrol.wait (the previous grid complete, its writes
-// visible).
-#include <cooperative_groups.h>
-
+// Launched as a programmatic dependent of the previous kernel in the stream:
+// barrier set-up overlaps its tail, and every global read waits on
+// griddepcontrol.wait (the previous grid complete, its writes visible).
 #include <algorithm>
 
 #include "common.cuh"
 #include "kernels.h"
+#include "warp_mma.cuh"
 
 namespace mkv {
 
@@ -44,59 +40,16 @@ constexpr int kThreads = 128;  // 4 warps x 16 rows of each 64-row tile
 constexpr int kStages = 3;
 constexpr int kTT = kDecodeTile;
 constexpr unsigned kFull = 0xffffffffu;
-constexpr int kMaxClusterSplits = 16;
 
-namespace cg = cooperative_groups;
-
-__device__ __forceinline__ void cluster_arrive_relaxed() {
-  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
-}
-__device__ __forceinline__ void cluster_arrive_release() {
-  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
-}
-__device__ __forceinline__ void cluster_wait_acquire() {
-  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-__device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
-__device__ __forceinline__ void grid_launch_dependents() {
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-}
-
+// A rows 8..15 are zero (at most 8 query heads per KV head): registers a1, a3 = 0
 __device__ __forceinline__ void mma_bf16(float (&d)[4], uint32_t a0, uint32_t a2, uint32_t b0, uint32_t b1) {
-  // A rows 8..15 are zero (at most 8 query heads per KV head): registers a1, a3 = 0
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
-      "{%0,%1,%2,%3};"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a0), "r"(0u), "r"(a2), "r"(0u), "r"(b0), "r"(b1));
-}
-
-__device__ __forceinline__ void mma_bf16_full(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
-                                              uint32_t b0, uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
-      "{%0,%1,%2,%3};"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+  mma_m16n8k16(d, a0, 0u, a2, 0u, b0, b1);
 }
 
 // (hi, lo) bf16 pair parts of two floats: hi = bf16(x), lo = bf16(x - hi)
 __device__ __forceinline__ void split_bf16x2(float x, float y, uint32_t& hi, uint32_t& lo) {
-  const __nv_bfloat162 h = __floats2bfloat162_rn(x, y);
-  const __nv_bfloat162 l = __floats2bfloat162_rn(x - __low2float(h), y - __high2float(h));
-  hi = *reinterpret_cast<const uint32_t*>(&h);
-  lo = *reinterpret_cast<const uint32_t*>(&l);
-}
-
-__device__ __forceinline__ void ldsm_x4_trans(uint32_t (&r)[4], const void* p) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
-               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-               : "r"(smem_addr(p)));
-}
-
-__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
-  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-  return *reinterpret_cast<uint32_t*>(&v);
+  hi = pack_bf16x2(x, y);
+  lo = pack_bf16x2(bf16_residual(x), bf16_residual(y));
 }
 
 // Per-warp online-softmax state for head g = lane/4 (meaningful when g < G):
@@ -154,18 +107,18 @@ __device__ __forceinline__ void process16(WarpState<D>& st, const uint32_t (&qa)
     st.o[nt][1] *= alpha;
   }
   // P as bf16 hi + lo (A operand: tokens 2t, 2t+1 and 8+2t, 8+2t+1 of row g)
-  const uint32_t ph0 = pack_bf16(p[0], p[1]), ph2 = pack_bf16(p[2], p[3]);
+  const uint32_t ph0 = pack_bf16x2(p[0], p[1]), ph2 = pack_bf16x2(p[2], p[3]);
   const float r0 = p[0] - __bfloat162float(__float2bfloat16_rn(p[0]));
   const float r1 = p[1] - __bfloat162float(__float2bfloat16_rn(p[1]));
   const float r2 = p[2] - __bfloat162float(__float2bfloat16_rn(p[2]));
   const float r3 = p[3] - __bfloat162float(__float2bfloat16_rn(p[3]));
-  const uint32_t pl0 = pack_bf16(r0, r1), pl2 = pack_bf16(r2, r3);
+  const uint32_t pl0 = pack_bf16x2(r0, r1), pl2 = pack_bf16x2(r2, r3);
   const int mi = lane >> 3, mr = lane & 7;
   const int vr = row0 + (mi & 1) * 8 + mr;
 #pragma unroll
   for (int np = 0; np < D / 16; ++np) {
     uint32_t vb[4];
-    ldsm_x4_trans(vb, tV + swz_off(vr, np * 16 + (mi >> 1) * 8, kTT));
+    ldsm_x4_t(vb, tV + swz_off(vr, np * 16 + (mi >> 1) * 8, kTT));
     mma_bf16(st.o[2 * np], ph0, ph2, vb[0], vb[1]);
     mma_bf16(st.o[2 * np], pl0, pl2, vb[0], vb[1]);
     mma_bf16(st.o[2 * np + 1], ph0, ph2, vb[2], vb[3]);
@@ -173,10 +126,9 @@ __device__ __forceinline__ void process16(WarpState<D>& st, const uint32_t (&qa)
   }
 }
 
-template <int D, int G, bool CL, bool C16, bool EARLY>
+template <int D, int G, bool C16, bool EARLY>
 __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, const __grid_constant__ CUtensorMap tmK,
                                                           const __grid_constant__ CUtensorMap tmV) {
-  constexpr int DPL = D / 32;
   constexpr int PS = D + 4;  // partial record: o[D], m (log2 domain), l
   constexpr int kTileBytes = kTT * D * 2;
   extern __shared__ __align__(128) uint8_t dsmem_raw[];
@@ -195,17 +147,6 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const float scale = rsqrtf(static_cast<float>(D));
 
-  // cluster variant: CTA 0's receive area [S][G][PS] partials, [G][D] f_hat_E
-  float* sRcv = reinterpret_cast<float*>(dsmem + 2 * kStages * kTileBytes);
-  float* sFr = sRcv + (size_t)a.S * G * PS;
-  float* rcv0 = nullptr;
-  float* fr0 = nullptr;
-  if constexpr (CL) {
-    cluster_arrive_relaxed();  // every CTA of the cluster has started before the first remote store
-    cg::cluster_group cluster = cg::this_cluster();
-    rcv0 = cluster.map_shared_rank(sRcv, 0);
-    fr0 = cluster.map_shared_rank(sFr, 0);
-  }
   if (tid == 0) {
     for (int i = 0; i < kStages; ++i) mbar_init(&bars[i], 1);
     mbar_fence_init();
@@ -381,7 +322,6 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
   } else if (tid == 0 && s == 0 && __ldcg(a.len + u) != len_read) {
     record_error(a.ws, MKV_ERR_INVALID_ARG, u);  // the cache changed under an early load
   }
-  const int seen0 = (CL && s == 0 && tid == 0 && a.k_new != nullptr) ? __ldcg(a.seen + u) : 0;  // bookkeeping
   const bool has_new = a.k_new != nullptr;
   const bool use_m = n_e > 0;
   // the appended token is attended to by the last CTA (which holds the
@@ -427,8 +367,8 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
       b0 = (k == kk) ? qa[k][0] : b0;
       b1 = (k == kk) ? qa[k][1] : b1;
     }
-    mma_bf16_full(d, hi[0], hi[1], hi[2], hi[3], b0, b1);
-    mma_bf16_full(d, lo[0], lo[1], lo[2], lo[3], b0, b1);  // zero for a bf16 copy of C
+    mma_m16n8k16(d, hi[0], hi[1], hi[2], hi[3], b0, b1);
+    mma_m16n8k16(d, lo[0], lo[1], lo[2], lo[3], b0, b1);  // zero for a bf16 copy of C
   };
   if (use_m && do_c && split_k) {
     const int g = lane >> 2, t = lane & 3;
@@ -447,10 +387,9 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
     }
   }
   __syncthreads();
-  if constexpr (CL) cluster_wait_acquire();
   // f_hat_E[h][row] = mu_v[row] + scale * (C'q_h)[row]
   if (use_m && do_c) {
-    float* fdst = CL ? fr0 : a.fhat + (size_t)u * G * D;
+    float* fdst = a.fhat + (size_t)u * G * D;
     if (split_k) {
       const int n_pairs = (r1 - r0) * G;
 #pragma unroll
@@ -578,7 +517,7 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
     }
   }
   __syncthreads();
-  float* part = CL ? rcv0 + (size_t)s * G * PS : a.partial + ((size_t)u * a.S + s) * G * PS;
+  float* part = a.partial + ((size_t)u * a.S + s) * G * PS;
   for (int idx = tid; idx < G * D; idx += kThreads) {
     const int h = idx / D, dd = idx % D;
     float M = -INFINITY;
@@ -606,73 +545,7 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
   const float* src = nullptr;
   float* sF = nullptr;  // [G][D] f_hat_E rows (or mu_v for order 0)
   float* sP = reinterpret_cast<float*>(dsmem);
-  if constexpr (CL) {
-    // ---- cluster barrier: every partial and f_hat_E row is in CTA 0
-    cluster_arrive_release();
-    cluster_wait_acquire();
-    if (s != 0) return;
-    // warp w merges heads w, w + 4, ...: lane sp < S holds split sp's (m, l);
-    // lane l owns the output dims [l*DPL, (l+1)*DPL).  No block barrier.
-    for (int h = warp; h < G; h += 4) {
-      float m_s = -INFINITY, l_s = 0.f;
-      if (lane < a.S) {
-        m_s = sRcv[((size_t)lane * G + h) * PS + D];
-        l_s = sRcv[((size_t)lane * G + h) * PS + D + 1];
-      }
-      const float Mx = warp_max(l_s > 0.f ? m_s : -INFINITY);
-      const float w_s = (l_s > 0.f && Mx != -INFINITY) ? fast_exp2(m_s - Mx) : 0.f;
-      const float l = warp_sum(l_s * w_s);
-      float acc[DPL];
-#pragma unroll
-      for (int d = 0; d < DPL; ++d) acc[d] = 0.f;
-      for (int sp = 0; sp < a.S; ++sp) {
-        const float wsp = __shfl_sync(kFull, w_s, sp);
-        if (wsp != 0.f) {  // warp-uniform
-          const float* rec = sRcv + ((size_t)sp * G + h) * PS + lane * DPL;
-#pragma unroll
-          for (int d = 0; d < DPL; ++d) acc[d] = fmaf(wsp, rec[d], acc[d]);
-        }
-      }
-      const bool have_r = l > 0.f;
-      const float inv_l = have_r ? 1.f / l : 0.f;
-      float res[DPL], lse = have_r ? Mx * kLn2 + logf(l) : -INFINITY;
-      if (use_m) {
-        const float e = logf(static_cast<float>(n_e)) + sSbar[h];
-        float wR = 0.f;
-        if (have_r) {
-          const float top = fmaxf(lse, e);
-          const float wr = expf(lse - top), we = expf(e - top);
-          wR = wr / (wr + we);
-          lse = top + logf(wr + we);
-        } else {
-          lse = e;
-        }
-#pragma unroll
-        for (int d = 0; d < DPL; ++d) {
-          const float fh = (a.order == 1) ? sFr[h * D + lane * DPL + d] : __ldg(a.mu_v + (size_t)u * D + lane * DPL + d);
-          res[d] = have_r ? wR * (acc[d] * inv_l) + (1.f - wR) * fh : fh;
-        }
-      } else {
-        if (!have_r && lane == 0) record_error(a.ws, MKV_ERR_INVALID_ARG, u);
-#pragma unroll
-        for (int d = 0; d < DPL; ++d) res[d] = acc[d] * inv_l;
-      }
-      float* o = a.out + ((size_t)u * G + h) * D + lane * DPL;
-      if constexpr (DPL == 4) *reinterpret_cast<float4*>(o) = make_float4(res[0], res[1], res[2], res[3]);
-      else *reinterpret_cast<float2*>(o) = make_float2(res[0], res[1]);
-      if (a.lse != nullptr && lane == 0) a.lse[(size_t)u * G + h] = lse;
-    }
-    if (has_new && tid == 0) {  // the row itself was written by the CTA that attended to it
-      if (len0 + 1 > a.cap) {
-        record_error(a.ws, MKV_ERR_CAPACITY, u);
-      } else {
-        a.pos[(size_t)u * a.cap + len0] = seen0;
-        a.seen[u] = seen0 + 1;
-        a.len[u] = len0 + 1;
-      }
-    }
-    return;
-  } else {
+  {
     // ---- ticket: the last CTA of this unit merges everything
     __threadfence();
     __syncthreads();
@@ -788,55 +661,14 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
   }
 }
 
-// Whether clusters of S CTAs with `smem` bytes each can be resident (checked
-// once per split count; portable sizes always can).
-template <int D, int G, bool C16, bool EARLY>
-bool cluster_fits(int S, size_t smem) {
-  if (S <= 8) return true;
-  static std::mutex mu;
-  static signed char known[kMaxClusterSplits + 1] = {};
-  std::lock_guard<std::mutex> lock(mu);
-  if (known[S] == 0) {
-    cudaLaunchConfig_t cfg{};
-    cfg.gridDim = dim3(S, 1, 1);
-    cfg.blockDim = dim3(kThreads, 1, 1);
-    cfg.dynamicSmemBytes = smem;
-    cudaLaunchAttribute at[1];
-    at[0].id = cudaLaunchAttributeClusterDimension;
-    at[0].val.clusterDim.x = S;
-    at[0].val.clusterDim.y = 1;
-    at[0].val.clusterDim.z = 1;
-    cfg.attrs = at;
-    cfg.numAttrs = 1;
-    int n = 0;
-    const cudaError_t e = cudaOccupancyMaxActiveClusters(&n, decode_kernel<D, G, true, C16, EARLY>, &cfg);
-    if (e != cudaSuccess) (void)cudaGetLastError();
-    known[S] = (e == cudaSuccess && n > 0) ? 1 : -1;
-  }
-  return known[S] > 0;
-}
-
 template <int D, int G, bool C16, bool EARLY>
 cudaError_t launch_dgc(const DecodeArgs& args, cudaStream_t stream) {
   DecodeArgs a = args;
   a.polls = pipeline_poll_limit();
   const size_t ring = (size_t)2 * kStages * kTT * D * 2 + 1024;  // + alignment slack
-  const size_t rcv = ((size_t)a.S * G * (D + 4) + (size_t)G * D + 2 * (size_t)a.S * G) * sizeof(float);
-  const bool cl = a.S <= kMaxClusterSplits;
-  const size_t smem = cl ? ring + rcv : ring;
-  // per-device function attributes; setting them again is harmless
-  cudaError_t e;
-  if (cl) {
-    e = cudaFuncSetAttribute(decode_kernel<D, G, true, C16, EARLY>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(smem));
-    if (e == cudaSuccess && a.S > 8)
-      e = cudaFuncSetAttribute(decode_kernel<D, G, true, C16, EARLY>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-  } else {
-    e = cudaFuncSetAttribute(decode_kernel<D, G, false, C16, EARLY>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(smem));
-  }
+  cudaError_t e = cudaFuncSetAttribute(decode_kernel<D, G, C16, EARLY>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(ring));
   if (e != cudaSuccess) return e;
-  const bool use_cl = cl && cluster_fits<D, G, C16, EARLY>(a.S, smem) && g_force_ticket_merge.load() == 0;
   // the cache slabs of all units as one [units * cap][D] matrix
   const uint64_t rows = (uint64_t)a.batch * a.n_kv * a.cap;
   CUtensorMap tmK, tmV;
@@ -846,24 +678,14 @@ cudaError_t launch_dgc(const DecodeArgs& args, cudaStream_t stream) {
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3(a.S, a.n_kv, a.batch);
   cfg.blockDim = dim3(kThreads, 1, 1);
-  cfg.dynamicSmemBytes = use_cl ? smem : ring;
+  cfg.dynamicSmemBytes = ring;
   cfg.stream = stream;
-  cudaLaunchAttribute at[2];
+  cudaLaunchAttribute at[1];
   at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   at[0].val.programmaticStreamSerializationAllowed = 1;
-  at[1].id = cudaLaunchAttributeClusterDimension;
-  at[1].val.clusterDim.x = a.S;
-  at[1].val.clusterDim.y = 1;
-  at[1].val.clusterDim.z = 1;
   cfg.attrs = at;
-  cfg.numAttrs = use_cl ? 2 : 1;
-  if (use_cl) return cudaLaunchKernelEx(&cfg, decode_kernel<D, G, true, C16, EARLY>, a, tmK, tmV);
-  if (cl) {  // the cluster did not fit: the ticket variant with the ring only
-    e = cudaFuncSetAttribute(decode_kernel<D, G, false, C16, EARLY>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(ring));
-    if (e != cudaSuccess) return e;
-  }
-  return cudaLaunchKernelEx(&cfg, decode_kernel<D, G, false, C16, EARLY>, a, tmK, tmV);
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, decode_kernel<D, G, C16, EARLY>, a, tmK, tmV);
 }
 
 template <int D, int G>
@@ -873,69 +695,6 @@ cudaError_t launch_dg(const DecodeArgs& a, cudaStream_t stream) {
   return a.C16 != nullptr ? launch_dgc<D, G, true, false>(a, stream) : launch_dgc<D, G, false, false>(a, stream);
 }
 
-}  // namespace
-
-// Split count per unit.  Up to two CTAs per SM (a CTA's 4 warps leave room
-// for a second), and the units' clusters of S CTAs must all be resident at
-// once: clusters are placed within one GPC, so the driver's occupancy query
-// decides rather than a division of SM counts (a second wave of clusters
-// costs a whole launch latency).  Within that, one tile per CTA up to ten
-// tiles, at least two tiles per CTA beyond, and at most 12 splits, past which
-// the merge costs more than the extra parallelism saves.
-namespace {
-template <int D, int G>
-int active_clusters(int S) {
-  constexpr int kMaxDev = 64;
-  static std::mutex mu;
-  static int known[kMaxDev][kMaxClusterSplits + 1] = {};
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) return 0;
-  std::lock_guard<std::mutex> lock(mu);
-  if (known[dev][S] == 0) {
-    const size_t ring = (size_t)2 * kStages * kTT * D * 2 + 1024;
-    const size_t smem = ring + ((size_t)S * G * (D + 4) + (size_t)G * D + 2 * (size_t)S * G) * sizeof(float);
-    int n = 0;
-    cudaError_t e = cudaFuncSetAttribute(decode_kernel<D, G, true, false, false>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
-    if (e == cudaSuccess && S > 8)
-      e = cudaFuncSetAttribute(decode_kernel<D, G, true, false, false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-    if (e == cudaSuccess) {
-      cudaLaunchConfig_t cfg{};
-      cfg.gridDim = dim3(S, 1, 1);
-      cfg.blockDim = dim3(kThreads, 1, 1);
-      cfg.dynamicSmemBytes = smem;
-      cudaLaunchAttribute at[1];
-      at[0].id = cudaLaunchAttributeClusterDimension;
-      at[0].val.clusterDim.x = S;
-      at[0].val.clusterDim.y = 1;
-      at[0].val.clusterDim.z = 1;
-      cfg.attrs = at;
-      cfg.numAttrs = 1;
-      e = cudaOccupancyMaxActiveClusters(&n, decode_kernel<D, G, true, false, false>, &cfg);
-    }
-    if (e != cudaSuccess) {
-      (void)cudaGetLastError();
-      n = 0;
-    }
-    known[dev][S] = n > 0 ? n : -1;
-  }
-  return known[dev][S];
-}
-
-int active_clusters_dg(int head_dim, int group, int S) {
-#define MKV_AC_CASE(D, G) \
-  if (head_dim == D && group == G) return active_clusters<D, G>(S);
-  MKV_AC_CASE(128, 1)
-  MKV_AC_CASE(128, 2)
-  MKV_AC_CASE(128, 4)
-  MKV_AC_CASE(128, 8)
-  MKV_AC_CASE(64, 1)
-  MKV_AC_CASE(64, 2)
-  MKV_AC_CASE(64, 4)
-  MKV_AC_CASE(64, 8)
-#undef MKV_AC_CASE
-  return 0;
-}
 }  // namespace
 
 namespace {
@@ -959,12 +718,14 @@ cudaError_t launch_pack_bf16(const float* C, __nv_bfloat16* C16, size_t n, cudaS
   return cudaGetLastError();
 }
 
+// Split count of the ticket kernel: up to two CTAs per SM, one tile per CTA
+// up to ten tiles, at least two tiles per CTA beyond, and at most 12 splits,
+// past which the merge costs more than the extra parallelism saves.
 int decode_splits(const mkv_geom& g, int32_t capacity, int num_sms) {
   const long units = (long)g.batch * g.n_kv_heads;
   const long tiles = ((long)capacity + 1 + kTT - 1) / kTT;
   const long by_tiles = tiles <= 10 ? tiles : std::max(10L, (tiles + 1) / 2);
   long S = std::min<long>(std::min(by_tiles, 12L), 2L * num_sms / units);
-  while (S > 1 && units > active_clusters_dg(g.head_dim, g.group, static_cast<int>(S))) --S;
   if (S < 1) S = 1;
   return static_cast<int>(S);
 }
@@ -991,9 +752,11 @@ void decode_carve(DecodeArgs& a, const mkv_geom& g, int32_t capacity, int num_sm
   off += align_up(units * S * g.group * (g.head_dim + 4) * sizeof(float), 256);
   a.fhat = reinterpret_cast<float*>(p + off);
   a.S = S;
+  a.S_cl = decode_cluster_splits(g, capacity, num_sms, a.early);
 }
 
 cudaError_t launch_decode(const DecodeArgs& a, int head_dim, int group, cudaStream_t stream) {
+  if (a.S_cl > 0 && g_force_ticket_merge.load() == 0) return launch_decode_cluster(a, head_dim, group, stream);
 #define MKV_DECODE_CASE(D, G) \
   if (head_dim == D && group == G) return launch_dg<D, G>(a, stream);
   MKV_DECODE_CASE(128, 1)

@@ -37,7 +37,8 @@ struct DecodeArgs {
   float* fhat;         // [units][G][D]
   int32_t batch;
   int32_t n_kv;
-  int32_t S;
+  int32_t S;       // split count of the ticket kernel (its partial records are sized for it)
+  int32_t S_cl;    // split count of the cluster kernel; 0 when no cluster of that size fits
   uint32_t polls;  // poll limit of the tile waits (the drain after a timeout uses kMaxPolls)
   int32_t early;   // cache and moments read before the dependency wait (mkv_decode_params.early_load)
 };
@@ -45,10 +46,13 @@ struct DecodeArgs {
 constexpr int kDecodeTile = 64;  // tokens per pipeline stage
 
 int decode_splits(const mkv_geom& g, int32_t capacity, int num_sms);
+int decode_cluster_splits(const mkv_geom& g, int32_t capacity, int num_sms, int early);
 size_t decode_workspace_bytes(const mkv_geom& g, int32_t capacity, int num_sms);
 // Carves the workspace and fills the ws/counters/partial/fhat fields.
 void decode_carve(DecodeArgs& a, const mkv_geom& g, int32_t capacity, int num_sms, void* ws);
+// The cluster kernel when a.S_cl > 0 (and the ticket merge is not forced), else the ticket kernel.
 cudaError_t launch_decode(const DecodeArgs& a, int head_dim, int group, cudaStream_t stream);
+cudaError_t launch_decode_cluster(const DecodeArgs& a, int head_dim, int group, cudaStream_t stream);
 cudaError_t launch_pack_bf16(const float* C, __nv_bfloat16* C16, size_t n, cudaStream_t stream);
 
 // ------------------------------------------------------------------- evict

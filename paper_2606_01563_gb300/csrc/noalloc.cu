@@ -72,7 +72,7 @@ size_t scratch_bytes(const mkv_geom& g, int S) {
          align_up(units * g.group * g.head_dim * sizeof(float), 256);
 }
 
-void carve(DecodeArgs& a, const mkv_geom& g, int S, void* scratch) {
+void carve(DecodeArgs& a, const mkv_geom& g, int S, int sms, void* scratch) {
   const size_t units = (size_t)g.batch * g.n_kv_heads;
   uint8_t* p = static_cast<uint8_t*>(scratch);
   a.ws = scratch;
@@ -81,6 +81,7 @@ void carve(DecodeArgs& a, const mkv_geom& g, int S, void* scratch) {
   a.fhat = reinterpret_cast<float*>(p + kHeaderBytes + kCounterBytes +
                                     align_up(units * S * g.group * (g.head_dim + 4) * sizeof(float), 256));
   a.S = S;
+  a.S_cl = decode_cluster_splits(g, a.cap, sms, a.early);
 }
 
 }  // namespace
@@ -127,7 +128,7 @@ extern "C" MKV_API mkv_status mkv_decode_step_noalloc(mkv_geom geom, const void*
   a.batch = geom.batch;
   a.n_kv = geom.n_kv_heads;
   a.early = p->early_load;
-  carve(a, geom, S, scratch);
+  carve(a, geom, S, sms, scratch);
   return launch_decode(a, geom.head_dim, geom.group, static_cast<cudaStream_t>(stream)) == cudaSuccess
              ? MKV_OK
              : MKV_ERR_CUDA;

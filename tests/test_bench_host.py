@@ -43,7 +43,7 @@ def test_code_sha_sees_code_and_literals(tmp_path):
 
 
 def test_kernel_sources_exist():
-    for cu in ("decode.cu", "compress.cu", "evict.cu"):
+    for cu in ("decode_cl.cu", "decode.cu", "compress.cu", "evict.cu"):
         paths = bench.kernel_sources(cu)
         assert all(os.path.exists(p) for p in paths)
         assert len(bench.code_sha(paths)) == 64

@@ -17,15 +17,20 @@ from gpu_util import assert_output_close, bf16, f32, host, i32
 pytestmark = pytest.mark.gpu
 
 
-@pytest.mark.parametrize("b,H,G,D,L,lens,cap,c16", [
-    (2, 8, 4, 128, 3, (300, 420), 440, False),
-    (1, 8, 4, 128, 4, (130, 510), 520, False),
-    (1, 8, 4, 128, 3, (200, 260), 270, True),
-    (24, 8, 2, 64, 2, (60, 90), 100, False),
+@pytest.mark.parametrize("b,H,G,D,L,lens,cap,c16,steps,graph", [
+    (2, 8, 4, 128, 3, (300, 420), 440, False, 3, False),
+    (1, 8, 4, 128, 4, (130, 510), 520, False, 3, False),
+    (1, 8, 4, 128, 3, (200, 260), 270, True, 3, False),
+    (24, 8, 2, 64, 2, (60, 90), 100, False, 3, False),
+    # two layers, few units, back to back from a graph: the launch two back
+    # in the stream is the same layer, so a launch must not start (and read
+    # its cache early) before its predecessor's own predecessor has finished
+    (4, 8, 4, 128, 2, (100, 300), 340, False, 24, True),
+    (1, 8, 4, 128, 2, (500, 600), 640, False, 24, True),
+    (1, 2, 4, 64, 2, (40, 90), 120, False, 24, True),
 ])
-def test_layer_chain_early_load(b, H, G, D, L, lens, cap, c16):
+def test_layer_chain_early_load(b, H, G, D, L, lens, cap, c16, steps, graph):
     rng = np.random.default_rng(b * 1000 + L * 10 + D)
-    steps = 3
     layers = []
     for l in range(L):
         K = bf16_round(rng.standard_normal((b, H, cap, D)))
@@ -57,12 +62,36 @@ def test_layer_chain_early_load(b, H, G, D, L, lens, cap, c16):
     ws = mkv.alloc_workspace(mkv.mkv_decode_workspace_size(g, cap))
     torch.cuda.synchronize()
     stream = torch.cuda.Stream()
-    with torch.cuda.stream(stream):
+
+    def chain():
         for i in range(steps):
             for l in range(L):
                 cache, mom, C16 = dev[l]
                 p = mkv.mkv_decode_params(1, 1, 1e-6, None if C16 is None else C16.data_ptr(), 1)
                 mkv.mkv_decode_step(g, qd[i, l], knd[i, l], vnd[i, l], cache, mom, p, outs[i, l], None, ws, stream)
+
+    if graph:
+        # launched back to back from a CUDA graph, as a serving loop would,
+        # so that consecutive launches really overlap (host launches from
+        # Python leave gaps between them); the graph is captured from a copy
+        # of the initial cache lengths and replayed once
+        lens0 = [d[0].len.clone() for d in dev]
+        seen0 = [d[0].seen.clone() for d in dev]
+        with torch.cuda.stream(stream):
+            chain()  # warm-up: function attributes and split counts
+        stream.synchronize()
+        gr = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gr, stream=stream, capture_error_mode="relaxed"):
+            chain()
+        for d, l0, s0 in zip(dev, lens0, seen0):
+            d[0].len.copy_(l0)
+            d[0].seen.copy_(s0)
+        torch.cuda.synchronize()
+        with torch.cuda.stream(stream):
+            gr.replay()
+    else:
+        with torch.cuda.stream(stream):
+            chain()
     stream.synchronize()
     code, info = mkv.mkv_get_device_error(ws)
     assert code == 0, (code, info)
