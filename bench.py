@@ -59,7 +59,8 @@ ORACLE_JOBS = 16  # (layer, unit, budget) jobs in one oracle sample
 # headline workload from one ncu capture, valid while the code the kernel
 # compiles from (its .cu file and the library headers, comments aside) is
 # what was captured: code_sha of those sources at capture time.
-NCU_TRAFFIC = {}
+NCU_TRAFFIC = {"decode_cl_kernel": {"bytes": 15275530,
+                                     "code_sha": "26e3b083a0e780442182d4f543b13d8c1b63aaa5d179e8c29c8caf19514a577a"}}
 
 
 def parse():

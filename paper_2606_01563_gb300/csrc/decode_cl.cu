@@ -149,10 +149,14 @@ __global__ void __launch_bounds__(kClThreads, 2)
   const bool corr = a.correction != 0 && a.n != nullptr;
   const bool do_c = corr && a.order == 1;
   const bool has_new = a.k_new != nullptr;
+  // Moments and cache lengths are read again at every step while the cache
+  // rows stream through: the former stay in L2 (evict_last), the latter give
+  // way first (evict_first).
+  const uint64_t pol_keep = l2_evict_last(), pol_stream = l2_evict_first();
 
   // ---- state read before (EARLY) or after the dependency wait
   int len_read = 0, len0 = 0, n_tiles = 0, n_cached = 0, row_base = 0, seen0 = 0, n_e = 0, issued = 0;
-  float2 cf[KS][4];  // producer: C' fragments of one owned 16-row block, all k-steps
+  float2 cf[KS][4];  // side warps: C' fragments of one owned 16-row block, all k-steps
   auto load_cf = [&](int j) {
     const int ra = (mlo + j) * 16 + g, rb = ra + 8;
     const bool va = do_c && j < nmt;
@@ -161,8 +165,12 @@ __global__ void __launch_bounds__(kClThreads, 2)
       const int c0 = kk * 16 + 2 * t;
       auto ld = [&](int row, int col) -> float2 {
         const size_t off = ((size_t)u * D + row) * D + col;
-        if constexpr (C16) return __bfloat1622float2(__ldg(reinterpret_cast<const __nv_bfloat162*>(a.C16 + off)));
-        else return __ldg(reinterpret_cast<const float2*>(a.C + off));
+        if constexpr (C16) {
+          const uint32_t w = ldg_hint(reinterpret_cast<const uint32_t*>(a.C16 + off), pol_keep);
+          return __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w));
+        } else {
+          return ldg_hint(reinterpret_cast<const float2*>(a.C + off), pol_keep);
+        }
       };
       cf[kk][0] = va ? ld(ra, c0) : make_float2(0.f, 0.f);
       cf[kk][1] = va ? ld(rb, c0) : make_float2(0.f, 0.f);
@@ -176,12 +184,12 @@ __global__ void __launch_bounds__(kClThreads, 2)
     mbar_arrive_expect_tx(&full[st], 2u * kTileBytes);
 #pragma unroll
     for (int bx = 0; bx < D / 64; ++bx) {
-      tma_load_2d(dk + bx * kRows * 128, &tmK, bx * 64, row_base + i * kRows, &full[st]);
-      tma_load_2d(dk + kTileBytes + bx * kRows * 128, &tmV, bx * 64, row_base + i * kRows, &full[st]);
+      tma_load_2d_hint(dk + bx * kRows * 128, &tmK, bx * 64, row_base + i * kRows, &full[st], pol_stream);
+      tma_load_2d_hint(dk + kTileBytes + bx * kRows * 128, &tmV, bx * 64, row_base + i * kRows, &full[st], pol_stream);
     }
   };
   auto prologue = [&]() {
-    len_read = __ldcg(a.len + u);
+    len_read = ldcg_hint(a.len + u, pol_keep);
     len0 = len_read;
     if (len0 < 0 || len0 > a.cap) {  // corrupt cache state: never read past the slab
       if (tid == 0 && s == 0) record_error(a.ws, MKV_ERR_CAPACITY, u);
@@ -192,7 +200,7 @@ __global__ void __launch_bounds__(kClThreads, 2)
     n_tiles = te - tb;
     n_cached = max(0, min(len0, te * kRows) - tb * kRows);
     row_base = u * a.cap + tb * kRows;
-    n_e = corr ? __ldcg(a.n + u) : 0;
+    n_e = corr ? ldcg_hint(a.n + u, pol_keep) : 0;
     if (!side) return;
     if (producer) {
       if (lane == 0) {
@@ -214,7 +222,7 @@ __global__ void __launch_bounds__(kClThreads, 2)
           asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base),
                        "r"((uint32_t)((nmt - 2) * 16 * D * (C16 ? 2 : 4))) : "memory");
         }
-        if (s == 0 && has_new) seen0 = __ldcg(a.seen + u);
+        if (s == 0 && has_new) seen0 = ldcg_hint(a.seen + u, pol_keep);
       }
       if constexpr (EARLY) {
         // The query and the new token may be written by the kernel this
@@ -232,15 +240,17 @@ __global__ void __launch_bounds__(kClThreads, 2)
         if (line != nullptr) asm volatile("prefetch.global.L2 [%0];" ::"l"(line));
       }
     }
-    if (corr && n_e > 0) {
+    if (corr) {
       // this warp's first C' block (blocks alternate between the loader and
-      // moment warps), the owned mu_v rows and mu_k
+      // moment warps), issued without waiting for the count n (unused when
+      // n = 0); the moment warp also stages the owned mu_v rows and mu_k (its
+      // stores wait for those loads, the loader must not: its tile copies
+      // and refills come first)
       load_cf(warp - kLoaderWarp);
-      // the mu_v rows of this warp's own blocks (read by this warp only)
-      for (int j = warp - kLoaderWarp + 2 * (lane >> 4); j < nmt; j += 4)
-        sMuv[j * 16 + (lane & 15)] = __ldg(a.mu_v + (size_t)u * D + (mlo + j) * 16 + (lane & 15));
-      if (producer)
-        for (int i = lane; i < D; i += 32) sMuk[i] = __ldg(a.mu_k + (size_t)u * D + i);
+      if (!producer) {
+        for (int i = lane; i < own_d; i += 32) sMuv[i] = ldg_hint(a.mu_v + (size_t)u * D + mlo * 16 + i, pol_keep);
+        for (int i = lane; i < D; i += 32) sMuk[i] = ldg_hint(a.mu_k + (size_t)u * D + i, pol_keep);
+      }
     }
   };
   if constexpr (EARLY) prologue();
@@ -270,8 +280,6 @@ __global__ void __launch_bounds__(kClThreads, 2)
       kvc = reinterpret_cast<const uint4*>(
           reinterpret_cast<const __nv_bfloat16*>(lane < D / 8 ? a.k_new : a.v_new) + (size_t)u * D)[lane % (D / 8)];
     if (producer) {
-      if (EARLY && s == 0 && lane == 0 && __ldcg(a.len + u) != len_read)
-        record_error(a.ws, MKV_ERR_INVALID_ARG, u);  // the cache changed under an early load
       // refills: stage i % NST is free once the four attending warps released tile i - NST
       if (lane == 0) {
         for (; issued < n_tiles; ++issued) {
@@ -284,16 +292,19 @@ __global__ void __launch_bounds__(kClThreads, 2)
       }
       __syncwarp();
     }
-    __syncwarp();  // this warp's mu_v rows are in place
+    __syncwarp();
+    named_sync(3, 64);  // the moment warp's mu_v and mu_k rows are in place
     if (use_m) {
       // f_hat_E rows of the owned blocks, blocks alternating between the two
       // side warps: mu_v + scale C'q on the tensor cores (A = C' rows split
       // into bf16 hi + lo parts, clamp of Eq. fused applied here; B = the q
-      // fragments), written as sF[row][head]
+      // fragments), written as sF[row][head].  Four independent accumulator
+      // chains (k-step parity x part): these products share the tensor pipe
+      // with an attending warp's tiles.
       const float nf = static_cast<float>(n_e), tau = a.tau;
       for (int j = warp - kLoaderWarp; j < nmt; j += 2) {
         if (j > 1) load_cf(j);
-        float d[4] = {0.f, 0.f, 0.f, 0.f};
+        float dc[4][4] = {};
         if (do_c) {
 #pragma unroll
           for (int kk = 0; kk < KS; ++kk) {
@@ -305,10 +316,13 @@ __global__ void __launch_bounds__(kClThreads, 2)
               hi[i] = pack_bf16x2(x, y);
               lo[i] = pack_bf16x2(bf16_residual(x), bf16_residual(y));
             }
-            mma_m16n8k16(d, hi[0], hi[1], hi[2], hi[3], qa[kk][0], qa[kk][1]);
-            if constexpr (!C16) mma_m16n8k16(d, lo[0], lo[1], lo[2], lo[3], qa[kk][0], qa[kk][1]);
+            mma_m16n8k16(dc[kk & 1], hi[0], hi[1], hi[2], hi[3], qa[kk][0], qa[kk][1]);
+            if constexpr (!C16) mma_m16n8k16(dc[2 + (kk & 1)], lo[0], lo[1], lo[2], lo[3], qa[kk][0], qa[kk][1]);
           }
         }
+        float d[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) d[i] = (dc[0][i] + dc[1][i]) + (dc[2][i] + dc[3][i]);
         const int ra = j * 16 + g, rb = ra + 8;  // local rows (owned dims)
         const float mva = sMuv[ra], mvb = sMuv[rb];
         if (2 * t < G) {
@@ -344,17 +358,18 @@ __global__ void __launch_bounds__(kClThreads, 2)
       __syncwarp();
       // per head: log2 of the moment weight n exp(scale q.mu_k) and the new
       // token's logit (log2 domain), from this lane's q dims
-      float dm = 0.f, dn = 0.f;
+      float dm2[2] = {0.f, 0.f}, dn2[2] = {0.f, 0.f};
 #pragma unroll
       for (int kk = 0; kk < KS; ++kk) {
 #pragma unroll
         for (int hf = 0; hf < 2; ++hf) {
           const __nv_bfloat162 q2 = *reinterpret_cast<const __nv_bfloat162*>(&qa[kk][hf]);
           const int c = kk * 16 + hf * 8 + 2 * t;
-          if (use_m) dm = fmaf(__low2float(q2), sMuk[c], fmaf(__high2float(q2), sMuk[c + 1], dm));
-          if (has_new) dn = fmaf(__low2float(q2), sKn[c], fmaf(__high2float(q2), sKn[c + 1], dn));
+          if (use_m) dm2[hf] = fmaf(__low2float(q2), sMuk[c], fmaf(__high2float(q2), sMuk[c + 1], dm2[hf]));
+          if (has_new) dn2[hf] = fmaf(__low2float(q2), sKn[c], fmaf(__high2float(q2), sKn[c + 1], dn2[hf]));
         }
       }
+      float dm = dm2[0] + dm2[1], dn = dn2[0] + dn2[1];
       dm += __shfl_xor_sync(0xffffffffu, dm, 1);
       dm += __shfl_xor_sync(0xffffffffu, dm, 2);
       dn += __shfl_xor_sync(0xffffffffu, dn, 1);
@@ -364,6 +379,8 @@ __global__ void __launch_bounds__(kClThreads, 2)
         sSn[g] = has_new ? dn * qscale : kNegInf;
       }
     }
+    if (!producer && EARLY && s == 0 && lane == 0 && ldcg_hint(a.len + u, pol_keep) != len_read)
+      record_error(a.ws, MKV_ERR_INVALID_ARG, u);  // the cache changed under an early load
     cluster_wait_acquire();
   } else {
     // ---- attending warps: rows [warp*16, warp*16 + 16) of every tile
@@ -600,8 +617,8 @@ __global__ void __launch_bounds__(kClThreads, 2)
         record_error(a.ws, MKV_ERR_CAPACITY, u);
       } else {
         a.pos[(size_t)u * a.cap + len0] = seen0;
-        a.seen[u] = seen0 + 1;
-        a.len[u] = len0 + 1;
+        st_hint(a.seen + u, seen0 + 1, pol_keep);
+        st_hint(a.len + u, len0 + 1, pol_keep);
       }
     }
     if (sFail) {
