@@ -165,7 +165,7 @@ def test_workspace_reused_across_steps():
     assert mkv.mkv_get_device_error(ws)[0] == 0
 
 
-@pytest.mark.parametrize("batch", [1, 8, 64])
+@pytest.mark.parametrize("batch", [1, 8, 32, 64])
 @pytest.mark.parametrize("budget", [256, 1024, 4096])
 def test_decode_sweep_full_size(batch, budget):
     """Llama-3.1-8B geometry decode sweep cells (32 query heads, 8 KV heads,

@@ -28,6 +28,9 @@ pytestmark = pytest.mark.gpu
     (4, 8, 4, 128, 2, (100, 300), 340, False, 24, True),
     (1, 8, 4, 128, 2, (500, 600), 640, False, 24, True),
     (1, 2, 4, 64, 2, (40, 90), 120, False, 24, True),
+    # the headline geometry (32 units) at budget-1024 lengths: five or six
+    # tiles per CTA, so stages are refilled while the chain runs
+    (4, 8, 4, 128, 3, (1024, 1300), 1340, False, 6, True),
 ])
 def test_layer_chain_early_load(b, H, G, D, L, lens, cap, c16, steps, graph):
     rng = np.random.default_rng(b * 1000 + L * 10 + D)
