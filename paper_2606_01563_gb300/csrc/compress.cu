@@ -890,7 +890,7 @@ struct SelectArgs {
   int32_t* tile0;  // optional [groups][hs + 1] first kTok-row tile of each unit within its group, and the total
 };
 
-constexpr int kFinRB = 2;  // rows of C per finalize CTA
+constexpr int kFinRB = 16;  // rows of C per finalize CTA
 constexpr int kSelCL = 8;  // CTAs per selection group (one cluster), each over a contiguous range of pairs
 constexpr int kSelSmemKeys = 49152;  // keys of a CTA's range cached in shared memory (192 KB)
 constexpr int kMaxHs = 64;           // KV heads of a batch item with the adaptive budget
@@ -1207,96 +1207,155 @@ __global__ void __launch_bounds__(kGatherThreads) gather_kernel(const GatherArgs
 // R's centred record is then removed with the reverse pairwise formula.
 // merge_all = 1: the all-token set is the chunk records (its merge is kept
 // in L.mall); merge_all = 0: it is L.mall itself.
+//
+// Thread (row ar = tid / 16, lane group cq = tid % 16) takes the columns
+// cq*4 + 64h (h < D/64) of its row as float4s.  The counts and means of up to
+// kFinCH records of both sets are staged in one pass; then every record's
+// co-moment values are loaded with several records in flight.
+constexpr int kFinCH = 32;  // records staged per pass and set
 __global__ void __launch_bounds__(256) finalize_kernel(const Layout L, float* out_rec, mkv_moments out_mom,
                                                        int final_out, int merge_all) {
-  constexpr int NT = 256, RB = kFinRB, CHB = 32;
-  __shared__ float s_nc[CHB], s_dv[CHB][RB], s_dk[CHB][kDP];
-  __shared__ float s_x0v[RB], s_x0k[kDP];
+  constexpr int RB = kFinRB, NV = kDP / 64;  // NV float4s per thread (D = 128; one at D = 64)
+  __shared__ float s_n[2][kFinCH];
+  __shared__ __align__(16) float s_mv[2][kFinCH][RB];
+  __shared__ __align__(16) float s_mk[2][kFinCH][kDP];
   const int D = L.D;
+  const int nv = D / 64;
   const int rb = blockIdx.x, u = blockIdx.y, tid = threadIdx.x;
   const size_t rf = rec_floats(D);
-  const int ar = tid / D, c = tid % D;  // this thread's element (row rb*RB + ar, column c)
-  const bool act = tid < RB * D;
+  const int ar = tid / 16, cq = tid % 16;
   const int row = rb * RB + ar;
 
+  const int n_rec = merge_all ? L.n_chunks : 1;
+  const float* recA = merge_all ? L.mpart + (size_t)u * L.n_chunks * rf : L.mall + (size_t)u * rf;
+  const float* recR = L.rpart + (size_t)u * L.n_rchunks * rf;
+  // a joint selection leaves the unit's rows in its first ceil(cnt / kTok) records
+  const int n_rrec = L.hs > 1 ? min(L.n_rchunks, (L.cnt[u] + kTok - 1) / kTok) : L.n_rchunks;
+
   struct Set {
-    float n, sv, sk, M;
+    float n, sv, sk[4 * NV], M[4 * NV];
+    float x0v, x0k[4 * NV];
   };
-  // merge n_ch records starting at rbase for this thread's element
-  auto merge = [&](const float* rbase, int n_ch, float& x0v, float& x0k) -> Set {
-    Set st{0.f, 0.f, 0.f, 0.f};
-    __syncthreads();
-    if (tid < RB) s_x0v[tid] = n_ch > 0 ? rbase[4 + D + rb * RB + tid] : 0.f;
-    for (int i = tid; i < D; i += NT) s_x0k[i] = n_ch > 0 ? rbase[4 + i] : 0.f;
-    __syncthreads();
-    x0v = act ? s_x0v[ar] : 0.f;
-    x0k = s_x0k[act ? c : 0];
-    for (int g0 = 0; g0 < n_ch; g0 += CHB) {
-      const int nb = min(CHB, n_ch - g0);
-      if (g0 > 0) __syncthreads();
-      for (int i = tid; i < nb * (1 + RB + D); i += NT) {
-        const int ch = i / (1 + RB + D), j = i % (1 + RB + D);
-        const float* r = rbase + (size_t)(g0 + ch) * rf;
-        if (j == 0) s_nc[ch] = r[0];
-        else if (j <= RB) s_dv[ch][j - 1] = r[4 + D + rb * RB + j - 1] - s_x0v[j - 1];
-        else s_dk[ch][j - 1 - RB] = r[4 + (j - 1 - RB)] - s_x0k[j - 1 - RB];
-      }
-      __syncthreads();
-      if (act) {
-#pragma unroll 8
-        for (int ch = 0; ch < nb; ++ch) {
-          const float nc = s_nc[ch];
-          if (nc > 0.f) {  // an empty record's co-moment is never written
-            const float m = rbase[(size_t)(g0 + ch) * rf + 4 + 2 * D + (size_t)row * D + c];
-            const float dv = s_dv[ch][ar], dk = s_dk[ch][c];
-            st.n += nc;
-            st.sv = fmaf(nc, dv, st.sv);
-            st.sk = fmaf(nc, dk, st.sk);
-            st.M += m + nc * dv * dk;
+  Set A{}, R{};
+  auto merge = [&](Set& st, int set, const float* rbase, int g0, int nb) {
+#pragma unroll 4
+    for (int ch = 0; ch < nb; ++ch) {
+      const float* m = rbase + (size_t)(g0 + ch) * rf + 4 + 2 * D + (size_t)row * D;
+      float4 mv4[NV];
+#pragma unroll
+      for (int h = 0; h < NV; ++h)
+        mv4[h] = h < nv ? *reinterpret_cast<const float4*>(m + h * 64 + cq * 4) : make_float4(0.f, 0.f, 0.f, 0.f);
+      const float nc = s_n[set][ch];
+      if (nc > 0.f) {  // an empty record's co-moment is never written
+        const float dv = s_mv[set][ch][ar] - st.x0v;
+        st.n += nc;
+        st.sv = fmaf(nc, dv, st.sv);
+#pragma unroll
+        for (int h = 0; h < NV; ++h) {
+          if (h >= nv) break;
+          const float4 k4 = *reinterpret_cast<const float4*>(&s_mk[set][ch][h * 64 + cq * 4]);
+          const float kk[4] = {k4.x, k4.y, k4.z, k4.w}, mm[4] = {mv4[h].x, mv4[h].y, mv4[h].z, mv4[h].w};
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const float dk = kk[i] - st.x0k[h * 4 + i];
+            st.sk[h * 4 + i] = fmaf(nc, dk, st.sk[h * 4 + i]);
+            st.M[h * 4 + i] += mm[i] + nc * dv * dk;
           }
         }
       }
     }
-    return st;
   };
-  const int n_rec = merge_all ? L.n_chunks : 1;
-  const float* recs = merge_all ? L.mpart + (size_t)u * L.n_chunks * rf : L.mall + (size_t)u * rf;
-  // a joint selection leaves the unit's rows in its first ceil(cnt / kTok) records
-  const int n_rrec = L.hs > 1 ? min(L.n_rchunks, (L.cnt[u] + kTok - 1) / kTok) : L.n_rchunks;
-  float x0v, x0k, x0vR, x0kR;
-  const Set A = merge(recs, n_rec, x0v, x0k);
-  const Set R = merge(L.rpart + (size_t)u * L.n_rchunks * rf, n_rrec, x0vR, x0kR);
-  if (!act) return;
+  for (int g0 = 0; g0 < max(n_rec, n_rrec); g0 += kFinCH) {
+    const int nbA = max(0, min(kFinCH, n_rec - g0)), nbR = max(0, min(kFinCH, n_rrec - g0));
+    if (g0 > 0) __syncthreads();
+    // per record: (n, ...), the CTA's RB mu_v rows and mu_k as float4s;
+    // four loads per thread in flight before their stores
+    const int per = 1 + RB / 4 + D / 4, totA = nbA * per, tot = totA + nbR * per;
+    for (int i0 = 0; i0 < tot; i0 += 4 * 256) {
+      float4 v[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int i = i0 + k * 256 + tid;
+        if (i < tot) {
+          const int set = i >= totA, kk = set ? i - totA : i, ch = kk / per, j = kk % per;
+          const float* r = (set ? recR : recA) + (size_t)(g0 + ch) * rf;
+          const float* src = j == 0 ? r : (j <= RB / 4 ? r + 4 + D + rb * RB + (j - 1) * 4 : r + 4 + (j - 1 - RB / 4) * 4);
+          v[k] = *reinterpret_cast<const float4*>(src);
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int i = i0 + k * 256 + tid;
+        if (i < tot) {
+          const int set = i >= totA, kk = set ? i - totA : i, ch = kk / per, j = kk % per;
+          if (j == 0) s_n[set][ch] = v[k].x;
+          else if (j <= RB / 4) *reinterpret_cast<float4*>(&s_mv[set][ch][(j - 1) * 4]) = v[k];
+          else *reinterpret_cast<float4*>(&s_mk[set][ch][(j - 1 - RB / 4) * 4]) = v[k];
+        }
+      }
+    }
+    __syncthreads();
+    if (g0 == 0) {  // the first record's means (zero when a set has none)
+      A.x0v = nbA > 0 ? s_mv[0][0][ar] : 0.f;
+      R.x0v = nbR > 0 ? s_mv[1][0][ar] : 0.f;
+#pragma unroll
+      for (int h = 0; h < NV; ++h)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int c = h * 64 + cq * 4 + i;
+          A.x0k[h * 4 + i] = (nbA > 0 && h < nv) ? s_mk[0][0][c] : 0.f;
+          R.x0k[h * 4 + i] = (nbR > 0 && h < nv) ? s_mk[1][0][c] : 0.f;
+        }
+    }
+    merge(A, 0, recA, g0, nbA);
+    merge(R, 1, recR, g0, nbR);
+  }
+
   const float n = A.n, nR = R.n, nE = n - nR;
-  const float mv = x0v + A.sv / n, mk = x0k + A.sk / n;
-  const float M = A.M - A.sv * A.sk / n;
-  const float mvR = nR > 0.f ? x0vR + R.sv / nR : 0.f, mkR = nR > 0.f ? x0kR + R.sk / nR : 0.f;
-  const float MR = nR > 0.f ? R.M - R.sv * R.sk / nR : 0.f;
-  if (merge_all) {
-    float* mall = L.mall + (size_t)u * rf;
-    mall[4 + 2 * D + (size_t)row * D + c] = M;
-    if (rb == 0 && ar == 0) mall[4 + c] = mk;
-    if (c == 0) mall[4 + D + row] = mv;
-    if (rb == 0 && tid == 0) mall[0] = n;
+  const float mv = A.x0v + A.sv / n;
+  const float mvR = nR > 0.f ? R.x0v + R.sv / nR : 0.f;
+  const float mvE = nE > 0.f ? (n * mv - nR * mvR) / nE : 0.f;
+  float* mall = L.mall + (size_t)u * rf;
+  float* o = final_out ? nullptr : out_rec + (size_t)u * rf;
+#pragma unroll
+  for (int h = 0; h < NV; ++h) {
+    if (h >= nv) break;
+    float Mo[4], CE[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int j = h * 4 + i, c = h * 64 + cq * 4 + i;
+      const float mk = A.x0k[j] + A.sk[j] / n;
+      const float M = A.M[j] - A.sv * A.sk[j] / n;
+      const float mkR = nR > 0.f ? R.x0k[j] + R.sk[j] / nR : 0.f;
+      const float MR = nR > 0.f ? R.M[j] - R.sv * R.sk[j] / nR : 0.f;
+      Mo[i] = M;
+      CE[i] = 0.f;
+      float mkE = 0.f;
+      if (nE > 0.f) {
+        mkE = (n * mk - nR * mkR) / nE;
+        const float ME = M - MR - (nE * nR / n) * (mvR - mvE) * (mkR - mkE);
+        CE[i] = ME / nE;
+      }
+      if (rb == 0 && ar == 0) {  // the k means: row 0's threads
+        if (merge_all) mall[4 + c] = mk;
+        if (final_out) out_mom.mu_k[(size_t)u * D + c] = mkE;
+        else o[4 + c] = mkE;
+      }
+    }
+    const size_t e = (size_t)row * D + h * 64 + cq * 4;
+    if (merge_all) *reinterpret_cast<float4*>(mall + 4 + 2 * D + e) = make_float4(Mo[0], Mo[1], Mo[2], Mo[3]);
+    if (final_out) *reinterpret_cast<float4*>(out_mom.C + (size_t)u * D * D + e) = make_float4(CE[0], CE[1], CE[2], CE[3]);
+    else *reinterpret_cast<float4*>(o + 4 + 2 * D + e) = make_float4(CE[0], CE[1], CE[2], CE[3]);
   }
-  float CE = 0.f, mkE = 0.f, mvE = 0.f;
-  if (nE > 0.f) {
-    mkE = (n * mk - nR * mkR) / nE;
-    mvE = (n * mv - nR * mvR) / nE;
-    const float ME = M - MR - (nE * nR / n) * (mvR - mvE) * (mkR - mkE);
-    CE = ME / nE;
+  if (cq == 0) {  // the v means: one thread per row
+    if (merge_all) mall[4 + D + row] = mv;
+    if (final_out) out_mom.mu_v[(size_t)u * D + row] = mvE;
+    else o[4 + D + row] = mvE;
   }
-  if (final_out) {
-    out_mom.C[((size_t)u * D + row) * D + c] = CE;
-    if (c == 0) out_mom.mu_v[(size_t)u * D + row] = mvE;
-    if (rb == 0 && ar == 0) out_mom.mu_k[(size_t)u * D + c] = mkE;
-    if (rb == 0 && tid == 0) out_mom.n[u] = static_cast<int32_t>(nE);
-  } else {
-    float* o = out_rec + (size_t)u * rf;
-    o[4 + 2 * D + (size_t)row * D + c] = CE;
-    if (c == 0) o[4 + D + row] = mvE;
-    if (rb == 0 && ar == 0) o[4 + c] = mkE;
-    if (rb == 0 && tid == 0) o[0] = nE;
+  if (rb == 0 && tid == 0) {
+    if (merge_all) mall[0] = n;
+    if (final_out) out_mom.n[u] = static_cast<int32_t>(nE);
+    else o[0] = nE;
   }
 }
 

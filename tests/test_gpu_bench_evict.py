@@ -57,8 +57,8 @@ def test_bench_periodic_eviction_all_units():
         state[h] = dict(K=K[h][R], V=V[h][R], pos=R.astype(np.int64), m=evicted_moments(K[h], V[h], R))
     # 64 decode steps with append, then the eviction, as the bench runs them
     for i in range(every):
-        run.decode(i)
-    run.evict(every - 1)
+        run.decode(stack, i)
+    run.evict(stack, every - 1)
     code, info = mkv.mkv_get_device_error(run.ws_d)
     assert code == 0, (code, info)
     code, info = mkv.mkv_get_device_error(run.ws_e)
