@@ -61,8 +61,8 @@ ORACLE_JOBS = 16  # (layer, unit, budget) jobs in one oracle sample
 # headline workload from one ncu capture, valid while the code the kernel
 # compiles from (its .cu file and the library headers, comments aside) is
 # what was captured: code_sha of those sources at capture time.
-NCU_TRAFFIC = {"decode_cl_kernel": {"bytes": 15275530,
-                                     "code_sha": "26e3b083a0e780442182d4f543b13d8c1b63aaa5d179e8c29c8caf19514a577a"}}
+NCU_TRAFFIC = {"decode_cl_kernel": {"bytes": 15292836,
+                                     "code_sha": "9d69462747c1f8bffb7c37fcf5df73f0f2a83953d0808a02ddcb68ad837127a8"}}
 
 
 def parse():
@@ -276,13 +276,18 @@ class Run:
         self.g = mkv.geom(G.batch, G.n_kv_heads, G.group, G.head_dim)
         self.cap = budget + (evict_every if evict_every else stack.S)
         self.p = mkv.mkv_compress_params(budget, wl.window, wl.sink, wl.keep_window, wl.pool, 1, 1, TAU)
-        # a layer chain: the kernel before each decode launch belongs to another
-        # layer (or is a compress or eviction of another layer), so the launch
-        # may read its cache and moments before its dependency wait
-        self.dp = mkv.mkv_decode_params(1, 1, TAU, None, 1 if stack.L > 1 else 0)
         # with periodic eviction the caches keep y_j = S_tilde k_j across calls
         self.caches = [mkv.alloc_cache(self.g, self.cap, dev, evict_state=bool(evict_every)) for _ in range(stack.L)]
         self.moms = [mkv.alloc_moments(self.g, dev) for _ in range(stack.L)]
+        # each layer's C' in the decode's operand form (bf16 hi, lo words),
+        # packed whenever the layer's moments change (compress, eviction)
+        d = G.head_dim
+        self.csplit = [torch.empty(G.batch, G.n_kv_heads, d, d, dtype=torch.int32, device=dev) for _ in range(stack.L)]
+        # a layer chain: the kernel before each decode launch belongs to another
+        # layer (or is a compress, pack or eviction of another layer), so the
+        # launch may read its cache and moments before its dependency wait
+        early = 1 if stack.L > 1 else 0
+        self.dps = [mkv.mkv_decode_params(1, 1, TAU, None, early, c.data_ptr()) for c in self.csplit]
         # one workspace per kind, shared by the layers (the calls run one after another on one stream)
         self.ws_c = mkv.alloc_workspace(mkv.mkv_compress_workspace_size(self.g, wl.T, self.p), dev)
         self.ws_d = mkv.alloc_workspace(mkv.mkv_decode_workspace_size(self.g, self.cap), dev)
@@ -295,17 +300,19 @@ class Run:
         for l in range(s.L):
             self.mkv.mkv_compress(self.g, s.wl.T, s.K[l], s.V[l], s.Q[l], self.p, self.caches[l], self.moms[l],
                                   self.ws_c)
+            self.mkv.mkv_moments_pack_split(self.g, self.moms[l], TAU, self.csplit[l])
 
     def decode(self, s, i):
         for l in range(s.L):
             out = self.final[i] if l == s.L - 1 else self.out
             self.mkv.mkv_decode_step(self.g, s.q[i, l], s.kn[i, l], s.vn[i, l], self.caches[l], self.moms[l],
-                                     self.dp, out, None, self.ws_d)
+                                     self.dps[l], out, None, self.ws_d)
 
     def evict(self, s, i):
         for l in range(s.L):
             self.mkv.mkv_evict_append(self.g, s.q[i, l], None, None, self.B, self.caches[l], self.moms[l], TAU,
                                       self.ws_e)
+            self.mkv.mkv_moments_pack_split(self.g, self.moms[l], TAU, self.csplit[l])
 
     def parts(self, s):
         """(kind, callable) in step order, reading the inputs of stack `s`."""
@@ -338,10 +345,11 @@ class Run:
         self.graphs = self.graph_sets[0]
 
     def launches(self):
-        """Kernels of ours one pass launches (9 per per-unit compress)."""
+        """Kernels of ours one pass launches (9 per per-unit compress, one
+        pack of C' after each compress and eviction)."""
         s = self.st
         n_ev = (s.S // self.ev_every) if self.ev_every else 0
-        return s.L * (9 + s.S + n_ev)
+        return s.L * (9 + 1 + s.S + 2 * n_ev)
 
     def check_errors(self, stream):
         for ws in (self.ws_c, self.ws_d, self.ws_e):
@@ -630,6 +638,8 @@ def run_gpu(args):
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": dict(config_dict(stack.L), parallelism=f"replicas x{world}"),
             "graphs": "one CUDA graph per part (compress of all layers; 64 decode steps x all layers)",
+            "moment_c": "fp32 C; after each compress a pack writes C' (clamped) as the decode's bf16 hi + lo operand "
+                        "words, the same bytes and products as reading C",
             "e2e": e2e, "gpu_launches": sum(r.launches() for r in runs) * args.steps,
             "per_budget": {str(k): v for k, v in per_budget.items()},
             "roofline": roof, "clocks": clk, "setup_s": round(setup_s, 1),

@@ -176,6 +176,15 @@ typedef struct {
                       /* undefined); other violations go undetected.  0: every */
                       /* read waits (always safe).  mkv_decode_evict_step        */
                       /* ignores it (its own eviction kernel writes the cache). */
+  const void* C_split; /* optional [b, h_kv, d, d/2] pairs of 32-bit words from  */
+                       /* mkv_moments_pack_split: C' of Eq. fused (C with the     */
+                       /* App. C.2 clamp applied) split into bf16 hi and lo      */
+                       /* parts.  When set, the order-1 term reads it instead of */
+                       /* mkv_moments.C: the same bytes, and the same products,  */
+                       /* without the clamp and split at every step.  Valid     */
+                       /* while the moments and tau are those of the pack (the  */
+                       /* output is then bit-identical to the fp32-C path); not  */
+                       /* with C16; 16-byte aligned.                             */
 } mkv_decode_params;
 
 /*
@@ -186,6 +195,22 @@ typedef struct {
  * MKV_ERR_INVALID_ARG on null or misaligned pointers.
  */
 MKV_API mkv_status mkv_moments_pack_bf16(mkv_geom geom, const mkv_moments* mom, void* C16, void* stream);
+
+/*
+ * The decode's operand form of C' (Eq. fused, App. C.2), written once when the
+ * moments change instead of at every decode step: for every unit u, row a
+ * and column pair (c, c + 1), with x = C[u][a][c] and y = C[u][a][c + 1]
+ * each set to 0 where |n_u x| < tau (the clamp of S_tilde = n C), word 0 is
+ * bf16x2(x, y) and word 1 is bf16x2(x - bf16(x), y - bf16(y)) (round to nearest
+ * even; the first value in the low half).  One launch on `stream`.  C_split
+ * is caller-owned device memory of b * h_kv * d * d 32-bit words (as many bytes
+ * as C), 16-byte aligned; pass it as mkv_decode_params.C_split with the same
+ * tau, and pack again after every call that changes the moments
+ * (mkv_compress, mkv_evict_append).  Returns MKV_ERR_INVALID_ARG on null or
+ * misaligned pointers or a negative or NaN tau.
+ */
+MKV_API mkv_status mkv_moments_pack_split(mkv_geom geom, const mkv_moments* mom, float tau, void* C_split,
+                                          void* stream);
 
 /* Human-readable name of a status code (static string). */
 MKV_API const char* mkv_status_str(mkv_status s);
@@ -349,8 +374,8 @@ MKV_API size_t mkv_decode_evict_workspace_size(mkv_geom geom, int32_t capacity);
  *   k_new, v_new  bf16 [b, h_kv, d]     the token appended (both required)
  *   out           fp32 [b, g*h_kv, d]   corrected output
  *   lse           fp32 [b, g*h_kv]      optional, as in mkv_decode_step
- * Requirements: as mkv_evict_append and mkv_decode_step; p->C16 must be NULL
- * (the moments change inside the call).  q, out, k_new and v_new must be
+ * Requirements: as mkv_evict_append and mkv_decode_step; p->C16 and
+ * p->C_split must be NULL (the moments change inside the call).  q, out, k_new and v_new must be
  * 16-byte aligned.
  */
 MKV_API mkv_status mkv_decode_evict_step(mkv_geom geom, const void* q, const void* k_new, const void* v_new,

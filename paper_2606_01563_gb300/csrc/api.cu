@@ -50,7 +50,7 @@ const char* mkv_status_str(mkv_status s) {
   return "unknown status";
 }
 
-int32_t mkv_version(void) { return 201; }
+int32_t mkv_version(void) { return 202; }
 
 // ------------------------------------------------------------------ decode
 size_t mkv_decode_workspace_size(mkv_geom geom, int32_t capacity) {
@@ -82,6 +82,7 @@ mkv_status mkv_decode_step(mkv_geom geom, const void* q, const void* k_new, cons
   a.mu_v = p->correction ? mom->mu_v : nullptr;
   a.C = p->correction ? mom->C : nullptr;
   a.C16 = p->correction ? static_cast<const __nv_bfloat16*>(p->C16) : nullptr;
+  a.Cs = p->correction ? static_cast<const uint2*>(p->C_split) : nullptr;
   a.correction = p->correction;
   a.order = p->order;
   a.tau = p->tau;
@@ -92,6 +93,14 @@ mkv_status mkv_decode_step(mkv_geom geom, const void* q, const void* k_new, cons
   a.early = p->early_load;
   decode_carve(a, geom, cache->capacity, sms, workspace);
   return cuda_status(launch_decode(a, geom.head_dim, geom.group, static_cast<cudaStream_t>(stream)));
+}
+
+mkv_status mkv_moments_pack_split(mkv_geom geom, const mkv_moments* mom, float tau, void* C_split, void* stream) {
+  NvtxRange nvtx("mkv_moments_pack_split");
+  if (!geom_ok(geom)) return geom_status(geom);
+  if (!moments_ok(mom) || !C_split || !aligned(C_split, 16) || !(tau >= 0.f)) return MKV_ERR_INVALID_ARG;
+  return cuda_status(launch_pack_split(mom->C, mom->n, tau, static_cast<uint2*>(C_split),
+                                       geom.batch * geom.n_kv_heads, geom.head_dim, static_cast<cudaStream_t>(stream)));
 }
 
 mkv_status mkv_moments_pack_bf16(mkv_geom geom, const mkv_moments* mom, void* C16, void* stream) {
@@ -164,7 +173,7 @@ mkv_status mkv_decode_evict_step(mkv_geom geom, const void* q, const void* k_new
     return MKV_ERR_INVALID_ARG;
   if (!aligned(q, 16) || !aligned(out, 16) || !aligned(k_new, 16) || !aligned(v_new, 16)) return MKV_ERR_INVALID_ARG;
   if ((p->correction != 0 && p->correction != 1) || (p->order != 0 && p->order != 1) || !(p->tau >= 0.f) ||
-      p->C16 != nullptr || (p->early_load != 0 && p->early_load != 1))
+      p->C16 != nullptr || p->C_split != nullptr || (p->early_load != 0 && p->early_load != 1))
     return MKV_ERR_INVALID_ARG;
   if (cache->capacity > 65536) return MKV_ERR_SHAPE;
   const int sms = num_sms_current();

@@ -206,11 +206,14 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
   const int n_mt = (r1 - r0 + 15) / 16;
   const bool do_c = corr && a.order == 1;
   const bool split_k = n_mt <= 2;
-  // C[row][c0], C[row][c0 + 1] as float2, from C or from its bf16 copy
+  // C[row][c0], C[row][c0 + 1] as float2, from C or from its bf16 copy; with
+  // the operand form of C' (cs), the bits of its (hi, lo) words
   constexpr bool c16 = C16;  // moment rows read from the bf16 copy of C
+  const bool cs = !c16 && a.Cs != nullptr;
   auto ld_c2 = [&](int row, int c0) -> float2 {
     const size_t off = ((size_t)u * D + row) * D + c0;
     if constexpr (c16) return __bfloat1622float2(__ldg(reinterpret_cast<const __nv_bfloat162*>(a.C16 + off)));
+    else if (cs) return __ldg(reinterpret_cast<const float2*>(a.Cs + off / 2));
     else return __ldg(reinterpret_cast<const float2*>(a.C + off));
   };
   float2 cfr[2][KPW][4];
@@ -236,8 +239,9 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
       }
     }
     if (do_c && !split_k && tid == 0 && r1 > r0) {  // whole-tile case: the rows are read after the tiles
-      const void* base = c16 ? static_cast<const void*>(a.C16 + ((size_t)u * D + r0) * D)
-                             : static_cast<const void*>(a.C + ((size_t)u * D + r0) * D);
+      const void* base = c16  ? static_cast<const void*>(a.C16 + ((size_t)u * D + r0) * D)
+                         : cs ? static_cast<const void*>(a.Cs + ((size_t)u * D + r0) * D / 2)
+                              : static_cast<const void*>(a.C + ((size_t)u * D + r0) * D);
       asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base),
                    "r"((uint32_t)((r1 - r0) * D * (c16 ? 2 : 4)))
                    : "memory");
@@ -355,9 +359,14 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a, co
     uint32_t hi[4], lo[4];
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-      const float x = (fabsf(f[i].x * nf) < tau) ? 0.f : f[i].x;
-      const float y = (fabsf(f[i].y * nf) < tau) ? 0.f : f[i].y;
-      split_bf16x2(x, y, hi[i], lo[i]);
+      if (cs) {  // already clamped and split
+        hi[i] = __float_as_uint(f[i].x);
+        lo[i] = __float_as_uint(f[i].y);
+      } else {
+        const float x = (fabsf(f[i].x * nf) < tau) ? 0.f : f[i].x;
+        const float y = (fabsf(f[i].y * nf) < tau) ? 0.f : f[i].y;
+        split_bf16x2(x, y, hi[i], lo[i]);
+      }
     }
     // the q fragment of k-step kk, selected without indexing the register
     // array by a runtime value (which would move qa to local memory)
@@ -709,7 +718,36 @@ __global__ void __launch_bounds__(256) pack_bf16_kernel(const float* __restrict_
     reinterpret_cast<uint2*>(C16)[i] = w;
   }
 }
+// The operand form of C' (Eq. fused with the App. C.2 clamp): per column
+// pair, the (hi, lo) bf16x2 words the decode kernels feed to the tensor cores,
+// computed exactly as they compute them from C at a step (split_bf16x2 of the
+// clamped pair).  Grid-stride over float4s of C: two pairs each.
+__global__ void __launch_bounds__(256) pack_split_kernel(const float* __restrict__ C, const int32_t* __restrict__ n,
+                                                         float tau, uint2* __restrict__ Cs, size_t n4, int per_unit4) {
+  for (size_t i = (size_t)blockIdx.x * 256 + threadIdx.x; i < n4; i += (size_t)gridDim.x * 256) {
+    const float nf = static_cast<float>(n[i / per_unit4]);
+    const float4 v = reinterpret_cast<const float4*>(C)[i];
+    const float c[4] = {v.x, v.y, v.z, v.w};
+    uint32_t hi[2], lo[2];
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      const float x = (fabsf(c[2 * j] * nf) < tau) ? 0.f : c[2 * j];
+      const float y = (fabsf(c[2 * j + 1] * nf) < tau) ? 0.f : c[2 * j + 1];
+      split_bf16x2(x, y, hi[j], lo[j]);
+    }
+    reinterpret_cast<uint4*>(Cs)[i] = make_uint4(hi[0], lo[0], hi[1], lo[1]);
+  }
+}
 }  // namespace
+
+cudaError_t launch_pack_split(const float* C, const int32_t* n, float tau, uint2* Cs, int units, int D,
+                              cudaStream_t stream) {
+  const int per_unit4 = D * D / 4;
+  const size_t n4 = (size_t)units * per_unit4;
+  const int blocks = static_cast<int>(std::min<size_t>((n4 + 255) / 256, 65535));
+  if (n4 > 0) pack_split_kernel<<<blocks, 256, 0, stream>>>(C, n, tau, Cs, n4, per_unit4);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_pack_bf16(const float* C, __nv_bfloat16* C16, size_t n, cudaStream_t stream) {
   const size_t n4 = n / 4;  // d * d is a multiple of 4

@@ -157,6 +157,9 @@ __global__ void __launch_bounds__(kClThreads, 2)
   // ---- state read before (EARLY) or after the dependency wait
   int len_read = 0, len0 = 0, n_tiles = 0, n_cached = 0, row_base = 0, seen0 = 0, n_e = 0, issued = 0;
   float2 cf[KS][4];  // side warps: C' fragments of one owned 16-row block, all k-steps
+  // with the operand form of C' (mkv_moments_pack_split) a fragment's float2
+  // holds the bits of its (hi, lo) words, already clamped and split
+  const bool cs = !C16 && a.Cs != nullptr;
   auto load_cf = [&](int j) {
     const int ra = (mlo + j) * 16 + g, rb = ra + 8;
     const bool va = do_c && j < nmt;
@@ -169,7 +172,8 @@ __global__ void __launch_bounds__(kClThreads, 2)
           const uint32_t w = ldg_hint(reinterpret_cast<const uint32_t*>(a.C16 + off), pol_keep);
           return __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w));
         } else {
-          return ldg_hint(reinterpret_cast<const float2*>(a.C + off), pol_keep);
+          return ldg_hint(cs ? reinterpret_cast<const float2*>(a.Cs + off / 2) : reinterpret_cast<const float2*>(a.C + off),
+                          pol_keep);
         }
       };
       cf[kk][0] = va ? ld(ra, c0) : make_float2(0.f, 0.f);
@@ -217,8 +221,9 @@ __global__ void __launch_bounds__(kClThreads, 2)
                        "r"(bytes) : "memory");
         }
         if (do_c && nmt > 2) {  // C' rows past the first two blocks are read later: into L2 now
-          const void* base = C16 ? static_cast<const void*>(a.C16 + ((size_t)u * D + (mlo + 2) * 16) * D)
-                                 : static_cast<const void*>(a.C + ((size_t)u * D + (mlo + 2) * 16) * D);
+          const void* base = C16  ? static_cast<const void*>(a.C16 + ((size_t)u * D + (mlo + 2) * 16) * D)
+                             : cs ? static_cast<const void*>(a.Cs + ((size_t)u * D + (mlo + 2) * 16) * D / 2)
+                                  : static_cast<const void*>(a.C + ((size_t)u * D + (mlo + 2) * 16) * D);
           asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base),
                        "r"((uint32_t)((nmt - 2) * 16 * D * (C16 ? 2 : 4))) : "memory");
         }
@@ -297,15 +302,24 @@ __global__ void __launch_bounds__(kClThreads, 2)
     if (use_m) {
       // f_hat_E rows of the owned blocks, blocks alternating between the two
       // side warps: mu_v + scale C'q on the tensor cores (A = C' rows split
-      // into bf16 hi + lo parts, clamp of Eq. fused applied here; B = the q
-      // fragments), written as sF[row][head].  Four independent accumulator
+      // into bf16 hi + lo parts, clamp of Eq. fused applied here, or both
+      // read ready-made from the operand form; B = the q fragments), written
+      // as sF[row][head].  Four independent accumulator
       // chains (k-step parity x part): these products share the tensor pipe
       // with an attending warp's tiles.
       const float nf = static_cast<float>(n_e), tau = a.tau;
       for (int j = warp - kLoaderWarp; j < nmt; j += 2) {
         if (j > 1) load_cf(j);
         float dc[4][4] = {};
-        if (do_c) {
+        if (do_c && cs) {  // operand words as loaded
+#pragma unroll
+          for (int kk = 0; kk < KS; ++kk) {
+            mma_m16n8k16(dc[kk & 1], __float_as_uint(cf[kk][0].x), __float_as_uint(cf[kk][1].x),
+                         __float_as_uint(cf[kk][2].x), __float_as_uint(cf[kk][3].x), qa[kk][0], qa[kk][1]);
+            mma_m16n8k16(dc[2 + (kk & 1)], __float_as_uint(cf[kk][0].y), __float_as_uint(cf[kk][1].y),
+                         __float_as_uint(cf[kk][2].y), __float_as_uint(cf[kk][3].y), qa[kk][0], qa[kk][1]);
+          }
+        } else if (do_c) {
 #pragma unroll
           for (int kk = 0; kk < KS; ++kk) {
             uint32_t hi[4], lo[4];

@@ -26,6 +26,7 @@ struct DecodeArgs {
   const float* mu_v;
   const float* C;
   const __nv_bfloat16* C16;  // optional bf16 copy of C (read instead of C when set)
+  const uint2* Cs;           // optional operand form of C' (bf16x2 hi, lo words per column pair; read instead of C)
   int32_t correction;
   int32_t order;
   float tau;
@@ -54,6 +55,8 @@ void decode_carve(DecodeArgs& a, const mkv_geom& g, int32_t capacity, int num_sm
 cudaError_t launch_decode(const DecodeArgs& a, int head_dim, int group, cudaStream_t stream);
 cudaError_t launch_decode_cluster(const DecodeArgs& a, int head_dim, int group, cudaStream_t stream);
 cudaError_t launch_pack_bf16(const float* C, __nv_bfloat16* C16, size_t n, cudaStream_t stream);
+cudaError_t launch_pack_split(const float* C, const int32_t* n, float tau, uint2* Cs, int units, int D,
+                              cudaStream_t stream);
 
 // ------------------------------------------------------------------- evict
 struct EvictArgs {

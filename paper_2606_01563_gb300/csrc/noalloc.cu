@@ -120,6 +120,7 @@ extern "C" MKV_API mkv_status mkv_decode_step_noalloc(mkv_geom geom, const void*
   a.mu_v = p->correction ? mom->mu_v : nullptr;
   a.C = p->correction ? mom->C : nullptr;
   a.C16 = p->correction ? static_cast<const __nv_bfloat16*>(p->C16) : nullptr;
+  a.Cs = p->correction ? static_cast<const uint2*>(p->C_split) : nullptr;
   a.correction = p->correction;
   a.order = p->order;
   a.tau = p->tau;

@@ -64,6 +64,7 @@ inline mkv_status decode_args_status(const mkv_geom& geom, const void* q, const 
   if (p->correction && !moments_ok(mom)) return MKV_ERR_INVALID_ARG;
   if (!(p->tau >= 0.f)) return MKV_ERR_INVALID_ARG;
   if (p->C16 && !aligned(p->C16, 16)) return MKV_ERR_INVALID_ARG;
+  if (p->C_split && (!aligned(p->C_split, 16) || p->C16)) return MKV_ERR_INVALID_ARG;
   if (p->early_load != 0 && p->early_load != 1) return MKV_ERR_INVALID_ARG;
   return MKV_OK;
 }

@@ -45,7 +45,7 @@ class mkv_compress_diag(ctypes.Structure):
 
 class mkv_decode_params(ctypes.Structure):
     _fields_ = [("correction", c_i32), ("order", c_i32), ("tau", ctypes.c_float), ("C16", c_vp),
-                ("early_load", c_i32)]
+                ("early_load", c_i32), ("C_split", c_vp)]
 
 
 STATUS = {0: "MKV_OK", 1: "MKV_ERR_INVALID_ARG", 2: "MKV_ERR_SHAPE", 3: "MKV_ERR_CAPACITY",
@@ -54,7 +54,7 @@ STATUS = {0: "MKV_OK", 1: "MKV_ERR_INVALID_ARG", 2: "MKV_ERR_SHAPE", 3: "MKV_ERR
 EXPORTS = ("mkv_status_str", "mkv_version", "mkv_compress_workspace_size", "mkv_compress",
            "mkv_decode_workspace_size", "mkv_decode_step", "mkv_evict_workspace_size",
            "mkv_evict_append", "mkv_get_device_error", "mkv_decode_step_noalloc", "mkv_moments_pack_bf16",
-           "mkv_decode_evict_workspace_size", "mkv_decode_evict_step")
+           "mkv_decode_evict_workspace_size", "mkv_decode_evict_step", "mkv_moments_pack_split")
 # test hooks declared in include/mkv_debug.h
 DEBUG_EXPORTS = ("mkv_debug_set_poll_limit", "mkv_debug_force_ticket_merge")
 
@@ -108,6 +108,8 @@ def lib():
                                             c_vp, c_vp, c_vp, ctypes.c_size_t, c_vp]
         L.mkv_moments_pack_bf16.restype = c_i32
         L.mkv_moments_pack_bf16.argtypes = [mkv_geom, ctypes.POINTER(mkv_moments), c_vp, c_vp]
+        L.mkv_moments_pack_split.restype = c_i32
+        L.mkv_moments_pack_split.argtypes = [mkv_geom, ctypes.POINTER(mkv_moments), ctypes.c_float, c_vp, c_vp]
         L.mkv_debug_set_poll_limit.restype = ctypes.c_int64
         L.mkv_debug_set_poll_limit.argtypes = [ctypes.c_int64]
         L.mkv_debug_force_ticket_merge.restype = c_i32
@@ -274,6 +276,14 @@ def mkv_moments_pack_bf16(g, mom: Moments, C16, stream=None):
     """C16 (bf16 [b, h_kv, d, d]) = bf16(mom.C): the 16-bit copy mkv_decode_params.C16 points at."""
     m = mom.c()
     _check(lib().mkv_moments_pack_bf16(g, ctypes.byref(m), _ptr(C16), _stream(stream)), "mkv_moments_pack_bf16")
+
+
+def mkv_moments_pack_split(g, mom: Moments, tau, C_split, stream=None):
+    """C_split (int32 [b, h_kv, d, d], as many bytes as C) = the (hi, lo) bf16x2
+    operand words of the clamped C': what mkv_decode_params.C_split points at."""
+    m = mom.c()
+    _check(lib().mkv_moments_pack_split(g, ctypes.byref(m), float(tau), _ptr(C_split), _stream(stream)),
+           "mkv_moments_pack_split")
 
 
 def mkv_debug_set_poll_limit(polls):

@@ -41,7 +41,7 @@ int main(void) {
   const mkv_geom bad_group = {1, 2, 3, 128};
   mkv_cache c = {FAKE, FAKE, (int32_t*)FAKE, (int32_t*)FAKE, (int32_t*)FAKE, 64, NULL, NULL};
   mkv_moments m = {(int32_t*)FAKE, (float*)FAKE, (float*)FAKE, (float*)FAKE};
-  mkv_decode_params dp = {1, 1, 1e-6f, NULL, 0};
+  mkv_decode_params dp = {1, 1, 1e-6f, NULL, 0, NULL};
   mkv_compress_params cp = {128, 16, 1, 1, 1, 1, 1, 1e-6f, 0};
   mkv_compress_params small = cp;
   const size_t big = (size_t)1 << 30;
@@ -52,12 +52,12 @@ int main(void) {
   CHECK(sizeof(mkv_cache) == 64 && offsetof(mkv_cache, capacity) == 40 && offsetof(mkv_cache, y_len) == 56);
   CHECK(sizeof(mkv_compress_params) == 36);
   CHECK(offsetof(mkv_compress_params, tau) == 28 && offsetof(mkv_compress_params, adaptive) == 32);
-  CHECK(sizeof(mkv_decode_params) == 32 && offsetof(mkv_decode_params, C16) == 16 &&
-        offsetof(mkv_decode_params, early_load) == 24);
+  CHECK(sizeof(mkv_decode_params) == 40 && offsetof(mkv_decode_params, C16) == 16 &&
+        offsetof(mkv_decode_params, early_load) == 24 && offsetof(mkv_decode_params, C_split) == 32);
   CHECK(sizeof(mkv_compress_diag) == 24);
   CHECK(sizeof(mkv_status) == 4 && MKV_ERR_WORKSPACE == 7);
 
-  CHECK(mkv_version() == 201);
+  CHECK(mkv_version() == 202);
   CHECK(strcmp(mkv_status_str(MKV_OK), "ok") == 0);
   CHECK(strcmp(mkv_status_str((mkv_status)99), "unknown status") == 0);
 
@@ -75,6 +75,7 @@ int main(void) {
   CHECK(mkv_decode_step_noalloc(bad_dim, FAKE, NULL, NULL, &c, &m, &dp, (float*)FAKE, NULL, NULL) ==
         MKV_ERR_UNSUPPORTED);
   CHECK(mkv_moments_pack_bf16(g, &m, NULL, NULL) == MKV_ERR_INVALID_ARG);
+  CHECK(mkv_moments_pack_split(g, &m, 1e-6f, NULL, NULL) == MKV_ERR_INVALID_ARG);
 
   /* compress */
   CHECK(mkv_compress_workspace_size(g, 1024, &cp) > 0);
@@ -130,7 +131,7 @@ def test_header_compiles_as_cpp(tmp_path):
     if cxx is None:
         pytest.skip("no C++ compiler")
     src = tmp_path / "h.cpp"
-    src.write_text('#include "mkv.h"\nint main() { return mkv_version() == 201 ? 0 : 1; }\n')
+    src.write_text('#include "mkv.h"\nint main() { return mkv_version() == 202 ? 0 : 1; }\n')
     r = subprocess.run([cxx, "-std=c++17", "-Wall", "-Wextra", "-Werror", "-fsyntax-only", "-I", INCLUDE, str(src)],
                        capture_output=True, text=True)
     assert r.returncode == 0, r.stderr
@@ -144,6 +145,6 @@ def test_binding_structs_match_the_c_layout():
     assert mkv.mkv_cache.y.offset == 48 and mkv.mkv_cache.y_len.offset == 56
     assert ctypes.sizeof(mkv.mkv_compress_params) == 36
     assert mkv.mkv_compress_params.tau.offset == 28 and mkv.mkv_compress_params.adaptive.offset == 32
-    assert ctypes.sizeof(mkv.mkv_decode_params) == 32 and mkv.mkv_decode_params.C16.offset == 16
-    assert mkv.mkv_decode_params.early_load.offset == 24
+    assert ctypes.sizeof(mkv.mkv_decode_params) == 40 and mkv.mkv_decode_params.C16.offset == 16
+    assert mkv.mkv_decode_params.early_load.offset == 24 and mkv.mkv_decode_params.C_split.offset == 32
     assert ctypes.sizeof(mkv.mkv_compress_diag) == 24

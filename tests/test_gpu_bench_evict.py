@@ -3,7 +3,8 @@ every unit: the one-layer Llama-3.1-8B workload of the bench (T = 8192,
 budget 512, window 32, the bench's device-drawn inputs), compressed, 64
 decode steps that each append a token (576 rows), then one mkv_evict_append
 back to the budget: 64 evictions in one call, 8 units.  The calls are the
-bench's own (bench.Stack and bench.Run, run eagerly instead of from graphs).
+bench's own (bench.Stack and bench.Run, run eagerly instead of from graphs),
+so the decode steps read C' in the operand form the run packs.
 
 The oracle starts from the state the compress left (checked first against the
 oracle's compress, near ties continued from the kernel's choice), checks
@@ -45,6 +46,9 @@ def test_bench_periodic_eviction_all_units():
     i1 = torch.zeros(1, H, B, dtype=torch.int32, device=dev)
     mkv.mkv_compress(run.g, T, stack.K[0], stack.V[0], stack.Q[0], run.p, run.caches[0], run.moms[0], run.ws_c,
                      diag=(s, s2, i1))
+    # the run's decode steps read C' in its operand form: packed after every
+    # compress and eviction, as the run's own compress does
+    mkv.mkv_moments_pack_split(run.g, run.moms[0], TAU, run.csplit[0])
     c, m = run.caches[0], run.moms[0]
     comp = dict(K=host(c.K), V=host(c.V), pos=host(c.pos), len=host(c.len), seen=host(c.seen), n=host(m.n),
                 mu_k=host(m.mu_k), mu_v=host(m.mu_v), C=host(m.C), s=host(s), s2=host(s2), i1=host(i1))

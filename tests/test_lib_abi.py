@@ -27,7 +27,7 @@ def declared_functions(header="mkv.h"):
 
 def test_every_declared_symbol_is_exported(L):
     names = declared_functions()
-    assert len(names) == 13, names
+    assert len(names) == 14, names
     assert set(names) == set(mkv.EXPORTS)
     for n in names:
         assert hasattr(L, n), n
@@ -48,7 +48,7 @@ def test_debug_hooks_round_trip(L):
 
 
 def test_version_and_status_strings(L):
-    assert mkv.mkv_version() == 201
+    assert mkv.mkv_version() == 202
     for code in range(8):
         assert mkv.mkv_status_str(code)
     assert mkv.mkv_status_str(99) == "unknown status"
@@ -94,6 +94,8 @@ def test_decode_validation(L):
     assert decode(L, g, wsb=16) == 7
     assert decode(L, g, ws=FAKE + 8) == 7                    # misaligned workspace
     assert decode(L, g, p=mkv.mkv_decode_params(1, 1, 0.0, FAKE + 8)) == 1  # misaligned bf16 C copy
+    assert decode(L, g, p=mkv.mkv_decode_params(1, 1, 0.0, None, 0, FAKE + 8)) == 1  # misaligned operand form
+    assert decode(L, g, p=mkv.mkv_decode_params(1, 1, 0.0, FAKE, 0, FAKE)) == 1  # operand form with the bf16 copy
     assert decode(L, g, q=FAKE + 4) == 1                     # misaligned q
     assert decode(L, g, p=mkv.mkv_decode_params(1, 1, 0.0, None, 2)) == 1   # early_load not 0/1
     # mu_k is read as float2 and mu_v as float4: 4-byte alignment is not enough
@@ -122,7 +124,8 @@ def test_noalloc_validation_matches_decode(L):
              dict(mom=mkv.mkv_moments(FAKE, FAKE + 4, FAKE, FAKE)),
              dict(mom=mkv.mkv_moments(FAKE, FAKE, FAKE + 8, FAKE)),
              dict(cache=mkv.mkv_cache(FAKE + 2, FAKE, FAKE, FAKE, FAKE, 64)),
-             dict(p=mkv.mkv_decode_params(1, 2, 0.0)), dict(p=mkv.mkv_decode_params(1, 1, 0.0, FAKE + 8))]
+             dict(p=mkv.mkv_decode_params(1, 2, 0.0)), dict(p=mkv.mkv_decode_params(1, 1, 0.0, FAKE + 8)),
+             dict(p=mkv.mkv_decode_params(1, 1, 0.0, None, 0, FAKE + 4))]
     for kw in cases:
         gg = kw.pop("g", g)
         want = decode(L, gg, **kw)
@@ -139,6 +142,19 @@ def test_pack_bf16_validation(L):
     assert L.mkv_moments_pack_bf16(g, ctypes.byref(m), FAKE + 8, None) == 1
     assert L.mkv_moments_pack_bf16(g, None, FAKE, None) == 1
     assert L.mkv_moments_pack_bf16(mkv.geom(1, 2, 4, 96), ctypes.byref(m), FAKE, None) == 6
+
+
+def test_pack_split_validation(L):
+    g = mkv.geom(1, 2, 4, 128)
+    m = mkv.mkv_moments(FAKE, FAKE, FAKE, FAKE)
+    assert L.mkv_moments_pack_split(g, ctypes.byref(m), 1e-6, None, None) == 1
+    assert L.mkv_moments_pack_split(g, ctypes.byref(m), 1e-6, FAKE + 8, None) == 1
+    assert L.mkv_moments_pack_split(g, ctypes.byref(m), -1.0, FAKE, None) == 1
+    assert L.mkv_moments_pack_split(g, ctypes.byref(m), float("nan"), FAKE, None) == 1
+    assert L.mkv_moments_pack_split(g, None, 1e-6, FAKE, None) == 1
+    assert L.mkv_moments_pack_split(g, ctypes.byref(mkv.mkv_moments(FAKE, FAKE, FAKE, FAKE + 8)), 1e-6, FAKE,
+                                    None) == 1  # C misaligned
+    assert L.mkv_moments_pack_split(mkv.geom(1, 2, 4, 96), ctypes.byref(m), 1e-6, FAKE, None) == 6
 
 
 def test_workspace_sizes(L):
@@ -203,6 +219,7 @@ def test_decode_evict_validation(L):
     assert run(out=FAKE + 8) == 1                 # misaligned output
     assert run(p=P(order=2)) == 1
     assert run(p=P(C16=FAKE)) == 1                # a 16-bit copy of C would be stale
+    assert run(p=P(C_split=FAKE)) == 1            # so would the operand form of C'
     assert run(wsb=8) == 7
     assert run(g=mkv.geom(1, 2, 5, 64)) == 2
     n = L.mkv_decode_evict_workspace_size(g, 64)
