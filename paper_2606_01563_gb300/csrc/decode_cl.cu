@@ -91,7 +91,7 @@ __host__ __device__ constexpr size_t cl_smem_bytes(int D, int G, int S) {
   return cl_stages(D, G, S) * cl_stage_bytes(D) + cl_extra_bytes(D, G, S) + 1024;  // + alignment slack
 }
 
-template <int D, int G, bool C16, bool EARLY>
+template <int D, int G, bool C16, bool EARLY, bool CS>
 __global__ void __launch_bounds__(kClThreads, 2)
     decode_cl_kernel(const DecodeArgs a, const __grid_constant__ CUtensorMap tmK,
                      const __grid_constant__ CUtensorMap tmV) {
@@ -157,9 +157,11 @@ __global__ void __launch_bounds__(kClThreads, 2)
   // ---- state read before (EARLY) or after the dependency wait
   int len_read = 0, len0 = 0, n_tiles = 0, n_cached = 0, row_base = 0, seen0 = 0, n_e = 0, issued = 0;
   float2 cf[KS][4];  // side warps: C' fragments of one owned 16-row block, all k-steps
-  // with the operand form of C' (mkv_moments_pack_split) a fragment's float2
-  // holds the bits of its (hi, lo) words, already clamped and split
-  const bool cs = !C16 && a.Cs != nullptr;
+  // with the operand form of C' (mkv_moments_pack_split; the CS variant) a
+  // fragment's float2 holds the bits of its (hi, lo) words, already clamped
+  // and split
+  static_assert(!(C16 && CS), "one form of C");
+  constexpr bool cs = CS;
   auto load_cf = [&](int j) {
     const int ra = (mlo + j) * 16 + g, rb = ra + 8;
     const bool va = do_c && j < nmt;
@@ -171,9 +173,10 @@ __global__ void __launch_bounds__(kClThreads, 2)
         if constexpr (C16) {
           const uint32_t w = ldg_hint(reinterpret_cast<const uint32_t*>(a.C16 + off), pol_keep);
           return __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w));
+        } else if constexpr (CS) {
+          return ldg_hint(reinterpret_cast<const float2*>(a.Cs + off / 2), pol_keep);
         } else {
-          return ldg_hint(cs ? reinterpret_cast<const float2*>(a.Cs + off / 2) : reinterpret_cast<const float2*>(a.C + off),
-                          pol_keep);
+          return ldg_hint(reinterpret_cast<const float2*>(a.C + off), pol_keep);
         }
       };
       cf[kk][0] = va ? ld(ra, c0) : make_float2(0.f, 0.f);
@@ -311,13 +314,15 @@ __global__ void __launch_bounds__(kClThreads, 2)
       for (int j = warp - kLoaderWarp; j < nmt; j += 2) {
         if (j > 1) load_cf(j);
         float dc[4][4] = {};
-        if (do_c && cs) {  // operand words as loaded
+        if constexpr (CS) {
+          if (do_c) {  // operand words as loaded
 #pragma unroll
-          for (int kk = 0; kk < KS; ++kk) {
-            mma_m16n8k16(dc[kk & 1], __float_as_uint(cf[kk][0].x), __float_as_uint(cf[kk][1].x),
-                         __float_as_uint(cf[kk][2].x), __float_as_uint(cf[kk][3].x), qa[kk][0], qa[kk][1]);
-            mma_m16n8k16(dc[2 + (kk & 1)], __float_as_uint(cf[kk][0].y), __float_as_uint(cf[kk][1].y),
-                         __float_as_uint(cf[kk][2].y), __float_as_uint(cf[kk][3].y), qa[kk][0], qa[kk][1]);
+            for (int kk = 0; kk < KS; ++kk) {
+              mma_m16n8k16(dc[kk & 1], __float_as_uint(cf[kk][0].x), __float_as_uint(cf[kk][1].x),
+                           __float_as_uint(cf[kk][2].x), __float_as_uint(cf[kk][3].x), qa[kk][0], qa[kk][1]);
+              mma_m16n8k16(dc[2 + (kk & 1)], __float_as_uint(cf[kk][0].y), __float_as_uint(cf[kk][1].y),
+                           __float_as_uint(cf[kk][2].y), __float_as_uint(cf[kk][3].y), qa[kk][0], qa[kk][1]);
+            }
           }
         } else if (do_c) {
 #pragma unroll
@@ -655,7 +660,7 @@ int cl_active_clusters(int S) {
   if (known[dev][S] == 0) {
     const size_t smem = cl_smem_bytes(D, G, S);
     int n = 0;
-    cudaError_t e = cudaFuncSetAttribute(decode_cl_kernel<D, G, C16, EARLY>,
+    cudaError_t e = cudaFuncSetAttribute(decode_cl_kernel<D, G, C16, EARLY, false>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
     if (e == cudaSuccess) {
       cudaLaunchConfig_t cfg{};
@@ -669,7 +674,7 @@ int cl_active_clusters(int S) {
       at[0].val.clusterDim.z = 1;
       cfg.attrs = at;
       cfg.numAttrs = 1;
-      e = cudaOccupancyMaxActiveClusters(&n, decode_cl_kernel<D, G, C16, EARLY>, &cfg);
+      e = cudaOccupancyMaxActiveClusters(&n, decode_cl_kernel<D, G, C16, EARLY, false>, &cfg);
     }
     if (e != cudaSuccess) {
       (void)cudaGetLastError();
@@ -680,13 +685,13 @@ int cl_active_clusters(int S) {
   return known[dev][S];
 }
 
-template <int D, int G, bool C16, bool EARLY>
+template <int D, int G, bool C16, bool EARLY, bool CS>
 cudaError_t launch_cl(const DecodeArgs& args, cudaStream_t stream) {
   DecodeArgs a = args;
   a.S = a.S_cl;
   a.polls = pipeline_poll_limit();
   const size_t smem = cl_smem_bytes(D, G, a.S);
-  cudaError_t e = cudaFuncSetAttribute(decode_cl_kernel<D, G, C16, EARLY>,
+  cudaError_t e = cudaFuncSetAttribute(decode_cl_kernel<D, G, C16, EARLY, CS>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
   const uint64_t rows = (uint64_t)a.batch * a.n_kv * a.cap;  // the cache slabs of all units as one matrix
@@ -708,13 +713,18 @@ cudaError_t launch_cl(const DecodeArgs& args, cudaStream_t stream) {
   at[1].val.clusterDim.z = 1;
   cfg.attrs = at;
   cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, decode_cl_kernel<D, G, C16, EARLY>, a, tmK, tmV);
+  return cudaLaunchKernelEx(&cfg, decode_cl_kernel<D, G, C16, EARLY, CS>, a, tmK, tmV);
 }
 
+// C as fp32, as its bf16 copy, or in the operand form (validation rejects both copies at once)
 template <int D, int G>
 cudaError_t launch_cl_dg(const DecodeArgs& a, cudaStream_t stream) {
-  if (a.early) return a.C16 != nullptr ? launch_cl<D, G, true, true>(a, stream) : launch_cl<D, G, false, true>(a, stream);
-  return a.C16 != nullptr ? launch_cl<D, G, true, false>(a, stream) : launch_cl<D, G, false, false>(a, stream);
+  if (a.early) {
+    if (a.C16 != nullptr) return launch_cl<D, G, true, true, false>(a, stream);
+    return a.Cs != nullptr ? launch_cl<D, G, false, true, true>(a, stream) : launch_cl<D, G, false, true, false>(a, stream);
+  }
+  if (a.C16 != nullptr) return launch_cl<D, G, true, false, false>(a, stream);
+  return a.Cs != nullptr ? launch_cl<D, G, false, false, true>(a, stream) : launch_cl<D, G, false, false, false>(a, stream);
 }
 
 template <int D, int G>
