@@ -146,3 +146,51 @@ def test_clock_samples_and_throttle_reasons():
     assert bench.Clocks.stop(c)["reasons"] == ["hw_slowdown", "sw_thermal_slowdown"]
     c.proc = None
     assert c.stop()["sm_mhz"] is None
+
+
+class _CountingBinding:
+    """Stands in for the binding: counts the kernels each entry point launches
+    (a per-unit compress with T > budget: 9; a decode step, an eviction and a
+    pack of C': 1 each)."""
+    KERNELS = {"mkv_compress": 9, "mkv_decode_step": 1, "mkv_evict_append": 1, "mkv_moments_pack_split": 1}
+
+    def __init__(self):
+        self.launched = 0
+        self.calls = []
+
+    def __getattr__(self, name):
+        def call(*args, **kwargs):
+            self.calls.append(name)
+            self.launched += self.KERNELS[name]
+        return call
+
+
+class _Index:
+    def __getitem__(self, key):
+        return None
+
+
+def test_launch_count_matches_the_parts():
+    """Run.launches() (the bench's gpu_launches claim) equals the kernels one
+    pass over the run's parts launches, with and without periodic eviction."""
+    from paper_2606_01563_gb300.inputs import WORKLOADS
+    for name, B, S, L, every in (("qwen4b_t32k", 128, 512, 3, 0), ("llama8b_t128k", 128, 1024, 2, 64),
+                                 ("llama8b_layer_t8k", 512, 256, 1, 64)):
+        st = type("FakeStack", (), {})()
+        st.wl = WORKLOADS[name]
+        st.G, st.S, st.L = st.wl.geom, S, L
+        st.K = st.V = st.Q = [None] * L
+        st.q = st.kn = st.vn = _Index()
+        r = bench.Run.__new__(bench.Run)
+        fake = _CountingBinding()
+        r.mkv, r.st, r.G, r.B, r.ev_every = fake, st, st.G, B, every
+        r.block = every if every else 64
+        r.g = r.p = r.ws_c = r.ws_d = r.ws_e = r.out = None
+        r.caches, r.moms, r.csplit, r.dps = [None] * L, [None] * L, [None] * L, [None] * L
+        r.final = [None] * S
+        for _, fn in r.parts(st):
+            fn()
+        assert fake.launched == r.launches(), (name, fake.launched, r.launches())
+        # every change of the moments is followed by a pack of that layer's C'
+        changes = sum(c in ("mkv_compress", "mkv_evict_append") for c in fake.calls)
+        assert fake.calls.count("mkv_moments_pack_split") == changes
