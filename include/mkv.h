@@ -387,6 +387,15 @@ MKV_API mkv_status mkv_decode_evict_step(mkv_geom geom, const void* q, const voi
  * Synchronises `stream`, returns the first error a kernel recorded in this
  * workspace since the last call (MKV_OK if none) and clears it.  `info`
  * (host pointer, may be NULL) receives a detail word (e.g. the unit index).
+ *
+ * MKV_ERR_TIMEOUT: a wait on a tile copy or a tensor-core commit ran out
+ * (the poll limit is over a second).  The CTA then stops its pipeline,
+ * contributes an empty state, and before it exits waits again, with the full
+ * limit, for the copies it issued into its shared memory and for its last
+ * commit.  If that wait runs out too, the CTA exits with those copies
+ * possibly still in flight; the status stays MKV_ERR_TIMEOUT.  Outputs of the
+ * call are undefined after any timeout, and after one whose drain also ran
+ * out the CUDA context should not be trusted any more.
  */
 MKV_API mkv_status mkv_get_device_error(void* workspace, void* stream, int32_t* info);
 
