@@ -194,3 +194,23 @@ def test_launch_count_matches_the_parts():
         # every change of the moments is followed by a pack of that layer's C'
         changes = sum(c in ("mkv_compress", "mkv_evict_append") for c in fake.calls)
         assert fake.calls.count("mkv_moments_pack_split") == changes
+
+
+def test_twin_input_set_is_a_distinct_copy():
+    """The end-to-end leg's second input set: the same shapes and contents as
+    the first in separate storage (CPU tensors stand in for device ones)."""
+    import torch
+    from paper_2606_01563_gb300.inputs import WORKLOADS
+    st = bench.Stack.__new__(bench.Stack)
+    st.wl = WORKLOADS["llama8b_layer_t8k"]
+    st.G, st.L, st.S = st.wl.geom, 2, 4
+    g = torch.Generator().manual_seed(0)
+    rnd = lambda *s: torch.randn(*s, generator=g).bfloat16()
+    st.K, st.V, st.Q = [rnd(1, 2, 16, 8) for _ in range(2)], [rnd(1, 2, 16, 8) for _ in range(2)], \
+        [rnd(1, 2, 4, 8) for _ in range(2)]
+    st.q, st.kn, st.vn = rnd(4, 2, 1, 8, 8), rnd(4, 2, 1, 2, 8), rnd(4, 2, 1, 2, 8)
+    tw = st.twin()
+    assert (tw.wl, tw.G, tw.L, tw.S) == (st.wl, st.G, st.L, st.S)
+    assert tw.nbytes() == st.nbytes()
+    for a, b in zip(st.tensors(), tw.tensors()):
+        assert torch.equal(a, b) and a.data_ptr() != b.data_ptr()
